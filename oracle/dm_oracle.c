@@ -1,0 +1,884 @@
+/*
+ * dm_oracle.c -- plain, sequential CPU oracle of DualMap's per-batch routing
+ * (arxiv 2602.06502).  TEST INFRASTRUCTURE ONLY: only the test-suite, the
+ * smoke check and the benchmark's CPU-baseline leg may load this library.
+ * It shares no code, header, table or constant generator with the CUDA path.
+ *
+ * Every step follows the paper's statement of the method, with the details
+ * the paper leaves open fixed as listed below (the same readings the CUDA
+ * path implements; each is argued in the design notes):
+ *
+ *   Hashing (Sec. 3.2 "two independent hash functions over the prompt
+ *   prefix"; App. A.1.1 block-granular prefixes; App. A.3.2 per-block keys):
+ *     key material from SplitMix64(seed), drawn in this order:
+ *       K1[0..B) (low 32 bits of each draw), K2[0..B), G1|1, G2|1,
+ *       S_c, S_r1, S_r2, S_v1, S_v2;
+ *     block k of a prompt (tokens t_0..t_{B-1}) under function f:
+ *       nh^f_k = sum_{i<B/2} ((t_2i + K^f_2i) mod 2^32)((t_2i+1 + K^f_2i+1) mod 2^32)  mod 2^64
+ *       (the NH hash of Black et al., UMAC, CRYPTO 1999),
+ *       d^f_k  = fmix64(nh^f_k + (k+1) G^f)        (MurmurHash3 finaliser),
+ *       P^f_b  = sum_{k<=b} d^f_k  mod 2^64        (chained prefix value),
+ *     cache key of block b: key_b = fmix64(P^1_b xor S_c), 0 replaced by 1;
+ *     only full blocks are keyed (n_blk = floor(L/B));
+ *     route positions: K = min(K_route, n_blk), pos_f = fmix64(P^f_{K-1} xor S_rf).
+ *
+ *   Dual rings (Sec. 3.4; App. A.1.3): each live id owns V virtual nodes per
+ *     ring at vpos_f(id,v) = fmix64(mix64((id<<32)|v) xor S_vf), where mix64
+ *     is one SplitMix64 output step; ring sorted by (vpos, id, v); a position
+ *     p belongs to the first node with vpos >= p, wrapping to the first node
+ *     (arcs (A,B] -> B).
+ *
+ *   Distinct candidates (Sec. 3.2, the unnumbered equation): c1 = owner on
+ *     ring 1; c2 = owner on ring 2, or, if equal, the next live id after c1
+ *     in ascending order, cyclically ((id1+1) mod N for dense ids).
+ *
+ *   Hit length (App. A.3.2): h_f = B * (leading run of keys resident on c_f),
+ *     probed against the index as it was at the start of the batch.
+ *
+ *   TTFT and choice (Sec. 3.2 "SLO-aware strategy"; App. A.1.1 TTFT =
+ *     T_q + T_c): ttft_f = W[c_f] + c*(L - h_f) in integer us, W = queued
+ *     prefill work of the instance.  Equal hits: the less-loaded (by W, tie
+ *     c1).  Otherwise the higher-hit candidate a unless ttft_a > SLO, then
+ *     the less-loaded of the two (tie a), flagged "switched".  Loads update
+ *     in arrival order within the batch; the request joins the chosen
+ *     instance's FIFO queue with work c*(L - h_choice).
+ *
+ *   Time: batch time = arrival of the batch's last request; before routing,
+ *     every instance's queue drains by the elapsed microseconds.
+ *
+ *   Commit (App. A.3.2 "KV cache save"): after route (and rebalance), in
+ *     arrival order, each request touches its keys on its final instance,
+ *     block n_blk-1 down to 0, each with stamp ++clock; an exact LRU of
+ *     capacity C per instance.
+ *
+ *   Rebalance (Sec. 3.3, Eq. "rebalance"; App. A.1.2): hotspots are live
+ *     instances with hot_den*N*W_i > hot_num*sum(W), taken in descending W;
+ *     a queued, not-started request r on hotspot i with alternative j has
+ *     benefit B = TTFT_{r,i} - TTFT_{r,j}, TTFT_{r,i} = work queued up to and
+ *     including r, TTFT_{r,j} = W_j + c*(L - h_{r,j}); candidates sorted by
+ *     (B desc, seq asc); migrate if B > 0 (re-evaluated with current W_j)
+ *     and TTFT_{r,j} < SLO and j is live; stop once i is no longer a
+ *     hotspot.  Single round; a request moves at most once per call.
+ *
+ *   Scaling (Sec. 3.4; App. A.1.3): add inserts V nodes per ring; remove
+ *     deletes them, the instance keeps draining and takes no new work.
+ *
+ * Data structures are the obvious ones: sorted arrays rebuilt from scratch
+ * on every membership change, an LRU as hash map + recency list, queues as
+ * plain arrays.
+ */
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+enum {
+    OR_OK = 0, OR_ERR_INVALID_ARG = 1, OR_ERR_CAPACITY = 2, OR_ERR_NO_INSTANCES = 3,
+    OR_ERR_DUPLICATE_ID = 4, OR_ERR_UNKNOWN_ID = 5, OR_ERR_ORDER = 6, OR_ERR_OOM = 9
+};
+
+/* ------------------------------------------------------------------ */
+/* Published primitives                                                */
+/* ------------------------------------------------------------------ */
+
+/* SplitMix64 (Steele, Lea, Flood 2014): advance the state, return output. */
+uint64_t or_splitmix64_next(uint64_t *state)
+{
+    uint64_t z = (*state += 0x9E3779B97F4A7C15ULL);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+/* One SplitMix64 output step taken from state x (stateless mixer). */
+uint64_t or_mix64(uint64_t x)
+{
+    uint64_t s = x;
+    return or_splitmix64_next(&s);
+}
+
+/* MurmurHash3 64-bit finaliser (Appleby, public domain). */
+uint64_t or_fmix64(uint64_t k)
+{
+    k ^= k >> 33;
+    k *= 0xff51afd7ed558ccdULL;
+    k ^= k >> 33;
+    k *= 0xc4ceb9fe1a85ec53ULL;
+    k ^= k >> 33;
+    return k;
+}
+
+/* NH over one block of B tokens (B even) under key K. */
+uint64_t or_nh(const uint32_t *t, const uint32_t *K, uint32_t B)
+{
+    uint64_t s = 0;
+    for (uint32_t i = 0; i < B / 2; i++) {
+        uint32_t a = t[2 * i] + K[2 * i];          /* mod 2^32 */
+        uint32_t b = t[2 * i + 1] + K[2 * i + 1];  /* mod 2^32 */
+        s += (uint64_t)a * (uint64_t)b;            /* mod 2^64 */
+    }
+    return s;
+}
+
+/* ------------------------------------------------------------------ */
+/* Configuration and state                                             */
+/* ------------------------------------------------------------------ */
+
+typedef struct {
+    uint32_t block_tokens;
+    uint32_t route_prefix_blocks;
+    uint32_t vnodes_per_instance;
+    uint32_t max_instances;
+    uint64_t cache_capacity_blocks;
+    uint64_t slo_us;
+    uint32_t cost_us_per_token;
+    uint32_t hot_num, hot_den;
+    uint32_t max_batch;
+    uint64_t max_batch_tokens;
+    uint64_t seed;
+} or_config;
+
+typedef struct {
+    uint64_t key, stamp;
+    int64_t newer, older;   /* recency list */
+    int64_t chain;          /* bucket chain */
+} lru_node;
+
+typedef struct {
+    lru_node *nodes;
+    int64_t n_nodes, cap_nodes, free_head;
+    int64_t *bucket;
+    uint64_t nbucket;       /* power of two */
+    int64_t mru, lru;
+    uint64_t size;
+} lru_t;
+
+typedef struct {
+    uint64_t seq;
+    uint32_t L, c1, c2, h1, h2;
+    uint64_t work, remaining;
+    uint64_t moved_in_call;  /* rebalance call id that moved it here; 0 = none */
+} q_entry;
+
+typedef struct {
+    q_entry *e;
+    uint64_t head, len, cap;  /* entries e[head .. head+len) */
+} queue_t;
+
+typedef struct {
+    uint64_t pos;
+    uint32_t id, v;
+} vnode;
+
+enum { INST_ABSENT = 0, INST_LIVE = 1, INST_DRAINING = 2 };
+
+typedef struct {
+    or_config cfg;
+    uint32_t K1[64], K2[64];
+    uint64_t G1, G2, Sc, Sr1, Sr2, Sv1, Sv2;
+    uint8_t *state;     /* per id: absent / live / draining */
+    uint64_t *W;        /* queued work per id */
+    queue_t *q;
+    lru_t *cache;
+    vnode *ring[2];
+    uint32_t ring_len;
+    uint64_t clock, next_seq, t_prev;
+    int have_time;
+    uint64_t rebalance_calls;
+    /* the last routed batch, kept for commit */
+    uint32_t pend_n;
+    uint64_t pend_seq0;
+    uint32_t *pend_final, *pend_nblk;
+    uint64_t **pend_keys;
+    int pending;
+} or_state;
+
+/* ------------------------------------------------------------------ */
+/* LRU: hash map key -> node, doubly linked recency list               */
+/* ------------------------------------------------------------------ */
+
+static uint64_t lru_bucket_of(const lru_t *c, uint64_t key)
+{
+    return (key ^ (key >> 29)) & (c->nbucket - 1);
+}
+
+static void lru_free(lru_t *c)
+{
+    free(c->nodes);
+    free(c->bucket);
+    memset(c, 0, sizeof *c);
+}
+
+static int lru_init(lru_t *c)
+{
+    memset(c, 0, sizeof *c);
+    c->nbucket = 1024;
+    c->bucket = (int64_t *)malloc(c->nbucket * sizeof(int64_t));
+    if (!c->bucket) return OR_ERR_OOM;
+    for (uint64_t i = 0; i < c->nbucket; i++) c->bucket[i] = -1;
+    c->mru = c->lru = -1;
+    c->free_head = -1;
+    return OR_OK;
+}
+
+static int64_t lru_find(const lru_t *c, uint64_t key)
+{
+    int64_t i = c->bucket[lru_bucket_of(c, key)];
+    while (i >= 0 && c->nodes[i].key != key) i = c->nodes[i].chain;
+    return i;
+}
+
+static void lru_unlink(lru_t *c, int64_t i)
+{
+    lru_node *n = &c->nodes[i];
+    if (n->newer >= 0) c->nodes[n->newer].older = n->older; else c->mru = n->older;
+    if (n->older >= 0) c->nodes[n->older].newer = n->newer; else c->lru = n->newer;
+    n->newer = n->older = -1;
+}
+
+static void lru_push_mru(lru_t *c, int64_t i)
+{
+    lru_node *n = &c->nodes[i];
+    n->newer = -1;
+    n->older = c->mru;
+    if (c->mru >= 0) c->nodes[c->mru].newer = i;
+    c->mru = i;
+    if (c->lru < 0) c->lru = i;
+}
+
+static int lru_grow_buckets(lru_t *c)
+{
+    uint64_t nb = c->nbucket * 2;
+    int64_t *b = (int64_t *)malloc(nb * sizeof(int64_t));
+    if (!b) return OR_ERR_OOM;
+    for (uint64_t i = 0; i < nb; i++) b[i] = -1;
+    free(c->bucket);
+    c->bucket = b;
+    c->nbucket = nb;
+    /* re-chain every live node (walk the recency list) */
+    for (int64_t i = c->mru; i >= 0; i = c->nodes[i].older) {
+        uint64_t h = lru_bucket_of(c, c->nodes[i].key);
+        c->nodes[i].chain = c->bucket[h];
+        c->bucket[h] = i;
+    }
+    return OR_OK;
+}
+
+static void lru_remove(lru_t *c, int64_t i)
+{
+    uint64_t h = lru_bucket_of(c, c->nodes[i].key);
+    int64_t *link = &c->bucket[h];
+    while (*link != i) link = &c->nodes[*link].chain;
+    *link = c->nodes[i].chain;
+    lru_unlink(c, i);
+    c->nodes[i].chain = c->free_head;
+    c->free_head = i;
+    c->size--;
+}
+
+/* Touch `key` with `stamp` (insert if absent), then evict least recent
+ * entries until at most `cap` remain.  This is the textbook LRU. */
+static int lru_touch(lru_t *c, uint64_t key, uint64_t stamp, uint64_t cap)
+{
+    int64_t i = lru_find(c, key);
+    if (i >= 0) {
+        lru_unlink(c, i);
+    } else {
+        if (c->free_head >= 0) {
+            i = c->free_head;
+            c->free_head = c->nodes[i].chain;
+        } else {
+            if (c->n_nodes == c->cap_nodes) {
+                int64_t nc = c->cap_nodes ? 2 * c->cap_nodes : 1024;
+                lru_node *nn = (lru_node *)realloc(c->nodes, (size_t)nc * sizeof(lru_node));
+                if (!nn) return OR_ERR_OOM;
+                c->nodes = nn;
+                c->cap_nodes = nc;
+            }
+            i = c->n_nodes++;
+        }
+        c->nodes[i].key = key;
+        uint64_t h = lru_bucket_of(c, key);
+        c->nodes[i].chain = c->bucket[h];
+        c->bucket[h] = i;
+        c->size++;
+    }
+    c->nodes[i].stamp = stamp;
+    lru_push_mru(c, i);
+    if (c->size > c->nbucket) {     /* rehash walks the recency list: after linking */
+        int rc = lru_grow_buckets(c);
+        if (rc) return rc;
+    }
+    while (c->size > cap) lru_remove(c, c->lru);
+    return OR_OK;
+}
+
+static void lru_clear(lru_t *c)
+{
+    lru_free(c);
+    lru_init(c);
+}
+
+/* ------------------------------------------------------------------ */
+/* Key material, prompt hashing                                        */
+/* ------------------------------------------------------------------ */
+
+void or_derive_keys(uint64_t seed, uint32_t B, uint32_t *K1, uint32_t *K2, uint64_t *scalars)
+{
+    uint64_t s = seed;
+    for (uint32_t j = 0; j < B; j++) K1[j] = (uint32_t)or_splitmix64_next(&s);
+    for (uint32_t j = 0; j < B; j++) K2[j] = (uint32_t)or_splitmix64_next(&s);
+    scalars[0] = or_splitmix64_next(&s) | 1ULL; /* G1 */
+    scalars[1] = or_splitmix64_next(&s) | 1ULL; /* G2 */
+    for (int j = 2; j < 7; j++) scalars[j] = or_splitmix64_next(&s); /* Sc Sr1 Sr2 Sv1 Sv2 */
+}
+
+/* All block keys of one prompt (n_blk of them) and its two ring positions.
+ * Returns n_blk.  The per-block digests are summed in block order. */
+static uint32_t prompt_keys(const or_state *s, const uint32_t *tok, uint32_t L,
+                            uint64_t *keys, uint64_t *pos)
+{
+    const uint32_t B = s->cfg.block_tokens;
+    const uint32_t nblk = L / B;
+    uint32_t K = s->cfg.route_prefix_blocks < nblk ? s->cfg.route_prefix_blocks : nblk;
+    uint64_t P1 = 0, P2 = 0;
+    for (uint32_t k = 0; k < nblk; k++) {
+        const uint32_t *t = tok + (uint64_t)k * B;
+        uint64_t d1 = or_fmix64(or_nh(t, s->K1, B) + (uint64_t)(k + 1) * s->G1);
+        P1 += d1;
+        uint64_t key = or_fmix64(P1 ^ s->Sc);
+        keys[k] = key ? key : 1;
+        if (k < K) {
+            uint64_t d2 = or_fmix64(or_nh(t, s->K2, B) + (uint64_t)(k + 1) * s->G2);
+            P2 += d2;
+            if (k == K - 1) {
+                pos[0] = or_fmix64(P1 ^ s->Sr1);
+                pos[1] = or_fmix64(P2 ^ s->Sr2);
+            }
+        }
+    }
+    return nblk;
+}
+
+/* ------------------------------------------------------------------ */
+/* Rings                                                               */
+/* ------------------------------------------------------------------ */
+
+static int vnode_cmp(const void *a, const void *b)
+{
+    const vnode *x = (const vnode *)a, *y = (const vnode *)b;
+    if (x->pos != y->pos) return x->pos < y->pos ? -1 : 1;
+    if (x->id != y->id) return x->id < y->id ? -1 : 1;
+    if (x->v != y->v) return x->v < y->v ? -1 : 1;
+    return 0;
+}
+
+uint64_t or_vnode_pos(uint64_t Sv, uint32_t id, uint32_t v)
+{
+    return or_fmix64(or_mix64(((uint64_t)id << 32) | v) ^ Sv);
+}
+
+/* Index of the first entry with vpos >= p in a sorted array, 0 if none. */
+uint32_t or_ring_successor(const uint64_t *vpos, uint32_t R, uint64_t p)
+{
+    uint32_t lo = 0, hi = R;          /* answer in [lo, hi] */
+    while (lo < hi) {
+        uint32_t mid = lo + (hi - lo) / 2;
+        if (vpos[mid] < p) lo = mid + 1; else hi = mid;
+    }
+    return lo == R ? 0 : lo;
+}
+
+static uint32_t ring_owner(const or_state *s, int f, uint64_t p)
+{
+    /* binary search over the vnode records (same rule as or_ring_successor) */
+    const vnode *r = s->ring[f];
+    uint32_t lo = 0, hi = s->ring_len;
+    while (lo < hi) {
+        uint32_t mid = lo + (hi - lo) / 2;
+        if (r[mid].pos < p) lo = mid + 1; else hi = mid;
+    }
+    return r[lo == s->ring_len ? 0 : lo].id;
+}
+
+static int rebuild_rings(or_state *s)
+{
+    uint32_t n = 0;
+    for (uint32_t id = 0; id < s->cfg.max_instances; id++)
+        if (s->state[id] == INST_LIVE) n++;
+    uint32_t R = n * s->cfg.vnodes_per_instance;
+    for (int f = 0; f < 2; f++) {
+        free(s->ring[f]);
+        s->ring[f] = (vnode *)malloc((size_t)(R ? R : 1) * sizeof(vnode));
+        if (!s->ring[f]) return OR_ERR_OOM;
+        uint64_t Sv = f == 0 ? s->Sv1 : s->Sv2;
+        uint32_t k = 0;
+        for (uint32_t id = 0; id < s->cfg.max_instances; id++) {
+            if (s->state[id] != INST_LIVE) continue;
+            for (uint32_t v = 0; v < s->cfg.vnodes_per_instance; v++) {
+                s->ring[f][k].pos = or_vnode_pos(Sv, id, v);
+                s->ring[f][k].id = id;
+                s->ring[f][k].v = v;
+                k++;
+            }
+        }
+        qsort(s->ring[f], R, sizeof(vnode), vnode_cmp);
+    }
+    s->ring_len = R;
+    return OR_OK;
+}
+
+static uint32_t n_live(const or_state *s)
+{
+    uint32_t n = 0;
+    for (uint32_t id = 0; id < s->cfg.max_instances; id++) n += s->state[id] == INST_LIVE;
+    return n;
+}
+
+/* Next live id after `id` in ascending order, cyclically. */
+static uint32_t next_live_after(const or_state *s, uint32_t id)
+{
+    uint32_t M = s->cfg.max_instances;
+    for (uint32_t k = 1; k <= M; k++) {
+        uint32_t j = (id + k) % M;
+        if (s->state[j] == INST_LIVE) return j;
+    }
+    return id;
+}
+
+/* ------------------------------------------------------------------ */
+/* Queues                                                              */
+/* ------------------------------------------------------------------ */
+
+static int q_push(queue_t *q, const q_entry *x)
+{
+    if (q->head + q->len == q->cap) {
+        if (q->head > 0) {  /* slide to the front */
+            memmove(q->e, q->e + q->head, q->len * sizeof(q_entry));
+            q->head = 0;
+        }
+        if (q->len == q->cap) {
+            uint64_t nc = q->cap ? 2 * q->cap : 64;
+            q_entry *ne = (q_entry *)realloc(q->e, nc * sizeof(q_entry));
+            if (!ne) return OR_ERR_OOM;
+            q->e = ne;
+            q->cap = nc;
+        }
+    }
+    q->e[q->head + q->len] = *x;
+    q->len++;
+    return OR_OK;
+}
+
+/* Remove the entry at position k (0 = head) keeping order. */
+static void q_erase(queue_t *q, uint64_t k)
+{
+    q_entry *b = q->e + q->head;
+    memmove(b + k, b + k + 1, (q->len - k - 1) * sizeof(q_entry));
+    q->len--;
+}
+
+/* Run `delta` microseconds of prefill work off the head of the queue. */
+static void q_drain(queue_t *q, uint64_t *W, uint64_t delta)
+{
+    while (q->len > 0) {
+        q_entry *h = &q->e[q->head];
+        if (h->remaining <= delta) {
+            delta -= h->remaining;
+            *W -= h->remaining;
+            q->head++;
+            q->len--;
+        } else {
+            h->remaining -= delta;
+            *W -= delta;
+            break;
+        }
+    }
+    if (q->len == 0) q->head = 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Lifecycle                                                           */
+/* ------------------------------------------------------------------ */
+
+static void clear_pending(or_state *s)
+{
+    if (s->pend_keys)
+        for (uint32_t i = 0; i < s->pend_n; i++) free(s->pend_keys[i]);
+    free(s->pend_keys);
+    free(s->pend_final);
+    free(s->pend_nblk);
+    s->pend_keys = NULL;
+    s->pend_final = s->pend_nblk = NULL;
+    s->pend_n = 0;
+    s->pending = 0;
+}
+
+void or_destroy(or_state *s)
+{
+    if (!s) return;
+    clear_pending(s);
+    for (uint32_t i = 0; i < s->cfg.max_instances; i++) {
+        if (s->cache) lru_free(&s->cache[i]);
+        if (s->q) free(s->q[i].e);
+    }
+    free(s->cache);
+    free(s->q);
+    free(s->W);
+    free(s->state);
+    free(s->ring[0]);
+    free(s->ring[1]);
+    free(s);
+}
+
+int or_create(const or_config *cfg, or_state **out)
+{
+    *out = NULL;
+    uint32_t B = cfg->block_tokens;
+    if (B < 2 || B > 64 || (B & 1) || cfg->route_prefix_blocks < 1 ||
+        cfg->vnodes_per_instance < 1 || cfg->max_instances < 2 ||
+        cfg->cache_capacity_blocks < 1 || cfg->cost_us_per_token < 1 ||
+        cfg->hot_den < 1 || cfg->max_batch < 1 || cfg->max_batch_tokens < B)
+        return OR_ERR_INVALID_ARG;
+    or_state *s = (or_state *)calloc(1, sizeof(or_state));
+    if (!s) return OR_ERR_OOM;
+    s->cfg = *cfg;
+    uint64_t sc[7];
+    or_derive_keys(cfg->seed, B, s->K1, s->K2, sc);
+    s->G1 = sc[0]; s->G2 = sc[1]; s->Sc = sc[2]; s->Sr1 = sc[3]; s->Sr2 = sc[4];
+    s->Sv1 = sc[5]; s->Sv2 = sc[6];
+    uint32_t M = cfg->max_instances;
+    s->state = (uint8_t *)calloc(M, 1);
+    s->W = (uint64_t *)calloc(M, sizeof(uint64_t));
+    s->q = (queue_t *)calloc(M, sizeof(queue_t));
+    s->cache = (lru_t *)calloc(M, sizeof(lru_t));
+    if (!s->state || !s->W || !s->q || !s->cache) { or_destroy(s); return OR_ERR_OOM; }
+    for (uint32_t i = 0; i < M; i++)
+        if (lru_init(&s->cache[i])) { or_destroy(s); return OR_ERR_OOM; }
+    if (rebuild_rings(s)) { or_destroy(s); return OR_ERR_OOM; }
+    *out = s;
+    return OR_OK;
+}
+
+int or_add_instance(or_state *s, uint32_t id)
+{
+    if (id >= s->cfg.max_instances) return OR_ERR_INVALID_ARG;
+    if (s->state[id] == INST_LIVE) return OR_ERR_DUPLICATE_ID;
+    if (s->state[id] == INST_DRAINING && s->q[id].len > 0) return OR_ERR_DUPLICATE_ID;
+    s->state[id] = INST_LIVE;
+    lru_clear(&s->cache[id]);   /* a (re-)added instance starts with an empty index */
+    s->W[id] = 0;
+    return rebuild_rings(s);
+}
+
+int or_remove_instance(or_state *s, uint32_t id)
+{
+    if (id >= s->cfg.max_instances || s->state[id] != INST_LIVE) return OR_ERR_UNKNOWN_ID;
+    s->state[id] = INST_DRAINING;
+    return rebuild_rings(s);
+}
+
+/* ------------------------------------------------------------------ */
+/* The routing step                                                     */
+/* ------------------------------------------------------------------ */
+
+/* SLO-aware choice between the two candidates (Sec. 3.2).  Returns the
+ * chosen id and sets *switched when the SLO rule overrode cache affinity. */
+uint32_t or_choose(uint32_t c1, uint32_t c2, uint32_t h1, uint32_t h2, uint32_t L,
+                   uint64_t W1, uint64_t W2, uint64_t slo, uint32_t cost,
+                   uint64_t *ttft1, uint64_t *ttft2, uint8_t *switched)
+{
+    *ttft1 = W1 + (uint64_t)cost * (L - h1);
+    *ttft2 = W2 + (uint64_t)cost * (L - h2);
+    *switched = 0;
+    if (h1 == h2) return W2 < W1 ? c2 : c1;
+    int a_is_1 = h1 > h2;
+    uint64_t ttft_a = a_is_1 ? *ttft1 : *ttft2;
+    uint64_t Wa = a_is_1 ? W1 : W2, Wb = a_is_1 ? W2 : W1;
+    uint32_t a = a_is_1 ? c1 : c2, b = a_is_1 ? c2 : c1;
+    if (ttft_a <= slo) return a;
+    *switched = 1;
+    return Wb < Wa ? b : a;
+}
+
+static uint32_t leading_hits(const lru_t *c, const uint64_t *keys, uint32_t nblk)
+{
+    uint32_t m = 0;
+    while (m < nblk && lru_find(c, keys[m]) >= 0) m++;
+    return m;
+}
+
+int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
+                   const uint32_t *lengths, uint32_t n, uint64_t t_batch,
+                   uint32_t *cand1, uint32_t *cand2, uint32_t *hit1, uint32_t *hit2,
+                   uint64_t *ttft1, uint64_t *ttft2, uint32_t *chosen, uint8_t *switched)
+{
+    const or_config *cf = &s->cfg;
+    if (n > cf->max_batch) return OR_ERR_CAPACITY;
+    if (n_live(s) < 2) return OR_ERR_NO_INSTANCES;
+    if (s->have_time && t_batch < s->t_prev) return OR_ERR_ORDER;
+    uint64_t total = 0;
+    for (uint32_t r = 0; r < n; r++) {
+        if (lengths[r] < cf->block_tokens) return OR_ERR_INVALID_ARG;
+        total += lengths[r];
+    }
+    if (total > cf->max_batch_tokens) return OR_ERR_CAPACITY;
+
+    /* time advances; every instance's queue runs for the elapsed us */
+    uint64_t delta = s->have_time ? t_batch - s->t_prev : 0;
+    for (uint32_t id = 0; id < cf->max_instances; id++)
+        if (s->state[id] != INST_ABSENT) q_drain(&s->q[id], &s->W[id], delta);
+    s->t_prev = t_batch;
+    s->have_time = 1;
+
+    clear_pending(s);
+    s->pend_n = n;
+    s->pend_seq0 = s->next_seq;
+    s->pend_final = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
+    s->pend_nblk = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
+    s->pend_keys = (uint64_t **)calloc(n ? n : 1, sizeof(uint64_t *));
+    if (!s->pend_final || !s->pend_nblk || !s->pend_keys) return OR_ERR_OOM;
+
+    /* 1) hash, ring lookup, distinct fix, probes: all against batch-start state */
+    for (uint32_t r = 0; r < n; r++) {
+        uint32_t L = lengths[r];
+        uint64_t *keys = (uint64_t *)malloc((size_t)(L / cf->block_tokens) * sizeof(uint64_t));
+        if (!keys) return OR_ERR_OOM;
+        uint64_t pos[2];
+        uint32_t nblk = prompt_keys(s, tokens + offsets[r], L, keys, pos);
+        s->pend_keys[r] = keys;
+        s->pend_nblk[r] = nblk;
+        uint32_t c1 = ring_owner(s, 0, pos[0]);
+        uint32_t c2 = ring_owner(s, 1, pos[1]);
+        if (c2 == c1) c2 = next_live_after(s, c1);
+        cand1[r] = c1;
+        cand2[r] = c2;
+        hit1[r] = cf->block_tokens * leading_hits(&s->cache[c1], keys, nblk);
+        hit2[r] = cf->block_tokens * leading_hits(&s->cache[c2], keys, nblk);
+    }
+    /* 2) choices in arrival order; loads update as we go */
+    for (uint32_t r = 0; r < n; r++) {
+        uint32_t c1 = cand1[r], c2 = cand2[r];
+        uint32_t ch = or_choose(c1, c2, hit1[r], hit2[r], lengths[r], s->W[c1], s->W[c2],
+                                cf->slo_us, cf->cost_us_per_token, &ttft1[r], &ttft2[r],
+                                &switched[r]);
+        chosen[r] = ch;
+        uint32_t hch = ch == c1 ? hit1[r] : hit2[r];
+        q_entry e;
+        e.seq = s->next_seq++;
+        e.L = lengths[r]; e.c1 = c1; e.c2 = c2; e.h1 = hit1[r]; e.h2 = hit2[r];
+        e.work = e.remaining = (uint64_t)cf->cost_us_per_token * (lengths[r] - hch);
+        e.moved_in_call = 0;
+        if (q_push(&s->q[ch], &e)) return OR_ERR_OOM;
+        s->W[ch] += e.work;
+        s->pend_final[r] = ch;
+    }
+    s->pending = 1;
+    return OR_OK;
+}
+
+int or_commit(or_state *s)
+{
+    if (!s->pending) return OR_OK;
+    for (uint32_t r = 0; r < s->pend_n; r++) {
+        lru_t *c = &s->cache[s->pend_final[r]];
+        const uint64_t *keys = s->pend_keys[r];
+        for (uint32_t b = s->pend_nblk[r]; b-- > 0;) {
+            int rc = lru_touch(c, keys[b], ++s->clock, s->cfg.cache_capacity_blocks);
+            if (rc) return rc;
+        }
+    }
+    clear_pending(s);
+    return OR_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* Hotspot-aware rebalancing (Sec. 3.3)                                 */
+/* ------------------------------------------------------------------ */
+
+typedef struct {
+    int64_t benefit;
+    uint64_t seq;
+    uint64_t ttft_i;
+} mig_cand;
+
+static int mig_cmp(const void *a, const void *b)
+{
+    const mig_cand *x = (const mig_cand *)a, *y = (const mig_cand *)b;
+    if (x->benefit != y->benefit) return x->benefit > y->benefit ? -1 : 1;
+    if (x->seq != y->seq) return x->seq < y->seq ? -1 : 1;
+    return 0;
+}
+
+static int is_hot(const or_state *s, uint32_t i, uint64_t sumW, uint32_t N)
+{
+    /* hot_den * N * W_i > hot_num * sum(W), in 128-bit-safe form */
+    unsigned __int128 lhs = (unsigned __int128)s->cfg.hot_den * N * s->W[i];
+    unsigned __int128 rhs = (unsigned __int128)s->cfg.hot_num * sumW;
+    return lhs > rhs;
+}
+
+int or_rebalance(or_state *s, uint64_t *mig_seq, uint32_t *mig_from, uint32_t *mig_to,
+                 uint32_t cap, uint32_t *n_out)
+{
+    const or_config *cf = &s->cfg;
+    const uint32_t M = cf->max_instances;
+    uint64_t call = ++s->rebalance_calls;
+    uint32_t nmig = 0;
+    uint32_t N = n_live(s);
+    uint64_t sumW = 0;
+    for (uint32_t i = 0; i < M; i++) if (s->state[i] == INST_LIVE) sumW += s->W[i];
+
+    /* hotspots at the start of the call, by W descending, then id */
+    uint32_t *hot = (uint32_t *)malloc(M * sizeof(uint32_t));
+    if (!hot) return OR_ERR_OOM;
+    uint32_t nh = 0;
+    for (uint32_t i = 0; i < M; i++)
+        if (s->state[i] == INST_LIVE && is_hot(s, i, sumW, N)) hot[nh++] = i;
+    for (uint32_t a = 1; a < nh; a++) {      /* insertion sort, stable by id */
+        uint32_t x = hot[a], b = a;
+        while (b > 0 && s->W[hot[b - 1]] < s->W[x]) { hot[b] = hot[b - 1]; b--; }
+        hot[b] = x;
+    }
+
+    for (uint32_t hi = 0; hi < nh; hi++) {
+        uint32_t i = hot[hi];
+        queue_t *q = &s->q[i];
+        mig_cand *cand = (mig_cand *)malloc((q->len ? q->len : 1) * sizeof(mig_cand));
+        if (!cand) { free(hot); return OR_ERR_OOM; }
+        uint32_t nc = 0;
+        uint64_t ahead = 0;
+        for (uint64_t k = 0; k < q->len; k++) {
+            const q_entry *e = &q->e[q->head + k];
+            uint64_t ttft_i = ahead + e->remaining;   /* T_q + T_c on i */
+            ahead += e->remaining;
+            if (e->remaining != e->work || e->moved_in_call == call) continue;
+            uint32_t j = e->c1 == i ? e->c2 : e->c1;
+            uint32_t hj = j == e->c1 ? e->h1 : e->h2;
+            uint64_t ttft_j = s->W[j] + (uint64_t)cf->cost_us_per_token * (e->L - hj);
+            cand[nc].benefit = (int64_t)(ttft_i - ttft_j);
+            cand[nc].seq = e->seq;
+            cand[nc].ttft_i = ttft_i;
+            nc++;
+        }
+        qsort(cand, nc, sizeof(mig_cand), mig_cmp);
+        for (uint32_t a = 0; a < nc; a++) {
+            if (!is_hot(s, i, sumW, N)) break;
+            /* find the entry again (its position may have shifted) */
+            uint64_t k = 0;
+            while (k < q->len && q->e[q->head + k].seq != cand[a].seq) k++;
+            q_entry e = q->e[q->head + k];
+            uint32_t j = e.c1 == i ? e.c2 : e.c1;
+            if (s->state[j] != INST_LIVE) continue;
+            uint32_t hj = j == e.c1 ? e.h1 : e.h2;
+            uint64_t new_work = (uint64_t)cf->cost_us_per_token * (e.L - hj);
+            uint64_t ttft_j = s->W[j] + new_work;
+            if (!(cand[a].ttft_i > ttft_j && ttft_j < cf->slo_us)) continue;
+            q_erase(q, k);
+            s->W[i] -= e.work;
+            sumW -= e.work;
+            e.work = e.remaining = new_work;
+            e.moved_in_call = call;
+            if (q_push(&s->q[j], &e)) { free(cand); free(hot); return OR_ERR_OOM; }
+            s->W[j] += new_work;
+            sumW += new_work;
+            if (s->pending && e.seq >= s->pend_seq0 && e.seq < s->pend_seq0 + s->pend_n)
+                s->pend_final[e.seq - s->pend_seq0] = j;
+            if (nmig < cap) {
+                mig_seq[nmig] = e.seq;
+                mig_from[nmig] = i;
+                mig_to[nmig] = j;
+            }
+            nmig++;
+        }
+        free(cand);
+    }
+    free(hot);
+    *n_out = nmig;
+    return OR_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* Introspection (tests)                                               */
+/* ------------------------------------------------------------------ */
+
+void or_get_loads(const or_state *s, uint64_t *W) { memcpy(W, s->W, s->cfg.max_instances * sizeof(uint64_t)); }
+
+void or_get_state(const or_state *s, uint8_t *st) { memcpy(st, s->state, s->cfg.max_instances); }
+
+uint64_t or_clock(const or_state *s) { return s->clock; }
+
+void or_key_material(const or_state *s, uint32_t *K1, uint32_t *K2, uint64_t *scalars)
+{
+    memcpy(K1, s->K1, s->cfg.block_tokens * sizeof(uint32_t));
+    memcpy(K2, s->K2, s->cfg.block_tokens * sizeof(uint32_t));
+    uint64_t v[7] = {s->G1, s->G2, s->Sc, s->Sr1, s->Sr2, s->Sv1, s->Sv2};
+    memcpy(scalars, v, sizeof v);
+}
+
+/* Keys and route positions of one prompt under this state's key material. */
+uint32_t or_prompt_keys(const or_state *s, const uint32_t *tok, uint32_t L, uint64_t *keys, uint64_t *pos)
+{
+    pos[0] = pos[1] = 0;
+    if (L < s->cfg.block_tokens) return 0;
+    return prompt_keys(s, tok, L, keys, pos);
+}
+
+/* Raw ring owners of positions (before the distinct fix). */
+void or_ring_owners(const or_state *s, const uint64_t *pos, uint32_t n, int f, uint32_t *owner)
+{
+    for (uint32_t i = 0; i < n; i++) owner[i] = ring_owner(s, f, pos[i]);
+}
+
+uint32_t or_ring_dump(const or_state *s, int f, uint64_t *vpos, uint32_t *owner, uint32_t *vidx)
+{
+    for (uint32_t k = 0; k < s->ring_len; k++) {
+        if (vpos) vpos[k] = s->ring[f][k].pos;
+        if (owner) owner[k] = s->ring[f][k].id;
+        if (vidx) vidx[k] = s->ring[f][k].v;
+    }
+    return s->ring_len;
+}
+
+uint32_t or_next_live(const or_state *s, uint32_t id) { return next_live_after(s, id); }
+
+/* Resident keys of an instance, most recent first. */
+uint64_t or_cache_dump(const or_state *s, uint32_t id, uint64_t *keys, uint64_t *stamps, uint64_t cap)
+{
+    const lru_t *c = &s->cache[id];
+    uint64_t k = 0;
+    for (int64_t i = c->mru; i >= 0; i = c->nodes[i].older, k++)
+        if (k < cap) { keys[k] = c->nodes[i].key; stamps[k] = c->nodes[i].stamp; }
+    return c->size;
+}
+
+/* Queue of an instance, head first: seq, work, remaining per entry. */
+uint64_t or_queue_dump(const or_state *s, uint32_t id, uint64_t *seq, uint64_t *work,
+                       uint64_t *remaining, uint64_t cap)
+{
+    const queue_t *q = &s->q[id];
+    for (uint64_t k = 0; k < q->len && k < cap; k++) {
+        seq[k] = q->e[q->head + k].seq;
+        work[k] = q->e[q->head + k].work;
+        remaining[k] = q->e[q->head + k].remaining;
+    }
+    return q->len;
+}
+
+/* Append a hand-built entry to an instance's queue (test set-up). */
+int or_debug_enqueue(or_state *s, uint32_t id, uint64_t seq, uint32_t L, uint32_t c1, uint32_t c2,
+                     uint32_t h1, uint32_t h2, uint64_t work, uint64_t remaining)
+{
+    if (id >= s->cfg.max_instances) return OR_ERR_INVALID_ARG;
+    q_entry e = {seq, L, c1, c2, h1, h2, work, remaining, 0};
+    int rc = q_push(&s->q[id], &e);
+    if (!rc) s->W[id] += remaining;
+    if (seq >= s->next_seq) s->next_seq = seq + 1;
+    return rc;
+}
+
+/* Touch one key on one instance's LRU (test set-up of cache contents). */
+int or_debug_touch(or_state *s, uint32_t id, uint64_t key)
+{
+    if (id >= s->cfg.max_instances) return OR_ERR_INVALID_ARG;
+    return lru_touch(&s->cache[id], key, ++s->clock, s->cfg.cache_capacity_blocks);
+}
