@@ -1,0 +1,390 @@
+"""Benchmark of the DualMap batched routing path on GB300.
+
+One step = one batch through the whole path: queue drain, prompt hashing,
+dual-ring lookup + cache probes, SLO-aware choice, (rebalance when the
+workload has it) and the LRU cache commit.  Default workload: the
+long-context stress shape (128 instances, 512 prompts of 32,768-131,072
+uint32 tokens per batch, 64 shared 16k-token prefixes, Zipf 0.8), inputs
+resident in HBM (each batch ~168 MB, larger than L2).
+
+Prints one JSON line: routed requests/s (value), prompt GB/s hashed+probed,
+the hashing kernel's HBM roofline, the end-to-end number through the
+host-buffer entry point, the CPU oracle baseline and the SM clocks seen.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl dualmap|reference]
+  torchrun --nproc-per-node N bench.py --gpus N ...   (N independent replicas)
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "routed req/s & prompt GB/s hashed+probed on 1 GB300; % HBM roofline"
+HASH_SRC = os.path.join(ROOT, "paper_2602_06502_gb300", "csrc", "dm_hash.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "hash_longctx_traffic.json")
+
+
+def longctx_handle_kwargs(w):
+    """Handle sizes used for the long-context workload (bench and its parity test)."""
+    return dict(max_instances=w["n_instances"] + 8, max_batch=w["batch"],
+                max_batch_tokens=w["batch"] * w["len_hi"] + 4 * w["batch"],
+                max_touch_per_instance=1 << 20)
+
+
+def handle_kwargs(w, max_id):
+    if w["name"] == "longctx":
+        return longctx_handle_kwargs(w)
+    mb = w["batch"] * (w.get("len_hi") or w.get("max_prompt") or (w.get("prefix_hi", 0) + w.get("uniq_hi", 0)))
+    return dict(max_instances=max_id + 9, max_batch=w["batch"], max_batch_tokens=mb + 4 * w["batch"],
+                max_touch_per_instance=min(mb // w["block_tokens"], 1 << 21))
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def file_sha(p):
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def traffic_per_launch():
+    """DRAM bytes per hashing launch from the committed ncu capture, or None
+    when the kernel source changed since it was taken."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            t = json.load(f)
+        if t.get("dm_hash_sha256") != file_sha(HASH_SRC):
+            return None
+        return float(t["bytes_per_launch_full_batch"])
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled in the background."""
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index):
+        self.rows = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                          "-i", str(dev_index), "-lms", "50"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+            self.th = threading.Thread(target=self._read, daemon=True)
+            self.th.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                self.rows.append((time.time(), parts))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        inside = [p for (t, p) in self.rows if t0 <= t <= t1]
+        window = "timed region"
+        if not inside:
+            inside = [p for (t, p) in self.rows if t0 - 1.0 <= t <= t1 + 1.0]
+            window = "timed region +-1 s (region shorter than the sampling interval)"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "window": "none"}
+        sm = [float(p[1]) for p in inside if p[1].replace(".", "").isdigit()]
+        mx = [float(p[2]) for p in inside if p[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for p in inside for k in range(4) if p[5 + k].lower() == "active"})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(inside), "window": window}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def cpu_oracle_run(tr, w, warm, timed, get_tokens, max_id):
+    """Time the CPU oracle (as it stands, one thread) over the `timed` batches,
+    after routing the `warm` batches untimed on the same state."""
+    from oracle import oracle as O
+    ora = O.Oracle(**O.config_from_workload(w, max_instances=max_id + 9, max_batch_tokens=1 << 40))
+    for i in range(w["n_instances"]):
+        ora.add_instance(i)
+    events = {}
+    for b, kind, i in tr.events:
+        events.setdefault(b, []).append((kind, i))
+    spent = 0.0
+    nreq = 0
+    for k, b in enumerate(list(warm) + list(timed)):
+        s, e, off, lens, ntok = tr.batch_layout(b)
+        tok = get_tokens(b)
+        t0 = time.perf_counter()
+        for kind, i in events.get(b, []):
+            (ora.add_instance if kind == "add" else ora.remove_instance)(i)
+        rc, _ = ora.route_batch(tok, off, lens, tr.batch_time(b))
+        assert rc == 0
+        if w.get("rebalance"):
+            ora.rebalance()
+        ora.commit()
+        if k >= len(warm):
+            spent += time.perf_counter() - t0
+            nreq += e - s
+    return nreq, spent
+
+
+def run_reference(args, world, rank):
+    """--impl reference: the CPU oracle timed on the host cores."""
+    from tracegen import Trace, workload
+    if rank != 0:
+        return
+    w = workload(args.workload)
+    tr = Trace(w)
+    nb = len(tr.batches)
+    k = max(1, min(args.steps, args.ref_max_batches))
+    warm = list(range(min(args.warmup, 2)))
+    timed = [len(warm) + j for j in range(min(k, nb - len(warm)))]
+    k = len(timed)
+    nreq, spent = cpu_oracle_run(tr, w, warm, timed, tr.batch_tokens, tr.max_instance_id())
+    val = nreq / spent
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "req/s", "n_gpus": args.gpus,
+            "steps": k, "warmup": len(warm), "ms_per_step": 1e3 * spent / k, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32/u64 integer", "data": "synthetic",
+            "config": {"workload": f"{w['name']}: {w['n_instances']} instances, batch {w['batch']}",
+                       "note": "reference arm = the plain-C CPU oracle, one host thread"},
+            "cpu_baseline": {"value": val, "unit": "req/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{k} batches of {w['batch']} requests (first {k} of the trace)"},
+            "e2e": {"value": val, "unit": "req/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=120)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", default="dualmap", choices=["dualmap", "reference"])
+    ap.add_argument("--workload", default="longctx")
+    ap.add_argument("--e2e-steps", type=int, default=24)
+    ap.add_argument("--cpu-batches", type=int, default=6)
+    ap.add_argument("--ref-max-batches", type=int, default=24)
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+
+    import torch
+    import torch.distributed as dist
+    from paper_2602_06502_gb300 import dualmap as D
+    from paper_2602_06502_gb300.scheduler import Scheduler, OUT_FIELDS
+    import tracegen.device as TD
+    from tracegen import Trace, workload
+
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = workload(args.workload)
+    W, K = max(args.warmup, 3), args.steps
+    tr = Trace(w)
+    nb = len(tr.batches)
+    kw = handle_kwargs(w, tr.max_instance_id())
+
+    # all batches' tokens resident in HBM (a pass longer than the trace replays it cyclically)
+    used = min(nb, W + K)
+    ntok = int(tr.req_off[tr.batches[used - 1][1]])
+    tokens = torch.empty(ntok + 4, dtype=torch.int32, device=dev)
+    for b0 in range(0, used, 16):
+        b1 = min(used, b0 + 16)
+        s0, e1 = tr.batches[b0][0], tr.batches[b1 - 1][1]
+        TD.fill_range(tr, s0, e1, tokens[int(tr.req_off[s0]):int(tr.req_off[e1])])
+    meta = []
+    for b in range(used):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        meta.append((s, e, torch.from_numpy(off.view(np.int64)).to(dev),
+                     torch.from_numpy(lens.view(np.int32)).to(dev), nt, int(tr.req_off[s])))
+    span = int(tr.arrival_us[-1]) + 1
+    events = {}
+    for b, kind, i in tr.events:
+        events.setdefault(b, []).append((kind, i))
+
+    def make_sched():
+        g = Scheduler(block_tokens=w["block_tokens"], route_prefix_blocks=w["route_prefix_blocks"],
+                      vnodes=w["vnodes"], capacity=w["capacity"], slo_us=w["slo_us"], cost_us=w["cost_us"],
+                      seed=w["seed"], **kw)
+        for i in range(w["n_instances"]):
+            assert g.add_instance(i) == 0
+        return g
+
+    def step(g, j, host=None):
+        b = j % used
+        cyc = j // used
+        for kind, i in (events.get(b, []) if cyc == 0 else []):
+            assert (g.add_instance(i) if kind == "add" else g.remove_instance(i)) == 0
+        s, e, doff, dlen, nt, t0 = meta[b]
+        tb = tr.batch_time(b) + cyc * span
+        if host is None:
+            g.route(tokens[t0:t0 + nt + 4], doff, dlen, e - s, nt, tb)
+        else:
+            hb = D.make_batch(host["tok"][b], host["off"][b], host["len"][b], e - s, nt, tb)
+            rc = D.dm_route_batch_host(g.h, hb, host["out_struct"])
+            assert rc == 0, rc
+        if w.get("rebalance"):
+            g.rebalance()
+        g.commit()
+        return e - s
+
+    # -- device-resident run -------------------------------------------------
+    g = make_sched()
+    for j in range(W):
+        step(g, j)
+    torch.cuda.synchronize()
+    assert g.last_error() == 0
+    D.dm_get_stage_times(g.h, reset=True)
+    D.dm_set_profiling(g.h, True)
+    sampler = ClockSampler(local)
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    wall0 = time.time()
+    ev0.record()
+    nreq = 0
+    prompt_bytes = 0
+    for j in range(W, W + K):
+        nreq += step(g, j)
+        b = j % used
+        prompt_bytes += 4 * int(tr.L[tr.batches[b][0]:tr.batches[b][1]].sum())
+    ev1.record()
+    torch.cuda.synchronize()
+    wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    sampler.stop()
+    ms = ev0.elapsed_time(ev1)
+    st = D.dm_get_stage_times(g.h, reset=True)
+    D.dm_set_profiling(g.h, False)
+    err = g.last_error()
+    assert err == 0, D.status_string(err)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * nreq / (ms / 1e3)
+    hash_ms, hash_calls = st["hash"]
+    probe_ms, _ = st["probe"]
+    hash_avg_s = hash_ms / 1e3 / max(hash_calls, 1)
+    bytes_per_launch = prompt_bytes / max(hash_calls, 1)
+    peak, peak_kind = peaks()
+    achieved = bytes_per_launch / hash_avg_s / 1e9
+    prompt_gbps = prompt_bytes / ((hash_ms + probe_ms) / 1e3) / 1e9
+    # route: setup, drain, hash, probe, choice; commit: count, maintain, prep, touch, evict
+    launches_per_step = 5 + 5 + (1 if w.get("rebalance") else 0)
+    clocks = sampler.summary(wall0, wall1)
+    g.close()
+    del g
+
+    # -- end-to-end through the host-buffer entry point ----------------------
+    e2e = None
+    if rank == 0 or world > 1:
+        Ke = max(1, min(args.e2e_steps, K))
+        g = make_sched()
+        need = sorted({j % used for j in range(W + Ke)})
+        host = {"tok": {}, "off": {}, "len": {}}
+        for b in need:
+            s, e, doff, dlen, nt, t0 = meta[b]
+            ht = torch.empty(nt + 4, dtype=torch.int32, pin_memory=True)
+            ht.copy_(tokens[t0:t0 + nt + 4])
+            host["tok"][b] = ht
+            host["off"][b] = doff.cpu().pin_memory()
+            host["len"][b] = dlen.cpu().pin_memory()
+        hout = {name: torch.zeros(w["batch"], dtype=t, pin_memory=True) for name, t in OUT_FIELDS}
+        host["out_struct"] = D.make_out(*[hout[name] for name, _ in OUT_FIELDS])
+        for j in range(W):
+            step(g, j, host)
+        torch.cuda.synchronize()
+        h2d = d2h = 0
+        t0 = time.perf_counter()
+        ne = 0
+        for j in range(W, W + Ke):
+            n = step(g, j, host)
+            ne += n
+            b = j % used
+            h2d += 4 * (meta[b][4]) + 12 * n
+            d2h += 41 * n
+        torch.cuda.synchronize()
+        te = time.perf_counter() - t0
+        assert g.last_error() == 0
+        g.close()
+        e2e = {"value": world * ne / te, "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
+               "d2h_bytes_per_step": d2h // Ke, "steps": Ke}
+
+    # -- CPU oracle baseline (rank 0, N=1 only) ------------------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cb = list(range(min(args.cpu_batches, used)))
+
+        def host_tokens(b):
+            s, e, doff, dlen, nt, t0 = meta[b]
+            return tokens[t0:t0 + nt].cpu().numpy().view(np.uint32)
+
+        n_cpu, t_cpu = cpu_oracle_run(tr, w, [], cb, host_tokens, tr.max_instance_id())
+        cpu = {"value": n_cpu / t_cpu, "unit": "req/s", "cores": 1, "kind": "oracle",
+               "sample": f"first {len(cb)} batches ({n_cpu} requests) of the same trace, "
+                         f"route+commit, {t_cpu:.1f} s"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "req/s", "n_gpus": world, "steps": K, "warmup": W,
+            "ms_per_step": ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "u32 tokens / u64 integer arithmetic", "data": "synthetic",
+            "prompt_GBps": prompt_gbps,
+            "config": {"workload": f"{w['name']}: {w['n_instances']} instances x {w['vnodes']} vnodes, "
+                                   f"batches of {w['batch']} prompts of {w['len_lo']}-{w['len_hi']} tokens "
+                                   f"(~{bytes_per_launch / 1e6:.0f} MB per batch)",
+                       "global_batch": w["batch"], "parallelism": f"replicas x{world}",
+                       "l2": "inputs larger than L2 (each batch > 129 MB, distinct per step)",
+                       "replay": "steps beyond the trace replay its batches cyclically" if W + K > nb else "none"},
+            "roofline": {"bound": "hbm", "kernel": "k_hash (prompt hashing)", "achieved": achieved,
+                         "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": traffic_per_launch(), "bytes_per_launch": bytes_per_launch,
+                         "avg_launch_ms": hash_avg_s * 1e3},
+            "stage_ms_per_step": {k: v[0] / max(v[1], 1) for k, v in st.items()},
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches_per_step * K, "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,257 @@
+/*
+ * dualmap.h -- C ABI of a GB300 (sm_103a) implementation of DualMap's batched
+ * request-routing path (arxiv 2602.06502, "DualMap: Enabling Both Cache
+ * Affinity and Load Balancing for Distributed LLM Serving").
+ *
+ * One handle is one global scheduler (Sec. 3.1): a cluster of up to
+ * `max_instances` inference instances, two consistent-hash rings, a per-
+ * instance index of cached prefix blocks, and per-instance FIFO queues of
+ * pending prefill work.  All state lives in device memory owned by the
+ * handle.  Work is enqueued on the handle's CUDA stream; calls return as soon
+ * as the work is enqueued unless stated otherwise.
+ *
+ * Conventions
+ *   - "device" pointers are CUDA device (or managed) memory, "host" pointers
+ *     are host memory.  The caller owns every buffer passed in; it must stay
+ *     valid until the handle's stream has executed the call.
+ *   - Synchronous argument checks return an error and change nothing.
+ *   - Checks that need device data (prompt lengths, offsets, capacities) run
+ *     in the kernels: a failure is recorded as a sticky device error, the
+ *     rest of that call's kernels do nothing, and every later call returns
+ *     the error (see dm_last_error).  The handle must then be destroyed.
+ *   - One handle must be used from one host thread at a time.
+ *
+ * Readings of details the paper leaves open (block size, hash family, ring
+ * layout, tie rules, time model) are fixed once here and implemented
+ * identically by the independent CPU oracle used in the tests.
+ */
+#ifndef DUALMAP_H
+#define DUALMAP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define DM_API __attribute__((visibility("default")))
+#else
+#define DM_API
+#endif
+
+typedef struct dm_handle dm_handle;
+
+typedef enum {
+    DM_OK = 0,
+    DM_ERR_INVALID_ARG = 1,   /* bad argument (null pointer, prompt < 1 block, misaligned offset...) */
+    DM_ERR_CAPACITY = 2,      /* a max_* bound of dm_config would be exceeded */
+    DM_ERR_NO_INSTANCES = 3,  /* routing needs at least two live instances */
+    DM_ERR_DUPLICATE_ID = 4,  /* id already live, or removed and still draining */
+    DM_ERR_UNKNOWN_ID = 5,    /* id not live */
+    DM_ERR_ORDER = 6,         /* batch time earlier than the previous batch's */
+    DM_ERR_CUDA = 7,          /* a CUDA runtime call failed */
+    DM_ERR_TIMEOUT = 8,       /* a bounded device-side loop gave up (state is corrupt) */
+    DM_ERR_OOM = 9            /* device or host allocation failed */
+} dm_status;
+
+/* Scheduler configuration (copied at dm_create). */
+typedef struct {
+    /* Tokens per block, B.  One of 4, 8, 16, 32, 64.  Blocks are the unit of
+     * prefix keys and of the cache index (App. A.1.1 uses 512-token hash
+     * blocks, App. A.3.2 128-token KV blocks; a single block size serves both
+     * here).  Only full blocks are keyed. */
+    uint32_t block_tokens;
+    /* Blocks hashed into the ring key, K_route in 1..256 (Sec. 3.2 "how long
+     * a prefix"); a prompt with fewer full blocks uses all of them. */
+    uint32_t route_prefix_blocks;
+    /* Virtual nodes per instance on each ring, V >= 1 (Sec. 3.4). */
+    uint32_t vnodes_per_instance;
+    /* Instance ids are 0 .. max_instances-1; 2 <= max_instances <= 8192. */
+    uint32_t max_instances;
+    /* Cache index capacity per instance in blocks, C >= 1 (exact LRU). */
+    uint64_t cache_capacity_blocks;
+    /* TTFT SLO in integer microseconds (Sec. 3.2). */
+    uint64_t slo_us;
+    /* Prefill cost in integer microseconds per uncached token, >= 1. */
+    uint32_t cost_us_per_token;
+    /* Hotspot rule of dm_rebalance: instance i is hot when
+     * hot_den * N * W_i > hot_num * sum(W) (3/2 = 1.5x the mean). */
+    uint32_t hot_num, hot_den;
+    /* Largest batch, in requests (>= 1). */
+    uint32_t max_batch;
+    /* Largest token buffer of a batch (dm_batch.total_tokens), >= B. */
+    uint64_t max_batch_tokens;
+    /* Largest number of blocks one commit may touch on one instance; 0 means
+     * max_batch_tokens / B.  Sizes each instance's index (2 x (C + this),
+     * rounded up to a power of two, 16 bytes a slot) and recency log. */
+    uint64_t max_touch_per_instance;
+    /* Queue capacity per instance in entries (power of two); 0 = 65536. */
+    uint32_t max_queue;
+    uint32_t reserved0;   /* must be 0 */
+    /* Seed of all hash key material (SplitMix64). */
+    uint64_t seed;
+    /* cudaStream_t for all work of this handle; NULL = legacy default stream. */
+    void *stream;
+} dm_config;
+
+/* One batch of requests in arrival order.
+ * Prompt r is tokens[offsets[r] .. offsets[r] + lengths[r]) (uint32 token
+ * ids).  For the device entry points `tokens` must be 16-byte aligned
+ * (DM_ERR_INVALID_ARG otherwise).  Every offsets[r] must be a multiple of 4
+ * (prompts start on 16-byte boundaries) and offsets[r] + lengths[r] <=
+ * total_tokens; prompts may overlap or share tokens.  lengths[r] >=
+ * block_tokens. */
+typedef struct {
+    const uint32_t *tokens;     /* device (host for dm_route_batch_host) */
+    const uint64_t *offsets;    /* device (host ...), n entries */
+    const uint32_t *lengths;    /* device (host ...), n entries */
+    uint32_t n;                 /* requests, <= max_batch; 0 = only advance time */
+    uint32_t reserved0;         /* must be 0 */
+    uint64_t total_tokens;      /* extent of tokens[], <= max_batch_tokens */
+    uint64_t batch_time_us;     /* arrival time of the batch's last request */
+} dm_batch;
+
+/* Per-request results of dm_route_batch (n entries each, device memory;
+ * host memory for dm_route_batch_host). */
+typedef struct {
+    uint32_t *cand1;     /* first candidate: owner of pos1 on ring 1 */
+    uint32_t *cand2;     /* second candidate (distinct from cand1) */
+    uint32_t *hit1;      /* cached-prefix tokens on cand1 (multiple of B) */
+    uint32_t *hit2;      /* cached-prefix tokens on cand2 */
+    uint64_t *ttft1;     /* estimated TTFT on cand1, us */
+    uint64_t *ttft2;     /* estimated TTFT on cand2, us */
+    uint32_t *chosen;    /* instance the request is queued on */
+    uint8_t *switched;   /* 1 when the SLO rule overrode cache affinity */
+} dm_route_out;
+
+typedef struct {
+    uint64_t req_seq;    /* global request sequence number (0-based, arrival order) */
+    uint32_t from, to;
+} dm_migration;
+
+/* Stages timed by dm_get_stage_times. */
+enum {
+    DM_STAGE_SETUP = 0,    /* batch validation and per-request prefix sums */
+    DM_STAGE_DRAIN = 1,    /* queue draining to the batch time */
+    DM_STAGE_HASH = 2,     /* token hashing into chained block prefix values */
+    DM_STAGE_PROBE = 3,    /* ring lookup, distinct fix, cache probes */
+    DM_STAGE_CHOICE = 4,   /* sequential SLO-aware choice */
+    DM_STAGE_COMMIT = 5,   /* cache commit with LRU eviction */
+    DM_STAGE_REBALANCE = 6,/* hotspot-aware rebalancing */
+    DM_STAGE_COUNT = 7
+};
+
+/* Create a scheduler with no instances.  Allocates all device state except
+ * the per-instance indices (allocated on first dm_add_instance of an id).
+ * Derives the hash key material from cfg->seed.  Synchronous. */
+DM_API dm_status dm_create(const dm_config *cfg, dm_handle **out);
+
+/* Destroy a handle, synchronising its stream first.  NULL is ignored. */
+DM_API void dm_destroy(dm_handle *h);
+
+/* Add instance `id` (Sec. 3.4, App. A.1.3): inserts its V virtual nodes into
+ * both rings (only keys on its new arcs remap) and gives it an empty index
+ * and queue.  DM_ERR_DUPLICATE_ID if it is live, or removed but its queue
+ * has not drained yet.  Synchronous (it reads the queue state). */
+DM_API dm_status dm_add_instance(dm_handle *h, uint32_t id);
+
+/* Remove instance `id`: deletes its virtual nodes from both rings; its
+ * queued work keeps draining, it receives no new requests and no
+ * migrations.  DM_ERR_UNKNOWN_ID if not live.  Asynchronous. */
+DM_API dm_status dm_remove_instance(dm_handle *h, uint32_t id);
+
+/* Route one batch (Sec. 3.2, App. A.1.1):
+ *   1. every queue drains by batch_time_us minus the previous batch time;
+ *   2. each prompt is hashed block by block into chained 64-bit prefix
+ *      values under two independent hash functions; the first
+ *      min(K_route, n_blk) blocks give two ring positions;
+ *   3. each position's successor virtual node on its ring gives a candidate;
+ *      equal candidates are separated by taking the next live id;
+ *   4. each candidate's index is probed for the leading run of resident
+ *      block keys (index state as of the start of the batch);
+ *   5. in arrival order: TTFT_f = W[c_f] + cost * (L - hit_f); the higher-hit
+ *      candidate unless its TTFT exceeds the SLO, then the less-loaded one;
+ *      equal hits take the less-loaded one; the request is queued there.
+ * The batch is kept for dm_commit_cache.  Asynchronous. */
+DM_API dm_status dm_route_batch(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
+
+/* Same as dm_route_batch with every pointer of `batch` and `out` in host
+ * memory (pinned memory is faster).  The library copies the inputs to its
+ * own device staging buffers, routes, copies the results back and
+ * synchronises the stream before returning. */
+DM_API dm_status dm_route_batch_host(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
+
+/* Hotspot-aware rebalancing (Sec. 3.3, Eq. "rebalance"; App. A.1.2), to be
+ * called after dm_route_batch and before dm_commit_cache.  Hot instances
+ * are visited in descending W; their queued, not-started requests are
+ * ranked by migration benefit B = TTFT_{r,i} - TTFT_{r,j} (j the request's
+ * other candidate) and moved to j while i stays hot, B > 0 and
+ * TTFT_{r,j} < SLO.  Writes up to `cap` migrations to out_dev (device) and
+ * the total count to *n_out_dev (device).  Asynchronous. */
+DM_API dm_status dm_rebalance(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev);
+
+/* Cache save (App. A.3.2) of the last routed batch: in arrival order, each
+ * request touches its block keys on its final instance (block n_blk-1 down
+ * to 0, one global clock tick each); each index then keeps its C most
+ * recently touched keys (exact LRU).  A no-op when the last batch is
+ * already committed.  Asynchronous. */
+DM_API dm_status dm_commit_cache(dm_handle *h);
+
+/* Chained block keys and ring positions of a batch without touching any
+ * scheduler state: keys_dev receives, for request r, its n_blk(r) = L/B
+ * cache keys at positions key_off[r] .. key_off[r] + n_blk(r), where
+ * key_off (device, n+1 entries, written by the call) is the exclusive prefix
+ * sum of n_blk; pos_dev (device, 2n entries) receives (pos1, pos2) per
+ * request.  keys_dev must hold sum(n_blk) entries (at most
+ * total_tokens / B).  Asynchronous. */
+DM_API dm_status dm_hash_prompts(dm_handle *h, const dm_batch *batch, uint64_t *keys_dev,
+                          uint64_t *key_off_dev, uint64_t *pos_dev);
+
+/* Raw ring owners (before the distinct fix) of n positions: pos_dev holds
+ * (pos1, pos2) pairs as written by dm_hash_prompts; owner1_dev/owner2_dev
+ * receive the successor's owner on ring 1 / ring 2.  Asynchronous. */
+DM_API dm_status dm_ring_lookup(dm_handle *h, const uint64_t *pos_dev, uint32_t n,
+                         uint32_t *owner1_dev, uint32_t *owner2_dev);
+
+/* Queued work W (us) of ids 0 .. min(cap, max_instances)-1.  Synchronous. */
+DM_API dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap);
+
+/* Resident (key, last-touch stamp) pairs of instance `id`, in unspecified
+ * order; *n_out = resident count (entries beyond cap are not written).
+ * Synchronous. */
+DM_API dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys_host, uint64_t *stamps_host,
+                          uint64_t cap, uint64_t *n_out);
+
+/* Queue of instance `id`, head first: sequence number, work and remaining
+ * work (us) of each entry; *n_out = queue length.  Synchronous. */
+DM_API dm_status dm_export_queue(dm_handle *h, uint32_t id, uint64_t *seq_host, uint64_t *work_host,
+                          uint64_t *remaining_host, uint64_t cap, uint64_t *n_out);
+
+/* Ring f (0 or 1) as sorted (position, owner) arrays; *n_out = its length.
+ * Synchronous. */
+DM_API dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos_host, uint32_t *owner_host,
+                         uint32_t cap, uint32_t *n_out);
+
+/* Value of the global commit clock (number of block touches so far). */
+DM_API dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host);
+
+/* Synchronise the stream and return the sticky error (DM_OK if none). */
+DM_API dm_status dm_last_error(dm_handle *h);
+
+/* Per-stage CUDA-event timing of every subsequent call (on = 1) or none. */
+DM_API dm_status dm_set_profiling(dm_handle *h, int on);
+
+/* Synchronise, then return the summed milliseconds and call counts of each
+ * stage since the last reset (arrays of DM_STAGE_COUNT); reset = 1 clears. */
+DM_API dm_status dm_get_stage_times(dm_handle *h, double *ms_host, uint64_t *calls_host, int reset);
+
+/* Human-readable name of a status code. */
+DM_API const char *dm_status_string(dm_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DUALMAP_H */

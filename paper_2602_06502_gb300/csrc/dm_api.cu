@@ -1,0 +1,648 @@
+// dm_api.cu -- host side of the C ABI declared in include/dualmap.h:
+// argument checks, device memory ownership, stream ordering, error mapping.
+// Every computation of the routing path runs in the kernels of the other
+// translation units; this file only validates, allocates and enqueues.
+#include <cstdio>
+#include <cstring>
+#include <utility>
+#include <vector>
+
+#include "dm_internal.cuh"
+
+using dm::DevState;
+using dm::QEntry;
+using dm::Slot;
+
+struct StageEvent {
+    int stage;
+    cudaEvent_t a, b;
+};
+
+struct dm_handle {
+    dm_config cfg{};
+    DevState d{};            // main scheduler state (kernel parameter)
+    DevState dh{};           // same, with the scratch of dm_hash_prompts
+    cudaStream_t st = nullptr;
+    std::vector<uint8_t> state;   // host mirror: 0 absent, 1 live, 2 draining
+    uint32_t n_live = 0;
+    uint64_t seq_next = 0, t_prev = 0;
+    bool have_time = false;
+    bool pending = false;
+    uint32_t pending_n = 0;
+    uint64_t pending_seq0 = 0;
+    uint32_t rebalance_calls = 0;
+    int hash_grid = 0;
+    uint64_t *vpos_buf[2][2] = {};
+    uint32_t *owner_buf[2][2] = {}, *vidx_buf[2][2] = {};
+    int cur[2] = {0, 0};
+    uint64_t *ring_spos = nullptr;
+    uint32_t *ring_svidx = nullptr;
+    std::vector<Slot *> tables, logs;
+    std::vector<void *> allocs;    // every cudaMalloc of the handle
+    // staging of dm_route_batch_host
+    uint32_t *h_tokens = nullptr, *h_lengths = nullptr;
+    uint64_t *h_offsets = nullptr;
+    dm_route_out h_out{};
+    bool profiling = false;
+    std::vector<StageEvent> events;
+    double stage_ms[DM_STAGE_COUNT] = {};
+    uint64_t stage_calls[DM_STAGE_COUNT] = {};
+    dm_status sticky = DM_OK;
+};
+
+namespace {
+
+template <typename T>
+cudaError_t dalloc(dm_handle *h, T **p, size_t count) {
+    void *q = nullptr;
+    cudaError_t e = cudaMalloc(&q, count ? count * sizeof(T) : 16);
+    if (e != cudaSuccess) { *p = nullptr; return e; }
+    h->allocs.push_back(q);
+    *p = static_cast<T *>(q);
+    return cudaSuccess;
+}
+
+uint64_t pow2_at_least(uint64_t x) {
+    uint64_t p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+dm_status map_cuda(dm_handle *h, cudaError_t e) {
+    if (e == cudaSuccess) return DM_OK;
+    if (h->sticky == DM_OK) h->sticky = (e == cudaErrorMemoryAllocation) ? DM_ERR_OOM : DM_ERR_CUDA;
+    return h->sticky;
+}
+
+// Split R into the levels of the 32-ary search tree.
+void set_levels(DevState &d, uint32_t R) {
+    d.R = R;
+    d.lev_n[0] = R;
+    uint32_t k = 0;
+    while (d.lev_n[k] > 32 && k + 1 < (uint32_t)dm::kMaxLevels) {
+        d.lev_n[k + 1] = (d.lev_n[k] + 31) / 32;
+        ++k;
+    }
+    d.nlev = k + 1;
+    d.lev_off[1] = 0;
+    for (uint32_t j = 1; j + 1 < d.nlev; ++j) d.lev_off[j + 1] = d.lev_off[j] + d.lev_n[j];
+}
+
+struct Stage {
+    dm_handle *h;
+    int s;
+    cudaEvent_t a = nullptr, b = nullptr;
+    Stage(dm_handle *h_, int s_) : h(h_), s(s_) {
+        if (h->profiling && cudaEventCreate(&a) == cudaSuccess && cudaEventCreate(&b) == cudaSuccess)
+            cudaEventRecord(a, h->st);
+    }
+    ~Stage() {
+        if (a && b) {
+            cudaEventRecord(b, h->st);
+            h->events.push_back(StageEvent{s, a, b});
+        }
+    }
+};
+
+uint64_t splitmix_next(uint64_t &s) {
+    uint64_t z = (s += 0x9E3779B97F4A7C15ULL);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+dm_status check_live(dm_handle *h) {
+    if (!h) return DM_ERR_INVALID_ARG;
+    return h->sticky;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *dm_status_string(dm_status s) {
+    switch (s) {
+        case DM_OK: return "ok";
+        case DM_ERR_INVALID_ARG: return "invalid argument";
+        case DM_ERR_CAPACITY: return "capacity exceeded";
+        case DM_ERR_NO_INSTANCES: return "fewer than two live instances";
+        case DM_ERR_DUPLICATE_ID: return "instance id already live or still draining";
+        case DM_ERR_UNKNOWN_ID: return "instance id not live";
+        case DM_ERR_ORDER: return "batch time earlier than the previous batch";
+        case DM_ERR_CUDA: return "CUDA runtime error";
+        case DM_ERR_TIMEOUT: return "bounded device loop gave up";
+        case DM_ERR_OOM: return "out of memory";
+    }
+    return "unknown status";
+}
+
+void dm_destroy(dm_handle *h) {
+    if (!h) return;
+    cudaStreamSynchronize(h->st);
+    for (auto &ev : h->events) { cudaEventDestroy(ev.a); cudaEventDestroy(ev.b); }
+    for (void *p : h->allocs) cudaFree(p);
+    delete h;
+}
+
+dm_status dm_create(const dm_config *cfg, dm_handle **out) {
+    if (!cfg || !out) return DM_ERR_INVALID_ARG;
+    *out = nullptr;
+    const dm_config &c = *cfg;
+    const uint32_t B = c.block_tokens;
+    if (!(B == 4 || B == 8 || B == 16 || B == 32 || B == 64)) return DM_ERR_INVALID_ARG;
+    if (c.route_prefix_blocks < 1 || c.route_prefix_blocks > dm::kMaxRouteBlocks) return DM_ERR_INVALID_ARG;
+    if (c.vnodes_per_instance < 1 || c.vnodes_per_instance > 65536) return DM_ERR_INVALID_ARG;
+    if (c.max_instances < 2 || c.max_instances > dm::kMaxInstances) return DM_ERR_INVALID_ARG;
+    if (uint64_t(c.max_instances) * c.vnodes_per_instance > (1ull << 31)) return DM_ERR_INVALID_ARG;
+    if (c.cache_capacity_blocks < 1 || c.cost_us_per_token < 1 || c.hot_den < 1) return DM_ERR_INVALID_ARG;
+    if (c.max_batch < 1 || c.max_batch > (1u << 24) || c.max_batch_tokens < B) return DM_ERR_INVALID_ARG;
+    if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
+    if (c.reserved0) return DM_ERR_INVALID_ARG;
+
+    dm_handle *h = new dm_handle();
+    h->cfg = c;
+    h->st = static_cast<cudaStream_t>(c.stream);
+    DevState &d = h->d;
+    d.B = B;
+    d.Kroute = c.route_prefix_blocks;
+    d.V = c.vnodes_per_instance;
+    d.M = c.max_instances;
+    d.C = c.cache_capacity_blocks;
+    d.slo = c.slo_us;
+    d.cost = c.cost_us_per_token;
+    d.hot_num = c.hot_num;
+    d.hot_den = c.hot_den;
+    d.max_batch = c.max_batch;
+    d.max_blocks = c.max_batch_tokens / B;
+    d.max_segs = d.max_blocks / dm::kSegBlocks + c.max_batch;
+    d.T = c.max_touch_per_instance ? c.max_touch_per_instance : d.max_blocks;
+    d.S = pow2_at_least(2 * (d.C + d.T));
+    d.logcap = pow2_at_least(2 * (d.C + d.T));
+    d.Q = c.max_queue ? c.max_queue : 65536;
+    d.rb_cap = (uint32_t)pow2_at_least(d.Q > d.M ? d.Q : d.M);
+    // key material: SplitMix64(seed) -> K1[0..B), K2[0..B), G1|1, G2|1, Sc, Sr1, Sr2, Sv1, Sv2
+    uint64_t s = c.seed;
+    for (uint32_t j = 0; j < B; ++j) d.K1[j] = (uint32_t)splitmix_next(s);
+    for (uint32_t j = 0; j < B; ++j) d.K2[j] = (uint32_t)splitmix_next(s);
+    d.G1 = splitmix_next(s) | 1ull;
+    d.G2 = splitmix_next(s) | 1ull;
+    d.Sc = splitmix_next(s);
+    d.Sr1 = splitmix_next(s);
+    d.Sr2 = splitmix_next(s);
+    d.Sv1 = splitmix_next(s);
+    d.Sv2 = splitmix_next(s);
+
+    const uint64_t M = d.M, Rmax = M * d.V;
+    cudaError_t e = cudaSuccess;
+    auto A = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
+    for (int f = 0; f < 2; ++f)
+        for (int b = 0; b < 2; ++b) {
+            A(dalloc(h, &h->vpos_buf[f][b], Rmax));
+            A(dalloc(h, &h->owner_buf[f][b], Rmax));
+            A(dalloc(h, &h->vidx_buf[f][b], Rmax));
+        }
+    uint64_t tree_n = 0;
+    for (uint64_t n = Rmax; n > 32;) { n = (n + 31) / 32; tree_n += n; }
+    for (int f = 0; f < 2; ++f) A(dalloc(h, &d.ring[f].tree, tree_n + 32));
+    uint32_t P = 1;
+    while (P < d.V) P <<= 1;
+    A(dalloc(h, &h->ring_spos, 2ull * P));
+    A(dalloc(h, &h->ring_svidx, 2ull * P));
+    A(dalloc(h, &d.inst_state, M));
+    A(dalloc(h, &d.next_live, M));
+    A(dalloc(h, &d.W, M));
+    A(dalloc(h, &d.q_head, M));
+    A(dalloc(h, &d.q_tail, M));
+    A(dalloc(h, &d.q, M * d.Q));
+    A(dalloc(h, &d.table, M));
+    A(dalloc(h, &d.logbuf, M));
+    A(dalloc(h, &d.log_front, M));
+    A(dalloc(h, &d.log_tail, M));
+    A(dalloc(h, &d.live, M));
+    A(dalloc(h, &d.used, M));
+    A(dalloc(h, &d.touch_cnt, M));
+    A(dalloc(h, &d.clock, 1));
+    A(dalloc(h, &d.err, 1));
+    A(dalloc(h, &d.seq_next, 1));
+    A(dalloc(h, &d.rb_key, d.rb_cap));
+    A(dalloc(h, &d.rb_seq, d.rb_cap));
+    A(dalloc(h, &d.rb_ttft, d.rb_cap));
+    A(dalloc(h, &d.rb_pos, d.rb_cap));
+    // two sets of batch scratch: routing and dm_hash_prompts
+    for (DevState *x : {&h->d, &h->dh}) {
+        if (x == &h->dh) {
+            const DevState keep = h->d;
+            *x = keep;
+        }
+        A(dalloc(h, &x->r_L, c.max_batch));
+        A(dalloc(h, &x->r_nblk, c.max_batch));
+        A(dalloc(h, &x->r_segoff, c.max_batch));
+        A(dalloc(h, &x->r_tokoff, c.max_batch));
+        A(dalloc(h, &x->r_blkoff, c.max_batch));
+        A(dalloc(h, &x->seg_req, d.max_segs));
+        A(dalloc(h, &x->seg_total, d.max_segs));
+        A(dalloc(h, &x->seg_carry, d.max_segs));
+        A(dalloc(h, &x->plocal, d.max_blocks));
+        A(dalloc(h, &x->r_pos, 2ull * c.max_batch));
+        A(dalloc(h, &x->r_c1, c.max_batch));
+        A(dalloc(h, &x->r_c2, c.max_batch));
+        A(dalloc(h, &x->r_h1, c.max_batch));
+        A(dalloc(h, &x->r_h2, c.max_batch));
+        A(dalloc(h, &x->r_final, c.max_batch));
+        A(dalloc(h, &x->r_touchoff, c.max_batch));
+        A(dalloc(h, &x->info, 1));
+    }
+    if (e != cudaSuccess) {
+        dm_destroy(h);
+        return e == cudaErrorMemoryAllocation ? DM_ERR_OOM : DM_ERR_CUDA;
+    }
+    for (int f = 0; f < 2; ++f) {
+        d.ring[f].vpos = h->vpos_buf[f][0];
+        d.ring[f].owner = h->owner_buf[f][0];
+        d.ring[f].vidx = h->vidx_buf[f][0];
+        h->dh.ring[f] = d.ring[f];
+    }
+    set_levels(d, 0);
+    A(cudaMemsetAsync(d.inst_state, 0, M, h->st));
+    A(cudaMemsetAsync(d.W, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.q_head, 0, M * 4, h->st));
+    A(cudaMemsetAsync(d.q_tail, 0, M * 4, h->st));
+    A(cudaMemsetAsync(d.table, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.logbuf, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.log_front, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.log_tail, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.live, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.used, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.clock, 0, 8, h->st));
+    A(cudaMemsetAsync(d.err, 0, 4, h->st));
+    A(cudaMemsetAsync(h->d.info, 0, sizeof(dm::BatchInfo), h->st));
+    A(cudaMemsetAsync(h->dh.info, 0, sizeof(dm::BatchInfo), h->st));
+    A(dm::launch_next_live(d, h->st));
+    A(cudaStreamSynchronize(h->st));
+    if (e != cudaSuccess) {
+        dm_destroy(h);
+        return DM_ERR_CUDA;
+    }
+    h->state.assign(M, 0);
+    h->tables.assign(M, nullptr);
+    h->logs.assign(M, nullptr);
+    h->hash_grid = dm::hash_grid_size();
+    *out = h;
+    return DM_OK;
+}
+
+// Keep the hash-prompts copy in step with the ring / instance state.
+static void sync_copy(dm_handle *h) {
+    DevState keep = h->dh;
+    h->dh = h->d;
+    h->dh.r_L = keep.r_L; h->dh.r_nblk = keep.r_nblk; h->dh.r_segoff = keep.r_segoff;
+    h->dh.r_tokoff = keep.r_tokoff; h->dh.r_blkoff = keep.r_blkoff; h->dh.seg_req = keep.seg_req;
+    h->dh.seg_total = keep.seg_total; h->dh.seg_carry = keep.seg_carry; h->dh.plocal = keep.plocal;
+    h->dh.r_pos = keep.r_pos; h->dh.r_c1 = keep.r_c1; h->dh.r_c2 = keep.r_c2; h->dh.r_h1 = keep.r_h1;
+    h->dh.r_h2 = keep.r_h2; h->dh.r_final = keep.r_final; h->dh.r_touchoff = keep.r_touchoff;
+    h->dh.info = keep.info;
+}
+
+static dm_status ring_change(dm_handle *h, uint32_t id, bool add) {
+    DevState &d = h->d;
+    const uint32_t newR = add ? d.R + d.V : d.R - d.V;
+    uint64_t *nv[2];
+    uint32_t *no[2], *ni[2];
+    for (int f = 0; f < 2; ++f) {
+        const int nb = 1 - h->cur[f];
+        nv[f] = h->vpos_buf[f][nb];
+        no[f] = h->owner_buf[f][nb];
+        ni[f] = h->vidx_buf[f][nb];
+    }
+    cudaError_t e = dm::launch_ring_update(d, id, add, newR, h->ring_spos, nullptr, h->ring_svidx, nv, no, ni,
+                                           h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    for (int f = 0; f < 2; ++f) {
+        h->cur[f] = 1 - h->cur[f];
+        d.ring[f].vpos = nv[f];
+        d.ring[f].owner = no[f];
+        d.ring[f].vidx = ni[f];
+    }
+    set_levels(d, newR);
+    e = dm::launch_tree_build(d, h->st);
+    if (e == cudaSuccess) e = dm::launch_set_state(d, id, add ? 1 : 2, h->st);
+    if (e == cudaSuccess) e = dm::launch_next_live(d, h->st);
+    sync_copy(h);
+    return map_cuda(h, e);
+}
+
+dm_status dm_add_instance(dm_handle *h, uint32_t id) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    DevState &d = h->d;
+    if (id >= d.M) return DM_ERR_INVALID_ARG;
+    if (h->state[id] == 1) return DM_ERR_DUPLICATE_ID;
+    cudaError_t e = cudaSuccess;
+    if (h->state[id] == 2) {
+        uint32_t ht[2];
+        e = cudaMemcpyAsync(&ht[0], d.q_head + id, 4, cudaMemcpyDeviceToHost, h->st);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&ht[1], d.q_tail + id, 4, cudaMemcpyDeviceToHost, h->st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+        if (e != cudaSuccess) return map_cuda(h, e);
+        if (ht[0] != ht[1]) return DM_ERR_DUPLICATE_ID;
+    }
+    if (!h->tables[id]) {
+        Slot *t = nullptr, *lg = nullptr;
+        e = dalloc(h, &t, d.S);
+        if (e == cudaSuccess) e = dalloc(h, &lg, d.logcap);
+        if (e != cudaSuccess) { cudaGetLastError(); return DM_ERR_OOM; }
+        h->tables[id] = t;
+        h->logs[id] = lg;
+        e = cudaMemcpyAsync(d.table + id, &h->tables[id], sizeof(Slot *), cudaMemcpyHostToDevice, h->st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(d.logbuf + id, &h->logs[id], sizeof(Slot *), cudaMemcpyHostToDevice, h->st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+        if (e != cudaSuccess) return map_cuda(h, e);
+    }
+    // a (re-)added instance starts empty
+    e = cudaMemsetAsync(h->tables[id], 0, d.S * sizeof(Slot), h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.log_front + id, 0, 8, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.log_tail + id, 0, 8, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.live + id, 0, 8, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.used + id, 0, 8, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.W + id, 0, 8, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.q_head + id, 0, 4, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d.q_tail + id, 0, 4, h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    s = ring_change(h, id, true);
+    if (s) return s;
+    h->state[id] = 1;
+    h->n_live++;
+    return DM_OK;
+}
+
+dm_status dm_remove_instance(dm_handle *h, uint32_t id) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (id >= h->d.M || h->state[id] != 1) return DM_ERR_UNKNOWN_ID;
+    s = ring_change(h, id, false);
+    if (s) return s;
+    h->state[id] = 2;
+    h->n_live--;
+    return DM_OK;
+}
+
+static dm_status check_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!b || b->reserved0) return DM_ERR_INVALID_ARG;
+    if (b->n > 0 && (!b->tokens || !b->offsets || !b->lengths)) return DM_ERR_INVALID_ARG;
+    if (o && b->n > 0 &&
+        (!o->cand1 || !o->cand2 || !o->hit1 || !o->hit2 || !o->ttft1 || !o->ttft2 || !o->chosen || !o->switched))
+        return DM_ERR_INVALID_ARG;
+    if (b->n > h->d.max_batch || b->total_tokens > h->cfg.max_batch_tokens) return DM_ERR_CAPACITY;
+    return DM_OK;
+}
+
+// The hashing kernel reads prompts with 16-byte loads.
+static bool tokens_aligned(const dm_batch *b) {
+    return b->n == 0 || (reinterpret_cast<uintptr_t>(b->tokens) & 15) == 0;
+}
+
+dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    dm_status s = check_batch(h, b, o);
+    if (s) return s;
+    if (!tokens_aligned(b)) return DM_ERR_INVALID_ARG;
+    if (!o) return DM_ERR_INVALID_ARG;
+    if (h->n_live < 2) return DM_ERR_NO_INSTANCES;
+    if (h->have_time && b->batch_time_us < h->t_prev) return DM_ERR_ORDER;
+    const uint64_t delta = h->have_time ? b->batch_time_us - h->t_prev : 0;
+    h->t_prev = b->batch_time_us;
+    h->have_time = true;
+    const DevState &d = h->d;
+    cudaError_t e;
+    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup(d, *b, h->st); }
+    if (e == cudaSuccess) { Stage st(h, DM_STAGE_DRAIN); e = dm::launch_drain(d, delta, h->st); }
+    if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_HASH); e = dm::launch_hash(d, *b, h->hash_grid, h->st); }
+    if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_PROBE); e = dm::launch_route_probe(d, *b, *o, h->st); }
+    if (e == cudaSuccess && b->n) {
+        Stage st(h, DM_STAGE_CHOICE);
+        e = dm::launch_choice(d, *o, b->n, h->seq_next, h->st);
+    }
+    if (e != cudaSuccess) return map_cuda(h, e);
+    h->pending = true;
+    h->pending_n = b->n;
+    h->pending_seq0 = h->seq_next;
+    h->seq_next += b->n;
+    return DM_OK;
+}
+
+dm_status dm_route_batch_host(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    dm_status s = check_batch(h, b, o);
+    if (s) return s;
+    if (!o) return DM_ERR_INVALID_ARG;
+    cudaError_t e = cudaSuccess;
+    const uint32_t mb = h->d.max_batch;
+    if (!h->h_tokens) {
+        auto A = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
+        A(dalloc(h, &h->h_tokens, h->cfg.max_batch_tokens));
+        A(dalloc(h, &h->h_offsets, mb));
+        A(dalloc(h, &h->h_lengths, mb));
+        A(dalloc(h, &h->h_out.cand1, mb));
+        A(dalloc(h, &h->h_out.cand2, mb));
+        A(dalloc(h, &h->h_out.hit1, mb));
+        A(dalloc(h, &h->h_out.hit2, mb));
+        A(dalloc(h, &h->h_out.ttft1, mb));
+        A(dalloc(h, &h->h_out.ttft2, mb));
+        A(dalloc(h, &h->h_out.chosen, mb));
+        A(dalloc(h, &h->h_out.switched, mb));
+        if (e != cudaSuccess) { cudaGetLastError(); h->h_tokens = nullptr; return DM_ERR_OOM; }
+    }
+    const uint32_t n = b->n;
+    if (n) {
+        e = cudaMemcpyAsync(h->h_tokens, b->tokens, b->total_tokens * 4, cudaMemcpyHostToDevice, h->st);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_offsets, b->offsets, n * 8ull, cudaMemcpyHostToDevice, h->st);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_lengths, b->lengths, n * 4ull, cudaMemcpyHostToDevice, h->st);
+        if (e != cudaSuccess) return map_cuda(h, e);
+    }
+    dm_batch db = *b;
+    db.tokens = h->h_tokens;
+    db.offsets = h->h_offsets;
+    db.lengths = h->h_lengths;
+    s = dm_route_batch(h, &db, &h->h_out);
+    if (s) return s;
+    if (n) {
+        const dm_route_out &x = h->h_out;
+        struct { void *dst; const void *src; size_t bytes; } cp[] = {
+            {o->cand1, x.cand1, n * 4ull}, {o->cand2, x.cand2, n * 4ull}, {o->hit1, x.hit1, n * 4ull},
+            {o->hit2, x.hit2, n * 4ull}, {o->ttft1, x.ttft1, n * 8ull}, {o->ttft2, x.ttft2, n * 8ull},
+            {o->chosen, x.chosen, n * 4ull}, {o->switched, x.switched, n * 1ull}};
+        for (auto &c : cp) {
+            e = cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyDeviceToHost, h->st);
+            if (e != cudaSuccess) return map_cuda(h, e);
+        }
+    }
+    e = cudaStreamSynchronize(h->st);
+    return map_cuda(h, e);
+}
+
+dm_status dm_rebalance(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!n_out_dev || (cap && !out_dev)) return DM_ERR_INVALID_ARG;
+    const uint32_t n = h->pending ? h->pending_n : 0;
+    cudaError_t e;
+    {
+        Stage st(h, DM_STAGE_REBALANCE);
+        e = dm::launch_rebalance(h->d, n, h->pending_seq0, ++h->rebalance_calls, out_dev, cap, n_out_dev, h->st);
+    }
+    return map_cuda(h, e);
+}
+
+dm_status dm_commit_cache(dm_handle *h) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!h->pending) return DM_OK;
+    cudaError_t e;
+    {
+        Stage st(h, DM_STAGE_COMMIT);
+        e = dm::launch_commit(h->d, h->pending_n, h->st);
+    }
+    h->pending = false;
+    return map_cuda(h, e);
+}
+
+dm_status dm_hash_prompts(dm_handle *h, const dm_batch *b, uint64_t *keys_dev, uint64_t *key_off_dev,
+                          uint64_t *pos_dev) {
+    dm_status s = check_batch(h, b, nullptr);
+    if (s) return s;
+    if (b->n && (!keys_dev || !key_off_dev || !pos_dev)) return DM_ERR_INVALID_ARG;
+    if (!tokens_aligned(b)) return DM_ERR_INVALID_ARG;
+    if (b->n == 0) return DM_OK;
+    cudaError_t e = dm::launch_setup(h->dh, *b, h->st);
+    if (e == cudaSuccess) e = dm::launch_hash(h->dh, *b, h->hash_grid, h->st);
+    if (e == cudaSuccess) e = dm::launch_hash_keys(h->dh, b->n, keys_dev, key_off_dev, pos_dev, h->st);
+    return map_cuda(h, e);
+}
+
+dm_status dm_ring_lookup(dm_handle *h, const uint64_t *pos_dev, uint32_t n, uint32_t *o1, uint32_t *o2) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (n && (!pos_dev || !o1 || !o2)) return DM_ERR_INVALID_ARG;
+    if (n && h->d.R == 0) return DM_ERR_NO_INSTANCES;
+    return map_cuda(h, dm::launch_ring_lookup(h->d, pos_dev, n, o1, o2, h->st));
+}
+
+dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!W_host && cap) return DM_ERR_INVALID_ARG;
+    const uint32_t k = cap < h->d.M ? cap : h->d.M;
+    cudaError_t e = cudaMemcpyAsync(W_host, h->d.W, k * 8ull, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    return map_cuda(h, e);
+}
+
+dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys, uint64_t *stamps, uint64_t cap,
+                          uint64_t *n_out) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (id >= h->d.M || !n_out || (cap && (!keys || !stamps))) return DM_ERR_INVALID_ARG;
+    *n_out = 0;
+    if (!h->tables[id]) return DM_OK;
+    std::vector<Slot> t(h->d.S);
+    cudaError_t e = cudaMemcpyAsync(t.data(), h->tables[id], h->d.S * sizeof(Slot), cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    uint64_t k = 0;
+    for (const Slot &x : t) {
+        if (x.key == 0 || x.stamp == 0) continue;
+        if (k < cap) { keys[k] = x.key; stamps[k] = x.stamp; }
+        ++k;
+    }
+    *n_out = k;
+    return DM_OK;
+}
+
+dm_status dm_export_queue(dm_handle *h, uint32_t id, uint64_t *seq, uint64_t *work, uint64_t *rem, uint64_t cap,
+                          uint64_t *n_out) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (id >= h->d.M || !n_out || (cap && (!seq || !work || !rem))) return DM_ERR_INVALID_ARG;
+    uint32_t ht[2];
+    std::vector<QEntry> q(h->d.Q);
+    cudaError_t e = cudaMemcpyAsync(&ht[0], h->d.q_head + id, 4, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&ht[1], h->d.q_tail + id, 4, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(q.data(), h->d.q + uint64_t(id) * h->d.Q, h->d.Q * sizeof(QEntry),
+                            cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    uint64_t k = 0;
+    for (uint32_t p = ht[0]; p != ht[1]; ++p) {
+        const QEntry &x = q[p & (h->d.Q - 1)];
+        if (x.moved == dm::kTomb) continue;
+        if (k < cap) { seq[k] = x.seq; work[k] = x.work; rem[k] = x.remaining; }
+        ++k;
+    }
+    *n_out = k;
+    return DM_OK;
+}
+
+dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos, uint32_t *owner, uint32_t cap, uint32_t *n_out) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if ((f != 0 && f != 1) || !n_out || (cap && (!vpos || !owner))) return DM_ERR_INVALID_ARG;
+    const uint32_t k = cap < h->d.R ? cap : h->d.R;
+    cudaError_t e = cudaMemcpyAsync(vpos, h->d.ring[f].vpos, k * 8ull, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(owner, h->d.ring[f].owner, k * 4ull, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    *n_out = h->d.R;
+    return map_cuda(h, e);
+}
+
+dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!clock_host) return DM_ERR_INVALID_ARG;
+    cudaError_t e = cudaMemcpyAsync(clock_host, h->d.clock, 8, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    return map_cuda(h, e);
+}
+
+dm_status dm_last_error(dm_handle *h) {
+    if (!h) return DM_ERR_INVALID_ARG;
+    if (h->sticky) return h->sticky;
+    uint32_t err = 0;
+    cudaError_t e = cudaMemcpyAsync(&err, h->d.err, 4, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    if (err) h->sticky = static_cast<dm_status>(err);
+    return h->sticky;
+}
+
+dm_status dm_set_profiling(dm_handle *h, int on) {
+    if (!h) return DM_ERR_INVALID_ARG;
+    h->profiling = on != 0;
+    return DM_OK;
+}
+
+dm_status dm_get_stage_times(dm_handle *h, double *ms, uint64_t *calls, int reset) {
+    if (!h) return DM_ERR_INVALID_ARG;
+    cudaError_t e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    for (auto &ev : h->events) {
+        float t = 0.f;
+        if (cudaEventElapsedTime(&t, ev.a, ev.b) == cudaSuccess) {
+            h->stage_ms[ev.stage] += t;
+            h->stage_calls[ev.stage] += 1;
+        }
+        cudaEventDestroy(ev.a);
+        cudaEventDestroy(ev.b);
+    }
+    h->events.clear();
+    for (int i = 0; i < DM_STAGE_COUNT; ++i) {
+        if (ms) ms[i] = h->stage_ms[i];
+        if (calls) calls[i] = h->stage_calls[i];
+    }
+    if (reset)
+        for (int i = 0; i < DM_STAGE_COUNT; ++i) { h->stage_ms[i] = 0; h->stage_calls[i] = 0; }
+    return DM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,221 @@
+// dm_internal.cuh -- device state layout and device helpers shared by the
+// kernels of the DualMap routing library (sm_103a).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/dualmap.h"
+
+namespace dm {
+
+constexpr int kWarp = 32;
+constexpr uint32_t kSegBlocks = 256;       // blocks hashed by one warp task
+constexpr uint32_t kMaxInstances = 8192;
+constexpr uint32_t kMaxRouteBlocks = 256;
+constexpr uint32_t kTomb = 0xFFFFFFFFu;    // QEntry::moved of an entry migrated away
+constexpr int kMaxLevels = 8;
+constexpr uint64_t kSpinLimit = 1ull << 26; // bound of every data-dependent device loop
+
+// One queued request (48 bytes).
+struct QEntry {
+    uint64_t seq, work, remaining;
+    uint32_t L, c1, c2, h1, h2;
+    uint32_t moved;   // 0, or the rebalance call that moved it here, or kTomb
+};
+
+// One index slot / one recency-log record (16 bytes).  In the index, key 0
+// means empty and stamp 0 means "evicted" (the key stays, so a later touch
+// revives the slot in place).
+struct Slot {
+    uint64_t key, stamp;
+};
+
+// Per-batch values produced on the device.
+struct BatchInfo {
+    uint64_t total_blocks;
+    uint32_t total_segs;
+    uint32_t n;
+    uint64_t clock_base;    // commit clock before this batch's touches
+    uint32_t final_dirty;   // a rebalance moved a request of this batch
+    uint32_t pad;
+};
+
+struct Ring {
+    uint64_t *vpos;       // sorted positions, R entries
+    uint32_t *owner;      // owner id per entry
+    uint32_t *vidx;       // virtual-node index per entry (tie order)
+    uint64_t *tree;       // 32-ary search levels >= 1, concatenated
+};
+
+struct DevState {
+    // configuration
+    uint32_t B, Kroute, V, M;
+    uint64_t C, slo;
+    uint32_t cost, hot_num, hot_den, max_batch;
+    uint64_t max_blocks, max_segs, T, S, logcap;
+    uint32_t Q;
+    // key material
+    uint32_t K1[64], K2[64];
+    uint64_t G1, G2, Sc, Sr1, Sr2, Sv1, Sv2;
+    // rings (both have R entries)
+    Ring ring[2];
+    uint32_t R, nlev;
+    uint64_t lev_off[kMaxLevels];   // offset of level k (k >= 1) inside tree
+    uint64_t lev_n[kMaxLevels];     // entries in level k (lev_n[0] = R)
+    uint8_t *inst_state;            // 0 absent, 1 live, 2 draining
+    uint32_t *next_live;
+    // per instance
+    uint64_t *W;
+    uint32_t *q_head, *q_tail;
+    QEntry *q;                      // M x Q
+    Slot **table;                   // per id: S slots (null until first add)
+    Slot **logbuf;                  // per id: logcap records
+    uint64_t *log_front, *log_tail, *live, *used;
+    uint64_t *touch_cnt;            // per id: blocks touched by the pending commit
+    // batch scratch
+    uint32_t *r_L, *r_nblk, *r_segoff;
+    uint64_t *r_tokoff, *r_blkoff;
+    uint32_t *seg_req;
+    uint64_t *seg_total, *seg_carry, *plocal;
+    uint64_t *r_pos;                // 2 per request
+    uint32_t *r_c1, *r_c2, *r_h1, *r_h2, *r_final;
+    uint64_t *r_touchoff;
+    BatchInfo *info;
+    uint64_t *clock;
+    uint32_t *err;
+    uint64_t *seq_next;
+    // rebalance scratch
+    uint64_t *rb_key;               // sort keys (benefit, biased) per candidate
+    uint64_t *rb_seq;
+    uint64_t *rb_ttft;
+    uint32_t *rb_pos;               // queue position of the candidate
+    uint32_t rb_cap;                // candidates that fit (power of two)
+};
+
+// ---------------------------------------------------------------------------
+// Published mixers.
+// MurmurHash3 64-bit finaliser (Appleby, public domain).
+__device__ __host__ __forceinline__ uint64_t fmix64(uint64_t k) {
+    k ^= k >> 33;
+    k *= 0xff51afd7ed558ccdULL;
+    k ^= k >> 33;
+    k *= 0xc4ceb9fe1a85ec53ULL;
+    k ^= k >> 33;
+    return k;
+}
+
+// One SplitMix64 output step from state x (Steele, Lea & Flood 2014).
+__device__ __host__ __forceinline__ uint64_t splitmix_step(uint64_t x) {
+    uint64_t z = x + 0x9E3779B97F4A7C15ULL;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+    return z ^ (z >> 31);
+}
+
+// Cache key of a block from its chained prefix value (0 is the empty slot).
+__device__ __forceinline__ uint64_t cache_key(uint64_t P, uint64_t Sc) {
+    uint64_t k = fmix64(P ^ Sc);
+    return k ? k : 1ull;
+}
+
+// Virtual-node position of (id, v) on a ring with seed Sv.
+__device__ __host__ __forceinline__ uint64_t vnode_pos(uint64_t Sv, uint32_t id, uint32_t v) {
+    return fmix64(splitmix_step((uint64_t(id) << 32) | v) ^ Sv);
+}
+
+// First error wins; kernels of a call stop at entry once it is set.
+__device__ __forceinline__ void set_err(uint32_t *err, uint32_t code) {
+    atomicCAS(err, 0u, code);
+}
+
+__device__ __forceinline__ bool has_err(const uint32_t *err) {
+    return *(volatile const uint32_t *)err != 0u;
+}
+
+__device__ __forceinline__ uint64_t shfl_u64(uint64_t v, int src) {
+    return __shfl_sync(0xffffffffu, v, src);
+}
+
+__device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t v, int m) {
+    return __shfl_xor_sync(0xffffffffu, v, m);
+}
+
+__device__ __forceinline__ uint64_t shfl_up_u64(uint64_t v, int d) {
+    return __shfl_up_sync(0xffffffffu, v, d);
+}
+
+// Inclusive warp scan of uint64 values (mod 2^64).
+__device__ __forceinline__ uint64_t warp_incl_scan(uint64_t v, int lane) {
+#pragma unroll
+    for (int d = 1; d < kWarp; d <<= 1) {
+        uint64_t u = shfl_up_u64(v, d);
+        if (lane >= d) v += u;
+    }
+    return v;
+}
+
+// 16-byte slot load that bypasses L1 (probes are random; L2 is the cache).
+__device__ __forceinline__ Slot load_slot(const Slot *p) {
+    Slot s;
+    asm volatile("ld.global.cg.v2.u64 {%0, %1}, [%2];"
+                 : "=l"(s.key), "=l"(s.stamp) : "l"(__cvta_generic_to_global(p)));
+    return s;
+}
+
+// Look key up in one instance's open-addressed (linear probing) index.
+// Returns the slot index holding the key (live or evicted) or -1.
+__device__ __forceinline__ int64_t table_find(const Slot *t, uint64_t mask, uint64_t key,
+                                              uint64_t *stamp, uint32_t *err) {
+    uint64_t i = key & mask;
+    for (uint64_t it = 0; it <= mask; ++it) {
+        Slot s = load_slot(t + i);
+        if (s.key == key) { *stamp = s.stamp; return (int64_t)i; }
+        if (s.key == 0) return -1;
+        i = (i + 1) & mask;
+    }
+    set_err(err, DM_ERR_TIMEOUT);
+    return -1;
+}
+
+// Carries of one request's segments (exclusive prefix of the segment
+// totals written by the hashing kernel), stored in seg_carry.  Whole warp.
+__device__ __forceinline__ void request_carries(const DevState &d, uint32_t r, int lane) {
+    const uint32_t s0 = d.r_segoff[r];
+    const uint32_t ns = (d.r_nblk[r] + kSegBlocks - 1) / kSegBlocks;
+    uint64_t carry = 0;
+    for (uint32_t b = 0; b < ns; b += 32) {
+        const uint32_t s = b + lane;
+        const uint64_t t = s < ns ? d.seg_total[s0 + s] : 0;
+        const uint64_t inc = warp_incl_scan(t, lane);
+        if (s < ns) d.seg_carry[s0 + s] = carry + inc - t;
+        carry += shfl_u64(inc, 31);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Host-side launchers (one translation unit each).
+cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st);
+cudaError_t launch_drain(const DevState &d, uint64_t delta, cudaStream_t st);
+cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st);
+int hash_grid_size();
+cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
+                               cudaStream_t st);
+cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, uint64_t seq0,
+                          cudaStream_t st);
+cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st);
+cudaError_t launch_rebalance(const DevState &d, uint32_t n, uint64_t seq0, uint32_t call,
+                             dm_migration *out, uint32_t cap, uint32_t *n_out, cudaStream_t st);
+cudaError_t launch_hash_keys(const DevState &d, uint32_t n, uint64_t *keys, uint64_t *key_off,
+                             uint64_t *pos, cudaStream_t st);
+cudaError_t launch_ring_lookup(const DevState &d, const uint64_t *pos, uint32_t n, uint32_t *o1,
+                               uint32_t *o2, cudaStream_t st);
+cudaError_t launch_ring_update(DevState &d, uint32_t id, bool add, uint32_t new_R,
+                               uint64_t *scratch_pos, uint32_t *scratch_owner,
+                               uint32_t *scratch_vidx, uint64_t *new_vpos[2],
+                               uint32_t *new_owner[2], uint32_t *new_vidx[2], cudaStream_t st);
+cudaError_t launch_tree_build(const DevState &d, cudaStream_t st);
+cudaError_t launch_next_live(const DevState &d, cudaStream_t st);
+cudaError_t launch_set_state(const DevState &d, uint32_t id, uint8_t s, cudaStream_t st);
+
+}  // namespace dm

@@ -1,0 +1,240 @@
+"""ctypes binding of libdualmap.so (include/dualmap.h).
+
+Argument marshalling only: every step of the routing path runs in the
+library's CUDA kernels.  PyTorch supplies device memory and streams.  There
+is no fallback: if the shared library is missing, importing the binding's
+functions raises.
+"""
+
+import ctypes as C
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libdualmap.so")
+
+DM_OK, DM_ERR_INVALID_ARG, DM_ERR_CAPACITY, DM_ERR_NO_INSTANCES = 0, 1, 2, 3
+DM_ERR_DUPLICATE_ID, DM_ERR_UNKNOWN_ID, DM_ERR_ORDER, DM_ERR_CUDA = 4, 5, 6, 7
+DM_ERR_TIMEOUT, DM_ERR_OOM = 8, 9
+STAGES = ["setup", "drain", "hash", "probe", "choice", "commit", "rebalance"]
+
+
+class dm_config(C.Structure):
+    _fields_ = [
+        ("block_tokens", C.c_uint32),
+        ("route_prefix_blocks", C.c_uint32),
+        ("vnodes_per_instance", C.c_uint32),
+        ("max_instances", C.c_uint32),
+        ("cache_capacity_blocks", C.c_uint64),
+        ("slo_us", C.c_uint64),
+        ("cost_us_per_token", C.c_uint32),
+        ("hot_num", C.c_uint32),
+        ("hot_den", C.c_uint32),
+        ("max_batch", C.c_uint32),
+        ("max_batch_tokens", C.c_uint64),
+        ("max_touch_per_instance", C.c_uint64),
+        ("max_queue", C.c_uint32),
+        ("reserved0", C.c_uint32),
+        ("seed", C.c_uint64),
+        ("stream", C.c_void_p),
+    ]
+
+
+class dm_batch(C.Structure):
+    _fields_ = [
+        ("tokens", C.c_void_p),
+        ("offsets", C.c_void_p),
+        ("lengths", C.c_void_p),
+        ("n", C.c_uint32),
+        ("reserved0", C.c_uint32),
+        ("total_tokens", C.c_uint64),
+        ("batch_time_us", C.c_uint64),
+    ]
+
+
+class dm_route_out(C.Structure):
+    _fields_ = [(name, C.c_void_p) for name in
+                ("cand1", "cand2", "hit1", "hit2", "ttft1", "ttft2", "chosen", "switched")]
+
+
+class dm_migration(C.Structure):
+    _fields_ = [("req_seq", C.c_uint64), ("from_", C.c_uint32), ("to", C.c_uint32)]
+
+
+class DualMapError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+_lib = None
+
+# name -> (restype, argtypes); the exported set is exactly include/dualmap.h
+SIGNATURES = {
+    "dm_create": (C.c_int, [C.POINTER(dm_config), C.POINTER(C.c_void_p)]),
+    "dm_destroy": (None, [C.c_void_p]),
+    "dm_add_instance": (C.c_int, [C.c_void_p, C.c_uint32]),
+    "dm_remove_instance": (C.c_int, [C.c_void_p, C.c_uint32]),
+    "dm_route_batch": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
+    "dm_route_batch_host": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
+    "dm_rebalance": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]),
+    "dm_commit_cache": (C.c_int, [C.c_void_p]),
+    "dm_hash_prompts": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.c_void_p, C.c_void_p, C.c_void_p]),
+    "dm_ring_lookup": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p]),
+    "dm_get_loads": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32]),
+    "dm_export_cache": (C.c_int, [C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p, C.c_uint64,
+                                  C.POINTER(C.c_uint64)]),
+    "dm_export_queue": (C.c_int, [C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_uint64,
+                                  C.POINTER(C.c_uint64)]),
+    "dm_export_ring": (C.c_int, [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_uint32,
+                                 C.POINTER(C.c_uint32)]),
+    "dm_get_clock": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64)]),
+    "dm_last_error": (C.c_int, [C.c_void_p]),
+    "dm_set_profiling": (C.c_int, [C.c_void_p, C.c_int]),
+    "dm_get_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int]),
+    "dm_status_string": (C.c_char_p, [C.c_int]),
+}
+
+
+def lib():
+    """The loaded shared library; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        L = C.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def status_string(s):
+    return lib().dm_status_string(s).decode()
+
+
+def _check(rc, where):
+    if rc != DM_OK:
+        raise DualMapError(rc, where)
+
+
+def _ptr(t):
+    """Device (or host) address of a torch tensor / numpy array, or None."""
+    if t is None:
+        return None
+    if hasattr(t, "data_ptr"):
+        return t.data_ptr()
+    return t.ctypes.data
+
+
+# -- the C ABI, name for name ------------------------------------------------
+
+def dm_create(cfg):
+    h = C.c_void_p()
+    _check(lib().dm_create(C.byref(cfg), C.byref(h)), "dm_create")
+    return h
+
+
+def dm_destroy(h):
+    lib().dm_destroy(h)
+
+
+def dm_add_instance(h, i):
+    return lib().dm_add_instance(h, i)
+
+
+def dm_remove_instance(h, i):
+    return lib().dm_remove_instance(h, i)
+
+
+def make_batch(tokens, offsets, lengths, n, total_tokens, batch_time_us):
+    return dm_batch(_ptr(tokens), _ptr(offsets), _ptr(lengths), n, 0, total_tokens, batch_time_us)
+
+
+def make_out(cand1, cand2, hit1, hit2, ttft1, ttft2, chosen, switched):
+    return dm_route_out(*[_ptr(x) for x in (cand1, cand2, hit1, hit2, ttft1, ttft2, chosen, switched)])
+
+
+def dm_route_batch(h, batch, out):
+    return lib().dm_route_batch(h, C.byref(batch), C.byref(out))
+
+
+def dm_route_batch_host(h, batch, out):
+    return lib().dm_route_batch_host(h, C.byref(batch), C.byref(out))
+
+
+def dm_rebalance(h, out_dev, cap, n_out_dev):
+    return lib().dm_rebalance(h, _ptr(out_dev), cap, _ptr(n_out_dev))
+
+
+def dm_commit_cache(h):
+    return lib().dm_commit_cache(h)
+
+
+def dm_hash_prompts(h, batch, keys_dev, key_off_dev, pos_dev):
+    return lib().dm_hash_prompts(h, C.byref(batch), _ptr(keys_dev), _ptr(key_off_dev), _ptr(pos_dev))
+
+
+def dm_ring_lookup(h, pos_dev, n, owner1_dev, owner2_dev):
+    return lib().dm_ring_lookup(h, _ptr(pos_dev), n, _ptr(owner1_dev), _ptr(owner2_dev))
+
+
+def dm_get_loads(h, M):
+    W = np.zeros(M, np.uint64)
+    _check(lib().dm_get_loads(h, W.ctypes.data, M), "dm_get_loads")
+    return W
+
+
+def dm_export_cache(h, i):
+    n = C.c_uint64()
+    _check(lib().dm_export_cache(h, i, None, None, 0, C.byref(n)), "dm_export_cache")
+    k = np.zeros(max(n.value, 1), np.uint64)
+    s = np.zeros(max(n.value, 1), np.uint64)
+    _check(lib().dm_export_cache(h, i, k.ctypes.data, s.ctypes.data, n.value, C.byref(n)), "dm_export_cache")
+    return k[:n.value], s[:n.value]
+
+
+def dm_export_queue(h, i, cap=1 << 20):
+    n = C.c_uint64()
+    seq = np.zeros(cap, np.uint64)
+    work = np.zeros(cap, np.uint64)
+    rem = np.zeros(cap, np.uint64)
+    _check(lib().dm_export_queue(h, i, seq.ctypes.data, work.ctypes.data, rem.ctypes.data, cap, C.byref(n)),
+           "dm_export_queue")
+    m = min(n.value, cap)
+    return seq[:m], work[:m], rem[:m]
+
+
+def dm_export_ring(h, f, cap):
+    n = C.c_uint32()
+    vp = np.zeros(max(cap, 1), np.uint64)
+    ow = np.zeros(max(cap, 1), np.uint32)
+    _check(lib().dm_export_ring(h, f, vp.ctypes.data, ow.ctypes.data, cap, C.byref(n)), "dm_export_ring")
+    m = min(n.value, cap)
+    return vp[:m], ow[:m]
+
+
+def dm_get_clock(h):
+    c = C.c_uint64()
+    _check(lib().dm_get_clock(h, C.byref(c)), "dm_get_clock")
+    return c.value
+
+
+def dm_last_error(h):
+    return lib().dm_last_error(h)
+
+
+def dm_set_profiling(h, on):
+    return lib().dm_set_profiling(h, 1 if on else 0)
+
+
+def dm_get_stage_times(h, reset=False):
+    ms = np.zeros(len(STAGES), np.float64)
+    calls = np.zeros(len(STAGES), np.uint64)
+    _check(lib().dm_get_stage_times(h, ms.ctypes.data, calls.ctypes.data, 1 if reset else 0),
+           "dm_get_stage_times")
+    return {s: (float(ms[i]), int(calls[i])) for i, s in enumerate(STAGES)}

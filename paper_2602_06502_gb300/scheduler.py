@@ -1,0 +1,88 @@
+"""Convenience wrapper of one dm_handle with torch-owned device buffers.
+
+Only marshalling: it allocates output tensors on the device, builds the
+C structs, calls the C ABI and raises on error statuses.
+"""
+
+import ctypes as C
+
+import torch
+
+from . import dualmap as D
+
+OUT_FIELDS = [("cand1", torch.int32), ("cand2", torch.int32), ("hit1", torch.int32), ("hit2", torch.int32),
+              ("ttft1", torch.int64), ("ttft2", torch.int64), ("chosen", torch.int32), ("switched", torch.uint8)]
+
+
+class Scheduler:
+    def __init__(self, *, block_tokens=16, route_prefix_blocks=16, vnodes=64, max_instances=16,
+                 capacity=65536, slo_us=2_000_000, cost_us=1, hot_num=3, hot_den=2, max_batch=4096,
+                 max_batch_tokens=1 << 24, max_touch_per_instance=0, max_queue=0, seed=0, stream=None,
+                 device="cuda"):
+        self.device = torch.device(device)
+        self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
+        self.cfg = D.dm_config(block_tokens, route_prefix_blocks, vnodes, max_instances, capacity, slo_us,
+                               cost_us, hot_num, hot_den, max_batch, max_batch_tokens, max_touch_per_instance,
+                               max_queue, 0, seed, C.c_void_p(self.stream.cuda_stream))
+        self.h = D.dm_create(self.cfg)
+        self.M = max_instances
+        self.max_batch = max_batch
+        self.out = {k: torch.zeros(max_batch, dtype=t, device=self.device) for k, t in OUT_FIELDS}
+        self.out_struct = D.make_out(*[self.out[k] for k, _ in OUT_FIELDS])
+        self.mig = torch.zeros(1 << 16, 2, dtype=torch.int64, device=self.device)   # 16-byte records
+        self.mig_n = torch.zeros(1, dtype=torch.int32, device=self.device)
+
+    def close(self):
+        if self.h:
+            D.dm_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def add_instance(self, i):
+        return D.dm_add_instance(self.h, i)
+
+    def remove_instance(self, i):
+        return D.dm_remove_instance(self.h, i)
+
+    def route(self, tokens, offsets, lengths, n, total_tokens, t_batch, check=True):
+        """Route one batch held in device tensors; returns the status."""
+        b = D.make_batch(tokens, offsets, lengths, n, total_tokens, t_batch)
+        rc = D.dm_route_batch(self.h, b, self.out_struct)
+        if check and rc:
+            raise D.DualMapError(rc, "dm_route_batch")
+        return rc
+
+    def results(self, n):
+        """Host copies (numpy) of the last batch's outputs."""
+        torch.cuda.synchronize(self.device)
+        return {k: self.out[k][:n].cpu().numpy() for k, _ in OUT_FIELDS}
+
+    def rebalance(self):
+        rc = D.dm_rebalance(self.h, self.mig, self.mig.shape[0], self.mig_n)
+        if rc:
+            raise D.DualMapError(rc, "dm_rebalance")
+
+    def migrations(self):
+        torch.cuda.synchronize(self.device)
+        n = int(self.mig_n.item())
+        m = self.mig[:min(n, self.mig.shape[0])].cpu().numpy()
+        seq = m[:, 0].astype("uint64")
+        fr = (m[:, 1].astype("uint64") & 0xFFFFFFFF).astype("uint32")
+        to = (m[:, 1].astype("uint64") >> 32).astype("uint32")
+        return n, (seq, fr, to)
+
+    def commit(self):
+        rc = D.dm_commit_cache(self.h)
+        if rc:
+            raise D.DualMapError(rc, "dm_commit_cache")
+
+    def last_error(self):
+        return D.dm_last_error(self.h)
+
+    def loads(self):
+        return D.dm_get_loads(self.h, self.M)

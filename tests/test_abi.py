@@ -1,0 +1,91 @@
+"""The C-ABI library loads without a GPU, exports exactly the entry points
+include/dualmap.h declares, and the binding's struct layouts match the
+header's as compiled by the host C compiler."""
+
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HDR = os.path.join(ROOT, "include", "dualmap.h")
+
+
+@pytest.fixture(scope="module")
+def built():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2602_06502_gb300 import dualmap as D
+    return D
+
+
+def declared():
+    txt = open(HDR).read()
+    return sorted(set(re.findall(r"^DM_API [^(]*?\b(dm_\w+)\(", txt, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared()
+    for must in ("dm_create", "dm_destroy", "dm_add_instance", "dm_remove_instance", "dm_route_batch",
+                 "dm_commit_cache", "dm_rebalance"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(built):
+    D = built
+    exported = subprocess.run(["nm", "-D", "--defined-only", D.LIB_PATH], capture_output=True, text=True,
+                              check=True).stdout
+    syms = set(re.findall(r"\sT\s(dm_\w+)", exported))
+    assert set(declared()) == syms
+    assert set(D.SIGNATURES) == syms
+    lib = C.CDLL(D.LIB_PATH)
+    for s in declared():
+        assert getattr(lib, s) is not None
+
+
+def test_status_strings_without_gpu(built):
+    D = built
+    assert D.status_string(0) == "ok"
+    assert "instances" in D.status_string(3)
+
+
+def test_create_rejects_bad_config_without_touching_gpu(built):
+    """Synchronous argument checks run before any CUDA call."""
+    D = built
+    bad = D.dm_config(17, 16, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)   # B = 17
+    h = C.c_void_p()
+    assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
+    bad2 = D.dm_config(16, 0, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)   # K_route = 0
+    assert D.lib().dm_create(C.byref(bad2), C.byref(h)) == D.DM_ERR_INVALID_ARG
+    bad3 = D.dm_config(16, 16, 8, 1, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)  # one instance
+    assert D.lib().dm_create(C.byref(bad3), C.byref(h)) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
+
+
+def test_struct_layouts_match_header(built, tmp_path):
+    D = built
+    prog = tmp_path / "layout.c"
+    fields = {
+        "dm_config": [f for f, _ in D.dm_config._fields_],
+        "dm_batch": [f for f, _ in D.dm_batch._fields_],
+        "dm_route_out": [f for f, _ in D.dm_route_out._fields_],
+        "dm_migration": ["req_seq", "from", "to"],
+    }
+    lines = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HDR}"', "int main(void) {"]
+    for st, fs in fields.items():
+        lines.append(f'printf("{st} %zu\\n", sizeof({st}));')
+        for f in fs:
+            lines.append(f'printf("{st}.{f} %zu\\n", offsetof({st}, {f}));')
+    lines.append("return 0; }")
+    prog.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", str(prog), "-o", str(exe)], check=True)
+    out = dict(l.rsplit(" ", 1) for l in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                        check=True).stdout.split("\n") if l)
+    for st, cls in (("dm_config", D.dm_config), ("dm_batch", D.dm_batch), ("dm_route_out", D.dm_route_out),
+                    ("dm_migration", D.dm_migration)):
+        assert int(out[st]) == C.sizeof(cls), st
+        for (py, _), cn in zip(cls._fields_, fields[st]):
+            assert int(out[f"{st}.{cn}"]) == getattr(cls, py).offset, (st, cn)

@@ -1,0 +1,333 @@
+"""Bit-exact parity of the CUDA routing path (through the C ABI) with the CPU
+oracle on seeded synthetic traces of all five workload shapes, plus edge
+cases and error behaviour."""
+
+import numpy as np
+import pytest
+
+from parity_harness import Pair, lib_ready, run_trace
+from tracegen import Trace, workload
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    lib_ready()
+
+
+def _torch():
+    import torch
+    return torch
+
+
+# -- inputs and hashing ------------------------------------------------------------
+
+def test_device_token_filler_matches_host():
+    torch = _torch()
+    import tracegen.device as TD
+    tr = Trace(workload("multiturn", n_requests=300, batch=100))
+    r0, r1 = 37, 211
+    n = int(tr.req_off[r1] - tr.req_off[r0])
+    buf = torch.zeros(n + 4, dtype=torch.int32, device="cuda")
+    TD.fill_range(tr, r0, r1, buf)
+    got = buf.cpu().numpy().view(np.uint32)
+    for r in range(r0, r1):
+        o = int(tr.req_off[r] - tr.req_off[r0])
+        assert np.array_equal(got[o:o + tr.L[r]], tr.request_tokens(r)), r
+
+
+def _lengths_mix(B, rng):
+    """Edge lengths (exactly one block, one block + 1, segment boundaries of
+    256 blocks, a ragged tail) plus random lengths spanning several segments."""
+    fixed = [B, B + 1, 2 * B - 1, 31 * B, 32 * B, 33 * B + 3, 256 * B, 256 * B + 1, 257 * B, 600 * B + 5]
+    return fixed + rng.integers(B, 900 * B, size=40).tolist()
+
+
+@pytest.mark.parametrize("B,K", [(16, 16), (4, 1), (8, 40), (32, 7), (64, 256), (16, 256)])
+def test_hash_prompts_parity(B, K):
+    torch = _torch()
+    from oracle import oracle as O
+    from paper_2602_06502_gb300 import dualmap as D
+    from paper_2602_06502_gb300.scheduler import Scheduler
+    rng = np.random.default_rng(B * 1000 + K)
+    lens = np.array(_lengths_mix(B, rng), np.uint32)
+    off = np.zeros(len(lens), np.uint64)
+    off[1:] = np.cumsum((lens[:-1] + 3) // 4 * 4)
+    ntok = int(off[-1] + lens[-1])
+    tok = rng.integers(0, 1 << 32, size=ntok, dtype=np.uint64).astype(np.uint32)
+    seed = 77 + B
+    ora = O.Oracle(block_tokens=B, route_prefix_blocks=K, vnodes_per_instance=4, max_instances=4,
+                   cache_capacity_blocks=16, slo_us=1, cost_us_per_token=1, hot_num=3, hot_den=2,
+                   max_batch=len(lens), max_batch_tokens=1 << 24, seed=seed)
+    g = Scheduler(block_tokens=B, route_prefix_blocks=K, vnodes=4, max_instances=4, capacity=16,
+                  max_batch=len(lens), max_batch_tokens=ntok + 64, seed=seed)
+    dt = torch.from_numpy(tok.view(np.int32)).cuda()
+    do = torch.from_numpy(off.view(np.int64)).cuda()
+    dl = torch.from_numpy(lens.view(np.int32)).cuda()
+    nblk = lens // B
+    keys = torch.zeros(int(nblk.sum()) + 1, dtype=torch.int64, device="cuda")
+    koff = torch.zeros(len(lens) + 1, dtype=torch.int64, device="cuda")
+    pos = torch.zeros(2 * len(lens), dtype=torch.int64, device="cuda")
+    b = D.make_batch(dt, do, dl, len(lens), ntok, 0)
+    assert D.dm_hash_prompts(g.h, b, keys, koff, pos) == 0
+    assert g.last_error() == 0
+    keys = keys.cpu().numpy().view(np.uint64)
+    koff = koff.cpu().numpy().view(np.uint64)
+    pos = pos.cpu().numpy().view(np.uint64).reshape(-1, 2)
+    assert np.array_equal(np.diff(koff.astype(np.int64)), nblk.astype(np.int64))
+    for r in range(len(lens)):
+        want_k, want_p = ora.prompt_keys(tok[int(off[r]):int(off[r]) + int(lens[r])])
+        got_k = keys[int(koff[r]):int(koff[r + 1])]
+        assert np.array_equal(got_k, want_k), (r, int(lens[r]))
+        assert np.array_equal(pos[r], want_p), r
+    g.close()
+
+
+def test_ring_parity_add_remove_lookup():
+    torch = _torch()
+    from oracle import oracle as O
+    from paper_2602_06502_gb300 import dualmap as D
+    w = workload("tiny", vnodes=37)
+    p = Pair(w, max_instances=20)
+    rng = np.random.default_rng(4)
+    pos = rng.integers(0, 2**63, size=2000, dtype=np.int64).astype(np.uint64) * np.uint64(2)
+
+    def check():
+        for f in (0, 1):
+            vp, ow, _ = p.ora.ring(f)
+            gv, go = D.dm_export_ring(p.gpu.h, f, len(vp) + 8)
+            assert np.array_equal(gv, vp) and np.array_equal(go, ow)
+        dpos = torch.from_numpy(pos.view(np.int64)).cuda()
+        o1 = torch.zeros(len(pos) // 2, dtype=torch.int32, device="cuda")
+        o2 = torch.zeros_like(o1)
+        assert D.dm_ring_lookup(p.gpu.h, dpos, len(pos) // 2, o1, o2) == 0
+        pr = pos.reshape(-1, 2)
+        assert np.array_equal(o1.cpu().numpy().astype(np.uint32), p.ora.ring_owners(pr[:, 0].copy(), 0))
+        assert np.array_equal(o2.cpu().numpy().astype(np.uint32), p.ora.ring_owners(pr[:, 1].copy(), 1))
+        # a position equal to a vnode position belongs to that vnode
+        vp, ow, _ = p.ora.ring(0)
+        eq = np.repeat(vp[:200], 2)
+        deq = torch.from_numpy(eq.view(np.int64)).cuda()
+        assert D.dm_ring_lookup(p.gpu.h, deq, 200, o1, o2) == 0
+        assert np.array_equal(o1[:200].cpu().numpy().astype(np.uint32), ow[:200])
+
+    for i in [0, 3, 1, 7]:
+        p.add(i)
+        check()
+    for i in range(8, 20):
+        p.add(i)
+    check()
+    for i in [3, 19, 8, 0]:
+        p.remove(i)
+        check()
+    p.add(19)   # removed, nothing queued: may be re-added
+    check()
+
+
+# -- whole traces -------------------------------------------------------------------
+
+@pytest.mark.parametrize("seed", [1001, 1, 2, 3, 4, 5, 6])
+def test_tiny_trace_parity(seed):
+    tr = Trace(workload("tiny"), seed=seed)
+    run_trace(Pair(tr.cfg), tr, state_every=4)
+
+
+def test_tiny_trace_with_rebalance_and_small_cache():
+    """Eviction every batch, log compaction and index rebuilds (small C and
+    touch bound), rebalancing after every batch."""
+    w = workload("tiny", n_requests=2000, batch=100, capacity=700, zipf_s=1.3, rho=1.2)
+    tr = Trace(w)
+    p = Pair(w, max_touch=2600)
+    run_trace(p, tr, rebalance=True, state_every=5)
+
+
+def test_multiturn_parity():
+    tr = Trace(workload("multiturn", n_requests=6144))
+    p = Pair(tr.cfg, max_batch_tokens=1 << 25, capacity=60_000, max_touch=200_000)
+    run_trace(p, tr, state_every=3)
+
+
+def test_agent_parity():
+    tr = Trace(workload("agent", n_requests=3 * 4096))
+    p = Pair(tr.cfg, max_batch_tokens=40_000_000, max_touch=1 << 20)
+    run_trace(p, tr)
+    assert p.n_switched > 0      # the tight load makes the SLO rule fire
+
+
+def test_longctx_parity():
+    tr = Trace(workload("longctx", n_requests=3 * 512))
+    p = Pair(tr.cfg, max_batch_tokens=70_000_000, max_touch=1 << 20, capacity=200_000)
+    run_trace(p, tr)
+
+
+def test_scaling_parity_with_events():
+    """256 instances x 1,024 vnodes, rebalancing after every batch, an instance
+    added or removed between batches."""
+    w = workload("scaling", n_requests=5 * 4096, scale_every=4096, capacity=20_000)
+    tr = Trace(w)
+    assert len(tr.events) >= 3
+    p = Pair(tr.cfg, max_instances=w["n_instances"] + 4, max_batch_tokens=40_000_000, max_touch=1 << 20)
+    run_trace(p, tr, rebalance=True)
+
+
+# -- edge cases ---------------------------------------------------------------------
+
+def _mk(**kw):
+    base = dict(workload("tiny"))
+    base.update(kw)
+    return base
+
+
+def _batch(prompts):
+    lens = np.array([len(x) for x in prompts], np.uint32)
+    off = np.zeros(len(prompts), np.uint64)
+    if len(prompts) > 1:
+        off[1:] = np.cumsum((lens[:-1].astype(np.uint64) + 3) // 4 * 4)
+    tot = int(off[-1] + lens[-1]) if len(prompts) else 0
+    tok = np.zeros(max(tot, 4), np.uint32)
+    for o, x in zip(off, prompts):
+        tok[int(o):int(o) + len(x)] = x
+    return tok, off, lens
+
+
+def test_edge_cases_small_clusters():
+    rng = np.random.default_rng(12)
+    w = _mk(n_instances=2, vnodes=1, capacity=50, batch=64)
+    p = Pair(w, max_instances=3)
+    p.add(0)
+    p.add(1)
+    same = rng.integers(0, 32000, size=16 * 9, dtype=np.uint32)
+    t = 0
+    for step in range(6):
+        prompts = [same] * 5 + [rng.integers(0, 32000, size=int(L), dtype=np.uint32)
+                                for L in (16, 17, 31, 32, 48, 16 * 64)]
+        tok, off, lens = _batch(prompts)
+        p.route(tok, off, lens, t, tag=f"step {step}")
+        p.rebalance()
+        p.commit()
+        p.check_state()
+        t += 7
+    # a batch of one, then an empty batch (time only), then identical time
+    tok, off, lens = _batch([same])
+    p.route(tok, off, lens, t)
+    p.commit()
+    p.route(np.zeros(4, np.uint32), np.zeros(0, np.uint64), np.zeros(0, np.uint32), t + 100)
+    p.commit()
+    p.check_state()
+    p.add(2)
+    p.remove(0)            # remove down to two live instances
+    tok, off, lens = _batch([same] * 3)
+    p.route(tok, off, lens, t + 100)
+    p.commit()
+    p.check_state()
+
+
+def test_zero_load_and_non_dense_ids():
+    rng = np.random.default_rng(13)
+    w = _mk(vnodes=16, capacity=10_000, batch=128)
+    p = Pair(w, max_instances=12)
+    for i in (1, 4, 5, 9, 11):
+        p.add(i)
+    prompts = [rng.integers(0, 32000, size=int(L), dtype=np.uint32) for L in rng.integers(16, 3000, size=100)]
+    tok, off, lens = _batch(prompts)
+    p.route(tok, off, lens, 0)             # W = 0 everywhere at the start
+    p.commit()
+    p.remove(5)
+    p.route(tok, off, lens, 10**9)          # everything drained: W = 0 again
+    p.rebalance()
+    p.commit()
+    p.check_state()
+
+
+def test_error_statuses_match_oracle():
+    from paper_2602_06502_gb300 import dualmap as D
+    rng = np.random.default_rng(14)
+    w = _mk(batch=4)
+    p = Pair(w, max_instances=6)
+    tok, off, lens = _batch([rng.integers(0, 32000, size=64, dtype=np.uint32)])
+    dt, do, dl = p.to_dev(tok, off, lens)
+    assert p.gpu.route(dt, do, dl, 1, len(tok), 0, check=False) == D.DM_ERR_NO_INSTANCES
+    assert p.add(0) == 0
+    assert p.add(0) == D.DM_ERR_DUPLICATE_ID
+    assert p.add(6) == D.DM_ERR_INVALID_ARG
+    assert p.remove(3) == D.DM_ERR_UNKNOWN_ID
+    assert p.add(1) == 0
+    p.route(tok, off, lens, 50)
+    assert p.gpu.route(dt, do, dl, 1, len(tok), 49, check=False) == D.DM_ERR_ORDER
+    assert p.ora.route_batch(tok, off, lens, 49)[0] == D.DM_ERR_ORDER
+    tok5, off5, lens5 = _batch([tok[:16]] * 5)
+    d5 = p.to_dev(tok5, off5, lens5)
+    assert p.gpu.route(*d5, 5, len(tok5), 60, check=False) == D.DM_ERR_CAPACITY
+    # a removed instance with queued work cannot come back until drained
+    busy = int(p.gpu.results(1)["chosen"][0])
+    assert p.remove(busy) == 0
+    assert p.add(busy) == D.DM_ERR_DUPLICATE_ID
+    assert p.gpu.last_error() == 0
+
+
+def test_device_side_validation_is_sticky():
+    """A prompt shorter than one block is rejected in the set-up kernel: the
+    call's kernels do nothing and the handle reports the error."""
+    torch = _torch()
+    from paper_2602_06502_gb300 import dualmap as D
+    from paper_2602_06502_gb300.scheduler import Scheduler
+    g = Scheduler(vnodes=8, max_instances=4, max_batch=4, max_batch_tokens=1 << 12, seed=3)
+    g.add_instance(0)
+    g.add_instance(1)
+    tok = torch.zeros(64, dtype=torch.int32, device="cuda")
+    off = torch.tensor([0, 16], dtype=torch.int64, device="cuda")
+    ln = torch.tensor([32, 15], dtype=torch.int32, device="cuda")
+    assert g.route(tok, off, ln, 2, 64, 0, check=False) == 0
+    assert g.last_error() == D.DM_ERR_INVALID_ARG
+    assert np.all(g.loads() == 0)                 # nothing was queued
+    assert g.route(tok, off, ln, 2, 64, 1, check=False) == D.DM_ERR_INVALID_ARG
+    g.close()
+    g = Scheduler(vnodes=8, max_instances=4, max_batch=4, max_batch_tokens=1 << 12, seed=3)
+    g.add_instance(0)
+    g.add_instance(1)
+    off = torch.tensor([0, 18], dtype=torch.int64, device="cuda")    # not 16-byte aligned
+    ln = torch.tensor([16, 16], dtype=torch.int32, device="cuda")
+    assert g.route(tok, off, ln, 2, 64, 0, check=False) == 0
+    assert g.last_error() == D.DM_ERR_INVALID_ARG
+    g.close()
+
+
+def test_host_buffer_entry_point_matches_device_path():
+    from paper_2602_06502_gb300 import dualmap as D
+    from paper_2602_06502_gb300.scheduler import OUT_FIELDS
+    tr = Trace(workload("tiny", n_requests=768, batch=256))
+    a = Pair(tr.cfg)
+    b = Pair(tr.cfg)
+    for i in range(tr.cfg["n_instances"]):
+        a.add(i)
+        b.add(i)
+    for k in range(len(tr.batches)):
+        s, e, off, lens, ntok = tr.batch_layout(k)
+        tok = tr.batch_tokens(k)
+        want = a.route(tok, off, lens, tr.batch_time(k))
+        n = e - s
+        host = {name: np.zeros(n, dtype={"int32": np.uint32, "int64": np.uint64, "uint8": np.uint8}[str(t).split(".")[1]])
+                for name, t in OUT_FIELDS}
+        bt = D.make_batch(tok, off, lens, n, ntok, tr.batch_time(k))
+        out = D.make_out(*[host[name] for name, _ in OUT_FIELDS])
+        assert D.dm_route_batch_host(b.gpu.h, bt, out) == 0
+        b.ora.route_batch(tok, off, lens, tr.batch_time(k))
+        for name in want:
+            assert np.array_equal(host[name], want[name]), name
+        a.commit()
+        b.commit()
+    b.check_state()
+
+
+def test_longctx_full_size_batches():
+    """The long-context workload at its real sizes (512 prompts of 32k-131k
+    tokens per batch) in the launch configuration the benchmark uses: the
+    first batches compared in full."""
+    from bench import longctx_handle_kwargs
+    tr = Trace(workload("longctx"))
+    kw = longctx_handle_kwargs(tr.cfg)
+    p = Pair(tr.cfg, max_instances=kw["max_instances"], max_batch_tokens=kw["max_batch_tokens"],
+             max_touch=kw["max_touch_per_instance"])
+    run_trace(p, tr, batches=2, check_state_end=False)
+    p.check_state(ids=range(0, 128, 9))
