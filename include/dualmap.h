@@ -17,8 +17,10 @@
  *   - Synchronous argument checks return an error and change nothing.
  *   - Checks that need device data (prompt lengths, offsets, capacities) run
  *     in the kernels: a failure is recorded as a sticky device error, the
- *     rest of that call's kernels do nothing, and every later call returns
- *     the error (see dm_last_error).  The handle must then be destroyed.
+ *     rest of that call's kernels do nothing, and every later call that
+ *     changes state returns the error (see dm_last_error); the read-only
+ *     calls (dm_get_loads, dm_export_*, dm_get_clock) keep working.  The
+ *     handle must then be destroyed.
  *   - One handle must be used from one host thread at a time.
  *
  * Readings of details the paper leaves open (block size, hash family, ring

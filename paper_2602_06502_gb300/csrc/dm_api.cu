@@ -116,6 +116,11 @@ dm_status check_live(dm_handle *h) {
     return h->sticky;
 }
 
+// Read-only introspection keeps working after a sticky error.
+dm_status check_handle(dm_handle *h) {
+    return h ? DM_OK : DM_ERR_INVALID_ARG;
+}
+
 }  // namespace
 
 extern "C" {
@@ -529,7 +534,7 @@ dm_status dm_ring_lookup(dm_handle *h, const uint64_t *pos_dev, uint32_t n, uint
 }
 
 dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap) {
-    dm_status s = check_live(h);
+    dm_status s = check_handle(h);
     if (s) return s;
     if (!W_host && cap) return DM_ERR_INVALID_ARG;
     const uint32_t k = cap < h->d.M ? cap : h->d.M;
@@ -540,7 +545,7 @@ dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap) {
 
 dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys, uint64_t *stamps, uint64_t cap,
                           uint64_t *n_out) {
-    dm_status s = check_live(h);
+    dm_status s = check_handle(h);
     if (s) return s;
     if (id >= h->d.M || !n_out || (cap && (!keys || !stamps))) return DM_ERR_INVALID_ARG;
     *n_out = 0;
@@ -561,7 +566,7 @@ dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys, uint64_t *s
 
 dm_status dm_export_queue(dm_handle *h, uint32_t id, uint64_t *seq, uint64_t *work, uint64_t *rem, uint64_t cap,
                           uint64_t *n_out) {
-    dm_status s = check_live(h);
+    dm_status s = check_handle(h);
     if (s) return s;
     if (id >= h->d.M || !n_out || (cap && (!seq || !work || !rem))) return DM_ERR_INVALID_ARG;
     uint32_t ht[2];
@@ -585,7 +590,7 @@ dm_status dm_export_queue(dm_handle *h, uint32_t id, uint64_t *seq, uint64_t *wo
 }
 
 dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos, uint32_t *owner, uint32_t cap, uint32_t *n_out) {
-    dm_status s = check_live(h);
+    dm_status s = check_handle(h);
     if (s) return s;
     if ((f != 0 && f != 1) || !n_out || (cap && (!vpos || !owner))) return DM_ERR_INVALID_ARG;
     const uint32_t k = cap < h->d.R ? cap : h->d.R;
@@ -597,7 +602,7 @@ dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos, uint32_t *owner, u
 }
 
 dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host) {
-    dm_status s = check_live(h);
+    dm_status s = check_handle(h);
     if (s) return s;
     if (!clock_host) return DM_ERR_INVALID_ARG;
     cudaError_t e = cudaMemcpyAsync(clock_host, h->d.clock, 8, cudaMemcpyDeviceToHost, h->st);
