@@ -38,7 +38,7 @@ def longctx_handle_kwargs(w):
     """Handle sizes used for the long-context workload (bench and its parity test)."""
     return dict(max_instances=w["n_instances"] + 8, max_batch=w["batch"],
                 max_batch_tokens=w["batch"] * w["len_hi"] + 4 * w["batch"],
-                max_touch_per_instance=1 << 20)
+                max_touch_per_instance=1 << 20, index_slots_log2=23)
 
 
 def handle_kwargs(w, max_id):
@@ -196,6 +196,9 @@ def main():
     ap.add_argument("--cpu-batches", type=int, default=6)
     ap.add_argument("--ref-max-batches", type=int, default=24)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE",
+                    help="override a workload field (small cases for profiling)")
+    ap.add_argument("--max-touch", type=int, default=0, help="override max_touch_per_instance")
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":
@@ -212,11 +215,13 @@ def main():
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = workload(args.workload)
+    w = workload(args.workload, **{k: int(v) for k, v in (x.split("=", 1) for x in args.set)})
     W, K = max(args.warmup, 3), args.steps
     tr = Trace(w)
     nb = len(tr.batches)
     kw = handle_kwargs(w, tr.max_instance_id())
+    if args.max_touch:
+        kw["max_touch_per_instance"] = args.max_touch
 
     # all batches' tokens resident in HBM (a pass longer than the trace replays it cyclically)
     used = min(nb, W + K)
@@ -315,7 +320,7 @@ def main():
 
     # -- end-to-end through the host-buffer entry point ----------------------
     e2e = None
-    if rank == 0 or world > 1:
+    if args.e2e_steps > 0:
         Ke = max(1, min(args.e2e_steps, K))
         g = make_sched()
         need = sorted({j % used for j in range(W + Ke)})

@@ -91,7 +91,11 @@ typedef struct {
     uint64_t max_touch_per_instance;
     /* Queue capacity per instance in entries (power of two); 0 = 65536. */
     uint32_t max_queue;
-    uint32_t reserved0;   /* must be 0 */
+    /* log2 of the index slots per instance; 0 = automatic, the smallest
+     * power of two >= 2 x (C + max_touch_per_instance).  A larger index is
+     * rebuilt less often (it is rebuilt when half full, counting the slots
+     * evicted keys keep).  Never smaller than the automatic size; <= 40. */
+    uint32_t index_slots_log2;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */

@@ -11,6 +11,7 @@
 
 using dm::DevState;
 using dm::QEntry;
+using dm::Rec;
 using dm::Slot;
 
 struct StageEvent {
@@ -37,7 +38,9 @@ struct dm_handle {
     int cur[2] = {0, 0};
     uint64_t *ring_spos = nullptr;
     uint32_t *ring_svidx = nullptr;
-    std::vector<Slot *> tables, logs;
+    std::vector<Slot *> tables, tables2;   // both index buffers of each id (host copies)
+    std::vector<Rec *> logs, logs2;        // both log buffers
+    std::vector<uint8_t *> stales, stales2;
     std::vector<void *> allocs;    // every cudaMalloc of the handle
     // staging of dm_route_batch_host
     uint32_t *h_tokens = nullptr, *h_lengths = nullptr;
@@ -45,6 +48,7 @@ struct dm_handle {
     dm_route_out h_out{};
     bool profiling = false;
     std::vector<StageEvent> events;
+    std::vector<cudaEvent_t> ev_pool;
     double stage_ms[DM_STAGE_COUNT] = {};
     uint64_t stage_calls[DM_STAGE_COUNT] = {};
     dm_status sticky = DM_OK;
@@ -88,18 +92,36 @@ void set_levels(DevState &d, uint32_t R) {
     for (uint32_t j = 1; j + 1 < d.nlev; ++j) d.lev_off[j + 1] = d.lev_off[j] + d.lev_n[j];
 }
 
+// Events come from a pool that dm_get_stage_times refills, so timing a
+// stage costs two cudaEventRecord calls.
+cudaEvent_t pool_event(dm_handle *h) {
+    if (h->ev_pool.empty()) {
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        return e;
+    }
+    cudaEvent_t e = h->ev_pool.back();
+    h->ev_pool.pop_back();
+    return e;
+}
+
 struct Stage {
     dm_handle *h;
     int s;
     cudaEvent_t a = nullptr, b = nullptr;
     Stage(dm_handle *h_, int s_) : h(h_), s(s_) {
-        if (h->profiling && cudaEventCreate(&a) == cudaSuccess && cudaEventCreate(&b) == cudaSuccess)
-            cudaEventRecord(a, h->st);
+        if (!h->profiling) return;
+        a = pool_event(h);
+        b = pool_event(h);
+        if (a && b) cudaEventRecord(a, h->st);
     }
     ~Stage() {
         if (a && b) {
             cudaEventRecord(b, h->st);
             h->events.push_back(StageEvent{s, a, b});
+        } else {
+            if (a) h->ev_pool.push_back(a);
+            if (b) h->ev_pool.push_back(b);
         }
     }
 };
@@ -145,6 +167,7 @@ void dm_destroy(dm_handle *h) {
     if (!h) return;
     cudaStreamSynchronize(h->st);
     for (auto &ev : h->events) { cudaEventDestroy(ev.a); cudaEventDestroy(ev.b); }
+    for (auto e : h->ev_pool) cudaEventDestroy(e);
     for (void *p : h->allocs) cudaFree(p);
     delete h;
 }
@@ -162,7 +185,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.cache_capacity_blocks < 1 || c.cost_us_per_token < 1 || c.hot_den < 1) return DM_ERR_INVALID_ARG;
     if (c.max_batch < 1 || c.max_batch > (1u << 24) || c.max_batch_tokens < B) return DM_ERR_INVALID_ARG;
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
-    if (c.reserved0) return DM_ERR_INVALID_ARG;
+    if (c.index_slots_log2 > 40) return DM_ERR_INVALID_ARG;
 
     dm_handle *h = new dm_handle();
     h->cfg = c;
@@ -182,6 +205,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.max_segs = d.max_blocks / dm::kSegBlocks + c.max_batch;
     d.T = c.max_touch_per_instance ? c.max_touch_per_instance : d.max_blocks;
     d.S = pow2_at_least(2 * (d.C + d.T));
+    if (c.index_slots_log2 && (1ull << c.index_slots_log2) > d.S) d.S = 1ull << c.index_slots_log2;
     d.logcap = pow2_at_least(2 * (d.C + d.T));
     d.Q = c.max_queue ? c.max_queue : 65536;
     d.rb_cap = (uint32_t)pow2_at_least(d.Q > d.M ? d.Q : d.M);
@@ -221,11 +245,32 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.q, M * d.Q));
     A(dalloc(h, &d.table, M));
     A(dalloc(h, &d.logbuf, M));
+    A(dalloc(h, &d.table_alt, M));
+    A(dalloc(h, &d.logbuf_alt, M));
+    A(dalloc(h, &d.stale, M));
+    A(dalloc(h, &d.stale_alt, M));
+    A(dalloc(h, &d.mt_flags, M));
+    A(dalloc(h, &d.mt_newtail, M));
+    A(dalloc(h, &d.mc_chunk_off, M + 1));
+    A(dalloc(h, &d.mr_chunk_off, M + 1));
+    d.mc_cap = M * (d.logcap / dm::kEvChunk + 1);
+    A(dalloc(h, &d.mc_chunk_live, d.mc_cap));
     A(dalloc(h, &d.log_front, M));
     A(dalloc(h, &d.log_tail, M));
     A(dalloc(h, &d.live, M));
     A(dalloc(h, &d.used, M));
     A(dalloc(h, &d.touch_cnt, M));
+    A(dalloc(h, &d.log_adv, M));
+    A(dalloc(h, &d.log_base, M));
+    A(dalloc(h, &d.ev_excess, M));
+    A(dalloc(h, &d.ev_win, M));
+    A(dalloc(h, &d.ev_front_new, M));
+    A(dalloc(h, &d.ev_rem, M));
+    A(dalloc(h, &d.ev_chunk_off, M + 1));
+    // eviction windows: sum over ids of (2 x excess + 2048) rounded up to chunks,
+    // and excess <= blocks touched by one commit <= max_blocks
+    d.ev_cap = 2 * d.max_blocks + (2048 + 2 * dm::kEvChunk) * M;
+    A(dalloc(h, &d.ev_chunk_live, d.ev_cap / dm::kEvChunk + 1));
     A(dalloc(h, &d.clock, 1));
     A(dalloc(h, &d.err, 1));
     A(dalloc(h, &d.seq_next, 1));
@@ -247,8 +292,10 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         A(dalloc(h, &x->seg_req, d.max_segs));
         A(dalloc(h, &x->seg_total, d.max_segs));
         A(dalloc(h, &x->seg_carry, d.max_segs));
+        A(dalloc(h, &x->seg_total2, d.max_segs));
+        A(dalloc(h, &x->seg_newly, d.max_segs));
+        A(dalloc(h, &x->seg_claims, d.max_segs));
         A(dalloc(h, &x->plocal, d.max_blocks));
-        A(dalloc(h, &x->r_pos, 2ull * c.max_batch));
         A(dalloc(h, &x->r_c1, c.max_batch));
         A(dalloc(h, &x->r_c2, c.max_batch));
         A(dalloc(h, &x->r_h1, c.max_batch));
@@ -274,6 +321,11 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(cudaMemsetAsync(d.q_tail, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.table, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.logbuf, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.table_alt, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.logbuf_alt, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.stale, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.stale_alt, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.mt_flags, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.log_front, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.log_tail, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.live, 0, M * 8, h->st));
@@ -291,6 +343,10 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     h->state.assign(M, 0);
     h->tables.assign(M, nullptr);
     h->logs.assign(M, nullptr);
+    h->tables2.assign(M, nullptr);
+    h->logs2.assign(M, nullptr);
+    h->stales.assign(M, nullptr);
+    h->stales2.assign(M, nullptr);
     h->hash_grid = dm::hash_grid_size();
     *out = h;
     return DM_OK;
@@ -303,7 +359,10 @@ static void sync_copy(dm_handle *h) {
     h->dh.r_L = keep.r_L; h->dh.r_nblk = keep.r_nblk; h->dh.r_segoff = keep.r_segoff;
     h->dh.r_tokoff = keep.r_tokoff; h->dh.r_blkoff = keep.r_blkoff; h->dh.seg_req = keep.seg_req;
     h->dh.seg_total = keep.seg_total; h->dh.seg_carry = keep.seg_carry; h->dh.plocal = keep.plocal;
-    h->dh.r_pos = keep.r_pos; h->dh.r_c1 = keep.r_c1; h->dh.r_c2 = keep.r_c2; h->dh.r_h1 = keep.r_h1;
+    h->dh.seg_total2 = keep.seg_total2;
+    h->dh.seg_newly = keep.seg_newly;
+    h->dh.seg_claims = keep.seg_claims;
+    h->dh.r_c1 = keep.r_c1; h->dh.r_c2 = keep.r_c2; h->dh.r_h1 = keep.r_h1;
     h->dh.r_h2 = keep.r_h2; h->dh.r_final = keep.r_final; h->dh.r_touchoff = keep.r_touchoff;
     h->dh.info = keep.info;
 }
@@ -352,20 +411,36 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         if (ht[0] != ht[1]) return DM_ERR_DUPLICATE_ID;
     }
     if (!h->tables[id]) {
-        Slot *t = nullptr, *lg = nullptr;
+        Slot *t = nullptr, *t2 = nullptr;
+        Rec *lg = nullptr, *lg2 = nullptr;
+        uint8_t *sf = nullptr, *sf2 = nullptr;
         e = dalloc(h, &t, d.S);
+        if (e == cudaSuccess) e = dalloc(h, &t2, d.S);
         if (e == cudaSuccess) e = dalloc(h, &lg, d.logcap);
+        if (e == cudaSuccess) e = dalloc(h, &lg2, d.logcap);
+        if (e == cudaSuccess) e = dalloc(h, &sf, d.logcap);
+        if (e == cudaSuccess) e = dalloc(h, &sf2, d.logcap);
         if (e != cudaSuccess) { cudaGetLastError(); return DM_ERR_OOM; }
         h->tables[id] = t;
+        h->tables2[id] = t2;
         h->logs[id] = lg;
-        e = cudaMemcpyAsync(d.table + id, &h->tables[id], sizeof(Slot *), cudaMemcpyHostToDevice, h->st);
-        if (e == cudaSuccess)
-            e = cudaMemcpyAsync(d.logbuf + id, &h->logs[id], sizeof(Slot *), cudaMemcpyHostToDevice, h->st);
-        if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
-        if (e != cudaSuccess) return map_cuda(h, e);
+        h->logs2[id] = lg2;
+        h->stales[id] = sf;
+        h->stales2[id] = sf2;
     }
-    // a (re-)added instance starts empty
+    // a (re-)added instance starts empty, both buffers of each
+    struct { void *dst; const void *src; } ptrs[] = {
+        {d.table + id, &h->tables[id]}, {d.table_alt + id, &h->tables2[id]},
+        {d.logbuf + id, &h->logs[id]}, {d.logbuf_alt + id, &h->logs2[id]},
+        {d.stale + id, &h->stales[id]}, {d.stale_alt + id, &h->stales2[id]}};
+    for (auto &pp : ptrs)
+        if (e == cudaSuccess) e = cudaMemcpyAsync(pp.dst, pp.src, sizeof(void *), cudaMemcpyHostToDevice, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
     e = cudaMemsetAsync(h->tables[id], 0, d.S * sizeof(Slot), h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->tables2[id], 0, d.S * sizeof(Slot), h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->stales[id], 0, d.logcap, h->st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->stales2[id], 0, d.logcap, h->st);
     if (e == cudaSuccess) e = cudaMemsetAsync(d.log_front + id, 0, 8, h->st);
     if (e == cudaSuccess) e = cudaMemsetAsync(d.log_tail + id, 0, 8, h->st);
     if (e == cudaSuccess) e = cudaMemsetAsync(d.live + id, 0, 8, h->st);
@@ -550,14 +625,28 @@ dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys, uint64_t *s
     if (id >= h->d.M || !n_out || (cap && (!keys || !stamps))) return DM_ERR_INVALID_ARG;
     *n_out = 0;
     if (!h->tables[id]) return DM_OK;
+    Slot *cur = nullptr;   // the buffers in use (rebuilds and compactions swap them)
+    Rec *lcur = nullptr;
+    uint64_t front = 0;
+    cudaError_t e = cudaMemcpyAsync(&cur, h->d.table + id, sizeof(Slot *), cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&lcur, h->d.logbuf + id, sizeof(Rec *), cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&front, h->d.log_front + id, 8, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
     std::vector<Slot> t(h->d.S);
-    cudaError_t e = cudaMemcpyAsync(t.data(), h->tables[id], h->d.S * sizeof(Slot), cudaMemcpyDeviceToHost, h->st);
+    std::vector<Rec> lg(h->d.logcap);
+    e = cudaMemcpyAsync(t.data(), cur, h->d.S * sizeof(Slot), cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(lg.data(), lcur, h->d.logcap * sizeof(Rec), cudaMemcpyDeviceToHost, h->st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
     if (e != cudaSuccess) return map_cuda(h, e);
     uint64_t k = 0;
     for (const Slot &x : t) {
-        if (x.key == 0 || x.stamp == 0) continue;
-        if (k < cap) { keys[k] = x.key; stamps[k] = x.stamp; }
+        if (x.key == 0 || x.pos1 == 0 || x.pos1 - 1 < front) continue;   // empty or evicted
+        if (k < cap) {
+            keys[k] = x.key;
+            stamps[k] = lg[(x.pos1 - 1) & (h->d.logcap - 1)].stamp;
+        }
         ++k;
     }
     *n_out = k;
@@ -637,8 +726,8 @@ dm_status dm_get_stage_times(dm_handle *h, double *ms, uint64_t *calls, int rese
             h->stage_ms[ev.stage] += t;
             h->stage_calls[ev.stage] += 1;
         }
-        cudaEventDestroy(ev.a);
-        cudaEventDestroy(ev.b);
+        h->ev_pool.push_back(ev.a);
+        h->ev_pool.push_back(ev.b);
     }
     h->events.clear();
     for (int i = 0; i < DM_STAGE_COUNT; ++i) {

@@ -5,10 +5,12 @@
 // increasing head/tail counters; W[i] is the sum of remaining work.
 //
 // Choice: the decision for a request depends on the loads left by every
-// earlier request of the batch, so one CTA walks the batch in arrival order
-// with W in shared memory; everything that does not depend on W (uncached
-// work, which candidate has more hits) is precomputed in parallel, and the
-// queue writes and outputs are emitted in parallel afterwards.
+// earlier request of the batch that shares one of its candidates.  One CTA
+// keeps W in shared memory; one warp decides 32 requests at a time in
+// dependency rounds (a request waits only for earlier requests of the window
+// sharing an instance with it); everything that does not depend on W is
+// precomputed in parallel, and queue writes and outputs are emitted in
+// parallel afterwards.
 #include "dm_internal.cuh"
 
 namespace dm {
@@ -60,23 +62,44 @@ cudaError_t launch_drain(const DevState &d, uint64_t delta, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-constexpr uint32_t kChoiceChunk = 512;
+constexpr uint32_t kChoiceChunk = 1024;
 
-// Single CTA (1024 threads).  Dynamic shared memory: W[M] (u64), tail[M] (u32).
+// Single CTA (1024 threads).  Dynamic shared memory: per instance W (u64),
+// a packed counter PT = (log records this batch << 32) | queue tail, so one
+// 64-bit add per request advances both, and a lane mask used to find
+// conflicts inside a window; then the per-chunk request staging.
+//
+// Each request is staged as (a, b): a = the candidate with more cached
+// blocks (c1 on equal hits), u = uncached work on each, and
+// thr = SLO - u_a (-1 when u_a alone exceeds the SLO or the hits are equal),
+// so the rule of Sec. 3.2 becomes: choose b iff W_b < W_a and W_a > thr
+// (ttft_a = W_a + u_a > SLO); the SLO switch fired iff hits differ and
+// W_a > thr.
+struct ChoiceStage {
+    uint64_t ua[kChoiceChunk], ub[kChoiceChunk];
+    int64_t thr[kChoiceChunk];
+    uint64_t Wa[kChoiceChunk], Wb[kChoiceChunk], pt[kChoiceChunk];
+    uint32_t ab[kChoiceChunk];     // a | b << 14 | (a is c2) << 28 | (hits differ) << 29
+    uint32_t nb[kChoiceChunk];
+    uint8_t pickb[kChoiceChunk];
+};
+
+// W and PT (8 bytes each), the lane masks padded to a multiple of 4 entries
+// so that the staging block starts on a 16-byte boundary for any M.
+__host__ __device__ inline size_t choice_lanes(uint32_t M) { return (size_t(M) + 3) / 4 * 4; }
+size_t choice_smem(uint32_t M) { return size_t(M) * 16 + choice_lanes(M) * 4 + sizeof(ChoiceStage); }
+
 __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uint32_t n, uint64_t seq0) {
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ uint32_t s_c1[kChoiceChunk], s_c2[kChoiceChunk];
-    __shared__ uint64_t s_u1[kChoiceChunk], s_u2[kChoiceChunk];
-    __shared__ uint8_t s_cls[kChoiceChunk];      // 0: equal hits, 1: c1 has more, 2: c2 has more
-    __shared__ uint32_t s_ch[kChoiceChunk], s_slot[kChoiceChunk];
-    __shared__ uint64_t s_t1[kChoiceChunk], s_t2[kChoiceChunk];
-    __shared__ uint8_t s_sw[kChoiceChunk];
     if (has_err(d.err)) return;
     uint64_t *W = reinterpret_cast<uint64_t *>(smem);
-    uint32_t *tail = reinterpret_cast<uint32_t *>(W + d.M);
+    uint64_t *PT = W + d.M;
+    uint32_t *lanes = reinterpret_cast<uint32_t *>(PT + d.M);
+    ChoiceStage &S = *reinterpret_cast<ChoiceStage *>(lanes + choice_lanes(d.M));
     for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
         W[i] = d.W[i];
-        tail[i] = d.q_tail[i];
+        PT[i] = d.q_tail[i];
+        lanes[i] = 0;
     }
     const uint64_t cost = d.cost, slo = d.slo;
     for (uint32_t base = 0; base < n; base += kChoiceChunk) {
@@ -85,65 +108,83 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
         for (uint32_t k = threadIdx.x; k < m; k += blockDim.x) {
             const uint32_t r = base + k;
             const uint32_t L = d.r_L[r], h1 = d.r_h1[r], h2 = d.r_h2[r];
-            s_c1[k] = d.r_c1[r];
-            s_c2[k] = d.r_c2[r];
-            s_u1[k] = cost * (L - h1);
-            s_u2[k] = cost * (L - h2);
-            s_cls[k] = h1 == h2 ? 0 : (h1 > h2 ? 1 : 2);
+            const uint32_t c1 = d.r_c1[r], c2 = d.r_c2[r];
+            const bool a2 = h2 > h1;
+            const uint64_t ua = cost * (L - (a2 ? h2 : h1)), ub = cost * (L - (a2 ? h1 : h2));
+            S.ua[k] = ua;
+            S.ub[k] = ub;
+            S.thr[k] = (h1 == h2 || ua > slo) ? -1 : (int64_t)(slo - ua);
+            S.ab[k] = (a2 ? c2 : c1) | ((a2 ? c1 : c2) << 14) | (uint32_t(a2) << 28) | (uint32_t(h1 != h2) << 29);
+            S.nb[k] = d.r_nblk[r];
         }
         __syncthreads();
-        if (threadIdx.x == 0) {
-            for (uint32_t k = 0; k < m; ++k) {
-                const uint32_t c1 = s_c1[k], c2 = s_c2[k];
-                const uint64_t W1 = W[c1], W2 = W[c2];
-                const uint64_t u1 = s_u1[k], u2 = s_u2[k];
-                const uint32_t cls = s_cls[k];
-                const uint64_t t1 = W1 + u1, t2 = W2 + u2;
-                bool pick2;
-                uint8_t sw = 0;
-                if (cls == 0) {
-                    pick2 = W2 < W1;
-                } else {
-                    const bool a2 = cls == 2;          // a = higher-hit candidate
-                    const uint64_t ta = a2 ? t2 : t1;
-                    const uint64_t Wa = a2 ? W2 : W1, Wb = a2 ? W1 : W2;
-                    if (ta <= slo) {
-                        pick2 = a2;
-                    } else {
-                        sw = 1;
-                        pick2 = (Wb < Wa) ? !a2 : a2;
-                    }
+        if (threadIdx.x < 32) {
+            // Warp 0 takes 32 requests at a time.  A lane may decide once
+            // every earlier lane sharing one of its candidates has decided;
+            // lanes decided in the same round share no instance, so reading
+            // W and writing W[choice] then equals arrival order exactly.
+            const int lane = threadIdx.x;
+            for (uint32_t w0 = 0; w0 < m; w0 += 32) {
+                const uint32_t k = w0 + lane;
+                const bool valid = k < m;
+                const uint32_t ab = valid ? S.ab[k] : 0;
+                const uint32_t a = ab & 0x3FFF, b = (ab >> 14) & 0x3FFF;
+                if (valid) {
+                    atomicOr(&lanes[a], 1u << lane);
+                    atomicOr(&lanes[b], 1u << lane);
                 }
-                const uint32_t ch = pick2 ? c2 : c1;
-                W[ch] = (pick2 ? W2 : W1) + (pick2 ? u2 : u1);
-                s_ch[k] = ch;
-                s_slot[k] = tail[ch]++;
-                s_t1[k] = t1;
-                s_t2[k] = t2;
-                s_sw[k] = sw;
+                __syncwarp();
+                const uint32_t conf = valid ? (lanes[a] | lanes[b]) & ((1u << lane) - 1) : 0;
+                __syncwarp();
+                if (valid) { lanes[a] = 0; lanes[b] = 0; }
+                const uint64_t ua = valid ? S.ua[k] : 0, ub = valid ? S.ub[k] : 0;
+                const int64_t thr = valid ? S.thr[k] : 0;
+                uint32_t done = __ballot_sync(0xffffffffu, !valid);
+                while (done != 0xffffffffu) {
+                    const bool ready = !((done >> lane) & 1u) && (conf & ~done) == 0;
+                    if (ready) {
+                        const uint64_t Wa = W[a], Wb = W[b], Pa = PT[a], Pb = PT[b];
+                        const bool pb = Wb < Wa && (int64_t)Wa > thr;
+                        const uint32_t ch = pb ? b : a;
+                        const uint64_t Pold = pb ? Pb : Pa;
+                        W[ch] = pb ? Wb + ub : Wa + ua;
+                        PT[ch] = Pold + (uint64_t(S.nb[k]) << 32) + 1;
+                        S.Wa[k] = Wa;
+                        S.Wb[k] = Wb;
+                        S.pt[k] = Pold;
+                        S.pickb[k] = pb;
+                    }
+                    __syncwarp();
+                    done |= __ballot_sync(0xffffffffu, ready);
+                }
             }
         }
         __syncthreads();
         for (uint32_t k = threadIdx.x; k < m; k += blockDim.x) {
             const uint32_t r = base + k;
-            const uint32_t ch = s_ch[k];
-            const bool pick2 = ch == s_c2[k];
-            o.ttft1[r] = s_t1[k];
-            o.ttft2[r] = s_t2[k];
+            const uint32_t ab = S.ab[k];
+            const uint32_t a = ab & 0x3FFF, b = (ab >> 14) & 0x3FFF;
+            const bool a_is_c2 = (ab >> 28) & 1, differ = (ab >> 29) & 1;
+            const bool pb = S.pickb[k];
+            const uint32_t ch = pb ? b : a;
+            const uint64_t ta = S.Wa[k] + S.ua[k], tb = S.Wb[k] + S.ub[k];
+            o.ttft1[r] = a_is_c2 ? tb : ta;
+            o.ttft2[r] = a_is_c2 ? ta : tb;
             o.chosen[r] = ch;
-            o.switched[r] = s_sw[k];
+            o.switched[r] = differ && (int64_t)S.Wa[k] > S.thr[k];
             d.r_final[r] = ch;
-            const uint32_t slot = s_slot[k];
+            d.r_touchoff[r] = S.pt[k] >> 32;          // offset among this batch's records of ch
+            const uint32_t slot = (uint32_t)S.pt[k];
             if (slot - d.q_head[ch] >= d.Q) {
                 set_err(d.err, DM_ERR_CAPACITY);
                 continue;
             }
             QEntry e;
             e.seq = seq0 + r;
-            e.work = e.remaining = pick2 ? s_u2[k] : s_u1[k];
+            e.work = e.remaining = pb ? S.ub[k] : S.ua[k];
             e.L = d.r_L[r];
-            e.c1 = s_c1[k];
-            e.c2 = s_c2[k];
+            e.c1 = a_is_c2 ? b : a;
+            e.c2 = a_is_c2 ? a : b;
             e.h1 = d.r_h1[r];
             e.h2 = d.r_h2[r];
             e.moved = 0;
@@ -153,14 +194,16 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
     __syncthreads();
     for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
         d.W[i] = W[i];
-        d.q_tail[i] = tail[i];
+        d.q_tail[i] = (uint32_t)PT[i];
+        d.log_adv[i] = PT[i] >> 32;
     }
+    if (threadIdx.x == 0) d.info->final_dirty = 0;
 }
 
 cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, uint64_t seq0,
                           cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    const size_t smem = size_t(d.M) * (sizeof(uint64_t) + sizeof(uint32_t));
+    const size_t smem = choice_smem(d.M);
     static size_t configured = 0;
     if (smem > configured) {
         cudaError_t e = cudaFuncSetAttribute(k_choice, cudaFuncAttributeMaxDynamicSharedMemorySize,

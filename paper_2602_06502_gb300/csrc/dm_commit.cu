@@ -4,155 +4,369 @@
 // Sequential definition: in arrival order, each request of the batch touches
 // its block keys on its final instance from block n_blk-1 down to 0, one
 // global clock tick per touch, and an LRU of capacity C evicts on overflow.
-// An LRU holds exactly the C distinct keys with the latest last touch, so the
-// GPU applies all touches of the batch at once (slot stamp = atomicMax of the
-// touch stamps) and then evicts each instance's oldest keys down to C.
+// An LRU holds exactly the C distinct keys with the latest last touch, so all
+// touches of a batch are applied at once and each instance then drops its
+// oldest keys down to C.
 //
-// Every instance keeps a recency log: the (key, stamp) of every touch in
-// stamp order.  A log record is live when its stamp is still the key's slot
-// stamp; evicting the k oldest keys = zeroing the slots of the first k live
-// records from the log front.  Stale records are dropped by compaction, and
-// the index (whose evicted keys keep their slots) is rebuilt from the
-// compacted log when too many slots are used.
+// Layout per instance: a recency log of (key, stamp) records in stamp order,
+// a stale flag per record (set when a later touch supersedes it), and an
+// open-addressed index key -> 1 + position of the key's latest record.  A
+// key is resident iff that record is at or after the log front, so evicting
+// the k oldest keys is moving the front past the k-th non-stale record: no
+// per-key write at all.  Evicted keys keep their index slots until the index
+// passes half full, when it is rebuilt from the log's live records; a log
+// about to overflow is compacted.  Both write into second buffers and swap.
 #include "dm_internal.cuh"
 
 namespace dm {
 
-// Touch key with stamp in an index: claims an empty slot for a new key, and
-// raises the stamp to the newest touch.  Returns true when the key becomes
-// resident (new, or previously evicted); *claimed when a slot was taken.
-__device__ __forceinline__ bool table_touch(Slot *t, uint64_t mask, uint64_t key, uint64_t stamp,
-                                            uint32_t *err, bool *claimed) {
-    uint64_t i = key & mask;
-    for (uint64_t it = 0; it <= mask; ++it) {
+constexpr int kMtThreads = 256;
+constexpr uint32_t kPrepChunk = 2048;
+constexpr uint32_t kFlagCompact = 1, kFlagRebuild = 2;
+constexpr uint32_t kZeroChunk = 4096;   // slots or flag bytes cleared per chunk
+
+// Slot of `key` given the result `prev` of a CAS(0 -> key) at its home slot
+// i0: the home slot when it was empty (claimed) or already held the key,
+// else continue probing from i0 + 1.
+__device__ __forceinline__ uint64_t slot_after_home_cas(Slot *t, uint64_t mask, uint64_t key, uint64_t i0,
+                                                        uint64_t prev, uint32_t *err, bool *claimed) {
+    if (prev == 0) { *claimed = true; return i0; }
+    if (prev == key) return i0;
+    uint64_t i = (i0 + 1) & mask;
+    for (uint64_t it = 1; it <= mask; ++it) {
         uint64_t k = *(volatile uint64_t *)&t[i].key;
         if (k == 0) {
-            const unsigned long long prev =
+            const unsigned long long pv =
                 atomicCAS(reinterpret_cast<unsigned long long *>(&t[i].key), 0ull, (unsigned long long)key);
-            if (prev == 0) { *claimed = true; k = key; } else { k = prev; }
+            if (pv == 0) { *claimed = true; return i; }
+            k = pv;
         }
-        if (k == key) {
-            const unsigned long long old =
-                atomicMax(reinterpret_cast<unsigned long long *>(&t[i].stamp), (unsigned long long)stamp);
-            return old == 0;
-        }
+        if (k == key) return i;
         i = (i + 1) & mask;
     }
     set_err(err, DM_ERR_TIMEOUT);
-    return false;
+    return i0;
 }
 
-// Blocks each instance receives from the pending batch.
-__global__ void k_commit_count(DevState d, uint32_t n) {
-    if (has_err(d.err)) return;
-    const uint32_t r = blockIdx.x * blockDim.x + threadIdx.x;
-    if (r < n) atomicAdd(reinterpret_cast<unsigned long long *>(&d.touch_cnt[d.r_final[r]]),
-                         (unsigned long long)d.r_nblk[r]);
+// Insert a key known to be absent (index rebuild: all keys distinct).
+__device__ __forceinline__ void table_insert_new(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint32_t *err) {
+    uint64_t j = key & mask;
+    for (uint64_t it = 0; it <= mask; ++it) {
+        const unsigned long long prev =
+            atomicCAS(reinterpret_cast<unsigned long long *>(&t[j].key), 0ull, (unsigned long long)key);
+        if (prev == 0) { t[j].pos1 = p1; return; }
+        j = (j + 1) & mask;
+    }
+    set_err(err, DM_ERR_TIMEOUT);
 }
 
-// Block-wide exclusive scan of 0/1 flags (blockDim.x == 1024).
-__device__ __forceinline__ uint32_t block_rank(bool f, uint32_t *s_w, uint32_t &total) {
+// Point an existing key at a new record position (log compaction).
+__device__ __forceinline__ void table_set_pos(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint32_t *err) {
+    uint64_t j = key & mask;
+    for (uint64_t it = 0; it <= mask; ++it) {
+        if (t[j].key == key) { t[j].pos1 = p1; return; }
+        if (t[j].key == 0) break;
+        j = (j + 1) & mask;
+    }
+    set_err(err, DM_ERR_TIMEOUT);
+}
+
+// Exclusive block scan of u32 counts (any block size up to 1024).
+__device__ __forceinline__ uint32_t block_excl_u32(uint32_t v, uint32_t *s_w, uint32_t &total) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    const uint32_t b = __ballot_sync(0xffffffffu, f);
-    const uint32_t before = __popc(b & ((1u << lane) - 1));
-    if (lane == 0) s_w[wid] = __popc(b);
+    uint32_t inc = v;
+#pragma unroll
+    for (int dd = 1; dd < 32; dd <<= 1) {
+        const uint32_t u = __shfl_up_sync(0xffffffffu, inc, dd);
+        if (lane >= dd) inc += u;
+    }
+    if (lane == 31) s_w[wid] = inc;
     __syncthreads();
     if (wid == 0) {
-        const uint32_t v = lane < (int)(blockDim.x >> 5) ? s_w[lane] : 0;
-        uint32_t inc = v;
+        const uint32_t x = lane < (int)(blockDim.x >> 5) ? s_w[lane] : 0;
+        uint32_t y = x;
 #pragma unroll
         for (int dd = 1; dd < 32; dd <<= 1) {
-            const uint32_t u = __shfl_up_sync(0xffffffffu, inc, dd);
-            if (lane >= dd) inc += u;
+            const uint32_t u = __shfl_up_sync(0xffffffffu, y, dd);
+            if (lane >= dd) y += u;
         }
-        s_w[lane] = inc - v;
-        if (lane == 31) s_w[32] = inc;
+        s_w[lane] = y - x;
+        if (lane == 31) s_w[32] = y;
     }
     __syncthreads();
-    const uint32_t r = s_w[wid] + before;
+    const uint32_t r = s_w[wid] + inc - v;
     total = s_w[32];
     __syncthreads();
     return r;
 }
 
-// Make room for the pending batch: compact an instance's log when it would
-// overflow, rebuild its index when too many slots are used.  CTA per id.
-__global__ void __launch_bounds__(1024) k_maintain(DevState d) {
-    __shared__ uint32_t s_w[33];
-    if (has_err(d.err)) return;
-    const uint32_t i = blockIdx.x;
-    Slot *t = d.table[i];
-    if (!t) return;
-    const uint64_t cnt = d.touch_cnt[i];
-    if (cnt > d.T) {
-        if (threadIdx.x == 0) set_err(d.err, DM_ERR_CAPACITY);
-        return;
+// Instance owning flat chunk c of a chunk-offset table (largest i with off[i] <= c).
+__device__ __forceinline__ uint32_t owner_of(const uint32_t *off, uint32_t M, uint32_t c) {
+    uint32_t lo = 0, hi = M;
+    while (hi - lo > 1) {
+        const uint32_t mid = (lo + hi) >> 1;
+        if (off[mid] <= c) lo = mid; else hi = mid;
     }
-    const uint64_t front = d.log_front[i], tail = d.log_tail[i];
-    const bool rebuild = d.used[i] + cnt > d.S - d.S / 4;
-    const bool compact = rebuild || (tail - front) + cnt > d.logcap;
-    if (!compact) return;
-    Slot *lg = d.logbuf[i];
-    const uint64_t mask = d.S - 1, lmask = d.logcap - 1;
-    uint64_t w = front;
-    for (uint64_t p0 = front; p0 < tail; p0 += blockDim.x) {
-        const uint64_t p = p0 + threadIdx.x;
-        Slot e{0, 0};
-        bool live = false;
-        if (p < tail) {
-            e = lg[p & lmask];
-            uint64_t st = 0;
-            live = table_find(t, mask, e.key, &st, d.err) >= 0 && st == e.stamp;
-        }
-        uint32_t tot;
-        const uint32_t rk = block_rank(live, s_w, tot);
-        if (live) lg[(w + rk) & lmask] = e;   // w + rk <= p: order-preserving, in place
-        __syncthreads();
-        w += tot;
-    }
-    if (threadIdx.x == 0) d.log_tail[i] = w;
-    if (!rebuild) return;
-    __syncthreads();
-    for (uint64_t s = threadIdx.x; s < d.S; s += blockDim.x) t[s] = Slot{0, 0};
-    __syncthreads();
-    for (uint64_t p = front + threadIdx.x; p < w; p += blockDim.x) {
-        const Slot e = lg[p & lmask];
-        bool claimed = false;
-        uint64_t j = e.key & mask;
-        for (uint64_t it = 0; it <= mask; ++it) {   // keys are distinct: claim the first empty slot
-            const unsigned long long prev =
-                atomicCAS(reinterpret_cast<unsigned long long *>(&t[j].key), 0ull, (unsigned long long)e.key);
-            if (prev == 0) { t[j].stamp = e.stamp; claimed = true; break; }
-            j = (j + 1) & mask;
-        }
-        if (!claimed) set_err(d.err, DM_ERR_TIMEOUT);
-    }
-    if (threadIdx.x == 0) d.used[i] = w - front;
+    return lo;
 }
 
-// Log positions of each request's touches (arrival order per instance), the
-// clock base of the batch, and the new log tails.  Single CTA; dynamic smem
-// holds one u64 tail per instance.
+// ---------------------------------------------------------------------------
+// Maintenance before the touches.
+//   plan  one CTA: blocks each instance receives, which instances need a
+//         compaction (log would overflow) or a rebuild (index would pass half
+//         full), and the chunk lists of both;
+//   a     grid: clear the second index (rebuild) / stale flags (compaction),
+//         count live records per 1024-record chunk of the log;
+//   scan  warp per compacting instance: chunk counts -> destination offsets;
+//   c     grid: walk the live records; compaction copies them in order into
+//         the second log (and repoints their index slots, or inserts them
+//         into the second index when rebuilding too); a rebuild alone
+//         inserts them with their current positions.
+
+__global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
+    extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ uint32_t s_w[33];
+    if (has_err(d.err)) return;
+    unsigned long long *cntv = reinterpret_cast<unsigned long long *>(smem);
+    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) cntv[i] = 0;
+    __syncthreads();
+    for (uint32_t r = threadIdx.x; r < n; r += blockDim.x)
+        atomicAdd(&cntv[d.r_final[r]], (unsigned long long)d.r_nblk[r]);
+    __syncthreads();
+    uint32_t cw = 0, cz = 0;
+    for (uint32_t base = 0; base < d.M; base += blockDim.x) {
+        const uint32_t i = base + threadIdx.x;
+        uint32_t nw = 0, nz = 0, fl = 0;
+        if (i < d.M && d.table[i]) {
+            const uint64_t cnt = cntv[i];
+            if (cnt > d.T) set_err(d.err, DM_ERR_CAPACITY);
+            const uint64_t len = d.log_tail[i] - d.log_front[i];
+            if (len + cnt > d.logcap) {
+                fl |= kFlagCompact;
+                nz += (uint32_t)((d.logcap + kZeroChunk - 1) / kZeroChunk);
+            }
+            if (d.used[i] + cnt > d.S / 2) {
+                fl |= kFlagRebuild;
+                nz += (uint32_t)((d.S + kZeroChunk - 1) / kZeroChunk);
+            }
+            if (fl) nw = (uint32_t)((len + kEvChunk - 1) / kEvChunk);
+            d.touch_cnt[i] = cnt;
+        }
+        uint32_t tw, tz;
+        const uint32_t ew = block_excl_u32(nw, s_w, tw);
+        const uint32_t ez = block_excl_u32(nz, s_w, tz);
+        if (i < d.M) {
+            d.mc_chunk_off[i] = cw + ew;
+            d.mr_chunk_off[i] = cz + ez;
+            d.mt_flags[i] = fl;
+        }
+        cw += tw;
+        cz += tz;
+    }
+    if (threadIdx.x == 0) {
+        d.mc_chunk_off[d.M] = cw;
+        d.mr_chunk_off[d.M] = cz;
+        d.info->mc_chunks = cw;
+        d.info->mr_chunks = cz;
+        if (cw > d.mc_cap) set_err(d.err, DM_ERR_CAPACITY);
+    }
+}
+
+__global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
+    __shared__ uint32_t s_i, s_cnt[kMtThreads / 32];
+    if (has_err(d.err)) return;
+    // clearing: a rebuilding instance's chunks cover its second index first,
+    // a compacting instance's (then) its second stale-flag array
+    const uint32_t nz = d.info->mr_chunks;
+    for (uint32_t c = blockIdx.x; c < nz; c += gridDim.x) {
+        if (threadIdx.x == 0) s_i = owner_of(d.mr_chunk_off, d.M, c);
+        __syncthreads();
+        const uint32_t i = s_i;
+        const uint32_t fl = d.mt_flags[i];
+        uint64_t k = uint64_t(c - d.mr_chunk_off[i]) * kZeroChunk;
+        const uint64_t tab = (fl & kFlagRebuild) ? d.S : 0;
+        const uint64_t tab_chunks_end = (tab + kZeroChunk - 1) / kZeroChunk * kZeroChunk;
+        if (k < tab_chunks_end) {
+            Slot *t = d.table_alt[i];
+            for (uint32_t q = threadIdx.x; q < kZeroChunk; q += kMtThreads)
+                if (k + q < tab) t[k + q] = Slot{0, 0};
+        } else {
+            k -= tab_chunks_end;
+            uint8_t *f = d.stale_alt[i];
+            for (uint32_t q = threadIdx.x; q < kZeroChunk; q += kMtThreads)
+                if (k + q < d.logcap) f[k + q] = 0;
+        }
+        __syncthreads();
+    }
+    // live records per log chunk of every instance being maintained
+    const uint32_t nw = d.info->mc_chunks;
+    const uint64_t lmask = d.logcap - 1;
+    for (uint32_t c = blockIdx.x; c < nw; c += gridDim.x) {
+        if (threadIdx.x == 0) s_i = owner_of(d.mc_chunk_off, d.M, c);
+        __syncthreads();
+        const uint32_t i = s_i;
+        const uint64_t tail = d.log_tail[i];
+        const uint64_t base = d.log_front[i] + uint64_t(c - d.mc_chunk_off[i]) * kEvChunk;
+        const uint8_t *st = d.stale[i];
+        uint32_t cnt = 0;
+        for (uint32_t k = threadIdx.x; k < kEvChunk; k += kMtThreads)
+            cnt += (base + k < tail && !st[(base + k) & lmask]);
+        cnt = __reduce_add_sync(0xffffffffu, cnt);
+        if ((threadIdx.x & 31) == 0) s_cnt[threadIdx.x >> 5] = cnt;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            uint32_t t = 0;
+            for (int w = 0; w < kMtThreads / 32; ++w) t += s_cnt[w];
+            d.mc_chunk_live[c] = t;
+        }
+        __syncthreads();
+    }
+}
+
+// Warp per compacting instance: chunk counts -> exclusive destination offsets.
+__global__ void k_compact_scan(DevState d) {
+    if (has_err(d.err)) return;
+    const int lane = threadIdx.x & 31;
+    const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (i >= d.M || !(d.mt_flags[i] & kFlagCompact)) return;
+    const uint32_t c0 = d.mc_chunk_off[i], c1 = d.mc_chunk_off[i + 1];
+    uint64_t carry = 0;
+    for (uint32_t cb = c0; cb < c1; cb += 32) {
+        const uint32_t c = cb + lane;
+        const uint64_t v = c < c1 ? d.mc_chunk_live[c] : 0;
+        const uint64_t inc = warp_incl_scan(v, lane);
+        if (c < c1) d.mc_chunk_live[c] = (uint32_t)(carry + inc - v);
+        carry += shfl_u64(inc, 31);
+    }
+    if (lane == 0) d.mt_newtail[i] = d.log_front[i] + carry;
+}
+
+__global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
+    __shared__ uint32_t s_i, s_w[kMtThreads / 32];
+    if (has_err(d.err)) return;
+    const uint32_t nw = d.info->mc_chunks;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const uint64_t lmask = d.logcap - 1, mask = d.S - 1;
+    for (uint32_t c = blockIdx.x; c < nw; c += gridDim.x) {
+        if (threadIdx.x == 0) s_i = owner_of(d.mc_chunk_off, d.M, c);
+        __syncthreads();
+        const uint32_t i = s_i;
+        const uint32_t fl = d.mt_flags[i];
+        const uint64_t front = d.log_front[i], tail = d.log_tail[i];
+        const uint64_t base = front + uint64_t(c - d.mc_chunk_off[i]) * kEvChunk;
+        const Rec *lg = d.logbuf[i];
+        const uint8_t *st = d.stale[i];
+        uint64_t out = front + ((fl & kFlagCompact) ? d.mc_chunk_live[c] : 0);
+        for (uint32_t k0 = 0; k0 < kEvChunk; k0 += kMtThreads) {   // keeps record order
+            const uint64_t p = base + k0 + threadIdx.x;
+            const bool live = p < tail && !st[p & lmask];
+            const uint32_t b = __ballot_sync(0xffffffffu, live);
+            if (lane == 0) s_w[wid] = __popc(b);
+            __syncthreads();
+            uint32_t before = 0, tot = 0;
+            for (int w = 0; w < kMtThreads / 32; ++w) {
+                before += w < wid ? s_w[w] : 0;
+                tot += s_w[w];
+            }
+            if (live) {
+                const Rec r = lg[p & lmask];
+                if (fl & kFlagCompact) {
+                    const uint64_t np = out + before + __popc(b & ((1u << lane) - 1));
+                    d.logbuf_alt[i][np & lmask] = r;
+                    if (fl & kFlagRebuild) table_insert_new(d.table_alt[i], mask, r.key, np + 1, d.err);
+                    else table_set_pos(d.table[i], mask, r.key, np + 1, d.err);
+                } else {
+                    table_insert_new(d.table_alt[i], mask, r.key, p + 1, d.err);
+                }
+            }
+            out += tot;
+            __syncthreads();
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Swap in compacted logs / rebuilt indices, fix each instance's log base for
+// this commit and advance its tail.  The choice kernel already placed every
+// request among its instance's records; only when a rebalance moved a
+// request of this batch are the offsets recomputed (arrival order per final
+// instance).  Single CTA; dynamic smem holds one u64 per instance.
 __global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
     extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ uint32_t s_f[kPrepChunk], s_nb[kPrepChunk];
+    __shared__ uint64_t s_off[kPrepChunk];
     if (has_err(d.err)) return;
-    uint64_t *tl = reinterpret_cast<uint64_t *>(smem);
-    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) tl[i] = d.log_tail[i];
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        for (uint32_t r = 0; r < n; ++r) {
-            const uint32_t f = d.r_final[r];
-            d.r_touchoff[r] = tl[f];
-            tl[f] += d.r_nblk[r];
+    uint64_t *adv = reinterpret_cast<uint64_t *>(smem);
+    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
+        const uint32_t fl = d.mt_flags[i];
+        if (fl & kFlagCompact) {
+            Rec *a = d.logbuf[i];
+            d.logbuf[i] = d.logbuf_alt[i];
+            d.logbuf_alt[i] = a;
+            uint8_t *f = d.stale[i];
+            d.stale[i] = d.stale_alt[i];
+            d.stale_alt[i] = f;
+            d.log_tail[i] = d.mt_newtail[i];
         }
+        if (fl & kFlagRebuild) {
+            Slot *a = d.table[i];
+            d.table[i] = d.table_alt[i];
+            d.table_alt[i] = a;
+            d.used[i] = d.live[i];
+        }
+        adv[i] = d.log_adv[i];
+    }
+    const bool dirty = d.info->final_dirty != 0;
+    if (dirty) {
+        __syncthreads();
+        for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) adv[i] = 0;
+        for (uint32_t base = 0; base < n; base += kPrepChunk) {
+            const uint32_t m = min(kPrepChunk, n - base);
+            __syncthreads();
+            for (uint32_t k = threadIdx.x; k < m; k += blockDim.x) {
+                s_f[k] = d.r_final[base + k];
+                s_nb[k] = d.r_nblk[base + k];
+            }
+            __syncthreads();
+            if (threadIdx.x == 0)
+                for (uint32_t k = 0; k < m; ++k) {
+                    const uint32_t f = s_f[k];
+                    const uint64_t o = adv[f];
+                    s_off[k] = o;
+                    adv[f] = o + s_nb[k];
+                }
+            __syncthreads();
+            for (uint32_t k = threadIdx.x; k < m; k += blockDim.x) d.r_touchoff[base + k] = s_off[k];
+        }
+        __syncthreads();
+    }
+    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
+        const uint64_t b = d.log_tail[i];
+        d.log_base[i] = b;
+        d.log_tail[i] = b + adv[i];
+    }
+    if (threadIdx.x == 0) {
         d.info->clock_base = *d.clock;
         *d.clock += d.info->total_blocks;
     }
-    __syncthreads();
-    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) d.log_tail[i] = tl[i];
 }
 
-// One warp per 256-block segment: cache keys, stamps, log records, index touches.
+// One warp per segment: cache keys, stamps, log records, index touches.  A
+// superseded record (the key's previous record, or this one when a later
+// touch of the batch already won) gets its stale flag.  Lane l handles
+// blocks l and l+32 of the segment together: the CAS at both home slots,
+// then both atomicMax, so their round trips overlap.
+__device__ __forceinline__ void touch_outcome(uint64_t old, uint64_t p, uint64_t front, uint8_t *st, uint64_t lmask,
+                                              uint32_t &newly) {
+    if (old == 0 || old - 1 < front) {
+        ++newly;                                  // new or evicted: resident again
+    } else if (old - 1 < p) {
+        st[(old - 1) & lmask] = 1;                // previous record superseded
+    } else {
+        st[p & lmask] = 1;                        // a later touch of this batch won
+    }
+}
+
 __global__ void __launch_bounds__(256) k_commit_touch(DevState d) {
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
@@ -166,63 +380,247 @@ __global__ void __launch_bounds__(256) k_commit_touch(DevState d) {
         const uint32_t nblk = d.r_nblk[r];
         const uint32_t f = d.r_final[r];
         const uint64_t carry = d.seg_carry[seg];
-        const uint64_t bo = d.r_blkoff[r], toff = d.r_touchoff[r];
+        const uint64_t bo = d.r_blkoff[r], toff = d.log_base[f] + d.r_touchoff[r];
+        const uint64_t front = d.log_front[f];
         Slot *t = d.table[f];
-        Slot *lg = d.logbuf[f];
+        Rec *lg = d.logbuf[f];
+        uint8_t *st = d.stale[f];
         const uint32_t b_end = min(nblk, (j + 1) * kSegBlocks);
         uint32_t newly = 0, claims = 0;
-        for (uint32_t b = j * kSegBlocks + lane; b < b_end; b += 32) {
-            const uint64_t key = cache_key(d.plocal[bo + b] + carry, d.Sc);
-            const uint64_t stamp = clock_base + bo + (nblk - b);   // block n_blk-1 is touched first
-            lg[(toff + (nblk - 1 - b)) & lmask] = Slot{key, stamp};
-            bool claimed = false;
-            newly += table_touch(t, mask, key, stamp, d.err, &claimed);
-            claims += claimed;
+        for (uint32_t b = j * kSegBlocks + lane; b < b_end; b += 64) {
+            const bool v1 = b + 32 < b_end;
+            const uint64_t k0 = cache_key(d.plocal[bo + b] + carry, d.Sc);
+            const uint64_t k1 = v1 ? cache_key(d.plocal[bo + b + 32] + carry, d.Sc) : 0;
+            const uint64_t p0 = toff + (nblk - 1 - b);              // block n_blk-1 is touched first
+            const uint64_t p1 = toff + (nblk - 1 - (b + 32));
+            lg[p0 & lmask] = Rec{k0, clock_base + bo + (nblk - b)};
+            if (v1) lg[p1 & lmask] = Rec{k1, clock_base + bo + (nblk - b - 32)};
+            const uint64_t i0 = k0 & mask, i1 = k1 & mask;
+            const unsigned long long c0 =
+                atomicCAS(reinterpret_cast<unsigned long long *>(&t[i0].key), 0ull, (unsigned long long)k0);
+            const unsigned long long c1 =
+                v1 ? atomicCAS(reinterpret_cast<unsigned long long *>(&t[i1].key), 0ull, (unsigned long long)k1) : 0;
+            bool cl0 = false, cl1 = false;
+            const uint64_t s0 = slot_after_home_cas(t, mask, k0, i0, c0, d.err, &cl0);
+            const uint64_t s1 = v1 ? slot_after_home_cas(t, mask, k1, i1, c1, d.err, &cl1) : 0;
+            const uint64_t o0 =
+                atomicMax(reinterpret_cast<unsigned long long *>(&t[s0].pos1), (unsigned long long)(p0 + 1));
+            const uint64_t o1 = v1 ? atomicMax(reinterpret_cast<unsigned long long *>(&t[s1].pos1),
+                                               (unsigned long long)(p1 + 1)) : 0;
+            touch_outcome(o0, p0, front, st, lmask, newly);
+            if (v1) touch_outcome(o1, p1, front, st, lmask, newly);
+            claims += cl0 + cl1;
         }
         newly = __reduce_add_sync(0xffffffffu, newly);
         claims = __reduce_add_sync(0xffffffffu, claims);
-        if (lane == 0) {
-            if (newly) atomicAdd(reinterpret_cast<unsigned long long *>(&d.live[f]), (unsigned long long)newly);
-            if (claims) atomicAdd(reinterpret_cast<unsigned long long *>(&d.used[f]), (unsigned long long)claims);
+        if (lane == 0) {   // summed per instance by the eviction plan (no hot-counter atomics)
+            d.seg_newly[seg] = newly;
+            d.seg_claims[seg] = claims;
         }
     }
 }
 
-// Evict the oldest resident keys of every instance above capacity.  CTA per id.
-__global__ void __launch_bounds__(1024) k_evict(DevState d) {
+// ---------------------------------------------------------------------------
+// Eviction.  Instance i drops its excess_i = live_i - C oldest resident keys
+// by moving its log front just past the excess_i-th non-stale record:
+//   plan   one CTA: a window of 2*excess_i + 2048 records from the front,
+//          cut into 1024-record chunks;
+//   count  grid over all chunks: non-stale records per chunk;
+//   cut    warp per instance: chunk and record where the count reaches
+//          excess_i;
+//   clear  grid over all chunks: reset the stale flags the front passes;
+//   walk   new fronts; an instance whose window held too few non-stale
+//          records continues record by record after it (rare).
+constexpr int kEvThreads = 256;
+
+// Warp per request: sum the touch kernel's counts over the request's
+// (contiguous) segments, one atomic per request and counter.
+__global__ void k_req_counts(DevState d, uint32_t n) {
+    if (has_err(d.err)) return;
+    const int lane = threadIdx.x & 31;
+    const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (r >= n) return;
+    const uint32_t s0 = d.r_segoff[r];
+    const uint32_t ns = (d.r_nblk[r] + kSegBlocks - 1) / kSegBlocks;
+    uint32_t a = 0, b = 0;
+    for (uint32_t j = lane; j < ns; j += 32) {
+        a += d.seg_newly[s0 + j];
+        b += d.seg_claims[s0 + j];
+    }
+    a = __reduce_add_sync(0xffffffffu, a);
+    b = __reduce_add_sync(0xffffffffu, b);
+    if (lane == 0) {
+        const uint32_t f = d.r_final[r];
+        if (a) atomicAdd(reinterpret_cast<unsigned long long *>(&d.live[f]), (unsigned long long)a);
+        if (b) atomicAdd(reinterpret_cast<unsigned long long *>(&d.used[f]), (unsigned long long)b);
+    }
+}
+
+__global__ void __launch_bounds__(1024) k_evict_plan(DevState d) {
+    __shared__ uint32_t s_w[33];
+    if (has_err(d.err)) return;
+    uint32_t carry = 0;
+    for (uint32_t base = 0; base < d.M; base += blockDim.x) {
+        const uint32_t i = base + threadIdx.x;
+        uint64_t excess = 0, win = 0;
+        if (i < d.M && d.table[i] && d.live[i] > d.C) {
+            excess = d.live[i] - d.C;
+            win = min(d.log_tail[i] - d.log_front[i], 2 * excess + 2048);
+        }
+        const uint32_t chunks = (uint32_t)((win + kEvChunk - 1) / kEvChunk);
+        uint32_t tot;
+        const uint32_t ex = block_excl_u32(chunks, s_w, tot);
+        if (i < d.M) {
+            d.ev_chunk_off[i] = carry + ex;
+            d.ev_excess[i] = excess;
+            d.ev_win[i] = win;
+            d.ev_rem[i] = 0;
+            d.ev_front_new[i] = d.log_front[i];
+        }
+        carry += tot;
+    }
+    if (threadIdx.x == 0) {
+        d.ev_chunk_off[d.M] = carry;
+        d.info->ev_chunks = carry;
+        if (uint64_t(carry) * kEvChunk > d.ev_cap) set_err(d.err, DM_ERR_CAPACITY);
+    }
+}
+
+__global__ void __launch_bounds__(kEvThreads) k_evict_count(DevState d) {
+    __shared__ uint32_t s_i;
+    __shared__ uint32_t s_cnt[kEvThreads / 32];
+    if (has_err(d.err)) return;
+    const uint32_t nchunks = d.info->ev_chunks;
+    const uint64_t lmask = d.logcap - 1;
+    for (uint32_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
+        if (threadIdx.x == 0) s_i = owner_of(d.ev_chunk_off, d.M, c);
+        __syncthreads();
+        const uint32_t i = s_i;
+        const uint64_t front = d.log_front[i];
+        const uint64_t end = front + d.ev_win[i];
+        const uint64_t base = front + uint64_t(c - d.ev_chunk_off[i]) * kEvChunk;
+        const uint8_t *st = d.stale[i];
+        uint32_t cnt = 0;
+        for (uint32_t k = threadIdx.x; k < kEvChunk; k += kEvThreads)
+            cnt += (base + k < end && !st[(base + k) & lmask]);
+        cnt = __reduce_add_sync(0xffffffffu, cnt);
+        if ((threadIdx.x & 31) == 0) s_cnt[threadIdx.x >> 5] = cnt;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            uint32_t tot = 0;
+            for (int w = 0; w < kEvThreads / 32; ++w) tot += s_cnt[w];
+            d.ev_chunk_live[c] = tot;
+        }
+        __syncthreads();
+    }
+}
+
+// Warp per instance: locate the record where the non-stale count reaches excess.
+__global__ void k_evict_cut(DevState d) {
+    if (has_err(d.err)) return;
+    const int lane = threadIdx.x & 31;
+    const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (i >= d.M) return;
+    const uint64_t excess = d.ev_excess[i];
+    if (excess == 0) return;
+    const uint32_t c0 = d.ev_chunk_off[i], c1 = d.ev_chunk_off[i + 1];
+    uint64_t cum = 0;
+    uint32_t cstar = c1;
+    uint64_t need = 0;
+    for (uint32_t cb = c0; cb < c1 && cstar == c1; cb += 32) {
+        const uint32_t c = cb + lane;
+        const uint64_t v = c < c1 ? d.ev_chunk_live[c] : 0;
+        const uint64_t inc = warp_incl_scan(v, lane) + cum;
+        const uint32_t hit = __ballot_sync(0xffffffffu, c < c1 && inc >= excess);
+        if (hit) {
+            const int l = __ffs(hit) - 1;
+            cstar = cb + l;
+            need = excess - (shfl_u64(inc, l) - shfl_u64(v, l));   // non-stale records needed in cstar
+        } else {
+            cum = shfl_u64(inc, 31);
+        }
+    }
+    const uint64_t front = d.log_front[i];
+    if (cstar == c1) {   // window too short: the walker continues after it
+        if (lane == 0) {
+            d.ev_front_new[i] = front + d.ev_win[i];
+            d.ev_rem[i] = excess - cum;
+        }
+        return;
+    }
+    // lane l owns records 32l .. 32l+31 of chunk cstar
+    const uint64_t cbase = front + uint64_t(cstar - c0) * kEvChunk + 32 * lane;
+    const uint64_t end = front + d.ev_win[i];
+    const uint8_t *st = d.stale[i];
+    uint32_t mbits = 0;
+#pragma unroll 8
+    for (int b = 0; b < 32; ++b) {
+        const uint64_t p = cbase + b;
+        mbits |= ((p < end && !st[p & (d.logcap - 1)]) ? 1u : 0u) << b;
+    }
+    const uint32_t cnt = __popc(mbits);
+    uint32_t inc = cnt;
+#pragma unroll
+    for (int dd = 1; dd < 32; dd <<= 1) {
+        const uint32_t u = __shfl_up_sync(0xffffffffu, inc, dd);
+        if (lane >= dd) inc += u;
+    }
+    const uint32_t ex = inc - cnt;
+    if (ex < need && need <= inc)   // exactly one lane
+        d.ev_front_new[i] = cbase + __fns(mbits, 0, (int)(need - ex)) + 1;
+}
+
+// Reset the stale flags of the records the front passes (those positions
+// will hold new records).
+__global__ void __launch_bounds__(kEvThreads) k_evict_clear(DevState d) {
+    __shared__ uint32_t s_i;
+    if (has_err(d.err)) return;
+    const uint32_t nchunks = d.info->ev_chunks;
+    const uint64_t lmask = d.logcap - 1;
+    for (uint32_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
+        if (threadIdx.x == 0) s_i = owner_of(d.ev_chunk_off, d.M, c);
+        __syncthreads();
+        const uint32_t i = s_i;
+        const uint64_t front = d.log_front[i];
+        const uint64_t cut = d.ev_front_new[i];
+        const uint64_t base = front + uint64_t(c - d.ev_chunk_off[i]) * kEvChunk;
+        uint8_t *st = d.stale[i];
+        for (uint32_t k = threadIdx.x; k < kEvChunk; k += kEvThreads)
+            if (base + k < cut) st[(base + k) & lmask] = 0;
+        __syncthreads();
+    }
+}
+
+__global__ void __launch_bounds__(1024) k_evict_walk(DevState d) {
     __shared__ uint32_t s_w[33];
     __shared__ uint64_t s_front;
     if (has_err(d.err)) return;
     const uint32_t i = blockIdx.x;
-    Slot *t = d.table[i];
-    if (!t) return;
-    const uint64_t live = d.live[i];
-    if (live <= d.C) return;
-    Slot *lg = d.logbuf[i];
-    const uint64_t mask = d.S - 1, lmask = d.logcap - 1;
+    if (d.ev_excess[i] == 0) return;
+    uint64_t remaining = d.ev_rem[i];
+    uint64_t front = d.ev_front_new[i];
+    if (remaining == 0) {
+        if (threadIdx.x == 0) {
+            d.log_front[i] = front;
+            d.live[i] = d.C;
+        }
+        return;
+    }
+    uint8_t *st = d.stale[i];
+    const uint64_t lmask = d.logcap - 1;
     const uint64_t tail = d.log_tail[i];
-    uint64_t front = d.log_front[i];
-    uint64_t remaining = live - d.C;
     while (remaining > 0 && front < tail) {
         const uint64_t p = front + threadIdx.x;
-        int64_t slot = -1;
-        bool is_live = false;
-        if (p < tail) {
-            const Slot e = lg[p & lmask];
-            uint64_t st = 0;
-            slot = table_find(t, mask, e.key, &st, d.err);
-            is_live = slot >= 0 && st == e.stamp;
-        }
+        const bool live = p < tail && !st[p & lmask];
         uint32_t tot;
-        const uint32_t rk = block_rank(is_live, s_w, tot);
+        const uint32_t rk = block_excl_u32(live ? 1u : 0u, s_w, tot);
         if (threadIdx.x == 0) s_front = min(front + blockDim.x, tail);
         __syncthreads();
-        if (is_live && rk < remaining) {
-            t[slot].stamp = 0;
-            if (rk == remaining - 1) s_front = p + 1;
-        }
+        if (live && rk == remaining - 1) s_front = p + 1;
         __syncthreads();
-        front = s_front;
+        const uint64_t nf = s_front;
+        if (p < nf) st[p & lmask] = 0;
+        front = nf;
         remaining -= remaining < (uint64_t)tot ? remaining : (uint64_t)tot;
         __syncthreads();
     }
@@ -230,25 +628,37 @@ __global__ void __launch_bounds__(1024) k_evict(DevState d) {
         if (remaining) set_err(d.err, DM_ERR_TIMEOUT);   // the log must cover every live key
         d.log_front[i] = front;
         d.live[i] = d.C;
+        d.ev_rem[i] = 0;
     }
 }
 
 cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    cudaError_t e = cudaMemsetAsync(d.touch_cnt, 0, sizeof(uint64_t) * d.M, st);
-    if (e != cudaSuccess) return e;
-    k_commit_count<<<(n + 255) / 256, 256, 0, st>>>(d, n);
-    k_maintain<<<d.M, 1024, 0, st>>>(d);
     const size_t smem = sizeof(uint64_t) * d.M;
     static size_t configured = 0;
     if (smem > configured) {
-        e = cudaFuncSetAttribute(k_commit_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(k_commit_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(k_maint_plan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+
         if (e != cudaSuccess) return e;
         configured = smem;
     }
+    static const int g_a = full_grid(k_maint_a, kMtThreads), g_c = full_grid(k_maint_c, kMtThreads),
+                     g_t = full_grid(k_commit_touch, 256), g_ec = full_grid(k_evict_count, kEvThreads),
+                     g_el = full_grid(k_evict_clear, kEvThreads);
+    k_maint_plan<<<1, 1024, smem, st>>>(d, n);
+    k_maint_a<<<g_a, kMtThreads, 0, st>>>(d);
+    k_compact_scan<<<(d.M + 7) / 8, 256, 0, st>>>(d);
+    k_maint_c<<<g_c, kMtThreads, 0, st>>>(d);
     k_commit_prep<<<1, 1024, smem, st>>>(d, n);
-    k_commit_touch<<<hash_grid_size(), 256, 0, st>>>(d);
-    k_evict<<<d.M, 1024, 0, st>>>(d);
+    k_commit_touch<<<g_t, 256, 0, st>>>(d);
+    k_req_counts<<<(n + 7) / 8, 256, 0, st>>>(d, n);
+    k_evict_plan<<<1, 1024, 0, st>>>(d);
+    k_evict_count<<<g_ec, kEvThreads, 0, st>>>(d);
+    k_evict_cut<<<(d.M + 7) / 8, 256, 0, st>>>(d);
+    k_evict_clear<<<g_el, kEvThreads, 0, st>>>(d);
+    k_evict_walk<<<d.M, 1024, 0, st>>>(d);
     return cudaGetLastError();
 }
 

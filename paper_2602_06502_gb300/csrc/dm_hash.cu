@@ -5,11 +5,11 @@
 //   nh^f_k = sum_i ((t_2i + K^f_2i) mod 2^32) * ((t_2i+1 + K^f_2i+1) mod 2^32)  mod 2^64
 //   d^f_k  = fmix64(nh^f_k + (k+1) G^f)
 //   P^f_b  = sum_{k<=b} d^f_k  mod 2^64
-// Because the chain is a plain prefix sum, every 256-block segment of every
+// Because the chain is a plain prefix sum, every 64-block segment of every
 // prompt is hashed independently (one warp each); a segment writes its local
-// prefix values and its total, and the probe kernel adds the carry of the
+// prefix values and its totals, and the probe kernel adds the carry of the
 // earlier segments.  f2 only runs over the first K = min(K_route, n_blk)
-// blocks, which always lie in a prompt's first segment.
+// blocks: segments below K write the sum of their f2 digests.
 #include "dm_internal.cuh"
 
 namespace dm {
@@ -94,17 +94,22 @@ __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off,
         d.info->n = n;
         if (carry_blk > d.max_blocks || carry_seg > d.max_segs) set_err(d.err, DM_ERR_CAPACITY);
     }
-    __syncthreads();
+}
+
+// Segment -> request map, one warp per request.
+__global__ void k_segmap(DevState d, uint32_t n) {
     if (has_err(d.err)) return;
-    for (uint32_t r = threadIdx.x; r < n; r += blockDim.x) {
-        uint32_t s0 = d.r_segoff[r];
-        uint32_t ns = (d.r_nblk[r] + kSegBlocks - 1) / kSegBlocks;
-        for (uint32_t j = 0; j < ns; ++j) d.seg_req[s0 + j] = r;
-    }
+    const int lane = threadIdx.x & 31;
+    const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (r >= n) return;
+    const uint32_t s0 = d.r_segoff[r];
+    const uint32_t ns = (d.r_nblk[r] + kSegBlocks - 1) / kSegBlocks;
+    for (uint32_t j = lane; j < ns; j += 32) d.seg_req[s0 + j] = r;
 }
 
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st) {
     k_setup<<<1, 1024, 0, st>>>(d, b.offsets, b.lengths, b.n, b.total_tokens);
+    if (b.n) k_segmap<<<(b.n + 7) / 8, 256, 0, st>>>(d, b.n);
     return cudaGetLastError();
 }
 
@@ -140,13 +145,16 @@ __device__ __forceinline__ uint64_t reduce_scatter(uint64_t (&p)[U], int q) {
     return p[0];
 }
 
-// One warp per segment of up to 256 blocks.  An iteration covers 32 blocks
-// (32*U uint4): load j of lane l reads uint4 j*32+l (fully coalesced), which
-// is quarter l%U of block j*(32/U)+l/U.  After the reduce-scatter lane l
+// One warp per segment of up to 64 blocks (two iterations of 32 blocks).
+// Iteration `it` covers 32 blocks (32*U uint4): load j of lane l reads uint4
+// j*32+l of the iteration (fully coalesced), which is quarter l%U of block
+// j*(32/U)+l/U.  Both iterations' loads are issued before any arithmetic
+// (4 KB in flight per warp at B = 16).  After the reduce-scatter lane l
 // holds block (l%U)*(32/U) + l/U; one shuffle puts block m on lane m for the
-// scan.
+// scan.  Segments below K also sum their f2 digests (blocks < K).
 template <int U>
 __global__ void __launch_bounds__(256) k_hash(DevState d, const uint32_t *__restrict__ tokens) {
+    constexpr int IT = kSegBlocks / 32;
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
@@ -170,19 +178,23 @@ __global__ void __launch_bounds__(256) k_hash(DevState d, const uint32_t *__rest
         const uint4 *src4 = reinterpret_cast<const uint4 *>(tokens + d.r_tokoff[r] + uint64_t(b0) * d.B);
         uint64_t *out = d.plocal + d.r_blkoff[r] + b0;
         const uint32_t K = min(d.Kroute, nblk);
-        uint64_t carry1 = 0, carry2 = 0;
-        for (uint32_t it = 0; it * 32 < nb; ++it) {
-            const uint32_t nvalid = min(32u, nb - it * 32);
-            uint4 v[U];
+        uint4 v[IT][U];
+#pragma unroll
+        for (int it = 0; it < IT; ++it)
 #pragma unroll
             for (int jj = 0; jj < U; ++jj) {
-                const uint32_t blk = jj * GPL + g;
-                v[jj] = blk < nvalid ? ld_stream(src4 + uint64_t(it) * 32 * U + jj * 32 + lane)
+                const uint32_t blk = it * 32 + jj * GPL + g;
+                v[it][jj] = blk < nb ? ld_stream(src4 + uint64_t(it) * 32 * U + jj * 32 + lane)
                                      : make_uint4(0, 0, 0, 0);
             }
+        uint64_t carry1 = 0, sum2 = 0;
+#pragma unroll
+        for (int it = 0; it < IT; ++it) {
+            if ((uint32_t)it * 32 >= nb) break;
+            const uint32_t nvalid = min(32u, nb - it * 32);
             uint64_t p1[U];
 #pragma unroll
-            for (int jj = 0; jj < U; ++jj) p1[jj] = nh4(v[jj], k1);
+            for (int jj = 0; jj < U; ++jj) p1[jj] = nh4(v[it][jj], k1);
             const uint64_t s1 = reduce_scatter<U>(p1, q);
             const uint32_t kb = b0 + it * 32 + bq;   // block index within the prompt
             uint64_t dg1 = (uint32_t)bq < nvalid ? fmix64(s1 + uint64_t(kb + 1) * G1) : 0;
@@ -190,22 +202,20 @@ __global__ void __launch_bounds__(256) k_hash(DevState d, const uint32_t *__rest
             const uint64_t P1 = warp_incl_scan(dg1, lane) + carry1;
             if ((uint32_t)lane < nvalid) out[it * 32 + lane] = P1;
             carry1 = shfl_u64(P1, 31);
-            if (j == 0 && it * 32 < K) {              // second function, first K blocks
+            if (b0 + it * 32 < K) {                   // second function, blocks < K
                 uint64_t p2[U];
 #pragma unroll
-                for (int jj = 0; jj < U; ++jj) p2[jj] = nh4(v[jj], k2);
+                for (int jj = 0; jj < U; ++jj) p2[jj] = nh4(v[it][jj], k2);
                 const uint64_t s2 = reduce_scatter<U>(p2, q);
-                uint64_t dg2 = kb < K ? fmix64(s2 + uint64_t(kb + 1) * G2) : 0;
-                dg2 = shfl_u64(dg2, src);
-                const uint64_t P2 = warp_incl_scan(dg2, lane) + carry2;
-                carry2 = shfl_u64(P2, 31);
-                if (it * 32 + lane == K - 1) {
-                    d.r_pos[2 * r] = fmix64(P1 ^ d.Sr1);
-                    d.r_pos[2 * r + 1] = fmix64(P2 ^ d.Sr2);
-                }
+                sum2 += ((uint32_t)bq < nvalid && kb < K) ? fmix64(s2 + uint64_t(kb + 1) * G2) : 0;
             }
         }
-        if (lane == 0) d.seg_total[seg] = carry1;
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) sum2 += shfl_xor_u64(sum2, o);
+        if (lane == 0) {
+            d.seg_total[seg] = carry1;
+            d.seg_total2[seg] = sum2;
+        }
     }
 }
 
@@ -246,10 +256,12 @@ __global__ void k_hash_keys(DevState d, uint32_t n, uint64_t *keys, uint64_t *ke
     const uint64_t bo = d.r_blkoff[r];
     for (uint32_t b = lane; b < nblk; b += 32)
         keys[bo + b] = cache_key(d.plocal[bo + b] + d.seg_carry[s0 + b / kSegBlocks], d.Sc);
+    uint64_t p1, p2;
+    route_positions(d, r, lane, p1, p2);
     if (lane == 0) {
         key_off[r] = bo;
-        pos[2 * r] = d.r_pos[2 * r];
-        pos[2 * r + 1] = d.r_pos[2 * r + 1];
+        pos[2 * r] = p1;
+        pos[2 * r + 1] = p2;
         if (r == n - 1) key_off[n] = bo + nblk;
     }
 }

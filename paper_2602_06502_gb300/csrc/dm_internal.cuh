@@ -10,11 +10,13 @@
 namespace dm {
 
 constexpr int kWarp = 32;
-constexpr uint32_t kSegBlocks = 256;       // blocks hashed by one warp task
+constexpr uint32_t kSegBlocks = 64;        // blocks hashed by one warp task
 constexpr uint32_t kMaxInstances = 8192;
 constexpr uint32_t kMaxRouteBlocks = 256;
 constexpr uint32_t kTomb = 0xFFFFFFFFu;    // QEntry::moved of an entry migrated away
 constexpr int kMaxLevels = 8;
+constexpr uint32_t kEvChunk = 1024;      // log records per eviction / compaction chunk
+constexpr uint32_t kRbChunk = 4096;      // index slots per rebuild chunk
 constexpr uint64_t kSpinLimit = 1ull << 26; // bound of every data-dependent device loop
 
 // One queued request (48 bytes).
@@ -24,10 +26,16 @@ struct QEntry {
     uint32_t moved;   // 0, or the rebalance call that moved it here, or kTomb
 };
 
-// One index slot / one recency-log record (16 bytes).  In the index, key 0
-// means empty and stamp 0 means "evicted" (the key stays, so a later touch
-// revives the slot in place).
+// One index slot (16 bytes): a block key and 1 + the position of its latest
+// record in the instance's recency log; key 0 marks an empty slot.  A key is
+// resident while that position is at or after the log front.
 struct Slot {
+    uint64_t key, pos1;
+};
+
+// One recency-log record (16 bytes): the block key and the global clock
+// stamp of the touch.  Records of an instance are in stamp order.
+struct Rec {
     uint64_t key, stamp;
 };
 
@@ -38,6 +46,9 @@ struct BatchInfo {
     uint32_t n;
     uint64_t clock_base;    // commit clock before this batch's touches
     uint32_t final_dirty;   // a rebalance moved a request of this batch
+    uint32_t ev_chunks;     // eviction window chunks of this commit
+    uint32_t mc_chunks;     // log-compaction chunks of this commit
+    uint32_t mr_chunks;     // index-rebuild chunks of this commit
     uint32_t pad;
 };
 
@@ -70,17 +81,35 @@ struct DevState {
     uint32_t *q_head, *q_tail;
     QEntry *q;                      // M x Q
     Slot **table;                   // per id: S slots (null until first add)
-    Slot **logbuf;                  // per id: logcap records
+    Rec **logbuf;                   // per id: logcap records
+    uint8_t **stale;                // per id: logcap flags, 1 = record superseded by a later touch
+    Slot **table_alt;               // per id: second index buffer (rebuild target)
+    Rec **logbuf_alt;               // per id: second log buffer (compaction target)
+    uint8_t **stale_alt;
     uint64_t *log_front, *log_tail, *live, *used;
     uint64_t *touch_cnt;            // per id: blocks touched by the pending commit
+    // eviction scratch: per id window plan and cut, per chunk live counts
+    uint64_t *ev_excess, *ev_win, *ev_front_new, *ev_rem;
+    uint32_t *ev_chunk_off;         // M + 1 entries
+    uint32_t *ev_chunk_live;
+    uint64_t ev_cap;                // window records that fit (chunks * kEvChunk)
+    // maintenance plan: per id flags / new log tail, chunk offsets and counts
+    uint32_t *mt_flags;
+    uint64_t *mt_newtail;
+    uint32_t *mc_chunk_off, *mr_chunk_off;   // M + 1 entries each
+    uint32_t *mc_chunk_live;
+    uint64_t mc_cap;                         // compaction chunks that fit
     // batch scratch
     uint32_t *r_L, *r_nblk, *r_segoff;
     uint64_t *r_tokoff, *r_blkoff;
     uint32_t *seg_req;
     uint64_t *seg_total, *seg_carry, *plocal;
-    uint64_t *r_pos;                // 2 per request
+    uint64_t *seg_total2;           // per segment: f2 digest sum over its blocks < K
+    uint32_t *seg_newly, *seg_claims;   // per segment: keys made resident / index slots taken by the commit
     uint32_t *r_c1, *r_c2, *r_h1, *r_h2, *r_final;
-    uint64_t *r_touchoff;
+    uint64_t *r_touchoff;           // per request: offset among its instance's records of the batch
+    uint64_t *log_adv;              // per id: log records the pending batch appends
+    uint64_t *log_base;             // per id: log tail when the commit starts
     BatchInfo *info;
     uint64_t *clock;
     uint32_t *err;
@@ -159,23 +188,22 @@ __device__ __forceinline__ uint64_t warp_incl_scan(uint64_t v, int lane) {
 __device__ __forceinline__ Slot load_slot(const Slot *p) {
     Slot s;
     asm volatile("ld.global.cg.v2.u64 {%0, %1}, [%2];"
-                 : "=l"(s.key), "=l"(s.stamp) : "l"(__cvta_generic_to_global(p)));
+                 : "=l"(s.key), "=l"(s.pos1) : "l"(__cvta_generic_to_global(p)));
     return s;
 }
 
 // Look key up in one instance's open-addressed (linear probing) index.
-// Returns the slot index holding the key (live or evicted) or -1.
-__device__ __forceinline__ int64_t table_find(const Slot *t, uint64_t mask, uint64_t key,
-                                              uint64_t *stamp, uint32_t *err) {
+// Returns 1 + log position of its latest record (0 if the key has no slot).
+__device__ __forceinline__ uint64_t table_pos1(const Slot *t, uint64_t mask, uint64_t key, uint32_t *err) {
     uint64_t i = key & mask;
     for (uint64_t it = 0; it <= mask; ++it) {
         Slot s = load_slot(t + i);
-        if (s.key == key) { *stamp = s.stamp; return (int64_t)i; }
-        if (s.key == 0) return -1;
+        if (s.key == key) return s.pos1;
+        if (s.key == 0) return 0;
         i = (i + 1) & mask;
     }
     set_err(err, DM_ERR_TIMEOUT);
-    return -1;
+    return 0;
 }
 
 // Carries of one request's segments (exclusive prefix of the segment
@@ -191,6 +219,34 @@ __device__ __forceinline__ void request_carries(const DevState &d, uint32_t r, i
         if (s < ns) d.seg_carry[s0 + s] = carry + inc - t;
         carry += shfl_u64(inc, 31);
     }
+}
+
+// The two ring positions of request r (after request_carries): P^1_{K-1}
+// from its local prefix value plus carry, P^2_{K-1} as the sum of the f2
+// segment partials (f2 only runs over blocks < K).  Whole warp; all lanes
+// return the same values.
+__device__ __forceinline__ void route_positions(const DevState &d, uint32_t r, int lane, uint64_t &pos1,
+                                                uint64_t &pos2) {
+    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
+    const uint32_t K = min(d.Kroute, nblk);
+    const uint32_t last = (K - 1) / kSegBlocks;   // segments holding blocks < K: 0..last
+    const uint64_t P1 = d.plocal[d.r_blkoff[r] + K - 1] + d.seg_carry[s0 + last];
+    uint64_t p2 = 0;
+    for (uint32_t j = lane; j <= last; j += 32) p2 += d.seg_total2[s0 + j];
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) p2 += shfl_xor_u64(p2, o);
+    pos1 = fmix64(P1 ^ d.Sr1);
+    pos2 = fmix64(p2 ^ d.Sr2);
+}
+
+// Grid of a grid-stride kernel: every SM filled to the kernel's occupancy.
+template <typename K>
+inline int full_grid(K kernel, int block) {
+    int dev = 0, sms = 0, per = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kernel, block, 0);
+    return sms * (per > 0 ? per : 1);
 }
 
 // ---------------------------------------------------------------------------

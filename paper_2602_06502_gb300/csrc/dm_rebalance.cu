@@ -82,7 +82,7 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
     __shared__ uint32_t s_w[33];
     __shared__ uint64_t s_u[33];
     __shared__ uint64_t s_sumW;
-    __shared__ uint32_t s_nhot, s_ncand, s_cnt;
+    __shared__ uint32_t s_nhot, s_cnt;
     if (has_err(d.err)) return;
     uint64_t *W = reinterpret_cast<uint64_t *>(smem);
     uint32_t *hotl = reinterpret_cast<uint32_t *>(W + d.M);

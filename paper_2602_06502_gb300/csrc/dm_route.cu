@@ -46,44 +46,70 @@ __device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uin
     lb2 = (uint32_t)(i2 + 1 == (int64_t)d.R ? 0 : i2 + 1);
 }
 
-// One warp per request: carries, candidates, hit lengths.
-__global__ void __launch_bounds__(128) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
+// One CTA of kProbeWarps warps per request.  Warp 0 computes the segment
+// carries, the two ring positions and candidates; then every round probes
+// 32 * kProbeWarps consecutive blocks on each candidate still running, and
+// the smallest missing block over the warps ends that candidate's run.
+constexpr int kProbeWarps = 8;
+
+__global__ void __launch_bounds__(kProbeWarps * 32) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
+    __shared__ uint32_t s_c[2];
+    __shared__ uint32_t s_miss[2][kProbeWarps];
     if (has_err(d.err)) return;
-    const int lane = threadIdx.x & 31;
-    const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (r >= n) return;
-    request_carries(d, r, lane);
-    __syncwarp();
-
-    uint32_t lb1, lb2;
-    ring_search2(d, d.r_pos[2 * r], d.r_pos[2 * r + 1], lane, lb1, lb2);
-    const uint32_t c1 = d.ring[0].owner[lb1];
-    const uint32_t raw2 = d.ring[1].owner[lb2];
-    const uint32_t c2 = raw2 != c1 ? raw2 : d.next_live[c1];
-
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const uint32_t r = blockIdx.x;
+    if (wid == 0) {
+        request_carries(d, r, lane);
+        __syncwarp();
+        uint64_t p1, p2;
+        route_positions(d, r, lane, p1, p2);
+        uint32_t lb1, lb2;
+        ring_search2(d, p1, p2, lane, lb1, lb2);
+        const uint32_t c1 = d.ring[0].owner[lb1];
+        const uint32_t raw2 = d.ring[1].owner[lb2];
+        if (lane == 0) {
+            s_c[0] = c1;
+            s_c[1] = raw2 != c1 ? raw2 : d.next_live[c1];
+        }
+    }
+    __syncthreads();
+    const uint32_t c1 = s_c[0], c2 = s_c[1];
     const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
     const uint64_t bo = d.r_blkoff[r];
     const Slot *t1 = d.table[c1];
     const Slot *t2 = d.table[c2];
+    const uint64_t f1 = d.log_front[c1], f2 = d.log_front[c2];   // resident: record at or after the front
     const uint64_t mask = d.S - 1;
+    constexpr uint32_t kRound = 32 * kProbeWarps;
     bool done1 = false, done2 = false;
     uint32_t h1 = 0, h2 = 0;
-    for (uint32_t it = 0; !(done1 && done2); ++it) {
-        const uint32_t b = it * 32 + lane;
+    for (uint32_t base = 0; !(done1 && done2); base += kRound) {
+        const uint32_t b = base + threadIdx.x;
         const bool inb = b < nblk;
         bool res1 = false, res2 = false;
         if (inb) {
             const uint64_t key = cache_key(d.plocal[bo + b] + d.seg_carry[s0 + b / kSegBlocks], d.Sc);
-            uint64_t st;
-            if (!done1) res1 = table_find(t1, mask, key, &st, d.err) >= 0 && st != 0;
-            if (!done2) res2 = table_find(t2, mask, key, &st, d.err) >= 0 && st != 0;
+            if (!done1) res1 = table_pos1(t1, mask, key, d.err) > f1;
+            if (!done2) res2 = table_pos1(t2, mask, key, d.err) > f2;
         }
         const uint32_t m1 = __ballot_sync(0xffffffffu, !res1);
         const uint32_t m2 = __ballot_sync(0xffffffffu, !res2);
-        if (!done1 && m1) { h1 = it * 32 + __ffs(m1) - 1; done1 = true; }
-        if (!done2 && m2) { h2 = it * 32 + __ffs(m2) - 1; done2 = true; }
+        if (lane == 0) {
+            s_miss[0][wid] = m1 ? wid * 32 + __ffs(m1) - 1 : kRound;
+            s_miss[1][wid] = m2 ? wid * 32 + __ffs(m2) - 1 : kRound;
+        }
+        __syncthreads();
+        uint32_t m1w = kRound, m2w = kRound;
+#pragma unroll
+        for (int w = 0; w < kProbeWarps; ++w) {
+            m1w = min(m1w, s_miss[0][w]);
+            m2w = min(m2w, s_miss[1][w]);
+        }
+        if (!done1 && m1w < kRound) { h1 = base + m1w; done1 = true; }
+        if (!done2 && m2w < kRound) { h2 = base + m2w; done2 = true; }
+        __syncthreads();
     }
-    if (lane == 0) {
+    if (threadIdx.x == 0) {
         const uint32_t hit1 = h1 * d.B, hit2 = h2 * d.B;
         d.r_c1[r] = c1;
         d.r_c2[r] = c2;
@@ -99,8 +125,7 @@ __global__ void __launch_bounds__(128) k_route_probe(DevState d, dm_route_out o,
 cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
                                cudaStream_t st) {
     if (b.n == 0) return cudaSuccess;
-    const uint32_t warps = 4;
-    k_route_probe<<<(b.n + warps - 1) / warps, warps * 32, 0, st>>>(d, o, b.n);
+    k_route_probe<<<b.n, kProbeWarps * 32, 0, st>>>(d, o, b.n);
     return cudaGetLastError();
 }
 

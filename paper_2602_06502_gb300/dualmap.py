@@ -35,7 +35,7 @@ class dm_config(C.Structure):
         ("max_batch_tokens", C.c_uint64),
         ("max_touch_per_instance", C.c_uint64),
         ("max_queue", C.c_uint32),
-        ("reserved0", C.c_uint32),
+        ("index_slots_log2", C.c_uint32),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]

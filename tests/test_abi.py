@@ -55,12 +55,14 @@ def test_create_rejects_bad_config_without_touching_gpu(built):
     """Synchronous argument checks run before any CUDA call."""
     D = built
     bad = D.dm_config(17, 16, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)   # B = 17
+    bad4 = D.dm_config(16, 16, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 41, 1, None)  # index > 2^40
     h = C.c_void_p()
     assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
     bad2 = D.dm_config(16, 0, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)   # K_route = 0
     assert D.lib().dm_create(C.byref(bad2), C.byref(h)) == D.DM_ERR_INVALID_ARG
     bad3 = D.dm_config(16, 16, 8, 1, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)  # one instance
     assert D.lib().dm_create(C.byref(bad3), C.byref(h)) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_create(C.byref(bad4), C.byref(h)) == D.DM_ERR_INVALID_ARG
     assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
 
 

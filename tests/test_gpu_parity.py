@@ -329,6 +329,6 @@ def test_longctx_full_size_batches():
     tr = Trace(workload("longctx"))
     kw = longctx_handle_kwargs(tr.cfg)
     p = Pair(tr.cfg, max_instances=kw["max_instances"], max_batch_tokens=kw["max_batch_tokens"],
-             max_touch=kw["max_touch_per_instance"])
+             max_touch=kw["max_touch_per_instance"], index_slots_log2=kw["index_slots_log2"])
     run_trace(p, tr, batches=2, check_state_end=False)
     p.check_state(ids=range(0, 128, 9))
