@@ -215,6 +215,34 @@ DM_API dm_status dm_commit_cache(dm_handle *h);
 DM_API dm_status dm_hash_prompts(dm_handle *h, const dm_batch *batch, uint64_t *keys_dev,
                           uint64_t *key_off_dev, uint64_t *pos_dev);
 
+/* Limits of dm_hash_prompts_noalloc: requests per call, and full blocks per
+ * call (total_tokens / block_tokens).  Its fixed scratch is about 2.2 MB. */
+#define DM_NOALLOC_MAX_REQUESTS 4096u
+#define DM_NOALLOC_MAX_BLOCKS 4194304ull
+
+/* dm_hash_prompts without any device allocation, and without a handle: the
+ * same block keys, key offsets and ring positions as dm_hash_prompts on a
+ * handle created with this block_tokens, route_prefix_blocks and seed.  The
+ * paper has no counterpart; it exists for callers that cannot allocate
+ * device memory at the point they hash, for example a serving process whose
+ * device memory is entirely owned by another allocator, or code on a path
+ * where cudaMalloc's implicit synchronisation is not acceptable.
+ * Working memory is one fixed array of about 2.2 MB inside the library, which
+ * every GPU that loads the library keeps until the process exits; keys_dev
+ * (which must hold sum(n_blk) entries) doubles as working space.
+ * Returns DM_ERR_CAPACITY without doing anything when n exceeds
+ * DM_NOALLOC_MAX_REQUESTS or total_tokens / block_tokens exceeds
+ * DM_NOALLOC_MAX_BLOCKS; device-side checks (prompt lengths and offsets, the
+ * exact block count) are reported by the return value, because the call
+ * synchronises `stream` (a cudaStream_t, NULL = legacy default stream) before
+ * returning.  The first call on each device looks up the array's device
+ * address and must come before any stream capture on that device.  Every call
+ * uses the same array: calls whose work overlaps on the GPU (other host
+ * threads, other streams) race and produce garbage. */
+DM_API dm_status dm_hash_prompts_noalloc(uint32_t block_tokens, uint32_t route_prefix_blocks, uint64_t seed,
+                                         const dm_batch *batch, uint64_t *keys_dev, uint64_t *key_off_dev,
+                                         uint64_t *pos_dev, void *stream);
+
 /* Raw ring owners (before the distinct fix) of n positions: pos_dev holds
  * (pos1, pos2) pairs as written by dm_hash_prompts; owner1_dev/owner2_dev
  * receive the successor's owner on ring 1 / ring 2.  Asynchronous. */

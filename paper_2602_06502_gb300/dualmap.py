@@ -81,6 +81,8 @@ SIGNATURES = {
     "dm_rebalance": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]),
     "dm_commit_cache": (C.c_int, [C.c_void_p]),
     "dm_hash_prompts": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.c_void_p, C.c_void_p, C.c_void_p]),
+    "dm_hash_prompts_noalloc": (C.c_int, [C.c_uint32, C.c_uint32, C.c_uint64, C.POINTER(dm_batch), C.c_void_p,
+                                          C.c_void_p, C.c_void_p, C.c_void_p]),
     "dm_ring_lookup": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p]),
     "dm_get_loads": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32]),
     "dm_export_cache": (C.c_int, [C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p, C.c_uint64,
@@ -177,6 +179,12 @@ def dm_commit_cache(h):
 
 def dm_hash_prompts(h, batch, keys_dev, key_off_dev, pos_dev):
     return lib().dm_hash_prompts(h, C.byref(batch), _ptr(keys_dev), _ptr(key_off_dev), _ptr(pos_dev))
+
+
+def dm_hash_prompts_noalloc(block_tokens, route_prefix_blocks, seed, batch, keys_dev, key_off_dev, pos_dev,
+                            stream=None):
+    return lib().dm_hash_prompts_noalloc(block_tokens, route_prefix_blocks, seed, C.byref(batch), _ptr(keys_dev),
+                                         _ptr(key_off_dev), _ptr(pos_dev), stream)
 
 
 def dm_ring_lookup(h, pos_dev, n, owner1_dev, owner2_dev):
