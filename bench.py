@@ -258,14 +258,52 @@ def main():
         tb = tr.batch_time(b) + cyc * span
         if host is None:
             g.route(tokens[t0:t0 + nt + 4], doff, dlen, e - s, nt, tb)
-        else:
+        else:   # pinned host buffers: upload, route and readback are enqueued; uploads overlap routing
             hb = D.make_batch(host["tok"][b], host["off"][b], host["len"][b], e - s, nt, tb)
-            rc = D.dm_route_batch_host(g.h, hb, host["out_struct"])
+            rc = D.dm_route_batch_host_async(g.h, hb, host["out_struct"][j % 2])
             assert rc == 0, rc
         if w.get("rebalance"):
             g.rebalance()
         g.commit()
         return e - s
+
+    # -- end-to-end through the host-buffer entry point ----------------------
+    # (first, while the process's host memory is fresh: pinned upload speed on
+    # this platform depends on where the pinned pages land)
+    e2e = None
+    if args.e2e_steps > 0:
+        Ke = max(1, min(args.e2e_steps, K))
+        g = make_sched()
+        need = sorted({j % used for j in range(W + Ke)})
+        host = {"tok": {}, "off": {}, "len": {}}
+        for b in need:
+            s, e, doff, dlen, nt, t0 = meta[b]
+            ht = torch.empty(nt + 4, dtype=torch.int32, pin_memory=True)
+            ht.copy_(tokens[t0:t0 + nt + 4])
+            host["tok"][b] = ht
+            host["off"][b] = doff.cpu().pin_memory()
+            host["len"][b] = dlen.cpu().pin_memory()
+        houts = [{name: torch.zeros(w["batch"], dtype=t, pin_memory=True) for name, t in OUT_FIELDS}
+                 for _ in range(2)]
+        host["out_struct"] = [D.make_out(*[ho[name] for name, _ in OUT_FIELDS]) for ho in houts]
+        for j in range(W):
+            step(g, j, host)
+        torch.cuda.synchronize()
+        h2d = d2h = 0
+        t0 = time.perf_counter()
+        ne = 0
+        for j in range(W, W + Ke):
+            n = step(g, j, host)
+            ne += n
+            b = j % used
+            h2d += 4 * (meta[b][4]) + 12 * n
+            d2h += 41 * n
+        assert g.last_error() == 0          # synchronises the handle's stream (all copies included)
+        torch.cuda.synchronize()
+        te = time.perf_counter() - t0
+        g.close()
+        e2e = {"value": world * ne / te, "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
+               "d2h_bytes_per_step": d2h // Ke, "steps": Ke}
 
     # -- device-resident run -------------------------------------------------
     g = make_sched()
@@ -312,46 +350,13 @@ def main():
     peak, peak_kind = peaks()
     achieved = bytes_per_launch / hash_avg_s / 1e9
     prompt_gbps = prompt_bytes / ((hash_ms + probe_ms) / 1e3) / 1e9
-    # route: setup, drain, hash, probe, choice; commit: count, maintain, prep, touch, evict
-    launches_per_step = 5 + 5 + (1 if w.get("rebalance") else 0)
+    # route: setup, segmap, drain, hash, probe, choice (6); commit: maint_plan, maint_a,
+    # compact_scan, maint_c, commit_prep, commit_touch, req_counts, evict_plan,
+    # evict_count, evict_cut, evict_clear, evict_walk (12); rebalance (1)
+    launches_per_step = 6 + 12 + (1 if w.get("rebalance") else 0)
     clocks = sampler.summary(wall0, wall1)
     g.close()
     del g
-
-    # -- end-to-end through the host-buffer entry point ----------------------
-    e2e = None
-    if args.e2e_steps > 0:
-        Ke = max(1, min(args.e2e_steps, K))
-        g = make_sched()
-        need = sorted({j % used for j in range(W + Ke)})
-        host = {"tok": {}, "off": {}, "len": {}}
-        for b in need:
-            s, e, doff, dlen, nt, t0 = meta[b]
-            ht = torch.empty(nt + 4, dtype=torch.int32, pin_memory=True)
-            ht.copy_(tokens[t0:t0 + nt + 4])
-            host["tok"][b] = ht
-            host["off"][b] = doff.cpu().pin_memory()
-            host["len"][b] = dlen.cpu().pin_memory()
-        hout = {name: torch.zeros(w["batch"], dtype=t, pin_memory=True) for name, t in OUT_FIELDS}
-        host["out_struct"] = D.make_out(*[hout[name] for name, _ in OUT_FIELDS])
-        for j in range(W):
-            step(g, j, host)
-        torch.cuda.synchronize()
-        h2d = d2h = 0
-        t0 = time.perf_counter()
-        ne = 0
-        for j in range(W, W + Ke):
-            n = step(g, j, host)
-            ne += n
-            b = j % used
-            h2d += 4 * (meta[b][4]) + 12 * n
-            d2h += 41 * n
-        torch.cuda.synchronize()
-        te = time.perf_counter() - t0
-        assert g.last_error() == 0
-        g.close()
-        e2e = {"value": world * ne / te, "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
-               "d2h_bytes_per_step": d2h // Ke, "steps": Ke}
 
     # -- CPU oracle baseline (rank 0, N=1 only) ------------------------------------
     cpu = None

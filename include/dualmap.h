@@ -189,6 +189,14 @@ DM_API dm_status dm_route_batch(dm_handle *h, const dm_batch *batch, const dm_ro
  * synchronises the stream before returning. */
 DM_API dm_status dm_route_batch_host(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
 
+/* Asynchronous dm_route_batch_host: returns once the work is enqueued.  The
+ * library alternates between two device staging buffers, uploading a batch
+ * on its own copy stream while the previous batch routes, so the caller's
+ * host input and output buffers must stay untouched until the handle's
+ * stream has been synchronised (dm_last_error does).  Use pinned host memory
+ * for the copies to overlap. */
+DM_API dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
+
 /* Hotspot-aware rebalancing (Sec. 3.3, Eq. "rebalance"; App. A.1.2), to be
  * called after dm_route_batch and before dm_commit_cache.  Hot instances
  * are visited in descending W; their queued, not-started requests are

@@ -42,10 +42,17 @@ struct dm_handle {
     std::vector<Rec *> logs, logs2;        // both log buffers
     std::vector<uint8_t *> stales, stales2;
     std::vector<void *> allocs;    // every cudaMalloc of the handle
-    // staging of dm_route_batch_host
-    uint32_t *h_tokens = nullptr, *h_lengths = nullptr;
-    uint64_t *h_offsets = nullptr;
-    dm_route_out h_out{};
+    // staging of the host-buffer entry points: two buffers, so the upload of
+    // one batch (on copy_st) overlaps the routing of the previous one
+    struct HostStage {
+        uint32_t *tokens = nullptr, *lengths = nullptr;
+        uint64_t *offsets = nullptr;
+        dm_route_out out{};
+        cudaEvent_t copied = nullptr, consumed = nullptr;
+        bool used = false;
+    } hs[2];
+    int hs_next = 0;
+    cudaStream_t copy_st = nullptr;
     bool profiling = false;
     std::vector<StageEvent> events;
     std::vector<cudaEvent_t> ev_pool;
@@ -166,6 +173,14 @@ const char *dm_status_string(dm_status s) {
 void dm_destroy(dm_handle *h) {
     if (!h) return;
     cudaStreamSynchronize(h->st);
+    if (h->copy_st) {
+        cudaStreamSynchronize(h->copy_st);
+        cudaStreamDestroy(h->copy_st);
+    }
+    for (auto &x : h->hs) {
+        if (x.copied) cudaEventDestroy(x.copied);
+        if (x.consumed) cudaEventDestroy(x.consumed);
+    }
     for (auto &ev : h->events) { cudaEventDestroy(ev.a); cudaEventDestroy(ev.b); }
     for (auto e : h->ev_pool) cudaEventDestroy(e);
     for (void *p : h->allocs) cudaFree(p);
@@ -512,53 +527,69 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
     return DM_OK;
 }
 
-dm_status dm_route_batch_host(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
     dm_status s = check_batch(h, b, o);
     if (s) return s;
     if (!o) return DM_ERR_INVALID_ARG;
     cudaError_t e = cudaSuccess;
     const uint32_t mb = h->d.max_batch;
-    if (!h->h_tokens) {
+    if (!h->copy_st) {
         auto A = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
-        A(dalloc(h, &h->h_tokens, h->cfg.max_batch_tokens));
-        A(dalloc(h, &h->h_offsets, mb));
-        A(dalloc(h, &h->h_lengths, mb));
-        A(dalloc(h, &h->h_out.cand1, mb));
-        A(dalloc(h, &h->h_out.cand2, mb));
-        A(dalloc(h, &h->h_out.hit1, mb));
-        A(dalloc(h, &h->h_out.hit2, mb));
-        A(dalloc(h, &h->h_out.ttft1, mb));
-        A(dalloc(h, &h->h_out.ttft2, mb));
-        A(dalloc(h, &h->h_out.chosen, mb));
-        A(dalloc(h, &h->h_out.switched, mb));
-        if (e != cudaSuccess) { cudaGetLastError(); h->h_tokens = nullptr; return DM_ERR_OOM; }
+        for (auto &x : h->hs) {
+            A(dalloc(h, &x.tokens, h->cfg.max_batch_tokens + 4));
+            A(dalloc(h, &x.offsets, mb));
+            A(dalloc(h, &x.lengths, mb));
+            A(dalloc(h, &x.out.cand1, mb));
+            A(dalloc(h, &x.out.cand2, mb));
+            A(dalloc(h, &x.out.hit1, mb));
+            A(dalloc(h, &x.out.hit2, mb));
+            A(dalloc(h, &x.out.ttft1, mb));
+            A(dalloc(h, &x.out.ttft2, mb));
+            A(dalloc(h, &x.out.chosen, mb));
+            A(dalloc(h, &x.out.switched, mb));
+            A(cudaEventCreateWithFlags(&x.copied, cudaEventDisableTiming));
+            A(cudaEventCreateWithFlags(&x.consumed, cudaEventDisableTiming));
+        }
+        A(cudaStreamCreateWithFlags(&h->copy_st, cudaStreamNonBlocking));
+        if (e != cudaSuccess) { cudaGetLastError(); h->copy_st = nullptr; return DM_ERR_OOM; }
     }
+    auto &x = h->hs[h->hs_next];
+    h->hs_next ^= 1;
     const uint32_t n = b->n;
     if (n) {
-        e = cudaMemcpyAsync(h->h_tokens, b->tokens, b->total_tokens * 4, cudaMemcpyHostToDevice, h->st);
-        if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_offsets, b->offsets, n * 8ull, cudaMemcpyHostToDevice, h->st);
-        if (e == cudaSuccess) e = cudaMemcpyAsync(h->h_lengths, b->lengths, n * 4ull, cudaMemcpyHostToDevice, h->st);
+        // the upload waits until kernels reading this buffer's last batch are done
+        if (x.used) e = cudaStreamWaitEvent(h->copy_st, x.consumed, 0);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(x.tokens, b->tokens, b->total_tokens * 4, cudaMemcpyHostToDevice, h->copy_st);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(x.offsets, b->offsets, n * 8ull, cudaMemcpyHostToDevice, h->copy_st);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(x.lengths, b->lengths, n * 4ull, cudaMemcpyHostToDevice, h->copy_st);
+        if (e == cudaSuccess) e = cudaEventRecord(x.copied, h->copy_st);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(h->st, x.copied, 0);
         if (e != cudaSuccess) return map_cuda(h, e);
     }
     dm_batch db = *b;
-    db.tokens = h->h_tokens;
-    db.offsets = h->h_offsets;
-    db.lengths = h->h_lengths;
-    s = dm_route_batch(h, &db, &h->h_out);
+    db.tokens = x.tokens;
+    db.offsets = x.offsets;
+    db.lengths = x.lengths;
+    s = dm_route_batch(h, &db, &x.out);
     if (s) return s;
     if (n) {
-        const dm_route_out &x = h->h_out;
+        e = cudaEventRecord(x.consumed, h->st);
+        x.used = true;
         struct { void *dst; const void *src; size_t bytes; } cp[] = {
-            {o->cand1, x.cand1, n * 4ull}, {o->cand2, x.cand2, n * 4ull}, {o->hit1, x.hit1, n * 4ull},
-            {o->hit2, x.hit2, n * 4ull}, {o->ttft1, x.ttft1, n * 8ull}, {o->ttft2, x.ttft2, n * 8ull},
-            {o->chosen, x.chosen, n * 4ull}, {o->switched, x.switched, n * 1ull}};
-        for (auto &c : cp) {
-            e = cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyDeviceToHost, h->st);
-            if (e != cudaSuccess) return map_cuda(h, e);
-        }
+            {o->cand1, x.out.cand1, n * 4ull}, {o->cand2, x.out.cand2, n * 4ull}, {o->hit1, x.out.hit1, n * 4ull},
+            {o->hit2, x.out.hit2, n * 4ull}, {o->ttft1, x.out.ttft1, n * 8ull}, {o->ttft2, x.out.ttft2, n * 8ull},
+            {o->chosen, x.out.chosen, n * 4ull}, {o->switched, x.out.switched, n * 1ull}};
+        for (auto &c : cp)
+            if (e == cudaSuccess) e = cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyDeviceToHost, h->st);
     }
-    e = cudaStreamSynchronize(h->st);
     return map_cuda(h, e);
+}
+
+dm_status dm_route_batch_host(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    dm_status s = dm_route_batch_host_async(h, b, o);
+    if (s) return s;
+    return map_cuda(h, cudaStreamSynchronize(h->st));
 }
 
 dm_status dm_rebalance(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev) {

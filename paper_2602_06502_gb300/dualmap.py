@@ -78,6 +78,7 @@ SIGNATURES = {
     "dm_remove_instance": (C.c_int, [C.c_void_p, C.c_uint32]),
     "dm_route_batch": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
     "dm_route_batch_host": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
+    "dm_route_batch_host_async": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
     "dm_rebalance": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]),
     "dm_commit_cache": (C.c_int, [C.c_void_p]),
     "dm_hash_prompts": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -167,6 +168,10 @@ def dm_route_batch(h, batch, out):
 
 def dm_route_batch_host(h, batch, out):
     return lib().dm_route_batch_host(h, C.byref(batch), C.byref(out))
+
+
+def dm_route_batch_host_async(h, batch, out):
+    return lib().dm_route_batch_host_async(h, C.byref(batch), C.byref(out))
 
 
 def dm_rebalance(h, out_dev, cap, n_out_dev):

@@ -332,3 +332,39 @@ def test_longctx_full_size_batches():
              max_touch=kw["max_touch_per_instance"], index_slots_log2=kw["index_slots_log2"])
     run_trace(p, tr, batches=2, check_state_end=False)
     p.check_state(ids=range(0, 128, 9))
+
+
+def test_host_async_pipeline_matches_oracle():
+    """Asynchronous host-buffer routing: several batches enqueued back to back
+    (uploads overlapping routing on the two staging buffers), one wait, every
+    batch's results equal to the oracle's."""
+    from paper_2602_06502_gb300 import dualmap as D
+    from paper_2602_06502_gb300.scheduler import OUT_FIELDS
+    import torch
+    tr = Trace(workload("tiny", n_requests=1280, batch=256))
+    p = Pair(tr.cfg)
+    for i in range(tr.cfg["n_instances"]):
+        p.add(i)
+    npdt = {"int32": np.uint32, "int64": np.uint64, "uint8": np.uint8}
+    keep, wants = [], []
+    for k in range(len(tr.batches)):
+        s, e, off, lens, ntok = tr.batch_layout(k)
+        tok = tr.batch_tokens(k)
+        rc, want = p.ora.route_batch(tok, off, lens, tr.batch_time(k))
+        assert rc == 0 and p.ora.commit() == 0
+        n = e - s
+        pin = {"tok": torch.from_numpy(tok.view(np.int32)).pin_memory(),
+               "off": torch.from_numpy(off.view(np.int64)).pin_memory(),
+               "len": torch.from_numpy(lens.view(np.int32)).pin_memory()}
+        host = {name: torch.zeros(n, dtype=t).pin_memory() for name, t in OUT_FIELDS}
+        bt = D.make_batch(pin["tok"], pin["off"], pin["len"], n, ntok, tr.batch_time(k))
+        assert D.dm_route_batch_host_async(p.gpu.h, bt, D.make_out(*[host[name] for name, _ in OUT_FIELDS])) == 0
+        p.gpu.commit()
+        keep.append((pin, host))
+        wants.append(want)
+    assert p.gpu.last_error() == 0
+    for (pin, host), want in zip(keep, wants):
+        for name, t in OUT_FIELDS:
+            got = host[name].numpy().view(npdt[str(t).split(".")[1]])
+            assert np.array_equal(got, want[name]), name
+    p.check_state()
