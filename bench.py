@@ -45,8 +45,11 @@ def handle_kwargs(w, max_id):
     if w["name"] == "longctx":
         return longctx_handle_kwargs(w)
     mb = w["batch"] * (w.get("len_hi") or w.get("max_prompt") or (w.get("prefix_hi", 0) + w.get("uniq_hi", 0)))
+    # blocks one commit may touch on one instance: the busiest pair of a batch
+    # takes well under half of it in every workload here
+    touch = min(mb // w["block_tokens"], 1 << 21 if w["n_instances"] <= 64 else 1 << 19)
     return dict(max_instances=max_id + 9, max_batch=w["batch"], max_batch_tokens=mb + 4 * w["batch"],
-                max_touch_per_instance=min(mb // w["block_tokens"], 1 << 21))
+                max_touch_per_instance=touch)
 
 
 def peaks():
@@ -124,6 +127,24 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(inside), "window": window}
 
 
+def max_over_ranks(x, device="cpu"):
+    """Largest value of x over the ranks of the default process group (x
+    itself when not distributed): step time is the slowest replica's."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(requests_per_rank, ms_max, world):
+    """Whole-job routed requests/s: every replica routes the same number of
+    requests, the job takes as long as its slowest replica."""
+    return world * requests_per_rank / (ms_max / 1e3)
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -194,7 +215,7 @@ def main():
     ap.add_argument("--workload", default="longctx")
     ap.add_argument("--e2e-steps", type=int, default=24)
     ap.add_argument("--cpu-batches", type=int, default=6)
-    ap.add_argument("--ref-max-batches", type=int, default=24)
+    ap.add_argument("--ref-max-batches", type=int, default=48)
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE",
                     help="override a workload field (small cases for profiling)")
@@ -302,7 +323,8 @@ def main():
         torch.cuda.synchronize()
         te = time.perf_counter() - t0
         g.close()
-        e2e = {"value": world * ne / te, "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
+        te = max_over_ranks(te * 1e3, device=dev) / 1e3
+        e2e = {"value": job_throughput(ne, te * 1e3, world), "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
                "d2h_bytes_per_step": d2h // Ke, "steps": Ke}
 
     # -- device-resident run -------------------------------------------------
@@ -338,11 +360,8 @@ def main():
     D.dm_set_profiling(g.h, False)
     err = g.last_error()
     assert err == 0, D.status_string(err)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * nreq / (ms / 1e3)
+    ms = max_over_ranks(ms, device=dev)
+    value = job_throughput(nreq, ms, world)
     hash_ms, hash_calls = st["hash"]
     probe_ms, _ = st["probe"]
     hash_avg_s = hash_ms / 1e3 / max(hash_calls, 1)
