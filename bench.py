@@ -52,6 +52,14 @@ def handle_kwargs(w, max_id):
                 max_touch_per_instance=touch)
 
 
+def describe_lengths(w):
+    if "len_lo" in w:
+        return f"{w['len_lo']}-{w['len_hi']}"
+    if w["kind"] == "template":
+        return f"{w['prefix_lo'] + w['uniq_lo']}-{w['prefix_hi'] + w['uniq_hi']}"
+    return f"{w['chunk_lo']}-{w['max_prompt']} (multi-turn)"
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -398,7 +406,7 @@ def main():
             "dtype": "u32 tokens / u64 integer arithmetic", "data": "synthetic",
             "prompt_GBps": prompt_gbps,
             "config": {"workload": f"{w['name']}: {w['n_instances']} instances x {w['vnodes']} vnodes, "
-                                   f"batches of {w['batch']} prompts of {w['len_lo']}-{w['len_hi']} tokens "
+                                   f"batches of {w['batch']} prompts of {describe_lengths(w)} tokens "
                                    f"(~{bytes_per_launch / 1e6:.0f} MB per batch)",
                        "global_batch": w["batch"], "parallelism": f"replicas x{world}",
                        "l2": "inputs larger than L2 (each batch > 129 MB, distinct per step)",

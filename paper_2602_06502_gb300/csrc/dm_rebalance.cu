@@ -3,7 +3,8 @@
 //
 // Hotspots (hot_den * N * W_i > hot_num * sum W over live instances) are
 // visited in descending W.  For hotspot i the CTA gathers, in parallel, every
-// queued request that has not started and was not moved in this call, with
+// queued request that has not started, was not moved in this call and could
+// still pass the move test, with
 // TTFT_{r,i} = work queued up to and including r and TTFT_{r,j} = W_j +
 // cost * (L - h_{r,j}) for its other candidate j; sorts them by (benefit
 // desc, sequence asc); then one thread walks the list, moving r to j while i
@@ -75,30 +76,85 @@ __device__ __forceinline__ uint64_t block_excl_u64(uint64_t v, uint64_t *s, uint
     return r;
 }
 
-// Single CTA of 1024 threads; dynamic smem: W[M] u64, hot list u32[M].
+constexpr uint32_t kRbStage = 1024;   // candidates staged per sequential pass
+
+// Sequential-pass staging of one chunk of sorted candidates.
+struct RbChunk {
+    uint64_t seq[kRbStage], work[kRbStage], ttft_i[kRbStage], new_work[kRbStage];
+    uint32_t pos[kRbStage], L[kRbStage], c1[kRbStage], c2[kRbStage], h1[kRbStage], h2[kRbStage];
+    uint32_t j[kRbStage];
+    // moves decided in this chunk: candidate index and target slot
+    uint32_t mv_k[kRbStage], mv_slot[kRbStage];
+};
+
+// Dynamic shared memory layout: per instance W (u64), queue tails (u32),
+// hot list (u32), state (u8, padded); then the chunk staging; then the sort
+// arrays (key u64, seq u64, ttft u64, pos u32) of up to `sort_cap` candidates.
+__host__ __device__ inline size_t rb_inst_bytes(uint32_t M) { return (size_t(M) * 17 + 15) / 16 * 16; }
+__host__ __device__ inline size_t rb_sort_bytes(uint32_t cap) { return size_t(cap) * 28; }
+
+// Bitonic sort of P (power of two) candidates by (key asc, seq asc) with
+// their payloads; the arrays are shared or global memory of this CTA.
+__device__ void bitonic_sort(uint64_t *key, uint64_t *seq, uint64_t *tt, uint32_t *pos, uint32_t P) {
+    for (uint32_t k = 2; k <= P; k <<= 1) {
+        for (uint32_t jj = k >> 1; jj > 0; jj >>= 1) {
+            for (uint32_t x = threadIdx.x; x < P; x += blockDim.x) {
+                const uint32_t y = x ^ jj;
+                if (y > x) {
+                    const bool asc = (x & k) == 0;
+                    const uint64_t kx = key[x], ky = key[y];
+                    const uint64_t sx = seq[x], sy = seq[y];
+                    const bool gt = kx > ky || (kx == ky && sx > sy);
+                    if (gt == asc) {
+                        key[x] = ky; key[y] = kx;
+                        seq[x] = sy; seq[y] = sx;
+                        const uint64_t t = tt[x]; tt[x] = tt[y]; tt[y] = t;
+                        const uint32_t q = pos[x]; pos[x] = pos[y]; pos[y] = q;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+}
+
+// Single CTA of 1024 threads.
 __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint64_t seq0, uint32_t call,
-                                                    dm_migration *out, uint32_t cap, uint32_t *n_out) {
+                                                    dm_migration *out, uint32_t cap, uint32_t *n_out,
+                                                    uint32_t sort_cap) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_w[33];
     __shared__ uint64_t s_u[33];
     __shared__ uint64_t s_sumW;
-    __shared__ uint32_t s_nhot, s_cnt;
+    __shared__ uint32_t s_nhot, s_cnt, s_nmv, s_stop;
     if (has_err(d.err)) return;
+    const uint32_t M = d.M;
     uint64_t *W = reinterpret_cast<uint64_t *>(smem);
-    uint32_t *hotl = reinterpret_cast<uint32_t *>(W + d.M);
+    uint32_t *tails = reinterpret_cast<uint32_t *>(W + M);
+    uint32_t *hotl = tails + M;
+    uint8_t *st = reinterpret_cast<uint8_t *>(hotl + M);
+    RbChunk &Ch = *reinterpret_cast<RbChunk *>(smem + rb_inst_bytes(M));
+    unsigned char *sort_base = smem + rb_inst_bytes(M) + sizeof(RbChunk);
+    uint64_t *sk = reinterpret_cast<uint64_t *>(sort_base);
+    uint64_t *ss = sk + sort_cap;
+    uint64_t *stt = ss + sort_cap;
+    uint32_t *sp = reinterpret_cast<uint32_t *>(stt + sort_cap);
+
     uint64_t myW = 0;
     uint32_t myN = 0;
-    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
+    for (uint32_t i = threadIdx.x; i < M; i += blockDim.x) {
         W[i] = d.W[i];
-        if (d.inst_state[i] == 1) { myW += W[i]; ++myN; }
+        tails[i] = d.q_tail[i];
+        st[i] = d.inst_state[i];
+        if (st[i] == 1) { myW += W[i]; ++myN; }
     }
     const uint64_t sumW0 = block_sum_u64(myW, s_u);
     const uint32_t N = (uint32_t)block_sum_u64(myN, s_u);
     // hot list (ids in ascending order), then ranks by (W desc, id asc)
     uint32_t nhot = 0;
-    for (uint32_t base = 0; base < d.M; base += blockDim.x) {
+    for (uint32_t base = 0; base < M; base += blockDim.x) {
         const uint32_t i = base + threadIdx.x;
-        const bool h = i < d.M && d.inst_state[i] == 1 && hot(W[i], sumW0, N, d.hot_num, d.hot_den);
+        const bool h = i < M && st[i] == 1 && hot(W[i], sumW0, N, d.hot_num, d.hot_den);
         uint32_t tot;
         const uint32_t rk = rank_in_block(h, s_w, tot);
         if (h) d.rb_pos[nhot + rk] = i;   // scratch: unsorted hot ids
@@ -119,11 +175,12 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
     const uint64_t cost = d.cost;
     for (uint32_t hi = 0; hi < s_nhot; ++hi) {
         const uint32_t i = hotl[hi];
-        const QEntry *qi = d.q + uint64_t(i) * d.Q;
-        const uint32_t head = d.q_head[i], tail = d.q_tail[i];
+        QEntry *qi = d.q + uint64_t(i) * d.Q;
+        const uint32_t head = d.q_head[i], tail = tails[i];
+        // 1) gather the candidates of hotspot i (parallel over its queue)
         uint64_t ahead = 0;
         uint32_t ncand = 0;
-        for (uint32_t p0 = head; p0 != tail && (uint32_t)(p0 - head) < (uint32_t)(tail - head);) {
+        for (uint32_t p0 = head; p0 != tail;) {
             const uint32_t p = p0 + threadIdx.x;
             const bool valid = (uint32_t)(p - head) < (uint32_t)(tail - head);
             QEntry e{};
@@ -131,7 +188,7 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
             uint64_t tot_rem;
             const uint64_t ex = block_excl_u64(valid ? e.remaining : 0, s_u, &tot_rem);
             const uint64_t ttft_i = ahead + ex + (valid ? e.remaining : 0);
-            const bool elig = valid && e.moved != kTomb && e.moved != call && e.remaining == e.work;
+            bool elig = valid && e.moved != kTomb && e.moved != call && e.remaining == e.work;
             uint64_t key = 0;
             if (elig) {
                 const uint32_t j = e.c1 == i ? e.c2 : e.c1;
@@ -139,6 +196,11 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
                 const uint64_t ttft_j = W[j] + cost * (e.L - hj);
                 const int64_t B = (int64_t)(ttft_i - ttft_j);
                 key = ~(uint64_t(B) ^ 0x8000000000000000ull);   // ascending = benefit descending
+                // While hotspot i is walked, W_j only grows (earlier hotspots
+                // are done; i's moves add to their targets), so a request
+                // that fails the move test now fails it at its turn too.
+                // Dropping it changes no move and no stop decision.
+                if (!(B > 0 && ttft_j < d.slo)) elig = false;
             }
             uint32_t tot;
             const uint32_t rk = rank_in_block(elig, s_w, tot);
@@ -153,90 +215,138 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
             }
             ncand += tot;
             ahead += tot_rem;
-            const uint32_t step = min((uint32_t)blockDim.x, (uint32_t)(tail - p0));
-            p0 += step;
+            p0 += min((uint32_t)blockDim.x, (uint32_t)(tail - p0));
         }
         if (ncand > d.rb_cap) {
             if (threadIdx.x == 0) set_err(d.err, DM_ERR_CAPACITY);
             return;
         }
-        // bitonic sort of the candidates by (key asc, seq asc), padded to a power of two
+        if (ncand == 0) continue;
+        // 2) sort by (benefit desc, sequence asc), in shared memory when it fits
         uint32_t P = 1;
         while (P < ncand) P <<= 1;
-        for (uint32_t c = ncand + threadIdx.x; c < P; c += blockDim.x) {
-            d.rb_key[c] = ~0ull;
-            d.rb_seq[c] = ~0ull;
+        if (P <= sort_cap) {
+            for (uint32_t c = threadIdx.x; c < P; c += blockDim.x) {
+                const bool v = c < ncand;
+                sk[c] = v ? d.rb_key[c] : ~0ull;
+                ss[c] = v ? d.rb_seq[c] : ~0ull;
+                stt[c] = v ? d.rb_ttft[c] : 0;
+                sp[c] = v ? d.rb_pos[c] : 0;
+            }
+            __syncthreads();
+            bitonic_sort(sk, ss, stt, sp, P);
+            for (uint32_t c = threadIdx.x; c < ncand; c += blockDim.x) {
+                d.rb_ttft[c] = stt[c];
+                d.rb_pos[c] = sp[c];
+            }
+        } else {
+            for (uint32_t c = ncand + threadIdx.x; c < P; c += blockDim.x) {
+                d.rb_key[c] = ~0ull;
+                d.rb_seq[c] = ~0ull;
+            }
+            __syncthreads();
+            bitonic_sort(d.rb_key, d.rb_seq, d.rb_ttft, d.rb_pos, P);
         }
         __syncthreads();
-        for (uint32_t k = 2; k <= P; k <<= 1) {
-            for (uint32_t jj = k >> 1; jj > 0; jj >>= 1) {
-                for (uint32_t x = threadIdx.x; x < P; x += blockDim.x) {
-                    const uint32_t y = x ^ jj;
-                    if (y > x) {
-                        const bool asc = (x & k) == 0;
-                        const uint64_t kx = d.rb_key[x], ky = d.rb_key[y];
-                        const uint64_t sx = d.rb_seq[x], sy = d.rb_seq[y];
-                        const bool gt = kx > ky || (kx == ky && sx > sy);
-                        if (gt == asc) {
-                            d.rb_key[x] = ky; d.rb_key[y] = kx;
-                            d.rb_seq[x] = sy; d.rb_seq[y] = sx;
-                            const uint64_t tx = d.rb_ttft[x];
-                            d.rb_ttft[x] = d.rb_ttft[y]; d.rb_ttft[y] = tx;
-                            const uint32_t px = d.rb_pos[x];
-                            d.rb_pos[x] = d.rb_pos[y]; d.rb_pos[y] = px;
-                        }
-                    }
-                }
-                __syncthreads();
-            }
-        }
-        if (threadIdx.x == 0) {
-            uint64_t sumW = s_sumW;
-            uint32_t cnt = s_cnt;
-            for (uint32_t c = 0; c < ncand; ++c) {
-                if (!hot(W[i], sumW, N, d.hot_num, d.hot_den)) break;
-                const uint32_t p = d.rb_pos[c];
-                QEntry *pe = d.q + uint64_t(i) * d.Q + (p & (d.Q - 1));
-                QEntry e = *pe;
+        // 3) walk the sorted candidates chunk by chunk: stage, decide (one
+        //    thread, shared memory only), apply the moves in parallel
+        if (threadIdx.x == 0) s_stop = 0;
+        __syncthreads();
+        for (uint32_t c0 = 0; c0 < ncand && !s_stop; c0 += kRbStage) {
+            const uint32_t m = min(kRbStage, ncand - c0);
+            for (uint32_t k = threadIdx.x; k < m; k += blockDim.x) {
+                const uint32_t p = d.rb_pos[c0 + k];
+                const QEntry e = qi[p & (d.Q - 1)];
                 const uint32_t j = e.c1 == i ? e.c2 : e.c1;
-                if (d.inst_state[j] != 1) continue;
                 const uint32_t hj = j == e.c1 ? e.h1 : e.h2;
-                const uint64_t new_work = cost * (e.L - hj);
-                const uint64_t ttft_j = W[j] + new_work;
-                if (!(d.rb_ttft[c] > ttft_j && ttft_j < d.slo)) continue;
-                const uint32_t slot = d.q_tail[j];
-                if (slot - d.q_head[j] >= d.Q) { set_err(d.err, DM_ERR_CAPACITY); break; }
-                pe->moved = kTomb;
-                pe->work = 0;
-                pe->remaining = 0;
-                W[i] -= e.work;
-                sumW -= e.work;
-                e.work = e.remaining = new_work;
+                Ch.seq[k] = e.seq;
+                Ch.work[k] = e.work;
+                Ch.ttft_i[k] = d.rb_ttft[c0 + k];
+                Ch.new_work[k] = cost * (e.L - hj);
+                Ch.pos[k] = p;
+                Ch.L[k] = e.L;
+                Ch.c1[k] = e.c1;
+                Ch.c2[k] = e.c2;
+                Ch.h1[k] = e.h1;
+                Ch.h2[k] = e.h2;
+                Ch.j[k] = j;
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                uint64_t sumW = s_sumW;
+                uint32_t nmv = 0, stop = 0;
+                for (uint32_t k = 0; k < m; ++k) {
+                    if (!hot(W[i], sumW, N, d.hot_num, d.hot_den)) { stop = 1; break; }
+                    const uint32_t j = Ch.j[k];
+                    if (st[j] != 1) continue;
+                    const uint64_t nw = Ch.new_work[k];
+                    const uint64_t ttft_j = W[j] + nw;
+                    if (!(Ch.ttft_i[k] > ttft_j && ttft_j < d.slo)) continue;
+                    const uint32_t slot = tails[j];
+                    if (slot - d.q_head[j] >= d.Q) { set_err(d.err, DM_ERR_CAPACITY); stop = 1; break; }
+                    tails[j] = slot + 1;
+                    W[i] -= Ch.work[k];
+                    sumW -= Ch.work[k];
+                    W[j] += nw;
+                    sumW += nw;
+                    Ch.mv_k[nmv] = k;
+                    Ch.mv_slot[nmv] = slot;
+                    ++nmv;
+                }
+                s_sumW = sumW;
+                s_nmv = nmv;
+                s_stop = stop;
+            }
+            __syncthreads();
+            const uint32_t cnt0 = s_cnt;
+            for (uint32_t t = threadIdx.x; t < s_nmv; t += blockDim.x) {
+                const uint32_t k = Ch.mv_k[t];
+                const uint32_t j = Ch.j[k];
+                QEntry *src = qi + (Ch.pos[k] & (d.Q - 1));
+                src->moved = kTomb;
+                src->work = 0;
+                src->remaining = 0;
+                QEntry e;
+                e.seq = Ch.seq[k];
+                e.work = e.remaining = Ch.new_work[k];
+                e.L = Ch.L[k];
+                e.c1 = Ch.c1[k];
+                e.c2 = Ch.c2[k];
+                e.h1 = Ch.h1[k];
+                e.h2 = Ch.h2[k];
                 e.moved = call;
-                d.q[uint64_t(j) * d.Q + (slot & (d.Q - 1))] = e;
-                d.q_tail[j] = slot + 1;
-                W[j] += new_work;
-                sumW += new_work;
+                d.q[uint64_t(j) * d.Q + (Ch.mv_slot[t] & (d.Q - 1))] = e;
                 if (e.seq >= seq0 && e.seq < seq0 + n) {
                     d.r_final[e.seq - seq0] = j;
                     d.info->final_dirty = 1;
                 }
-                if (cnt < cap) out[cnt] = dm_migration{e.seq, i, j};
-                ++cnt;
+                if (cnt0 + t < cap) out[cnt0 + t] = dm_migration{e.seq, i, j};
             }
-            s_sumW = sumW;
-            s_cnt = cnt;
+            __syncthreads();
+            if (threadIdx.x == 0) s_cnt = cnt0 + s_nmv;
+            __syncthreads();
         }
-        __syncthreads();
     }
     __syncthreads();
-    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) d.W[i] = W[i];
+    for (uint32_t i = threadIdx.x; i < M; i += blockDim.x) {
+        d.W[i] = W[i];
+        d.q_tail[i] = tails[i];
+    }
     if (threadIdx.x == 0) *n_out = s_cnt;
 }
 
 cudaError_t launch_rebalance(const DevState &d, uint32_t n, uint64_t seq0, uint32_t call,
                              dm_migration *out, uint32_t cap, uint32_t *n_out, cudaStream_t st) {
-    const size_t smem = size_t(d.M) * (sizeof(uint64_t) + sizeof(uint32_t));
+    // shared memory: per-instance arrays, chunk staging, then as many sort
+    // entries (power of two) as the 227 KB budget allows
+    const size_t budget = 227 * 1024 - 2048;
+    const size_t fixed = rb_inst_bytes(d.M) + sizeof(RbChunk);
+    uint32_t sort_cap = 0;
+    if (fixed + rb_sort_bytes(256) <= budget) {
+        sort_cap = 256;
+        while (sort_cap < 8192 && fixed + rb_sort_bytes(sort_cap * 2) <= budget) sort_cap *= 2;
+    }
+    const size_t smem = fixed + rb_sort_bytes(sort_cap);
     static size_t configured = 0;
     if (smem > configured) {
         cudaError_t e = cudaFuncSetAttribute(k_rebalance, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -244,7 +354,7 @@ cudaError_t launch_rebalance(const DevState &d, uint32_t n, uint64_t seq0, uint3
         if (e != cudaSuccess) return e;
         configured = smem;
     }
-    k_rebalance<<<1, 1024, smem, st>>>(d, n, seq0, call, out, cap, n_out);
+    k_rebalance<<<1, 1024, smem, st>>>(d, n, seq0, call, out, cap, n_out, sort_cap);
     return cudaGetLastError();
 }
 
