@@ -409,7 +409,9 @@ def main():
                                    f"batches of {w['batch']} prompts of {describe_lengths(w)} tokens "
                                    f"(~{bytes_per_launch / 1e6:.0f} MB per batch)",
                        "global_batch": w["batch"], "parallelism": f"replicas x{world}",
-                       "l2": "inputs larger than L2 (each batch > 129 MB, distinct per step)",
+                       "l2": ("inputs larger than L2 (each batch > 129 MB, distinct per step)"
+                              if bytes_per_launch > 129e6 else
+                              "batches smaller than L2, L2 not flushed between steps"),
                        "replay": "steps beyond the trace replay its batches cyclically" if W + K > nb else "none"},
             "roofline": {"bound": "hbm", "kernel": "k_hash (prompt hashing)", "achieved": achieved,
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
