@@ -228,6 +228,7 @@ def main():
     ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE",
                     help="override a workload field (small cases for profiling)")
     ap.add_argument("--max-touch", type=int, default=0, help="override max_touch_per_instance")
+    ap.add_argument("--index-slots-log2", type=int, default=0, help="override the index size (log2 slots)")
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":
@@ -251,6 +252,8 @@ def main():
     kw = handle_kwargs(w, tr.max_instance_id())
     if args.max_touch:
         kw["max_touch_per_instance"] = args.max_touch
+    if args.index_slots_log2:
+        kw["index_slots_log2"] = args.index_slots_log2
 
     # all batches' tokens resident in HBM (a pass longer than the trace replays it cyclically)
     used = min(nb, W + K)
@@ -342,7 +345,7 @@ def main():
     torch.cuda.synchronize()
     assert g.last_error() == 0
     D.dm_get_stage_times(g.h, reset=True)
-    D.dm_set_profiling(g.h, True)
+    D.dm_set_profiling(g.h, True, stages=["hash"])   # the roofline kernel only: events elsewhere cost time
     sampler = ClockSampler(local)
     time.sleep(0.3)
     if world > 1:
@@ -371,16 +374,25 @@ def main():
     ms = max_over_ranks(ms, device=dev)
     value = job_throughput(nreq, ms, world)
     hash_ms, hash_calls = st["hash"]
-    probe_ms, _ = st["probe"]
     hash_avg_s = hash_ms / 1e3 / max(hash_calls, 1)
     bytes_per_launch = prompt_bytes / max(hash_calls, 1)
     peak, peak_kind = peaks()
     achieved = bytes_per_launch / hash_avg_s / 1e9
-    prompt_gbps = prompt_bytes / ((hash_ms + probe_ms) / 1e3) / 1e9
+
+    # per-stage breakdown: a shorter run after the timed one, every stage timed
+    D.dm_set_profiling(g.h, True)
+    nb_stage = min(K, 30)
+    for j in range(W + K, W + K + nb_stage):
+        step(g, j)
+    st_all = D.dm_get_stage_times(g.h, reset=True)
+    D.dm_set_profiling(g.h, False)
+    assert g.last_error() == 0
+    stage_ms = {k: v[0] / max(v[1], 1) for k, v in st_all.items()}
+    prompt_gbps = bytes_per_launch / ((stage_ms["hash"] + stage_ms["probe"]) / 1e3) / 1e9
     # route: setup, segmap, drain, hash, probe, choice (6); commit: maint_plan, maint_a,
-    # compact_scan, maint_c, commit_prep, commit_touch, req_counts, evict_plan,
-    # evict_count, evict_cut, evict_clear, evict_walk (12); rebalance (1)
-    launches_per_step = 6 + 12 + (1 if w.get("rebalance") else 0)
+    # compact_scan, maint_c, commit_prep, commit_touch, touch_deferred, req_counts,
+    # evict_plan, evict_count, evict_cut, evict_clear, evict_walk (13); rebalance (1)
+    launches_per_step = 6 + 13 + (1 if w.get("rebalance") else 0)
     clocks = sampler.summary(wall0, wall1)
     g.close()
     del g
@@ -417,7 +429,7 @@ def main():
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic_per_launch(), "bytes_per_launch": bytes_per_launch,
                          "avg_launch_ms": hash_avg_s * 1e3},
-            "stage_ms_per_step": {k: v[0] / max(v[1], 1) for k, v in st.items()},
+            "stage_ms_per_step": stage_ms,
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches_per_step * K, "clocks": clocks,
         }
         print(json.dumps(line), flush=True)

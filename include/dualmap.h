@@ -94,7 +94,9 @@ typedef struct {
     /* log2 of the index slots per instance; 0 = automatic, the smallest
      * power of two >= 2 x (C + max_touch_per_instance).  A larger index is
      * rebuilt less often (it is rebuilt when half full, counting the slots
-     * evicted keys keep).  Never smaller than the automatic size; <= 40. */
+     * evicted keys keep).  Never smaller than the automatic size, nor than
+     * 64; <= 32.  dm_create returns DM_ERR_INVALID_ARG when the resulting
+     * index would exceed 2^32 slots (it records slot numbers as 32 bits). */
     uint32_t index_slots_log2;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
@@ -282,7 +284,11 @@ DM_API dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host);
 /* Synchronise the stream and return the sticky error (DM_OK if none). */
 DM_API dm_status dm_last_error(dm_handle *h);
 
-/* Per-stage CUDA-event timing of every subsequent call (on = 1) or none. */
+/* CUDA-event timing of the stages of every subsequent call: on = 0 none,
+ * 1 every stage, or DM_PROFILE_ONLY | (1 << DM_STAGE_x) | ... only the stages
+ * named.  Events between kernels cost a little time of their own; any other
+ * value returns DM_ERR_INVALID_ARG. */
+#define DM_PROFILE_ONLY 0x100
 DM_API dm_status dm_set_profiling(dm_handle *h, int on);
 
 /* Synchronise, then return the summed milliseconds and call counts of each

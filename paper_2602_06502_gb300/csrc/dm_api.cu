@@ -41,6 +41,7 @@ struct dm_handle {
     std::vector<Slot *> tables, tables2;   // both index buffers of each id (host copies)
     std::vector<Rec *> logs, logs2;        // both log buffers
     std::vector<uint8_t *> stales, stales2;
+    std::vector<uint32_t *> homes, homes2;  // both index-home logs
     std::vector<void *> allocs;    // every cudaMalloc of the handle
     // staging of the host-buffer entry points: two buffers, so the upload of
     // one batch (on copy_st) overlaps the routing of the previous one
@@ -53,7 +54,7 @@ struct dm_handle {
     } hs[2];
     int hs_next = 0;
     cudaStream_t copy_st = nullptr;
-    bool profiling = false;
+    uint32_t profiling = 0;   // bit s: time stage s
     std::vector<StageEvent> events;
     std::vector<cudaEvent_t> ev_pool;
     double stage_ms[DM_STAGE_COUNT] = {};
@@ -117,7 +118,7 @@ struct Stage {
     int s;
     cudaEvent_t a = nullptr, b = nullptr;
     Stage(dm_handle *h_, int s_) : h(h_), s(s_) {
-        if (!h->profiling) return;
+        if (!(h->profiling >> s & 1u)) return;
         a = pool_event(h);
         b = pool_event(h);
         if (a && b) cudaEventRecord(a, h->st);
@@ -200,7 +201,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.cache_capacity_blocks < 1 || c.cost_us_per_token < 1 || c.hot_den < 1) return DM_ERR_INVALID_ARG;
     if (c.max_batch < 1 || c.max_batch > (1u << 24) || c.max_batch_tokens < B) return DM_ERR_INVALID_ARG;
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
-    if (c.index_slots_log2 > 40) return DM_ERR_INVALID_ARG;
+    if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
 
     dm_handle *h = new dm_handle();
     h->cfg = c;
@@ -221,6 +222,11 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.T = c.max_touch_per_instance ? c.max_touch_per_instance : d.max_blocks;
     d.S = pow2_at_least(2 * (d.C + d.T));
     if (c.index_slots_log2 && (1ull << c.index_slots_log2) > d.S) d.S = 1ull << c.index_slots_log2;
+    if (d.S < 64) d.S = 64;   // at least a few whole groups
+    if (d.S > (1ull << 32)) {
+        delete h;
+        return DM_ERR_INVALID_ARG;
+    }
     d.logcap = pow2_at_least(2 * (d.C + d.T));
     d.Q = c.max_queue ? c.max_queue : 65536;
     d.rb_cap = (uint32_t)pow2_at_least(d.Q > d.M ? d.Q : d.M);
@@ -264,6 +270,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.logbuf_alt, M));
     A(dalloc(h, &d.stale, M));
     A(dalloc(h, &d.stale_alt, M));
+    A(dalloc(h, &d.loghome, M));
+    A(dalloc(h, &d.loghome_alt, M));
     A(dalloc(h, &d.mt_flags, M));
     A(dalloc(h, &d.mt_newtail, M));
     A(dalloc(h, &d.mc_chunk_off, M + 1));
@@ -293,6 +301,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.rb_seq, d.rb_cap));
     A(dalloc(h, &d.rb_ttft, d.rb_cap));
     A(dalloc(h, &d.rb_pos, d.rb_cap));
+    A(dalloc(h, &d.defer, d.max_segs * dm::kSegBlocks));
+    A(dalloc(h, &d.defer_n, d.max_segs));
     // two sets of batch scratch: routing and dm_hash_prompts
     for (DevState *x : {&h->d, &h->dh}) {
         if (x == &h->dh) {
@@ -340,6 +350,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(cudaMemsetAsync(d.logbuf_alt, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.stale, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.stale_alt, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.loghome, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.loghome_alt, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.mt_flags, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.log_front, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.log_tail, 0, M * 8, h->st));
@@ -362,6 +374,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     h->logs2.assign(M, nullptr);
     h->stales.assign(M, nullptr);
     h->stales2.assign(M, nullptr);
+    h->homes.assign(M, nullptr);
+    h->homes2.assign(M, nullptr);
     h->hash_grid = dm::hash_grid_size();
     *out = h;
     return DM_OK;
@@ -429,12 +443,15 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         Slot *t = nullptr, *t2 = nullptr;
         Rec *lg = nullptr, *lg2 = nullptr;
         uint8_t *sf = nullptr, *sf2 = nullptr;
+        uint32_t *hm = nullptr, *hm2 = nullptr;
         e = dalloc(h, &t, d.S);
         if (e == cudaSuccess) e = dalloc(h, &t2, d.S);
         if (e == cudaSuccess) e = dalloc(h, &lg, d.logcap);
         if (e == cudaSuccess) e = dalloc(h, &lg2, d.logcap);
         if (e == cudaSuccess) e = dalloc(h, &sf, d.logcap);
         if (e == cudaSuccess) e = dalloc(h, &sf2, d.logcap);
+        if (e == cudaSuccess) e = dalloc(h, &hm, d.logcap);
+        if (e == cudaSuccess) e = dalloc(h, &hm2, d.logcap);
         if (e != cudaSuccess) { cudaGetLastError(); return DM_ERR_OOM; }
         h->tables[id] = t;
         h->tables2[id] = t2;
@@ -442,12 +459,15 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         h->logs2[id] = lg2;
         h->stales[id] = sf;
         h->stales2[id] = sf2;
+        h->homes[id] = hm;
+        h->homes2[id] = hm2;
     }
     // a (re-)added instance starts empty, both buffers of each
     struct { void *dst; const void *src; } ptrs[] = {
         {d.table + id, &h->tables[id]}, {d.table_alt + id, &h->tables2[id]},
         {d.logbuf + id, &h->logs[id]}, {d.logbuf_alt + id, &h->logs2[id]},
-        {d.stale + id, &h->stales[id]}, {d.stale_alt + id, &h->stales2[id]}};
+        {d.stale + id, &h->stales[id]}, {d.stale_alt + id, &h->stales2[id]},
+        {d.loghome + id, &h->homes[id]}, {d.loghome_alt + id, &h->homes2[id]}};
     for (auto &pp : ptrs)
         if (e == cudaSuccess) e = cudaMemcpyAsync(pp.dst, pp.src, sizeof(void *), cudaMemcpyHostToDevice, h->st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
@@ -743,7 +763,12 @@ dm_status dm_last_error(dm_handle *h) {
 
 dm_status dm_set_profiling(dm_handle *h, int on) {
     if (!h) return DM_ERR_INVALID_ARG;
-    h->profiling = on != 0;
+    if (on == 0 || on == 1) {
+        h->profiling = on ? (1u << DM_STAGE_COUNT) - 1u : 0u;
+        return DM_OK;
+    }
+    if (!(on & DM_PROFILE_ONLY) || (on & ~(DM_PROFILE_ONLY | ((1 << DM_STAGE_COUNT) - 1)))) return DM_ERR_INVALID_ARG;
+    h->profiling = (uint32_t)on & ((1u << DM_STAGE_COUNT) - 1u);
     return DM_OK;
 }
 

@@ -17,6 +17,7 @@ namespace dm {
 
 // One warp per instance: run `delta` us of work off the queue head.
 __global__ void k_drain(DevState d, uint64_t delta) {
+    pdl_enter();
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -58,7 +59,7 @@ __global__ void k_drain(DevState d, uint64_t delta) {
 
 cudaError_t launch_drain(const DevState &d, uint64_t delta, cudaStream_t st) {
     const uint32_t warps = 8;
-    k_drain<<<(d.M + warps - 1) / warps, warps * 32, 0, st>>>(d, delta);
+    DM_TRY(launch_pdl(k_drain, (d.M + warps - 1) / warps, warps * 32, 0, st, d, delta));
     return cudaGetLastError();
 }
 
@@ -90,6 +91,7 @@ __host__ __device__ inline size_t choice_lanes(uint32_t M) { return (size_t(M) +
 size_t choice_smem(uint32_t M) { return size_t(M) * 16 + choice_lanes(M) * 4 + sizeof(ChoiceStage); }
 
 __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uint32_t n, uint64_t seq0) {
+    pdl_enter();
     extern __shared__ __align__(16) unsigned char smem[];
     if (has_err(d.err)) return;
     uint64_t *W = reinterpret_cast<uint64_t *>(smem);
@@ -211,7 +213,7 @@ cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, 
         if (e != cudaSuccess) return e;
         configured = smem;
     }
-    k_choice<<<1, 1024, smem, st>>>(d, o, n, seq0);
+    DM_TRY(launch_pdl(k_choice, 1, 1024, smem, st, d, o, n, seq0));
     return cudaGetLastError();
 }
 

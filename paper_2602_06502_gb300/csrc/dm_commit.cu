@@ -25,50 +25,93 @@ constexpr uint32_t kPrepChunk = 2048;
 constexpr uint32_t kFlagCompact = 1, kFlagRebuild = 2;
 constexpr uint32_t kZeroChunk = 4096;   // slots or flag bytes cleared per chunk
 
-// Slot of `key` given the result `prev` of a CAS(0 -> key) at its home slot
-// i0: the home slot when it was empty (claimed) or already held the key,
-// else continue probing from i0 + 1.
-__device__ __forceinline__ uint64_t slot_after_home_cas(Slot *t, uint64_t mask, uint64_t key, uint64_t i0,
-                                                        uint64_t prev, uint32_t *err, bool *claimed) {
-    if (prev == 0) { *claimed = true; return i0; }
-    if (prev == key) return i0;
-    uint64_t i = (i0 + 1) & mask;
-    for (uint64_t it = 1; it <= mask; ++it) {
-        uint64_t k = *(volatile uint64_t *)&t[i].key;
-        if (k == 0) {
-            const unsigned long long pv =
-                atomicCAS(reinterpret_cast<unsigned long long *>(&t[i].key), 0ull, (unsigned long long)key);
-            if (pv == 0) { *claimed = true; return i; }
-            k = pv;
+// 16-byte compare-and-swap of a whole index slot; returns its previous
+// contents.  Every slot access of the touch kernel goes through this, so key
+// and position change together and never tear.
+__device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
+    Slot old;
+    asm volatile(
+        "{\n\t.reg .b128 c, v, r;\n\t"
+        "mov.b128 c, {%2, %3};\n\t"
+        "mov.b128 v, {%4, %5};\n\t"
+        "atom.relaxed.gpu.global.cas.b128 r, [%6], c, v;\n\t"
+        "mov.b128 {%0, %1}, r;\n\t}"
+        : "=l"(old.key), "=l"(old.pos1)
+        : "l"(expect.key), "l"(expect.pos1), "l"(desired.key), "l"(desired.pos1),
+          "l"(__cvta_generic_to_global(s))
+        : "memory");
+    return old;
+}
+
+// Finish the touch of `key` at position value p1 (1 + log position), given
+// `old`, the result of CAS({0,0} -> {key, p1}) at its home slot.  An empty
+// slot was claimed by that CAS; a slot holding the key has its position
+// raised to p1 unless a larger one is already there (CAS loop: only a larger
+// value is written); a slot of another key moves on along the key's probe
+// order, using a snapshot of the bucket to skip the slots other keys hold
+// (slots never empty again, so only empty or matching ones are candidates).
+// Every touch of a key follows the same order, so concurrent first touches
+// meet at the same slot and one CAS wins.  Returns the position value the
+// key had before (0 if claimed now).
+__device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint64_t home,
+                                                  Slot old, uint32_t *err, bool *claimed) {
+    const uint32_t o = (uint32_t)(home & (kGroup - 1));
+    uint64_t R = home & ~uint64_t(kGroup - 1), i = home;
+    uint32_t step = 0;   // order position of slot i within bucket R
+    // at most one probe step per slot, and one retry per other touch of the
+    // key in the batch (each failed retry means another touch got in)
+    const uint64_t limit = mask + 1 + (1ull << 20);
+    for (uint64_t it = 0; it < limit; ++it) {
+        if (old.key == 0) { *claimed = true; return 0; }   // a CAS from {0,0} that failed returns a key
+        if (old.key == key) {
+            if (old.pos1 >= p1) return old.pos1;
+            const Slot now = slot_cas(&t[i], old, Slot{key, p1});
+            if (now.pos1 == old.pos1) return old.pos1;      // keys never change once set
+            old = now;
+            continue;
         }
-        if (k == key) return i;
-        i = (i + 1) & mask;
+        Slot sn[kGroup];
+#pragma unroll
+        for (int j = 0; j < (int)kGroup; ++j) sn[j] = load_slot(t + R + j);
+        uint32_t best = kGroup;
+        Slot bs{0, 0};
+#pragma unroll
+        for (int j = 0; j < (int)kGroup; ++j) {
+            const uint32_t q = (uint32_t(j) - o) & (kGroup - 1);
+            if ((sn[j].key == 0 || sn[j].key == key) && q > step && q < best) {
+                best = q;
+                bs = sn[j];
+            }
+        }
+        if (best < kGroup) {
+            step = best;
+        } else {
+            R = (R + kGroup) & mask;
+            step = 0;
+            bs = Slot{0, 0};
+        }
+        i = R + ((o + step) & (kGroup - 1));
+        old = bs.key == key ? bs : slot_cas(&t[i], Slot{0, 0}, Slot{key, p1});
     }
     set_err(err, DM_ERR_TIMEOUT);
-    return i0;
+    return 0;
 }
 
 // Insert a key known to be absent (index rebuild: all keys distinct).
-__device__ __forceinline__ void table_insert_new(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint32_t *err) {
-    uint64_t j = key & mask;
-    for (uint64_t it = 0; it <= mask; ++it) {
-        const unsigned long long prev =
-            atomicCAS(reinterpret_cast<unsigned long long *>(&t[j].key), 0ull, (unsigned long long)key);
-        if (prev == 0) { t[j].pos1 = p1; return; }
-        j = (j + 1) & mask;
-    }
-    set_err(err, DM_ERR_TIMEOUT);
+__device__ __forceinline__ void table_insert_new(Slot *t, uint64_t mask, uint64_t key, uint64_t home, uint64_t p1,
+                                                 uint32_t *err) {
+    bool cl = false;
+    touch_resolve(t, mask, key, p1, home, slot_cas(&t[home], Slot{0, 0}, Slot{key, p1}), err, &cl);
 }
 
-// Point an existing key at a new record position (log compaction).
-__device__ __forceinline__ void table_set_pos(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint32_t *err) {
-    uint64_t j = key & mask;
-    for (uint64_t it = 0; it <= mask; ++it) {
-        if (t[j].key == key) { t[j].pos1 = p1; return; }
-        if (t[j].key == 0) break;
-        j = (j + 1) & mask;
-    }
-    set_err(err, DM_ERR_TIMEOUT);
+// Point an existing key at a new record position (log compaction; no other
+// thread touches the key meanwhile).
+__device__ __forceinline__ void table_set_pos(Slot *t, uint64_t mask, uint64_t key, uint64_t home, uint64_t p1,
+                                              uint32_t *err) {
+    Slot s;
+    const uint64_t j = table_find(t, mask, key, home, err, &s);
+    if (j == kNoSlot) set_err(err, DM_ERR_TIMEOUT);
+    else t[j].pos1 = p1;
 }
 
 // Exclusive block scan of u32 counts (any block size up to 1024).
@@ -124,6 +167,7 @@ __device__ __forceinline__ uint32_t owner_of(const uint32_t *off, uint32_t M, ui
 //         inserts them with their current positions.
 
 __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
+    pdl_enter();
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_w[33];
     if (has_err(d.err)) return;
@@ -173,6 +217,7 @@ __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
 }
 
 __global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
+    pdl_enter();
     __shared__ uint32_t s_i, s_cnt[kMtThreads / 32];
     if (has_err(d.err)) return;
     // clearing: a rebuilding instance's chunks cover its second index first,
@@ -225,6 +270,7 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
 
 // Warp per compacting instance: chunk counts -> exclusive destination offsets.
 __global__ void k_compact_scan(DevState d) {
+    pdl_enter();
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -242,6 +288,7 @@ __global__ void k_compact_scan(DevState d) {
 }
 
 __global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
+    pdl_enter();
     __shared__ uint32_t s_i, s_w[kMtThreads / 32];
     if (has_err(d.err)) return;
     const uint32_t nw = d.info->mc_chunks;
@@ -270,13 +317,15 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
             }
             if (live) {
                 const Rec r = lg[p & lmask];
+                const uint32_t home = d.loghome[i][p & lmask];
                 if (fl & kFlagCompact) {
                     const uint64_t np = out + before + __popc(b & ((1u << lane) - 1));
                     d.logbuf_alt[i][np & lmask] = r;
-                    if (fl & kFlagRebuild) table_insert_new(d.table_alt[i], mask, r.key, np + 1, d.err);
-                    else table_set_pos(d.table[i], mask, r.key, np + 1, d.err);
+                    d.loghome_alt[i][np & lmask] = home;
+                    if (fl & kFlagRebuild) table_insert_new(d.table_alt[i], mask, r.key, home, np + 1, d.err);
+                    else table_set_pos(d.table[i], mask, r.key, home, np + 1, d.err);
                 } else {
-                    table_insert_new(d.table_alt[i], mask, r.key, p + 1, d.err);
+                    table_insert_new(d.table_alt[i], mask, r.key, home, p + 1, d.err);
                 }
             }
             out += tot;
@@ -292,6 +341,7 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
 // request of this batch are the offsets recomputed (arrival order per final
 // instance).  Single CTA; dynamic smem holds one u64 per instance.
 __global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
+    pdl_enter();
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_f[kPrepChunk], s_nb[kPrepChunk];
     __shared__ uint64_t s_off[kPrepChunk];
@@ -306,6 +356,9 @@ __global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
             uint8_t *f = d.stale[i];
             d.stale[i] = d.stale_alt[i];
             d.stale_alt[i] = f;
+            uint32_t *hm = d.loghome[i];
+            d.loghome[i] = d.loghome_alt[i];
+            d.loghome_alt[i] = hm;
             d.log_tail[i] = d.mt_newtail[i];
         }
         if (fl & kFlagRebuild) {
@@ -351,11 +404,8 @@ __global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
     }
 }
 
-// One warp per segment: cache keys, stamps, log records, index touches.  A
-// superseded record (the key's previous record, or this one when a later
-// touch of the batch already won) gets its stale flag.  Lane l handles
-// blocks l and l+32 of the segment together: the CAS at both home slots,
-// then both atomicMax, so their round trips overlap.
+// Index touches.  A superseded record (the key's previous record, or this
+// one when a later touch of the batch already won) gets its stale flag.
 __device__ __forceinline__ void touch_outcome(uint64_t old, uint64_t p, uint64_t front, uint8_t *st, uint64_t lmask,
                                               uint32_t &newly) {
     if (old == 0 || old - 1 < front) {
@@ -367,55 +417,158 @@ __device__ __forceinline__ void touch_outcome(uint64_t old, uint64_t p, uint64_t
     }
 }
 
-__global__ void __launch_bounds__(256) k_commit_touch(DevState d) {
+// Per-segment values of the touch kernel.  Within a segment, block e
+// (0..cnt-1) has log position p_first - e and stamp stamp_first - e: a
+// request touches its blocks from the last one down.
+struct TouchSeg {
+    uint64_t pidx;          // plocal index of the segment's first block
+    uint64_t p_first;       // log position of that block's record
+    uint64_t stamp_first;   // its clock stamp
+    uint64_t carry;         // prefix carry into the segment
+    uint64_t front;         // log front of the final instance
+    Slot *t;
+    Rec *lg;
+    uint8_t *st;
+    uint32_t *lh;           // index home of each record
+    uint32_t cnt, f;        // blocks in the segment, final instance
+};
+
+__device__ __forceinline__ TouchSeg touch_seg_load(const DevState &d, uint32_t seg, uint64_t clock_base) {
+    const uint32_t r = d.seg_req[seg];
+    const uint32_t first = (seg - d.r_segoff[r]) * kSegBlocks;
+    const uint32_t nblk = d.r_nblk[r], f = d.r_final[r];
+    const uint64_t bo = d.r_blkoff[r];
+    TouchSeg g;
+    g.pidx = bo + first;
+    g.p_first = d.log_base[f] + d.r_touchoff[r] + (nblk - 1 - first);
+    g.stamp_first = clock_base + bo + (nblk - first);
+    g.carry = d.seg_carry[seg];
+    g.front = d.log_front[f];
+    g.t = d.table[f];
+    g.lg = d.logbuf[f];
+    g.st = d.stale[f];
+    g.lh = d.loghome[f];
+    g.cnt = min(nblk - first, kSegBlocks);
+    g.f = f;
+    return g;
+}
+
+// Each warp takes a contiguous range of segments.  Its lanes load the
+// metadata of up to 32 of them at once into the warp's shared-memory slots
+// (request, final instance, offsets: one dependent chain per 32 segments
+// instead of per segment); then, segment by segment, lane l touches blocks l
+// and l+32: both home-slot CAS are issued before either result is used, and
+// the next segment's plocal values are loaded while they are in flight.  No
+// CTA barriers: a warp never waits for another.
+constexpr int kTouchThreads = 256;
+__global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
+    pdl_enter();
+    __shared__ TouchSeg s_seg[kTouchThreads / 32][32];
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
-    const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
+    const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
+    const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t total_segs = d.info->total_segs;
     const uint64_t clock_base = d.info->clock_base;
     const uint64_t mask = d.S - 1, lmask = d.logcap - 1;
-    for (uint32_t seg = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; seg < total_segs; seg += nwarps) {
-        const uint32_t r = d.seg_req[seg];
-        const uint32_t j = seg - d.r_segoff[r];
-        const uint32_t nblk = d.r_nblk[r];
-        const uint32_t f = d.r_final[r];
-        const uint64_t carry = d.seg_carry[seg];
-        const uint64_t bo = d.r_blkoff[r], toff = d.log_base[f] + d.r_touchoff[r];
-        const uint64_t front = d.log_front[f];
-        Slot *t = d.table[f];
-        Rec *lg = d.logbuf[f];
-        uint8_t *st = d.stale[f];
-        const uint32_t b_end = min(nblk, (j + 1) * kSegBlocks);
+    const uint32_t per = (total_segs + nw - 1) / nw;
+    const uint32_t lo = min(total_segs, gw * per), hi = min(total_segs, lo + per);
+    for (uint32_t c0 = lo; c0 < hi; c0 += 32) {
+        const uint32_t nc = min(32u, hi - c0);
+        TouchSeg *sg = s_seg[threadIdx.x >> 5];
+        if ((uint32_t)lane < nc) sg[lane] = touch_seg_load(d, c0 + lane, clock_base);
+        __syncwarp();
+        uint64_t x0 = lane < (int)sg[0].cnt ? d.plocal[sg[0].pidx + lane] : 0;
+        uint64_t x1 = lane + 32 < (int)sg[0].cnt ? d.plocal[sg[0].pidx + lane + 32] : 0;
+        for (uint32_t i = 0; i < nc; ++i) {
+            const TouchSeg &g = sg[i];
+            const bool v0 = lane < (int)g.cnt, v1 = lane + 32 < (int)g.cnt;
+            const uint64_t k0 = cache_key(x0 + g.carry, d.Sc), k1 = cache_key(x1 + g.carry, d.Sc);
+            const uint64_t h0 = group_home(group_anchor(k0, lane), lane, mask);   // segments start on a group boundary
+            const uint64_t h1 = group_home(group_anchor(k1, lane), lane, mask);
+            const uint64_t p0 = g.p_first - lane, p1 = g.p_first - lane - 32;
+            if (v0) {
+                g.lg[p0 & lmask] = Rec{k0, g.stamp_first - lane};
+                g.lh[p0 & lmask] = (uint32_t)h0;
+            }
+            if (v1) {
+                g.lg[p1 & lmask] = Rec{k1, g.stamp_first - lane - 32};
+                g.lh[p1 & lmask] = (uint32_t)h1;
+            }
+            const Slot c0s = v0 ? slot_cas(&g.t[h0], Slot{0, 0}, Slot{k0, p0 + 1}) : Slot{0, 0};
+            const Slot c1s = v1 ? slot_cas(&g.t[h1], Slot{0, 0}, Slot{k1, p1 + 1}) : Slot{0, 0};
+            if (i + 1 < nc) {   // next segment's blocks, loaded while the CAS are in flight
+                const uint64_t pi = sg[i + 1].pidx;
+                const uint32_t cn = sg[i + 1].cnt;
+                x0 = lane < (int)cn ? d.plocal[pi + lane] : 0;
+                x1 = lane + 32 < (int)cn ? d.plocal[pi + lane + 32] : 0;
+            }
+            // settled here: a claim of an empty home slot, or the key found
+            // there with a later position already; the rest is deferred
+            uint32_t newly = 0, claims = 0;
+            bool need0 = false, need1 = false;
+            if (v0) {
+                if (c0s.key == 0) { ++newly; ++claims; }
+                else if (c0s.key == k0 && c0s.pos1 > p0) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
+                else need0 = true;
+            }
+            if (v1) {
+                if (c1s.key == 0) { ++newly; ++claims; }
+                else if (c1s.key == k1 && c1s.pos1 > p1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
+                else need1 = true;
+            }
+            // deferred touches go to the segment's own slice of the queue
+            const uint32_t m0 = __ballot_sync(0xffffffffu, need0), m1 = __ballot_sync(0xffffffffu, need1);
+            const uint32_t below = (1u << lane) - 1u;
+            Deferred *dq = d.defer + uint64_t(c0 + i) * kSegBlocks;
+            if (need0) dq[__popc(m0 & below)] = Deferred{k0, p0, c0s.pos1, (uint32_t)h0, g.f, c0s.key == k0 ? 1u : 0u, 0};
+            if (need1)
+                dq[__popc(m0) + __popc(m1 & below)] =
+                    Deferred{k1, p1, c1s.pos1, (uint32_t)h1, g.f, c1s.key == k1 ? 1u : 0u, 0};
+            newly = __reduce_add_sync(0xffffffffu, newly);
+            claims = __reduce_add_sync(0xffffffffu, claims);
+            if (lane == 0) {   // summed per request by k_req_counts (no hot-counter atomics)
+                d.seg_newly[c0 + i] = newly;
+                d.seg_claims[c0 + i] = claims;
+                d.defer_n[c0 + i] = __popc(m0) + __popc(m1);
+            }
+        }
+        __syncwarp();   // the slots are refilled for the next 32 segments
+    }
+}
+
+// Second pass over the deferred touches, a warp per segment: raise the
+// position of a found key (CAS loop), or walk the probe order of a key whose
+// home slot holds another key.  Every record still ends up marked stale
+// exactly once unless it is its key's latest: the first pass only settled
+// claims (value 0 before) and touches that saw a later position (their own
+// record is stale), and the maxima taken here order the rest.
+__global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
+    pdl_enter();
+    if (has_err(d.err)) return;
+    const int lane = threadIdx.x & 31;
+    const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
+    const uint32_t total_segs = d.info->total_segs;
+    const uint64_t mask = d.S - 1, lmask = d.logcap - 1;
+    for (uint32_t seg = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; seg < total_segs; seg += nw) {
+        const uint32_t n = d.defer_n[seg];
+        if (n == 0) continue;
         uint32_t newly = 0, claims = 0;
-        for (uint32_t b = j * kSegBlocks + lane; b < b_end; b += 64) {
-            const bool v1 = b + 32 < b_end;
-            const uint64_t k0 = cache_key(d.plocal[bo + b] + carry, d.Sc);
-            const uint64_t k1 = v1 ? cache_key(d.plocal[bo + b + 32] + carry, d.Sc) : 0;
-            const uint64_t p0 = toff + (nblk - 1 - b);              // block n_blk-1 is touched first
-            const uint64_t p1 = toff + (nblk - 1 - (b + 32));
-            lg[p0 & lmask] = Rec{k0, clock_base + bo + (nblk - b)};
-            if (v1) lg[p1 & lmask] = Rec{k1, clock_base + bo + (nblk - b - 32)};
-            const uint64_t i0 = k0 & mask, i1 = k1 & mask;
-            const unsigned long long c0 =
-                atomicCAS(reinterpret_cast<unsigned long long *>(&t[i0].key), 0ull, (unsigned long long)k0);
-            const unsigned long long c1 =
-                v1 ? atomicCAS(reinterpret_cast<unsigned long long *>(&t[i1].key), 0ull, (unsigned long long)k1) : 0;
-            bool cl0 = false, cl1 = false;
-            const uint64_t s0 = slot_after_home_cas(t, mask, k0, i0, c0, d.err, &cl0);
-            const uint64_t s1 = v1 ? slot_after_home_cas(t, mask, k1, i1, c1, d.err, &cl1) : 0;
-            const uint64_t o0 =
-                atomicMax(reinterpret_cast<unsigned long long *>(&t[s0].pos1), (unsigned long long)(p0 + 1));
-            const uint64_t o1 = v1 ? atomicMax(reinterpret_cast<unsigned long long *>(&t[s1].pos1),
-                                               (unsigned long long)(p1 + 1)) : 0;
-            touch_outcome(o0, p0, front, st, lmask, newly);
-            if (v1) touch_outcome(o1, p1, front, st, lmask, newly);
-            claims += cl0 + cl1;
+        for (uint32_t j = lane; j < n; j += 32) {
+            const Deferred e = d.defer[uint64_t(seg) * kSegBlocks + j];
+            // the home slot as the first pass saw it (another key: any value
+            // other than 0 and e.key)
+            const Slot old = e.found ? Slot{e.key, e.x} : Slot{e.key == 1 ? 2ull : e.key ^ 1ull, 0};
+            bool cl = false;
+            const uint64_t o = touch_resolve(d.table[e.f], mask, e.key, e.p + 1, e.home, old, d.err, &cl);
+            touch_outcome(o, e.p, d.log_front[e.f], d.stale[e.f], lmask, newly);
+            claims += cl;
         }
         newly = __reduce_add_sync(0xffffffffu, newly);
         claims = __reduce_add_sync(0xffffffffu, claims);
-        if (lane == 0) {   // summed per instance by the eviction plan (no hot-counter atomics)
-            d.seg_newly[seg] = newly;
-            d.seg_claims[seg] = claims;
+        if (lane == 0) {   // this warp alone owns the segment's counters here
+            d.seg_newly[seg] += newly;
+            d.seg_claims[seg] += claims;
         }
     }
 }
@@ -436,6 +589,7 @@ constexpr int kEvThreads = 256;
 // Warp per request: sum the touch kernel's counts over the request's
 // (contiguous) segments, one atomic per request and counter.
 __global__ void k_req_counts(DevState d, uint32_t n) {
+    pdl_enter();
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -457,6 +611,7 @@ __global__ void k_req_counts(DevState d, uint32_t n) {
 }
 
 __global__ void __launch_bounds__(1024) k_evict_plan(DevState d) {
+    pdl_enter();
     __shared__ uint32_t s_w[33];
     if (has_err(d.err)) return;
     uint32_t carry = 0;
@@ -487,6 +642,7 @@ __global__ void __launch_bounds__(1024) k_evict_plan(DevState d) {
 }
 
 __global__ void __launch_bounds__(kEvThreads) k_evict_count(DevState d) {
+    pdl_enter();
     __shared__ uint32_t s_i;
     __shared__ uint32_t s_cnt[kEvThreads / 32];
     if (has_err(d.err)) return;
@@ -517,6 +673,7 @@ __global__ void __launch_bounds__(kEvThreads) k_evict_count(DevState d) {
 
 // Warp per instance: locate the record where the non-stale count reaches excess.
 __global__ void k_evict_cut(DevState d) {
+    pdl_enter();
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -573,6 +730,7 @@ __global__ void k_evict_cut(DevState d) {
 // Reset the stale flags of the records the front passes (those positions
 // will hold new records).
 __global__ void __launch_bounds__(kEvThreads) k_evict_clear(DevState d) {
+    pdl_enter();
     __shared__ uint32_t s_i;
     if (has_err(d.err)) return;
     const uint32_t nchunks = d.info->ev_chunks;
@@ -592,6 +750,7 @@ __global__ void __launch_bounds__(kEvThreads) k_evict_clear(DevState d) {
 }
 
 __global__ void __launch_bounds__(1024) k_evict_walk(DevState d) {
+    pdl_enter();
     __shared__ uint32_t s_w[33];
     __shared__ uint64_t s_front;
     if (has_err(d.err)) return;
@@ -645,20 +804,22 @@ cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
         configured = smem;
     }
     static const int g_a = full_grid(k_maint_a, kMtThreads), g_c = full_grid(k_maint_c, kMtThreads),
-                     g_t = full_grid(k_commit_touch, 256), g_ec = full_grid(k_evict_count, kEvThreads),
+                     g_t = full_grid(k_commit_touch, kTouchThreads), g_ec = full_grid(k_evict_count, kEvThreads),
+                     g_d = full_grid(k_touch_deferred, 256),
                      g_el = full_grid(k_evict_clear, kEvThreads);
-    k_maint_plan<<<1, 1024, smem, st>>>(d, n);
-    k_maint_a<<<g_a, kMtThreads, 0, st>>>(d);
-    k_compact_scan<<<(d.M + 7) / 8, 256, 0, st>>>(d);
-    k_maint_c<<<g_c, kMtThreads, 0, st>>>(d);
-    k_commit_prep<<<1, 1024, smem, st>>>(d, n);
-    k_commit_touch<<<g_t, 256, 0, st>>>(d);
-    k_req_counts<<<(n + 7) / 8, 256, 0, st>>>(d, n);
-    k_evict_plan<<<1, 1024, 0, st>>>(d);
-    k_evict_count<<<g_ec, kEvThreads, 0, st>>>(d);
-    k_evict_cut<<<(d.M + 7) / 8, 256, 0, st>>>(d);
-    k_evict_clear<<<g_el, kEvThreads, 0, st>>>(d);
-    k_evict_walk<<<d.M, 1024, 0, st>>>(d);
+    DM_TRY(launch_pdl(k_maint_plan, 1, 1024, smem, st, d, n));
+    DM_TRY(launch_pdl(k_maint_a, g_a, kMtThreads, 0, st, d));
+    DM_TRY(launch_pdl(k_compact_scan, (d.M + 7) / 8, 256, 0, st, d));
+    DM_TRY(launch_pdl(k_maint_c, g_c, kMtThreads, 0, st, d));
+    DM_TRY(launch_pdl(k_commit_prep, 1, 1024, smem, st, d, n));
+    DM_TRY(launch_pdl(k_commit_touch, g_t, kTouchThreads, 0, st, d));
+    DM_TRY(launch_pdl(k_touch_deferred, g_d, 256, 0, st, d));
+    DM_TRY(launch_pdl(k_req_counts, (n + 7) / 8, 256, 0, st, d, n));
+    DM_TRY(launch_pdl(k_evict_plan, 1, 1024, 0, st, d));
+    DM_TRY(launch_pdl(k_evict_count, g_ec, kEvThreads, 0, st, d));
+    DM_TRY(launch_pdl(k_evict_cut, (d.M + 7) / 8, 256, 0, st, d));
+    DM_TRY(launch_pdl(k_evict_clear, g_el, kEvThreads, 0, st, d));
+    DM_TRY(launch_pdl(k_evict_walk, d.M, 1024, 0, st, d));
     return cudaGetLastError();
 }
 

@@ -54,6 +54,7 @@ __device__ __forceinline__ void block_scan2(uint64_t a, uint32_t b, uint64_t &ea
 // Validate the batch and lay out per-request block / segment offsets.
 __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off, const uint32_t *len,
                                                 uint32_t n, uint64_t total_tokens) {
+    pdl_enter();
     __shared__ uint64_t sa[32];
     __shared__ uint32_t sb[32];
     if (has_err(d.err)) return;
@@ -98,6 +99,7 @@ __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off,
 
 // Segment -> request map, one warp per request.
 __global__ void k_segmap(DevState d, uint32_t n) {
+    pdl_enter();
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -108,8 +110,8 @@ __global__ void k_segmap(DevState d, uint32_t n) {
 }
 
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st) {
-    k_setup<<<1, 1024, 0, st>>>(d, b.offsets, b.lengths, b.n, b.total_tokens);
-    if (b.n) k_segmap<<<(b.n + 7) / 8, 256, 0, st>>>(d, b.n);
+    DM_TRY(launch_pdl(k_setup, 1, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens));
+    if (b.n) DM_TRY(launch_pdl(k_segmap, (b.n + 7) / 8, 256, 0, st, d, b.n));
     return cudaGetLastError();
 }
 
@@ -154,6 +156,7 @@ __device__ __forceinline__ uint64_t reduce_scatter(uint64_t (&p)[U], int q) {
 // scan.  Segments below K also sum their f2 digests (blocks < K).
 template <int U>
 __global__ void __launch_bounds__(256) k_hash(DevState d, const uint32_t *__restrict__ tokens) {
+    pdl_enter();
     constexpr int IT = kSegBlocks / 32;
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
@@ -233,11 +236,11 @@ int hash_grid_size() {
 
 cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st) {
     switch (d.B) {
-        case 4: k_hash<1><<<grid, 256, 0, st>>>(d, b.tokens); break;
-        case 8: k_hash<2><<<grid, 256, 0, st>>>(d, b.tokens); break;
-        case 16: k_hash<4><<<grid, 256, 0, st>>>(d, b.tokens); break;
-        case 32: k_hash<8><<<grid, 256, 0, st>>>(d, b.tokens); break;
-        case 64: k_hash<16><<<grid, 256, 0, st>>>(d, b.tokens); break;
+        case 4: DM_TRY(launch_pdl(k_hash<1>, grid, 256, 0, st, d, b.tokens)); break;
+        case 8: DM_TRY(launch_pdl(k_hash<2>, grid, 256, 0, st, d, b.tokens)); break;
+        case 16: DM_TRY(launch_pdl(k_hash<4>, grid, 256, 0, st, d, b.tokens)); break;
+        case 32: DM_TRY(launch_pdl(k_hash<8>, grid, 256, 0, st, d, b.tokens)); break;
+        case 64: DM_TRY(launch_pdl(k_hash<16>, grid, 256, 0, st, d, b.tokens)); break;
         default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();

@@ -18,6 +18,7 @@ constexpr int kMaxLevels = 8;
 constexpr uint32_t kEvChunk = 1024;      // log records per eviction / compaction chunk
 constexpr uint32_t kRbChunk = 4096;      // index slots per rebuild chunk
 constexpr uint64_t kSpinLimit = 1ull << 26; // bound of every data-dependent device loop
+constexpr uint32_t kGroup = 8;           // consecutive blocks of a prompt homed in one 128-byte index line
 
 // One queued request (48 bytes).
 struct QEntry {
@@ -29,7 +30,19 @@ struct QEntry {
 // One index slot (16 bytes): a block key and 1 + the position of its latest
 // record in the instance's recency log; key 0 marks an empty slot.  A key is
 // resident while that position is at or after the log front.
-struct Slot {
+//
+// Placement: the index is cut into buckets of kGroup slots (one 128-byte
+// line).  Block b of a prompt (b counted from the prompt's start) prefers
+// slot (b & 7) of bucket A & mask & ~7, A being the key of block b & ~7 of
+// the same prompt (its group anchor), so the 8 blocks of a group share one
+// line: one random DRAM access instead of 8 (random single-slot atomics
+// saturate far below line-local ones).  A key fixes its whole prefix and so
+// its anchor: every key has one home.  Probe order of a key: the slots of its
+// home bucket cyclically from its preferred one, then the next bucket's
+// likewise, and so on.  Inserts take the first slot of that order that is
+// empty, and slots never empty again (until the index is rebuilt into the
+// other buffer), so a lookup ends at the first bucket with an empty slot.
+struct __align__(16) Slot {
     uint64_t key, pos1;
 };
 
@@ -37,6 +50,15 @@ struct Slot {
 // stamp of the touch.  Records of an instance are in stamp order.
 struct Rec {
     uint64_t key, stamp;
+};
+
+// A touch the commit's first pass could not settle with one CAS at the
+// key's home slot (40 bytes): the key is there with an older position
+// (found = 1, x = the position value seen) or the home slot holds another
+// key (found = 0).  The second pass finishes it.
+struct Deferred {
+    uint64_t key, p, x;     // p: log position of the touch's record
+    uint32_t home, f, found, pad;
 };
 
 // Per-batch values produced on the device.
@@ -83,9 +105,11 @@ struct DevState {
     Slot **table;                   // per id: S slots (null until first add)
     Rec **logbuf;                   // per id: logcap records
     uint8_t **stale;                // per id: logcap flags, 1 = record superseded by a later touch
+    uint32_t **loghome;             // per id: logcap index home slots, one per record
     Slot **table_alt;               // per id: second index buffer (rebuild target)
     Rec **logbuf_alt;               // per id: second log buffer (compaction target)
     uint8_t **stale_alt;
+    uint32_t **loghome_alt;
     uint64_t *log_front, *log_tail, *live, *used;
     uint64_t *touch_cnt;            // per id: blocks touched by the pending commit
     // eviction scratch: per id window plan and cut, per chunk live counts
@@ -106,6 +130,8 @@ struct DevState {
     uint64_t *seg_total, *seg_carry, *plocal;
     uint64_t *seg_total2;           // per segment: f2 digest sum over its blocks < K
     uint32_t *seg_newly, *seg_claims;   // per segment: keys made resident / index slots taken by the commit
+    Deferred *defer;                // kSegBlocks per segment: touches left to the commit's second pass
+    uint32_t *defer_n;              // per segment: deferred touches
     uint32_t *r_c1, *r_c2, *r_h1, *r_h2, *r_final;
     uint64_t *r_touchoff;           // per request: offset among its instance's records of the batch
     uint64_t *log_adv;              // per id: log records the pending batch appends
@@ -121,6 +147,43 @@ struct DevState {
     uint32_t *rb_pos;               // queue position of the candidate
     uint32_t rb_cap;                // candidates that fit (power of two)
 };
+
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch.  The kernels of the routing and commit path
+// begin with pdl_enter(): the stream's next kernel may be launched as soon
+// as all of this kernel's CTAs are running (its CTAs then wait at their own
+// pdl_enter), and nothing here touches memory before the previous kernel
+// has completed with its writes visible.  So the order of the stream is
+// kept and only the launch latency between kernels is hidden.
+__device__ __forceinline__ void pdl_enter() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Return the first failing launch of a launcher function.
+#define DM_TRY(x)                            \
+    do {                                     \
+        const cudaError_t dm_e_ = (x);       \
+        if (dm_e_ != cudaSuccess) return dm_e_; \
+    } while (0)
+
+// Launch a kernel that begins with pdl_enter() with programmatic stream
+// serialization.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
+                              Args... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at{};
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
 
 // ---------------------------------------------------------------------------
 // Published mixers.
@@ -192,18 +255,53 @@ __device__ __forceinline__ Slot load_slot(const Slot *p) {
     return s;
 }
 
-// Look key up in one instance's open-addressed (linear probing) index.
-// Returns 1 + log position of its latest record (0 if the key has no slot).
-__device__ __forceinline__ uint64_t table_pos1(const Slot *t, uint64_t mask, uint64_t key, uint32_t *err) {
-    uint64_t i = key & mask;
-    for (uint64_t it = 0; it <= mask; ++it) {
-        Slot s = load_slot(t + i);
-        if (s.key == key) return s.pos1;
-        if (s.key == 0) return 0;
-        i = (i + 1) & mask;
+// Home slot of block b given its group anchor's key.
+__device__ __forceinline__ uint64_t group_home(uint64_t anchor, uint64_t b, uint64_t mask) {
+    return (anchor & mask & ~uint64_t(kGroup - 1)) | (b & (kGroup - 1));
+}
+
+// Key of the group anchor of the block held by this lane, when consecutive
+// lanes hold consecutive blocks and lane 0 holds a block of group boundary.
+// Whole warp.
+__device__ __forceinline__ uint64_t group_anchor(uint64_t key, int lane) {
+    return __shfl_sync(0xffffffffu, key, lane & ~int(kGroup - 1));
+}
+
+// Look key up in one instance's index from its home slot: its slot index
+// and contents, or kNoSlot.  The home slot is read first (it usually
+// settles the lookup); otherwise whole buckets are read at once.
+constexpr uint64_t kNoSlot = ~0ull;
+__device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uint64_t key, uint64_t home,
+                                               uint32_t *err, Slot *found) {
+    const Slot h = load_slot(t + home);
+    if (h.key == key) { *found = h; return home; }
+    if (h.key == 0) return kNoSlot;
+    uint64_t R = home & ~uint64_t(kGroup - 1);
+    for (uint64_t it = 0; it <= (mask >> 3); ++it) {
+        Slot sn[kGroup];
+#pragma unroll
+        for (int j = 0; j < (int)kGroup; ++j) sn[j] = load_slot(t + R + j);
+        bool empty = false;
+        uint64_t hit = kNoSlot;
+        Slot hs{0, 0};
+#pragma unroll
+        for (int j = 0; j < (int)kGroup; ++j) {
+            if (sn[j].key == key) { hit = R + j; hs = sn[j]; }
+            empty |= sn[j].key == 0;
+        }
+        if (hit != kNoSlot) { *found = hs; return hit; }
+        if (empty) return kNoSlot;
+        R = (R + kGroup) & mask;
     }
     set_err(err, DM_ERR_TIMEOUT);
-    return 0;
+    return kNoSlot;
+}
+
+// 1 + log position of key's latest record (0 if the key has no slot).
+__device__ __forceinline__ uint64_t table_pos1(const Slot *t, uint64_t mask, uint64_t key, uint64_t home,
+                                               uint32_t *err) {
+    Slot s;
+    return table_find(t, mask, key, home, err, &s) == kNoSlot ? 0 : s.pos1;
 }
 
 // Carries of one request's segments (exclusive prefix of the segment

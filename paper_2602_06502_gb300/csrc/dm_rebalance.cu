@@ -122,6 +122,7 @@ __device__ void bitonic_sort(uint64_t *key, uint64_t *seq, uint64_t *tt, uint32_
 __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint64_t seq0, uint32_t call,
                                                     dm_migration *out, uint32_t cap, uint32_t *n_out,
                                                     uint32_t sort_cap) {
+    pdl_enter();
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_w[33];
     __shared__ uint64_t s_u[33];
@@ -354,7 +355,7 @@ cudaError_t launch_rebalance(const DevState &d, uint32_t n, uint64_t seq0, uint3
         if (e != cudaSuccess) return e;
         configured = smem;
     }
-    k_rebalance<<<1, 1024, smem, st>>>(d, n, seq0, call, out, cap, n_out, sort_cap);
+    DM_TRY(launch_pdl(k_rebalance, 1, 1024, smem, st, d, n, seq0, call, out, cap, n_out, sort_cap));
     return cudaGetLastError();
 }
 

@@ -53,6 +53,7 @@ __device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uin
 constexpr int kProbeWarps = 8;
 
 __global__ void __launch_bounds__(kProbeWarps * 32) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
+    pdl_enter();
     __shared__ uint32_t s_c[2];
     __shared__ uint32_t s_miss[2][kProbeWarps];
     if (has_err(d.err)) return;
@@ -84,13 +85,14 @@ __global__ void __launch_bounds__(kProbeWarps * 32) k_route_probe(DevState d, dm
     bool done1 = false, done2 = false;
     uint32_t h1 = 0, h2 = 0;
     for (uint32_t base = 0; !(done1 && done2); base += kRound) {
-        const uint32_t b = base + threadIdx.x;
+        const uint32_t b = base + threadIdx.x;   // base is a multiple of the group size
         const bool inb = b < nblk;
         bool res1 = false, res2 = false;
+        const uint64_t key = inb ? cache_key(d.plocal[bo + b] + d.seg_carry[s0 + b / kSegBlocks], d.Sc) : 0;
+        const uint64_t home = group_home(group_anchor(key, lane), b, mask);
         if (inb) {
-            const uint64_t key = cache_key(d.plocal[bo + b] + d.seg_carry[s0 + b / kSegBlocks], d.Sc);
-            if (!done1) res1 = table_pos1(t1, mask, key, d.err) > f1;
-            if (!done2) res2 = table_pos1(t2, mask, key, d.err) > f2;
+            if (!done1) res1 = table_pos1(t1, mask, key, home, d.err) > f1;
+            if (!done2) res2 = table_pos1(t2, mask, key, home, d.err) > f2;
         }
         const uint32_t m1 = __ballot_sync(0xffffffffu, !res1);
         const uint32_t m2 = __ballot_sync(0xffffffffu, !res2);
@@ -125,7 +127,7 @@ __global__ void __launch_bounds__(kProbeWarps * 32) k_route_probe(DevState d, dm
 cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
                                cudaStream_t st) {
     if (b.n == 0) return cudaSuccess;
-    k_route_probe<<<b.n, kProbeWarps * 32, 0, st>>>(d, o, b.n);
+    DM_TRY(launch_pdl(k_route_probe, b.n, kProbeWarps * 32, 0, st, d, o, b.n));
     return cudaGetLastError();
 }
 

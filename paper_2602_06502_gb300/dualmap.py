@@ -241,7 +241,16 @@ def dm_last_error(h):
     return lib().dm_last_error(h)
 
 
-def dm_set_profiling(h, on):
+DM_PROFILE_ONLY = 0x100
+
+
+def dm_set_profiling(h, on, stages=None):
+    """on: time every stage; stages: names of STAGES to time instead (others untimed)."""
+    if stages is not None:
+        mode = DM_PROFILE_ONLY
+        for name in stages:
+            mode |= 1 << STAGES.index(name)
+        return lib().dm_set_profiling(h, mode)
     return lib().dm_set_profiling(h, 1 if on else 0)
 
 
