@@ -38,7 +38,7 @@ def longctx_handle_kwargs(w):
     """Handle sizes used for the long-context workload (bench and its parity test)."""
     return dict(max_instances=w["n_instances"] + 8, max_batch=w["batch"],
                 max_batch_tokens=w["batch"] * w["len_hi"] + 4 * w["batch"],
-                max_touch_per_instance=1 << 20, index_slots_log2=23)
+                max_touch_per_instance=1 << 20, index_slots_log2=24)
 
 
 def handle_kwargs(w, max_id):
@@ -391,8 +391,8 @@ def main():
     prompt_gbps = bytes_per_launch / ((stage_ms["hash"] + stage_ms["probe"]) / 1e3) / 1e9
     # route: setup, segmap, drain, hash, probe, choice (6); commit: maint_plan, maint_a,
     # compact_scan, maint_c, commit_prep, commit_touch, touch_deferred, req_counts,
-    # evict_plan, evict_count, evict_cut, evict_clear, evict_walk (13); rebalance (1)
-    launches_per_step = 6 + 13 + (1 if w.get("rebalance") else 0)
+    # evict (9); rebalance (1)
+    launches_per_step = 6 + 9 + (1 if w.get("rebalance") else 0)
     clocks = sampler.summary(wall0, wall1)
     g.close()
     del g

@@ -228,6 +228,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         return DM_ERR_INVALID_ARG;
     }
     d.logcap = pow2_at_least(2 * (d.C + d.T));
+    if (d.logcap < 1024) d.logcap = 1024;   // whole 16-byte flag groups (eviction reads flags 16 at a time)
     d.Q = c.max_queue ? c.max_queue : 65536;
     d.rb_cap = (uint32_t)pow2_at_least(d.Q > d.M ? d.Q : d.M);
     // key material: SplitMix64(seed) -> K1[0..B), K2[0..B), G1|1, G2|1, Sc, Sr1, Sr2, Sv1, Sv2
@@ -285,15 +286,6 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.touch_cnt, M));
     A(dalloc(h, &d.log_adv, M));
     A(dalloc(h, &d.log_base, M));
-    A(dalloc(h, &d.ev_excess, M));
-    A(dalloc(h, &d.ev_win, M));
-    A(dalloc(h, &d.ev_front_new, M));
-    A(dalloc(h, &d.ev_rem, M));
-    A(dalloc(h, &d.ev_chunk_off, M + 1));
-    // eviction windows: sum over ids of (2 x excess + 2048) rounded up to chunks,
-    // and excess <= blocks touched by one commit <= max_blocks
-    d.ev_cap = 2 * d.max_blocks + (2048 + 2 * dm::kEvChunk) * M;
-    A(dalloc(h, &d.ev_chunk_live, d.ev_cap / dm::kEvChunk + 1));
     A(dalloc(h, &d.clock, 1));
     A(dalloc(h, &d.err, 1));
     A(dalloc(h, &d.seq_next, 1));

@@ -16,7 +16,11 @@
 // per-key write at all.  Evicted keys keep their index slots until the index
 // passes half full, when it is rebuilt from the log's live records; a log
 // about to overflow is compacted.  Both write into second buffers and swap.
+#include <cooperative_groups.h>
+
 #include "dm_internal.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace dm {
 
@@ -575,16 +579,11 @@ __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
 
 // ---------------------------------------------------------------------------
 // Eviction.  Instance i drops its excess_i = live_i - C oldest resident keys
-// by moving its log front just past the excess_i-th non-stale record:
-//   plan   one CTA: a window of 2*excess_i + 2048 records from the front,
-//          cut into 1024-record chunks;
-//   count  grid over all chunks: non-stale records per chunk;
-//   cut    warp per instance: chunk and record where the count reaches
-//          excess_i;
-//   clear  grid over all chunks: reset the stale flags the front passes;
-//   walk   new fronts; an instance whose window held too few non-stale
-//          records continues record by record after it (rare).
-constexpr int kEvThreads = 256;
+// by moving its log front just past the excess_i-th non-stale record; the
+// stale flags it passes are reset (those positions will hold new records).
+// One CTA per instance walks its log from the front, 16 records per thread
+// and round (one 16-byte load of flags), with a block scan of the non-stale
+// counts locating the cut.
 
 // Warp per request: sum the touch kernel's counts over the request's
 // (contiguous) segments, one atomic per request and counter.
@@ -610,185 +609,151 @@ __global__ void k_req_counts(DevState d, uint32_t n) {
     }
 }
 
-__global__ void __launch_bounds__(1024) k_evict_plan(DevState d) {
+constexpr int kEvThreads = 1024;
+constexpr uint32_t kEvCluster = 4;                                // CTAs sharing one instance's walk
+constexpr uint32_t kEvVec = 4;                                    // 16-byte flag loads per thread and round
+constexpr uint32_t kEvPer = 16 * kEvVec;                          // records per thread and round
+constexpr uint64_t kEvCtaSpan = uint64_t(kEvThreads) * kEvPer;    // records per CTA and round
+constexpr uint64_t kEvRound = kEvCtaSpan * kEvCluster;            // records per cluster and round
+
+// A cluster of kEvCluster CTAs per instance (persistent: clusters loop over
+// instances).  Per round each CTA counts the non-stale records of its own
+// span and posts the count in shared memory; after one cluster barrier every
+// CTA reads all counts (distributed shared memory) and knows whether its
+// span lies wholly before the cut (reset all its flags), holds it (find the
+// exact record, reset up to it, write the new front) or lies after it.  The
+// posted counts alternate between two slots, so one barrier per round
+// suffices: a CTA cannot rewrite a slot before every CTA has passed the next
+// barrier, which it reaches only after reading that slot.
+__global__ void __cluster_dims__(kEvCluster, 1, 1) __launch_bounds__(kEvThreads) k_evict(DevState d) {
     pdl_enter();
+    cg::cluster_group cluster = cg::this_cluster();
     __shared__ uint32_t s_w[33];
-    if (has_err(d.err)) return;
-    uint32_t carry = 0;
-    for (uint32_t base = 0; base < d.M; base += blockDim.x) {
-        const uint32_t i = base + threadIdx.x;
-        uint64_t excess = 0, win = 0;
-        if (i < d.M && d.table[i] && d.live[i] > d.C) {
-            excess = d.live[i] - d.C;
-            win = min(d.log_tail[i] - d.log_front[i], 2 * excess + 2048);
-        }
-        const uint32_t chunks = (uint32_t)((win + kEvChunk - 1) / kEvChunk);
-        uint32_t tot;
-        const uint32_t ex = block_excl_u32(chunks, s_w, tot);
-        if (i < d.M) {
-            d.ev_chunk_off[i] = carry + ex;
-            d.ev_excess[i] = excess;
-            d.ev_win[i] = win;
-            d.ev_rem[i] = 0;
-            d.ev_front_new[i] = d.log_front[i];
-        }
-        carry += tot;
-    }
-    if (threadIdx.x == 0) {
-        d.ev_chunk_off[d.M] = carry;
-        d.info->ev_chunks = carry;
-        if (uint64_t(carry) * kEvChunk > d.ev_cap) set_err(d.err, DM_ERR_CAPACITY);
-    }
-}
-
-__global__ void __launch_bounds__(kEvThreads) k_evict_count(DevState d) {
-    pdl_enter();
-    __shared__ uint32_t s_i;
-    __shared__ uint32_t s_cnt[kEvThreads / 32];
-    if (has_err(d.err)) return;
-    const uint32_t nchunks = d.info->ev_chunks;
+    __shared__ uint32_t s_tot[2], s_go;
+    __shared__ uint64_t s_cut;
+    const uint32_t r = cluster.block_rank();
+    const uint32_t cid = blockIdx.x / kEvCluster, ncl = gridDim.x / kEvCluster;
+    // one decision for the whole cluster (rank 0's view of the error word)
+    if (threadIdx.x == 0) s_go = !has_err(d.err);
+    cluster.sync();
+    const uint32_t go = *cluster.map_shared_rank(&s_go, 0);
     const uint64_t lmask = d.logcap - 1;
-    for (uint32_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
-        if (threadIdx.x == 0) s_i = owner_of(d.ev_chunk_off, d.M, c);
-        __syncthreads();
-        const uint32_t i = s_i;
-        const uint64_t front = d.log_front[i];
-        const uint64_t end = front + d.ev_win[i];
-        const uint64_t base = front + uint64_t(c - d.ev_chunk_off[i]) * kEvChunk;
-        const uint8_t *st = d.stale[i];
-        uint32_t cnt = 0;
-        for (uint32_t k = threadIdx.x; k < kEvChunk; k += kEvThreads)
-            cnt += (base + k < end && !st[(base + k) & lmask]);
-        cnt = __reduce_add_sync(0xffffffffu, cnt);
-        if ((threadIdx.x & 31) == 0) s_cnt[threadIdx.x >> 5] = cnt;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            uint32_t tot = 0;
-            for (int w = 0; w < kEvThreads / 32; ++w) tot += s_cnt[w];
-            d.ev_chunk_live[c] = tot;
-        }
-        __syncthreads();
-    }
-}
-
-// Warp per instance: locate the record where the non-stale count reaches excess.
-__global__ void k_evict_cut(DevState d) {
-    pdl_enter();
-    if (has_err(d.err)) return;
-    const int lane = threadIdx.x & 31;
-    const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (i >= d.M) return;
-    const uint64_t excess = d.ev_excess[i];
-    if (excess == 0) return;
-    const uint32_t c0 = d.ev_chunk_off[i], c1 = d.ev_chunk_off[i + 1];
-    uint64_t cum = 0;
-    uint32_t cstar = c1;
-    uint64_t need = 0;
-    for (uint32_t cb = c0; cb < c1 && cstar == c1; cb += 32) {
-        const uint32_t c = cb + lane;
-        const uint64_t v = c < c1 ? d.ev_chunk_live[c] : 0;
-        const uint64_t inc = warp_incl_scan(v, lane) + cum;
-        const uint32_t hit = __ballot_sync(0xffffffffu, c < c1 && inc >= excess);
-        if (hit) {
-            const int l = __ffs(hit) - 1;
-            cstar = cb + l;
-            need = excess - (shfl_u64(inc, l) - shfl_u64(v, l));   // non-stale records needed in cstar
-        } else {
-            cum = shfl_u64(inc, 31);
-        }
-    }
-    const uint64_t front = d.log_front[i];
-    if (cstar == c1) {   // window too short: the walker continues after it
-        if (lane == 0) {
-            d.ev_front_new[i] = front + d.ev_win[i];
-            d.ev_rem[i] = excess - cum;
-        }
-        return;
-    }
-    // lane l owns records 32l .. 32l+31 of chunk cstar
-    const uint64_t cbase = front + uint64_t(cstar - c0) * kEvChunk + 32 * lane;
-    const uint64_t end = front + d.ev_win[i];
-    const uint8_t *st = d.stale[i];
-    uint32_t mbits = 0;
-#pragma unroll 8
-    for (int b = 0; b < 32; ++b) {
-        const uint64_t p = cbase + b;
-        mbits |= ((p < end && !st[p & (d.logcap - 1)]) ? 1u : 0u) << b;
-    }
-    const uint32_t cnt = __popc(mbits);
-    uint32_t inc = cnt;
-#pragma unroll
-    for (int dd = 1; dd < 32; dd <<= 1) {
-        const uint32_t u = __shfl_up_sync(0xffffffffu, inc, dd);
-        if (lane >= dd) inc += u;
-    }
-    const uint32_t ex = inc - cnt;
-    if (ex < need && need <= inc)   // exactly one lane
-        d.ev_front_new[i] = cbase + __fns(mbits, 0, (int)(need - ex)) + 1;
-}
-
-// Reset the stale flags of the records the front passes (those positions
-// will hold new records).
-__global__ void __launch_bounds__(kEvThreads) k_evict_clear(DevState d) {
-    pdl_enter();
-    __shared__ uint32_t s_i;
-    if (has_err(d.err)) return;
-    const uint32_t nchunks = d.info->ev_chunks;
-    const uint64_t lmask = d.logcap - 1;
-    for (uint32_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
-        if (threadIdx.x == 0) s_i = owner_of(d.ev_chunk_off, d.M, c);
-        __syncthreads();
-        const uint32_t i = s_i;
-        const uint64_t front = d.log_front[i];
-        const uint64_t cut = d.ev_front_new[i];
-        const uint64_t base = front + uint64_t(c - d.ev_chunk_off[i]) * kEvChunk;
+    uint32_t slot = 0;
+    for (uint32_t i = cid; go && i < d.M; i += ncl) {
+        if (!d.table[i] || d.live[i] <= d.C) continue;   // read alike by every CTA of the cluster
+        uint64_t remaining = d.live[i] - d.C;
         uint8_t *st = d.stale[i];
-        for (uint32_t k = threadIdx.x; k < kEvChunk; k += kEvThreads)
-            if (base + k < cut) st[(base + k) & lmask] = 0;
-        __syncthreads();
-    }
-}
-
-__global__ void __launch_bounds__(1024) k_evict_walk(DevState d) {
-    pdl_enter();
-    __shared__ uint32_t s_w[33];
-    __shared__ uint64_t s_front;
-    if (has_err(d.err)) return;
-    const uint32_t i = blockIdx.x;
-    if (d.ev_excess[i] == 0) return;
-    uint64_t remaining = d.ev_rem[i];
-    uint64_t front = d.ev_front_new[i];
-    if (remaining == 0) {
-        if (threadIdx.x == 0) {
-            d.log_front[i] = front;
+        const uint64_t tail = d.log_tail[i];
+        const uint64_t front0 = d.log_front[i];
+        uint64_t front = front0;
+        // rounds start on kEvPer-record boundaries (flags are read 16 at a
+        // time; logcap is a power of two >= kEvPer); records before the
+        // front in the first round do not count
+        uint64_t base = front & ~uint64_t(kEvPer - 1);
+        for (uint64_t it = 0; remaining > 0 && base < tail && it < kSpinLimit; ++it) {
+            const uint64_t p0 = base + r * kEvCtaSpan + uint64_t(threadIdx.x) * kEvPer;
+            // records [lo, hi) of the thread's kEvPer are after the front and before the tail
+            const uint32_t lo = front > p0 ? (uint32_t)min(front - p0, (uint64_t)kEvPer) : 0u;
+            const uint32_t hi = tail > p0 ? (uint32_t)min(tail - p0, (uint64_t)kEvPer) : 0u;
+            uint64_t live_bits = 0;
+#pragma unroll
+            for (uint32_t k = 0; k < kEvVec; ++k) {
+                if (16 * k >= hi) continue;
+                const uint4 v = *reinterpret_cast<const uint4 *>(st + ((p0 + 16 * k) & lmask));
+                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    // bit j of the nibble: flag byte j of the word is 0
+                    const uint32_t z = __vcmpeq4(w[q], 0u) & 0x01010101u;
+                    live_bits |= uint64_t((z * 0x10204080u) >> 28) << (16 * k + 4 * q);
+                }
+            }
+            const uint64_t below_hi = hi >= 64 ? ~0ull : (1ull << hi) - 1;
+            const uint64_t below_lo = lo >= 64 ? ~0ull : (1ull << lo) - 1;
+            live_bits &= below_hi & ~below_lo;
+            const uint32_t cnt = __popcll(live_bits);
+            uint32_t tot;
+            const uint32_t ex = block_excl_u32(cnt, s_w, tot);
+            if (threadIdx.x == 0) s_tot[slot] = tot;
+            cluster.sync();   // every span's count is visible
+            uint64_t pre = 0, all = 0;
+#pragma unroll
+            for (uint32_t q = 0; q < kEvCluster; ++q) {
+                const uint32_t t = *cluster.map_shared_rank(&s_tot[slot], q);
+                pre += q < r ? t : 0;
+                all += t;
+            }
+            slot ^= 1;
+            // end of the records this span evicts: all of them, up to the
+            // cut, or none
+            uint64_t cut;
+            if (pre + tot < remaining) {
+                cut = ~0ull;
+            } else if (pre < remaining) {
+                const uint64_t need = remaining - pre;
+                if (threadIdx.x == 0) s_cut = ~0ull;
+                __syncthreads();
+                if (ex < need && need <= ex + cnt) {   // exactly one thread
+                    const uint32_t lw = (uint32_t)live_bits, nlo = __popc(lw);
+                    const uint32_t m = (uint32_t)(need - ex);
+                    const uint32_t bit =
+                        m <= nlo ? __fns(lw, 0, (int)m) : 32 + __fns((uint32_t)(live_bits >> 32), 0, (int)(m - nlo));
+                    s_cut = p0 + bit + 1;
+                }
+                __syncthreads();
+                cut = s_cut;
+                if (threadIdx.x == 0) d.log_front[i] = cut;
+            } else {
+                cut = 0;
+            }
+            // reset the flags of the records the front passes: [lo, b) of the thread's
+            {
+                const uint32_t b = cut > p0 ? (uint32_t)min(cut - p0, (uint64_t)hi) : 0u;
+#pragma unroll
+                for (uint32_t k = 0; k < kEvVec; ++k) {
+                    const uint32_t k0 = 16 * k, k1 = k0 + 16;
+                    if (k1 <= lo || k0 >= b) continue;
+                    uint8_t *f = st + ((p0 + k0) & lmask);
+                    if (lo <= k0 && k1 <= b) {
+                        *reinterpret_cast<uint4 *>(f) = make_uint4(0, 0, 0, 0);
+                    } else {
+                        for (uint32_t q = max(lo, k0); q < min(b, k1); ++q) f[q - k0] = 0;
+                    }
+                }
+            }
+            remaining -= min(remaining, all);
+            base += kEvRound;
+            front = min(base, tail);
+        }
+        if (r == 0 && threadIdx.x == 0) {
+            if (remaining) {   // the log must cover every live key
+                set_err(d.err, DM_ERR_TIMEOUT);
+                d.log_front[i] = front;
+            }
             d.live[i] = d.C;
         }
-        return;
     }
-    uint8_t *st = d.stale[i];
-    const uint64_t lmask = d.logcap - 1;
-    const uint64_t tail = d.log_tail[i];
-    while (remaining > 0 && front < tail) {
-        const uint64_t p = front + threadIdx.x;
-        const bool live = p < tail && !st[p & lmask];
-        uint32_t tot;
-        const uint32_t rk = block_excl_u32(live ? 1u : 0u, s_w, tot);
-        if (threadIdx.x == 0) s_front = min(front + blockDim.x, tail);
-        __syncthreads();
-        if (live && rk == remaining - 1) s_front = p + 1;
-        __syncthreads();
-        const uint64_t nf = s_front;
-        if (p < nf) st[p & lmask] = 0;
-        front = nf;
-        remaining -= remaining < (uint64_t)tot ? remaining : (uint64_t)tot;
-        __syncthreads();
+    cluster.sync();   // no CTA leaves while another may still read its shared memory
+}
+
+// Clusters of the eviction kernel that can be resident at once (CTAs).
+static int evict_grid() {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(kEvCluster);
+    cfg.blockDim = dim3(kEvThreads);
+    cudaLaunchAttribute at{};
+    at.id = cudaLaunchAttributeClusterDimension;
+    at.val.clusterDim.x = kEvCluster;
+    at.val.clusterDim.y = 1;
+    at.val.clusterDim.z = 1;
+    cfg.attrs = &at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k_evict, &cfg) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = 1;
     }
-    if (threadIdx.x == 0) {
-        if (remaining) set_err(d.err, DM_ERR_TIMEOUT);   // the log must cover every live key
-        d.log_front[i] = front;
-        d.live[i] = d.C;
-        d.ev_rem[i] = 0;
-    }
+    return n * (int)kEvCluster;
 }
 
 cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
@@ -804,9 +769,8 @@ cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
         configured = smem;
     }
     static const int g_a = full_grid(k_maint_a, kMtThreads), g_c = full_grid(k_maint_c, kMtThreads),
-                     g_t = full_grid(k_commit_touch, kTouchThreads), g_ec = full_grid(k_evict_count, kEvThreads),
-                     g_d = full_grid(k_touch_deferred, 256),
-                     g_el = full_grid(k_evict_clear, kEvThreads);
+                     g_t = full_grid(k_commit_touch, kTouchThreads),
+                     g_d = full_grid(k_touch_deferred, 256), g_ev = evict_grid();
     DM_TRY(launch_pdl(k_maint_plan, 1, 1024, smem, st, d, n));
     DM_TRY(launch_pdl(k_maint_a, g_a, kMtThreads, 0, st, d));
     DM_TRY(launch_pdl(k_compact_scan, (d.M + 7) / 8, 256, 0, st, d));
@@ -815,11 +779,7 @@ cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
     DM_TRY(launch_pdl(k_commit_touch, g_t, kTouchThreads, 0, st, d));
     DM_TRY(launch_pdl(k_touch_deferred, g_d, 256, 0, st, d));
     DM_TRY(launch_pdl(k_req_counts, (n + 7) / 8, 256, 0, st, d, n));
-    DM_TRY(launch_pdl(k_evict_plan, 1, 1024, 0, st, d));
-    DM_TRY(launch_pdl(k_evict_count, g_ec, kEvThreads, 0, st, d));
-    DM_TRY(launch_pdl(k_evict_cut, (d.M + 7) / 8, 256, 0, st, d));
-    DM_TRY(launch_pdl(k_evict_clear, g_el, kEvThreads, 0, st, d));
-    DM_TRY(launch_pdl(k_evict_walk, d.M, 1024, 0, st, d));
+    DM_TRY(launch_pdl(k_evict, g_ev, kEvThreads, 0, st, d));
     return cudaGetLastError();
 }
 

@@ -68,7 +68,6 @@ struct BatchInfo {
     uint32_t n;
     uint64_t clock_base;    // commit clock before this batch's touches
     uint32_t final_dirty;   // a rebalance moved a request of this batch
-    uint32_t ev_chunks;     // eviction window chunks of this commit
     uint32_t mc_chunks;     // log-compaction chunks of this commit
     uint32_t mr_chunks;     // index-rebuild chunks of this commit
     uint32_t pad;
@@ -112,11 +111,6 @@ struct DevState {
     uint32_t **loghome_alt;
     uint64_t *log_front, *log_tail, *live, *used;
     uint64_t *touch_cnt;            // per id: blocks touched by the pending commit
-    // eviction scratch: per id window plan and cut, per chunk live counts
-    uint64_t *ev_excess, *ev_win, *ev_front_new, *ev_rem;
-    uint32_t *ev_chunk_off;         // M + 1 entries
-    uint32_t *ev_chunk_live;
-    uint64_t ev_cap;                // window records that fit (chunks * kEvChunk)
     // maintenance plan: per id flags / new log tail, chunk offsets and counts
     uint32_t *mt_flags;
     uint64_t *mt_newtail;
