@@ -52,7 +52,7 @@ __device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uin
 // the smallest missing block over the warps ends that candidate's run.
 constexpr int kProbeWarps = 8;
 
-__global__ void __launch_bounds__(kProbeWarps * 32) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
+__global__ void __launch_bounds__(kProbeWarps * 32, 4) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
     pdl_enter();
     __shared__ uint32_t s_c[2];
     __shared__ uint32_t s_miss[2][kProbeWarps];
