@@ -60,7 +60,8 @@ __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
 __device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint64_t home,
                                                   Slot old, uint32_t *err, bool *claimed) {
     const uint32_t o = (uint32_t)(home & (kGroup - 1));
-    uint64_t R = home & ~uint64_t(kGroup - 1), i = home;
+    const uint64_t R0 = home & ~uint64_t(kGroup - 1);
+    uint64_t R = R0, i = home, nbk = 0;   // nbk: position of bucket R in the probe order
     uint32_t step = 0;   // order position of slot i within bucket R
     // at most one probe step per slot, and one retry per other touch of the
     // key in the batch (each failed retry means another touch got in)
@@ -90,7 +91,7 @@ __device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64
         if (best < kGroup) {
             step = best;
         } else {
-            R = (R + kGroup) & mask;
+            R = probe_bucket(++nbk, R0, key, mask);
             step = 0;
             bs = Slot{0, 0};
         }

@@ -38,10 +38,15 @@ struct QEntry {
 // line: one random DRAM access instead of 8 (random single-slot atomics
 // saturate far below line-local ones).  A key fixes its whole prefix and so
 // its anchor: every key has one home.  Probe order of a key: the slots of its
-// home bucket cyclically from its preferred one, then the next bucket's
-// likewise, and so on.  Inserts take the first slot of that order that is
-// empty, and slots never empty again (until the index is rebuilt into the
-// other buffer), so a lookup ends at the first bucket with an empty slot.
+// home bucket cyclically from its preferred one; then those of the next
+// kLinearBuckets - 1 buckets (a group displaced from a full home bucket
+// moves on together, within a few hundred bytes); then the buckets from one
+// chosen by the key's own hash onwards, each likewise.  (Prompts that share
+// a prefix but diverge inside a group share that group's anchor: past the
+// first buckets the key hash spreads their overflow instead of piling it up.)
+// Inserts take the first slot of that order that is empty, and slots never
+// empty again (until the index is rebuilt into the other buffer), so a
+// lookup ends at the first bucket with an empty slot.
 struct __align__(16) Slot {
     uint64_t key, pos1;
 };
@@ -254,6 +259,15 @@ __device__ __forceinline__ uint64_t group_home(uint64_t anchor, uint64_t b, uint
     return (anchor & mask & ~uint64_t(kGroup - 1)) | (b & (kGroup - 1));
 }
 
+// Bucket j >= 1 of the probe order of key (bucket 0 is its home bucket R0):
+// the buckets after R0 while j < kLinearBuckets, then the bucket chosen by
+// the key's hash and those after it.
+constexpr uint64_t kLinearBuckets = 2;
+__device__ __forceinline__ uint64_t probe_bucket(uint64_t j, uint64_t R0, uint64_t key, uint64_t mask) {
+    if (j < kLinearBuckets) return (R0 + j * kGroup) & mask;
+    return ((fmix64(key) & mask & ~uint64_t(kGroup - 1)) + (j - kLinearBuckets) * kGroup) & mask;
+}
+
 // Key of the group anchor of the block held by this lane, when consecutive
 // lanes hold consecutive blocks and lane 0 holds a block of group boundary.
 // Whole warp.
@@ -270,8 +284,9 @@ __device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uin
     const Slot h = load_slot(t + home);
     if (h.key == key) { *found = h; return home; }
     if (h.key == 0) return kNoSlot;
-    uint64_t R = home & ~uint64_t(kGroup - 1);
-    for (uint64_t it = 0; it <= (mask >> 3); ++it) {
+    const uint64_t R0 = home & ~uint64_t(kGroup - 1);
+    uint64_t R = R0;
+    for (uint64_t j = 1; j <= (mask >> 3) + kLinearBuckets + 1; ++j) {
         Slot sn[kGroup];
 #pragma unroll
         for (int j = 0; j < (int)kGroup; ++j) sn[j] = load_slot(t + R + j);
@@ -285,7 +300,7 @@ __device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uin
         }
         if (hit != kNoSlot) { *found = hs; return hit; }
         if (empty) return kNoSlot;
-        R = (R + kGroup) & mask;
+        R = probe_bucket(j, R0, key, mask);
     }
     set_err(err, DM_ERR_TIMEOUT);
     return kNoSlot;
