@@ -74,15 +74,17 @@ def file_sha(p):
         return hashlib.sha256(f.read()).hexdigest()
 
 
-def traffic_per_launch():
-    """DRAM bytes per hashing launch from the committed ncu capture, or None
-    when the kernel source changed since it was taken."""
+def traffic_per_launch(token_bytes):
+    """DRAM bytes (read + write) per hashing launch of `token_bytes` of
+    prompts, scaled from the committed ncu capture of one full-size batch
+    (traffic grows in proportion to the tokens hashed); None when the kernel
+    source changed since the capture was taken."""
     try:
         with open(TRAFFIC_FILE) as f:
             t = json.load(f)
         if t.get("dm_hash_sha256") != file_sha(HASH_SRC):
             return None
-        return float(t["bytes_per_launch_full_batch"])
+        return float(t["dram_bytes_per_launch"]) * token_bytes / float(t["batch_token_bytes"])
     except Exception:
         return None
 
@@ -427,7 +429,7 @@ def main():
                        "replay": "steps beyond the trace replay its batches cyclically" if W + K > nb else "none"},
             "roofline": {"bound": "hbm", "kernel": "k_hash (prompt hashing)", "achieved": achieved,
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": traffic_per_launch(), "bytes_per_launch": bytes_per_launch,
+                         "traffic": traffic_per_launch(bytes_per_launch), "bytes_per_launch": bytes_per_launch,
                          "avg_launch_ms": hash_avg_s * 1e3},
             "stage_ms_per_step": stage_ms,
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches_per_step * K, "clocks": clocks,

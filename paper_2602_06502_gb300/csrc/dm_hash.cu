@@ -155,7 +155,7 @@ __device__ __forceinline__ uint64_t reduce_scatter(uint64_t (&p)[U], int q) {
 // holds block (l%U)*(32/U) + l/U; one shuffle puts block m on lane m for the
 // scan.  Segments below K also sum their f2 digests (blocks < K).
 template <int U>
-__global__ void __launch_bounds__(256) k_hash(DevState d, const uint32_t *__restrict__ tokens) {
+__global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__restrict__ tokens) {
     pdl_enter();
     constexpr int IT = kSegBlocks / 32;
     if (has_err(d.err)) return;
