@@ -391,10 +391,10 @@ def main():
     assert g.last_error() == 0
     stage_ms = {k: v[0] / max(v[1], 1) for k, v in st_all.items()}
     prompt_gbps = bytes_per_launch / ((stage_ms["hash"] + stage_ms["probe"]) / 1e3) / 1e9
-    # route: setup, segmap, drain, hash, probe, choice (6); commit: maint_plan, maint_a,
-    # compact_scan, maint_c, commit_prep, commit_touch, touch_deferred, req_counts,
-    # evict (9); rebalance (1)
-    launches_per_step = 6 + 9 + (1 if w.get("rebalance") else 0)
+    # route: setup (with the queue drain), segmap, hash, probe, choice (5); commit:
+    # maint_plan, maint_a, compact_scan, maint_c, commit_prep, commit_touch,
+    # touch_deferred, req_counts, evict (9); rebalance (1)
+    launches_per_step = 5 + 9 + (1 if w.get("rebalance") else 0)
     clocks = sampler.summary(wall0, wall1)
     g.close()
     del g

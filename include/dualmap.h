@@ -142,7 +142,8 @@ typedef struct {
 /* Stages timed by dm_get_stage_times. */
 enum {
     DM_STAGE_SETUP = 0,    /* batch validation and per-request prefix sums */
-    DM_STAGE_DRAIN = 1,    /* queue draining to the batch time */
+    DM_STAGE_DRAIN = 1,    /* queue draining to the batch time (runs inside the setup
+                              stage's kernel, so it is timed there; 0 calls) */
     DM_STAGE_HASH = 2,     /* token hashing into chained block prefix values */
     DM_STAGE_PROBE = 3,    /* ring lookup, distinct fix, cache probes */
     DM_STAGE_CHOICE = 4,   /* sequential SLO-aware choice */

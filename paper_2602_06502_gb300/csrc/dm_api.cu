@@ -523,8 +523,7 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
     h->have_time = true;
     const DevState &d = h->d;
     cudaError_t e;
-    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup(d, *b, h->st); }
-    if (e == cudaSuccess) { Stage st(h, DM_STAGE_DRAIN); e = dm::launch_drain(d, delta, h->st); }
+    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_drain(d, *b, delta, h->st); }   // drain included
     if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_HASH); e = dm::launch_hash(d, *b, h->hash_grid, h->st); }
     if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_PROBE); e = dm::launch_route_probe(d, *b, *o, h->st); }
     if (e == cudaSuccess && b->n) {

@@ -15,53 +15,6 @@
 
 namespace dm {
 
-// One warp per instance: run `delta` us of work off the queue head.
-__global__ void k_drain(DevState d, uint64_t delta) {
-    pdl_enter();
-    if (has_err(d.err)) return;
-    const int lane = threadIdx.x & 31;
-    const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (i >= d.M) return;
-    uint32_t head = d.q_head[i];
-    const uint32_t tail = d.q_tail[i];
-    if (head == tail) return;
-    const QEntry *qb = d.q + uint64_t(i) * d.Q;
-    uint64_t left = delta, used = 0;
-    while (head != tail) {
-        const uint32_t cnt = min(32u, tail - head);
-        const uint32_t idx = (head + lane) & (d.Q - 1);
-        const uint64_t rem = (uint32_t)lane < cnt ? qb[idx].remaining : 0;
-        const uint64_t inc = warp_incl_scan(rem, lane);
-        const uint32_t done = __ballot_sync(0xffffffffu, (uint32_t)lane < cnt && inc <= left);
-        const uint32_t ndone = __popc(done);   // a prefix of the lanes
-        if (ndone == cnt) {                    // whole chunk drained
-            const uint64_t tot = shfl_u64(inc, 31);
-            left -= tot;
-            used += tot;
-            head += cnt;
-            continue;
-        }
-        const uint64_t before = ndone ? shfl_u64(inc, ndone - 1) : 0;
-        if ((uint32_t)lane == ndone) {
-            const uint64_t take = left - before;   // < rem of this entry
-            d.q[uint64_t(i) * d.Q + idx].remaining = rem - take;
-        }
-        used += left;
-        left = 0;
-        head += ndone;
-        break;
-    }
-    if (lane == 0) {
-        d.q_head[i] = head;
-        d.W[i] -= used;
-    }
-}
-
-cudaError_t launch_drain(const DevState &d, uint64_t delta, cudaStream_t st) {
-    const uint32_t warps = 8;
-    DM_TRY(launch_pdl(k_drain, (d.M + warps - 1) / warps, warps * 32, 0, st, d, delta));
-    return cudaGetLastError();
-}
 
 constexpr uint32_t kChoiceChunk = 1024;
 

@@ -51,13 +51,20 @@ __device__ __forceinline__ void block_scan2(uint64_t a, uint32_t b, uint64_t &ea
     __syncthreads();
 }
 
-// Validate the batch and lay out per-request block / segment offsets.
+// CTA 0: validate the batch and lay out per-request block / segment
+// offsets.  CTAs 1.. (routing only): drain the queues by `delta` us, a warp
+// per instance (independent of the batch layout).
 __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off, const uint32_t *len,
-                                                uint32_t n, uint64_t total_tokens) {
+                                                uint32_t n, uint64_t total_tokens, uint64_t delta) {
     pdl_enter();
     __shared__ uint64_t sa[32];
     __shared__ uint32_t sb[32];
     if (has_err(d.err)) return;
+    if (blockIdx.x > 0) {
+        const uint32_t i = (blockIdx.x - 1) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+        if (i < d.M) drain_queue(d, i, delta, threadIdx.x & 31);
+        return;
+    }
     uint64_t carry_blk = 0;
     uint32_t carry_seg = 0;
     bool bad = false;
@@ -110,7 +117,14 @@ __global__ void k_segmap(DevState d, uint32_t n) {
 }
 
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st) {
-    DM_TRY(launch_pdl(k_setup, 1, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens));
+    DM_TRY(launch_pdl(k_setup, 1, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens, uint64_t(0)));
+    if (b.n) DM_TRY(launch_pdl(k_segmap, (b.n + 7) / 8, 256, 0, st, d, b.n));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, cudaStream_t st) {
+    const unsigned drain_ctas = (d.M + 31) / 32;
+    DM_TRY(launch_pdl(k_setup, 1 + drain_ctas, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens, delta));
     if (b.n) DM_TRY(launch_pdl(k_segmap, (b.n + 7) / 8, 256, 0, st, d, b.n));
     return cudaGetLastError();
 }

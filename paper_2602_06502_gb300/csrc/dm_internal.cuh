@@ -346,6 +346,44 @@ __device__ __forceinline__ void route_positions(const DevState &d, uint32_t r, i
     pos2 = fmix64(p2 ^ d.Sr2);
 }
 
+// Run `delta` us of prefill work off the head of instance i's queue (Sec.
+// 3.2: an instance's load is its pending prefill work).  Whole warp.
+__device__ __forceinline__ void drain_queue(const DevState &d, uint32_t i, uint64_t delta, int lane) {
+    uint32_t head = d.q_head[i];
+    const uint32_t tail = d.q_tail[i];
+    if (head == tail) return;
+    const QEntry *qb = d.q + uint64_t(i) * d.Q;
+    uint64_t left = delta, used = 0;
+    while (head != tail) {
+        const uint32_t cnt = min(32u, tail - head);
+        const uint32_t idx = (head + lane) & (d.Q - 1);
+        const uint64_t rem = (uint32_t)lane < cnt ? qb[idx].remaining : 0;
+        const uint64_t inc = warp_incl_scan(rem, lane);
+        const uint32_t done = __ballot_sync(0xffffffffu, (uint32_t)lane < cnt && inc <= left);
+        const uint32_t ndone = __popc(done);   // a prefix of the lanes
+        if (ndone == cnt) {                    // whole chunk drained
+            const uint64_t tot = shfl_u64(inc, 31);
+            left -= tot;
+            used += tot;
+            head += cnt;
+            continue;
+        }
+        const uint64_t before = ndone ? shfl_u64(inc, ndone - 1) : 0;
+        if ((uint32_t)lane == ndone) {
+            const uint64_t take = left - before;   // < rem of this entry
+            d.q[uint64_t(i) * d.Q + idx].remaining = rem - take;
+        }
+        used += left;
+        left = 0;
+        head += ndone;
+        break;
+    }
+    if (lane == 0) {
+        d.q_head[i] = head;
+        d.W[i] -= used;
+    }
+}
+
 // Grid of a grid-stride kernel: every SM filled to the kernel's occupancy.
 template <typename K>
 inline int full_grid(K kernel, int block) {
@@ -359,7 +397,7 @@ inline int full_grid(K kernel, int block) {
 // ---------------------------------------------------------------------------
 // Host-side launchers (one translation unit each).
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st);
-cudaError_t launch_drain(const DevState &d, uint64_t delta, cudaStream_t st);
+cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, cudaStream_t st);
 cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st);
 int hash_grid_size();
 cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
