@@ -282,6 +282,15 @@ DM_API dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos_host, uint32
 /* Value of the global commit clock (number of block touches so far). */
 DM_API dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host);
 
+/* Housekeeping of the per-instance cache indices since dm_create: how many
+ * times an instance's key index was rebuilt (it would have passed half full,
+ * counting the slots evicted keys keep) and how many times an instance's
+ * recency log was compacted (it would have overflowed).  The paper has no
+ * counterpart (its per-instance metadata store is opaque); neither changes
+ * any routing result.  For tests and monitoring; read-only, synchronous,
+ * works after a sticky error. */
+DM_API dm_status dm_get_maint_counts(dm_handle *h, uint64_t *rebuilds_host, uint64_t *compactions_host);
+
 /* Synchronise the stream and return the sticky error (DM_OK if none). */
 DM_API dm_status dm_last_error(dm_handle *h);
 

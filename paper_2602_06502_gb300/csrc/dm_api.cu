@@ -287,6 +287,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.log_adv, M));
     A(dalloc(h, &d.log_base, M));
     A(dalloc(h, &d.clock, 1));
+    A(dalloc(h, &d.maint_count, 2));
     A(dalloc(h, &d.err, 1));
     A(dalloc(h, &d.seq_next, 1));
     A(dalloc(h, &d.rb_key, d.rb_cap));
@@ -350,6 +351,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(cudaMemsetAsync(d.live, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.used, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.clock, 0, 8, h->st));
+    A(cudaMemsetAsync(d.maint_count, 0, 16, h->st));
     A(cudaMemsetAsync(d.err, 0, 4, h->st));
     A(cudaMemsetAsync(h->d.info, 0, sizeof(dm::BatchInfo), h->st));
     A(cudaMemsetAsync(h->dh.info, 0, sizeof(dm::BatchInfo), h->st));
@@ -739,6 +741,19 @@ dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host) {
     cudaError_t e = cudaMemcpyAsync(clock_host, h->d.clock, 8, cudaMemcpyDeviceToHost, h->st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
     return map_cuda(h, e);
+}
+
+dm_status dm_get_maint_counts(dm_handle *h, uint64_t *rebuilds_host, uint64_t *compactions_host) {
+    dm_status s = check_handle(h);
+    if (s) return s;
+    if (!rebuilds_host || !compactions_host) return DM_ERR_INVALID_ARG;
+    uint64_t c[2] = {0, 0};
+    cudaError_t e = cudaMemcpyAsync(c, h->d.maint_count, 16, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    *rebuilds_host = c[0];
+    *compactions_host = c[1];
+    return DM_OK;
 }
 
 dm_status dm_last_error(dm_handle *h) {

@@ -365,12 +365,14 @@ __global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
             d.loghome[i] = d.loghome_alt[i];
             d.loghome_alt[i] = hm;
             d.log_tail[i] = d.mt_newtail[i];
+            atomicAdd(reinterpret_cast<unsigned long long *>(&d.maint_count[1]), 1ull);
         }
         if (fl & kFlagRebuild) {
             Slot *a = d.table[i];
             d.table[i] = d.table_alt[i];
             d.table_alt[i] = a;
             d.used[i] = d.live[i];
+            atomicAdd(reinterpret_cast<unsigned long long *>(&d.maint_count[0]), 1ull);
         }
         adv[i] = d.log_adv[i];
     }

@@ -137,6 +137,7 @@ struct DevState {
     uint64_t *log_base;             // per id: log tail when the commit starts
     BatchInfo *info;
     uint64_t *clock;
+    uint64_t *maint_count;          // index rebuilds and log compactions so far (2 counters)
     uint32_t *err;
     uint64_t *seq_next;
     // rebalance scratch

@@ -93,6 +93,7 @@ SIGNATURES = {
     "dm_export_ring": (C.c_int, [C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_uint32,
                                  C.POINTER(C.c_uint32)]),
     "dm_get_clock": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64)]),
+    "dm_get_maint_counts": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
     "dm_last_error": (C.c_int, [C.c_void_p]),
     "dm_set_profiling": (C.c_int, [C.c_void_p, C.c_int]),
     "dm_get_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int]),
@@ -235,6 +236,13 @@ def dm_get_clock(h):
     c = C.c_uint64()
     _check(lib().dm_get_clock(h, C.byref(c)), "dm_get_clock")
     return c.value
+
+
+def dm_get_maint_counts(h):
+    """(index rebuilds, log compactions) since the handle was created."""
+    a, b = C.c_uint64(), C.c_uint64()
+    _check(lib().dm_get_maint_counts(h, C.byref(a), C.byref(b)), "dm_get_maint_counts")
+    return a.value, b.value
 
 
 def dm_last_error(h):

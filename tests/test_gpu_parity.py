@@ -368,3 +368,75 @@ def test_host_async_pipeline_matches_oracle():
             got = host[name].numpy().view(npdt[str(t).split(".")[1]])
             assert np.array_equal(got, want[name]), name
     p.check_state()
+
+
+# -- index maintenance and placement stress ----------------------------------------
+
+def _run_prompts(p, batches, t0=0, dt=10, rebalance=False, state_every=1):
+    t = t0
+    for k, prompts in enumerate(batches):
+        tok, off, lens = _batch(prompts)
+        p.route(tok, off, lens, t, tag=f"batch {k}")
+        if rebalance:
+            p.rebalance(tag=f"batch {k}")
+        p.commit()
+        p.check_loads(tag=f"batch {k}")
+        if state_every and (k + 1) % state_every == 0:
+            p.check_state(tag=f"batch {k}")
+        t += dt
+    return t
+
+
+def test_index_rebuild_and_log_compaction():
+    """Prompts that are only a few hot prefixes re-touch the same keys every
+    batch: the log fills with stale records while nothing is evicted, until it
+    must be compacted.  Batches of unique prompts then fill the index past
+    half, forcing rebuilds.  Both paths stay bit-exact, and the maintenance
+    counters show that each ran."""
+    from paper_2602_06502_gb300 import dualmap as D
+    rng = np.random.default_rng(21)
+    w = _mk(n_instances=2, vnodes=16, capacity=1000, batch=64)
+    p = Pair(w, max_instances=3, max_touch=4096)
+    p.add(0)
+    p.add(1)
+    hot = [rng.integers(0, 32000, size=16 * 64, dtype=np.uint32) for _ in range(4)]
+    batches = [[hot[int(i)] for i in rng.integers(0, 4, size=64)] for _ in range(12)]
+    t = _run_prompts(p, batches, state_every=3)
+    rebuilds0, compactions = D.dm_get_maint_counts(p.gpu.h)
+    assert compactions >= 1, (rebuilds0, compactions)
+    uniq = [[rng.integers(0, 32000, size=16 * 64, dtype=np.uint32) for _ in range(64)] for _ in range(8)]
+    _run_prompts(p, uniq, t0=t, state_every=2)
+    rebuilds, compactions2 = D.dm_get_maint_counts(p.gpu.h)
+    assert rebuilds > rebuilds0, (rebuilds, compactions2)
+
+
+def test_eviction_of_more_than_one_round():
+    """Each commit evicts about 327k records per instance, more than one
+    eviction round (4 CTAs x 65,536 records) covers."""
+    rng = np.random.default_rng(22)
+    w = _mk(n_instances=2, vnodes=16, capacity=1000, batch=80)
+    p = Pair(w, max_instances=3, max_touch=1 << 20, max_batch_tokens=1 << 24)
+    p.add(0)
+    p.add(1)
+    batches = [[rng.integers(0, 32000, size=16 * 8192, dtype=np.uint32) for _ in range(80)] for _ in range(3)]
+    _run_prompts(p, batches, dt=10**7, state_every=1)
+
+
+def test_shared_prefix_ending_inside_a_group():
+    """Hundreds of prompts share a 35-block prefix (it ends 3 blocks into an
+    8-block group) and diverge after it: their diverging blocks share that
+    group's anchor and so its home bucket, which overflows into the
+    key-hashed buckets.  A small index makes the overflow heavy."""
+    rng = np.random.default_rng(23)
+    w = _mk(n_instances=2, vnodes=16, capacity=2000, batch=200)
+    p = Pair(w, max_instances=3, max_touch=8192)
+    p.add(0)
+    p.add(1)
+    prefix = rng.integers(0, 32000, size=16 * 35, dtype=np.uint32)
+    batches = []
+    for _ in range(6):
+        prompts = []
+        for L in rng.integers(1, 21, size=200):
+            prompts.append(np.concatenate([prefix, rng.integers(0, 32000, size=16 * int(L), dtype=np.uint32)]))
+        batches.append(prompts)
+    _run_prompts(p, batches, state_every=2)
