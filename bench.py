@@ -381,10 +381,17 @@ def main():
     peak, peak_kind = peaks()
     achieved = bytes_per_launch / hash_avg_s / 1e9
 
-    # per-stage breakdown: a shorter run after the timed one, every stage timed
+    # per-stage breakdown: a fresh handle replays the same steps with every
+    # stage timed (events between kernels stop their launch overlap, so this
+    # run is not the headline)
+    g.close()
+    del g
+    g = make_sched()
+    for j in range(W):
+        step(g, j)
+    D.dm_get_stage_times(g.h, reset=True)
     D.dm_set_profiling(g.h, True)
-    nb_stage = min(K, 30)
-    for j in range(W + K, W + K + nb_stage):
+    for j in range(W, W + K):
         step(g, j)
     st_all = D.dm_get_stage_times(g.h, reset=True)
     D.dm_set_profiling(g.h, False)

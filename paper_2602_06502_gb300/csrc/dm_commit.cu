@@ -510,28 +510,41 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
                 x0 = lane < (int)cn ? d.plocal[pi + lane] : 0;
                 x1 = lane + 32 < (int)cn ? d.plocal[pi + lane + 32] : 0;
             }
-            // settled here: a claim of an empty home slot, or the key found
-            // there with a later position already; the rest is deferred
+            // a key found at its home with an older position: one attempt to
+            // raise it here (both lanes' attempts in flight together)
+            Slot r0 = c0s, r1 = c1s;
+            const bool up0 = v0 && c0s.key == k0 && c0s.pos1 <= p0;
+            const bool up1 = v1 && c1s.key == k1 && c1s.pos1 <= p1;
+            if (up0) r0 = slot_cas(&g.t[h0], c0s, Slot{k0, p0 + 1});
+            if (up1) r1 = slot_cas(&g.t[h1], c1s, Slot{k1, p1 + 1});
+            // settled here: a claim of an empty home slot, a raise that went
+            // through, or the key found with a later position already; the
+            // rest is deferred (x: the position value seen last)
             uint32_t newly = 0, claims = 0;
             bool need0 = false, need1 = false;
+            uint64_t x0 = c0s.pos1, x1 = c1s.pos1;
             if (v0) {
                 if (c0s.key == 0) { ++newly; ++claims; }
-                else if (c0s.key == k0 && c0s.pos1 > p0) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
-                else need0 = true;
+                else if (up0 && r0.pos1 == c0s.pos1) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
+                else if (up0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
+                else if (!up0 && c0s.key == k0) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
+                else { need0 = true; x0 = up0 ? r0.pos1 : c0s.pos1; }
             }
             if (v1) {
                 if (c1s.key == 0) { ++newly; ++claims; }
-                else if (c1s.key == k1 && c1s.pos1 > p1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
-                else need1 = true;
+                else if (up1 && r1.pos1 == c1s.pos1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
+                else if (up1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
+                else if (!up1 && c1s.key == k1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
+                else { need1 = true; x1 = up1 ? r1.pos1 : c1s.pos1; }
             }
             // deferred touches go to the segment's own slice of the queue
             const uint32_t m0 = __ballot_sync(0xffffffffu, need0), m1 = __ballot_sync(0xffffffffu, need1);
             const uint32_t below = (1u << lane) - 1u;
             Deferred *dq = d.defer + uint64_t(c0 + i) * kSegBlocks;
-            if (need0) dq[__popc(m0 & below)] = Deferred{k0, p0, c0s.pos1, (uint32_t)h0, g.f, c0s.key == k0 ? 1u : 0u, 0};
+            if (need0) dq[__popc(m0 & below)] = Deferred{k0, p0, x0, (uint32_t)h0, g.f, c0s.key == k0 ? 1u : 0u, 0};
             if (need1)
                 dq[__popc(m0) + __popc(m1 & below)] =
-                    Deferred{k1, p1, c1s.pos1, (uint32_t)h1, g.f, c1s.key == k1 ? 1u : 0u, 0};
+                    Deferred{k1, p1, x1, (uint32_t)h1, g.f, c1s.key == k1 ? 1u : 0u, 0};
             newly = __reduce_add_sync(0xffffffffu, newly);
             claims = __reduce_add_sync(0xffffffffu, claims);
             if (lane == 0) {   // summed per request by k_req_counts (no hot-counter atomics)
