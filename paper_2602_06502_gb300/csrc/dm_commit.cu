@@ -511,12 +511,37 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
                 x1 = lane + 32 < (int)cn ? d.plocal[pi + lane + 32] : 0;
             }
             // a key found at its home with an older position: one attempt to
-            // raise it here (both lanes' attempts in flight together)
+            // raise it here.  A key whose home slot holds another key, in a
+            // group whose 8 lanes found every slot of the home bucket taken
+            // and none holding the key, continues its probe order in the
+            // next bucket: one attempt there.  (Slots never empty again, so
+            // the key can never belong to that bucket.)  All these attempts
+            // are in flight together.
             Slot r0 = c0s, r1 = c1s;
             const bool up0 = v0 && c0s.key == k0 && c0s.pos1 <= p0;
             const bool up1 = v1 && c1s.key == k1 && c1s.pos1 <= p1;
+            bool mv0, mv1;
+            {
+                const int gbase = lane & ~(int)(kGroup - 1), me = lane & (int)(kGroup - 1);
+                const bool full0 = __shfl_sync(0xffffffffu, (int)v0, gbase + (int)kGroup - 1) != 0;
+                const bool full1 = __shfl_sync(0xffffffffu, (int)v1, gbase + (int)kGroup - 1) != 0;
+                const uint64_t seen0 = c0s.key == 0 ? k0 : c0s.key, seen1 = c1s.key == 0 ? k1 : c1s.key;
+                bool in0 = false, in1 = false;
+#pragma unroll
+                for (int j = 0; j < (int)kGroup; ++j) {
+                    const uint64_t s0 = shfl_u64(seen0, gbase + j), s1 = shfl_u64(seen1, gbase + j);
+                    in0 |= j != me && s0 == k0;
+                    in1 |= j != me && s1 == k1;
+                }
+                mv0 = v0 && full0 && c0s.key != 0 && c0s.key != k0 && !in0;
+                mv1 = v1 && full1 && c1s.key != 0 && c1s.key != k1 && !in1;
+            }
+            const uint64_t n0 = (((h0 & ~uint64_t(kGroup - 1)) + kGroup) & mask) | (h0 & (kGroup - 1));
+            const uint64_t n1 = (((h1 & ~uint64_t(kGroup - 1)) + kGroup) & mask) | (h1 & (kGroup - 1));
             if (up0) r0 = slot_cas(&g.t[h0], c0s, Slot{k0, p0 + 1});
+            else if (mv0) r0 = slot_cas(&g.t[n0], Slot{0, 0}, Slot{k0, p0 + 1});
             if (up1) r1 = slot_cas(&g.t[h1], c1s, Slot{k1, p1 + 1});
+            else if (mv1) r1 = slot_cas(&g.t[n1], Slot{0, 0}, Slot{k1, p1 + 1});
             // settled here: a claim of an empty home slot, a raise that went
             // through, or the key found with a later position already; the
             // rest is deferred (x: the position value seen last)
@@ -524,14 +549,18 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             bool need0 = false, need1 = false;
             uint64_t x0 = c0s.pos1, x1 = c1s.pos1;
             if (v0) {
-                if (c0s.key == 0) { ++newly; ++claims; }
+                if (c0s.key == 0 || (mv0 && r0.key == 0)) { ++newly; ++claims; }
+                else if (mv0 && r0.key == k0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
+                else if (mv0) need0 = true;
                 else if (up0 && r0.pos1 == c0s.pos1) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
                 else if (up0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
                 else if (!up0 && c0s.key == k0) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
                 else { need0 = true; x0 = up0 ? r0.pos1 : c0s.pos1; }
             }
             if (v1) {
-                if (c1s.key == 0) { ++newly; ++claims; }
+                if (c1s.key == 0 || (mv1 && r1.key == 0)) { ++newly; ++claims; }
+                else if (mv1 && r1.key == k1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
+                else if (mv1) need1 = true;
                 else if (up1 && r1.pos1 == c1s.pos1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
                 else if (up1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
                 else if (!up1 && c1s.key == k1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);

@@ -287,7 +287,7 @@ __device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uin
     if (h.key == 0) return kNoSlot;
     const uint64_t R0 = home & ~uint64_t(kGroup - 1);
     uint64_t R = R0;
-    for (uint64_t j = 1; j <= (mask >> 3) + kLinearBuckets + 1; ++j) {
+    for (uint64_t nbk = 1; nbk <= (mask >> 3) + kLinearBuckets + 1; ++nbk) {
         Slot sn[kGroup];
 #pragma unroll
         for (int j = 0; j < (int)kGroup; ++j) sn[j] = load_slot(t + R + j);
@@ -301,7 +301,7 @@ __device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uin
         }
         if (hit != kNoSlot) { *found = hs; return hit; }
         if (empty) return kNoSlot;
-        R = probe_bucket(j, R0, key, mask);
+        R = probe_bucket(nbk, R0, key, mask);
     }
     set_err(err, DM_ERR_TIMEOUT);
     return kNoSlot;
