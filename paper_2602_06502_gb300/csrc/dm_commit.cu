@@ -676,6 +676,7 @@ __global__ void __cluster_dims__(kEvCluster, 1, 1) __launch_bounds__(kEvThreads)
     __shared__ uint32_t s_w[33];
     __shared__ uint32_t s_tot[2], s_go;
     __shared__ uint64_t s_cut;
+    __shared__ uint32_t s_ev[kMaxInstances];   // instances over capacity
     const uint32_t r = cluster.block_rank();
     const uint32_t cid = blockIdx.x / kEvCluster, ncl = gridDim.x / kEvCluster;
     // one decision for the whole cluster (rank 0's view of the error word)
@@ -684,8 +685,20 @@ __global__ void __cluster_dims__(kEvCluster, 1, 1) __launch_bounds__(kEvThreads)
     const uint32_t go = *cluster.map_shared_rank(&s_go, 0);
     const uint64_t lmask = d.logcap - 1;
     uint32_t slot = 0;
-    for (uint32_t i = cid; go && i < d.M; i += ncl) {
-        if (!d.table[i] || d.live[i] <= d.C) continue;   // read alike by every CTA of the cluster
+    // the instances over capacity, in id order (every CTA builds the same
+    // list), dealt to the clusters in turn
+    uint32_t nev = 0;
+    for (uint32_t base = 0; go && base < d.M; base += blockDim.x) {
+        const uint32_t i = base + threadIdx.x;
+        const bool over = i < d.M && d.table[i] && d.live[i] > d.C;
+        uint32_t tot;
+        const uint32_t rk = block_excl_u32(over ? 1u : 0u, s_w, tot);
+        if (over) s_ev[nev + rk] = i;
+        nev += tot;
+    }
+    __syncthreads();
+    for (uint32_t e = cid; go && e < nev; e += ncl) {
+        const uint32_t i = s_ev[e];
         uint64_t remaining = d.live[i] - d.C;
         uint8_t *st = d.stale[i];
         const uint64_t tail = d.log_tail[i];
