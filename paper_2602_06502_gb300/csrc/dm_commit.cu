@@ -30,8 +30,9 @@ constexpr uint32_t kFlagCompact = 1, kFlagRebuild = 2;
 constexpr uint32_t kZeroChunk = 4096;   // slots or flag bytes cleared per chunk
 
 // 16-byte compare-and-swap of a whole index slot; returns its previous
-// contents.  Every slot access of the touch kernel goes through this, so key
-// and position change together and never tear.
+// contents.  Every slot update of the touch passes goes through this, so key
+// and position change together and never tear (whole-bucket reads are plain
+// 16-byte loads used only to pick the next slot to try).
 __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
     Slot old;
     asm volatile(
@@ -589,9 +590,10 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
 // Second pass over the deferred touches, a warp per segment: raise the
 // position of a found key (CAS loop), or walk the probe order of a key whose
 // home slot holds another key.  Every record still ends up marked stale
-// exactly once unless it is its key's latest: the first pass only settled
-// claims (value 0 before) and touches that saw a later position (their own
-// record is stale), and the maxima taken here order the rest.
+// exactly once unless it is its key's latest: the first pass settled only
+// touches whose outcome its own CAS fixed (a claim of an empty slot, a raise
+// that went through, a later position already there), and the maxima taken
+// here order the rest.
 __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
     pdl_enter();
     if (has_err(d.err)) return;
@@ -626,9 +628,8 @@ __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
 // Eviction.  Instance i drops its excess_i = live_i - C oldest resident keys
 // by moving its log front just past the excess_i-th non-stale record; the
 // stale flags it passes are reset (those positions will hold new records).
-// One CTA per instance walks its log from the front, 16 records per thread
-// and round (one 16-byte load of flags), with a block scan of the non-stale
-// counts locating the cut.
+// A cluster of CTAs walks an instance's log from the front (k_evict below);
+// first the touch passes' per-segment counts are summed per request.
 
 // Warp per request: sum the touch kernel's counts over the request's
 // (contiguous) segments, one atomic per request and counter.
