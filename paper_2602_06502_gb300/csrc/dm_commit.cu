@@ -59,10 +59,12 @@ __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
 // meet at the same slot and one CAS wins.  Returns the position value the
 // key had before (0 if claimed now).
 __device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint64_t home,
-                                                  Slot old, uint32_t *err, bool *claimed) {
+                                                  Slot old, uint32_t *err, bool *claimed, uint32_t nbk0 = 0) {
+    // `old` was seen at the preferred slot of bucket nbk0 of the key's order
     const uint32_t o = (uint32_t)(home & (kGroup - 1));
     const uint64_t R0 = home & ~uint64_t(kGroup - 1);
-    uint64_t R = R0, i = home, nbk = 0;   // nbk: position of bucket R in the probe order
+    uint64_t nbk = nbk0;   // position of bucket R in the probe order
+    uint64_t R = nbk0 ? probe_bucket(nbk0, R0, key, mask) : R0, i = R + o;
     uint32_t step = 0;   // order position of slot i within bucket R
     // at most one probe step per slot, and one retry per other touch of the
     // key in the batch (each failed retry means another touch got in)
@@ -552,7 +554,7 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             if (v0) {
                 if (c0s.key == 0 || (mv0 && r0.key == 0)) { ++newly; ++claims; }
                 else if (mv0 && r0.key == k0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
-                else if (mv0) need0 = true;
+                else if (mv0) { need0 = true; x0 = r0.pos1; }
                 else if (up0 && r0.pos1 == c0s.pos1) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
                 else if (up0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
                 else if (!up0 && c0s.key == k0) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
@@ -561,7 +563,7 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             if (v1) {
                 if (c1s.key == 0 || (mv1 && r1.key == 0)) { ++newly; ++claims; }
                 else if (mv1 && r1.key == k1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
-                else if (mv1) need1 = true;
+                else if (mv1) { need1 = true; x1 = r1.pos1; }
                 else if (up1 && r1.pos1 == c1s.pos1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
                 else if (up1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
                 else if (!up1 && c1s.key == k1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
@@ -571,10 +573,14 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             const uint32_t m0 = __ballot_sync(0xffffffffu, need0), m1 = __ballot_sync(0xffffffffu, need1);
             const uint32_t below = (1u << lane) - 1u;
             Deferred *dq = d.defer + uint64_t(c0 + i) * kSegBlocks;
-            if (need0) dq[__popc(m0 & below)] = Deferred{k0, p0, x0, (uint32_t)h0, g.f, c0s.key == k0 ? 1u : 0u, 0};
+            // found: the key sits at the preferred slot of the recorded bucket
+            // (its home, or the next bucket after a move) with position x
+            if (need0)
+                dq[__popc(m0 & below)] = Deferred{k0, p0, x0, (uint32_t)h0, g.f,
+                                                  (mv0 ? r0.key : c0s.key) == k0 ? 1u : 0u, mv0 ? 1u : 0u};
             if (need1)
-                dq[__popc(m0) + __popc(m1 & below)] =
-                    Deferred{k1, p1, x1, (uint32_t)h1, g.f, c1s.key == k1 ? 1u : 0u, 0};
+                dq[__popc(m0) + __popc(m1 & below)] = Deferred{k1, p1, x1, (uint32_t)h1, g.f,
+                                                               (mv1 ? r1.key : c1s.key) == k1 ? 1u : 0u, mv1 ? 1u : 0u};
             newly = __reduce_add_sync(0xffffffffu, newly);
             claims = __reduce_add_sync(0xffffffffu, claims);
             if (lane == 0) {   // summed per request by k_req_counts (no hot-counter atomics)
@@ -611,7 +617,7 @@ __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
             // other than 0 and e.key)
             const Slot old = e.found ? Slot{e.key, e.x} : Slot{e.key == 1 ? 2ull : e.key ^ 1ull, 0};
             bool cl = false;
-            const uint64_t o = touch_resolve(d.table[e.f], mask, e.key, e.p + 1, e.home, old, d.err, &cl);
+            const uint64_t o = touch_resolve(d.table[e.f], mask, e.key, e.p + 1, e.home, old, d.err, &cl, e.bucket);
             touch_outcome(o, e.p, d.log_front[e.f], d.stale[e.f], lmask, newly);
             claims += cl;
         }

@@ -57,13 +57,14 @@ struct Rec {
     uint64_t key, stamp;
 };
 
-// A touch the commit's first pass could not settle with one CAS at the
-// key's home slot (40 bytes): the key is there with an older position
-// (found = 1, x = the position value seen) or the home slot holds another
-// key (found = 0).  The second pass finishes it.
+// A touch the commit's first pass could not settle (40 bytes): the key is at
+// its home slot with an older position (found = 1, x = the position value
+// seen last) or the preferred slot of bucket `bucket` of its probe order (0:
+// the home bucket) holds another key (found = 0).  The second pass finishes
+// it from there.
 struct Deferred {
     uint64_t key, p, x;     // p: log position of the touch's record
-    uint32_t home, f, found, pad;
+    uint32_t home, f, found, bucket;
 };
 
 // Per-batch values produced on the device.
