@@ -539,8 +539,8 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
                 mv0 = v0 && full0 && c0s.key != 0 && c0s.key != k0 && !in0;
                 mv1 = v1 && full1 && c1s.key != 0 && c1s.key != k1 && !in1;
             }
-            const uint64_t n0 = (((h0 & ~uint64_t(kGroup - 1)) + kGroup) & mask) | (h0 & (kGroup - 1));
-            const uint64_t n1 = (((h1 & ~uint64_t(kGroup - 1)) + kGroup) & mask) | (h1 & (kGroup - 1));
+            const uint64_t n0 = probe_bucket(1, h0 & ~uint64_t(kGroup - 1), k0, mask) | (h0 & (kGroup - 1));
+            const uint64_t n1 = probe_bucket(1, h1 & ~uint64_t(kGroup - 1), k1, mask) | (h1 & (kGroup - 1));
             if (up0) r0 = slot_cas(&g.t[h0], c0s, Slot{k0, p0 + 1});
             else if (mv0) r0 = slot_cas(&g.t[n0], Slot{0, 0}, Slot{k0, p0 + 1});
             if (up1) r1 = slot_cas(&g.t[h1], c1s, Slot{k1, p1 + 1});

@@ -38,12 +38,14 @@ struct QEntry {
 // line: one random DRAM access instead of 8 (random single-slot atomics
 // saturate far below line-local ones).  A key fixes its whole prefix and so
 // its anchor: every key has one home.  Probe order of a key: the slots of its
-// home bucket cyclically from its preferred one; then those of the next
-// kLinearBuckets - 1 buckets (a group displaced from a full home bucket
-// moves on together, within a few hundred bytes); then the buckets from one
-// chosen by the key's own hash onwards, each likewise.  (Prompts that share
-// a prefix but diverge inside a group share that group's anchor: past the
-// first buckets the key hash spreads their overflow instead of piling it up.)
+// home bucket cyclically from its preferred one; then those of a second
+// bucket derived from the home bucket's index (a group displaced from a full
+// home bucket moves there together; a hashed bucket is far likelier to be
+// empty than the adjacent one, which earlier displaced groups fill); then
+// the buckets from one chosen by the key's own hash onwards, each likewise.
+// (Prompts that share a prefix but diverge inside a group share that group's
+// anchor: past the first two buckets the key hash spreads their overflow
+// instead of piling it up.)
 // Inserts take the first slot of that order that is empty, and slots never
 // empty again (until the index is rebuilt into the other buffer), so a
 // lookup ends at the first bucket with an empty slot.
@@ -262,11 +264,14 @@ __device__ __forceinline__ uint64_t group_home(uint64_t anchor, uint64_t b, uint
 }
 
 // Bucket j >= 1 of the probe order of key (bucket 0 is its home bucket R0):
-// the buckets after R0 while j < kLinearBuckets, then the bucket chosen by
-// the key's hash and those after it.
+// j = 1 the bucket derived from R0 (the one after R0 should they coincide);
+// j >= 2 the bucket chosen by the key's hash, then those after it.
 constexpr uint64_t kLinearBuckets = 2;
 __device__ __forceinline__ uint64_t probe_bucket(uint64_t j, uint64_t R0, uint64_t key, uint64_t mask) {
-    if (j < kLinearBuckets) return (R0 + j * kGroup) & mask;
+    if (j == 1) {
+        const uint64_t R1 = fmix64(R0 ^ 0x5bd1e995a4c3b2e1ull) & mask & ~uint64_t(kGroup - 1);
+        return R1 == R0 ? (R0 + kGroup) & mask : R1;
+    }
     return ((fmix64(key) & mask & ~uint64_t(kGroup - 1)) + (j - kLinearBuckets) * kGroup) & mask;
 }
 
