@@ -391,6 +391,27 @@ __device__ __forceinline__ void drain_queue(const DevState &d, uint32_t i, uint6
     }
 }
 
+// The same two ring positions without the stored carries: the carry of the
+// segment holding block K-1 is summed here from the (at most 4) segment
+// totals before it, so the ring search need not wait for request_carries.
+// Whole warp; all lanes return the same values.
+__device__ __forceinline__ void route_positions_direct(const DevState &d, uint32_t r, int lane, uint64_t &pos1,
+                                                       uint64_t &pos2) {
+    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
+    const uint32_t K = min(d.Kroute, nblk);
+    const uint32_t last = (K - 1) / kSegBlocks;   // <= 3 (K <= 256)
+    uint64_t c = (uint32_t)lane < last ? d.seg_total[s0 + lane] : 0;
+    uint64_t p2 = (uint32_t)lane <= last ? d.seg_total2[s0 + lane] : 0;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        c += shfl_xor_u64(c, o);
+        p2 += shfl_xor_u64(p2, o);
+    }
+    const uint64_t P1 = d.plocal[d.r_blkoff[r] + K - 1] + c;
+    pos1 = fmix64(P1 ^ d.Sr1);
+    pos2 = fmix64(p2 ^ d.Sr2);
+}
+
 // Grid of a grid-stride kernel: every SM filled to the kernel's occupancy.
 template <typename K>
 inline int full_grid(K kernel, int block) {

@@ -46,10 +46,11 @@ __device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uin
     lb2 = (uint32_t)(i2 + 1 == (int64_t)d.R ? 0 : i2 + 1);
 }
 
-// One CTA of kProbeWarps warps per request.  Warp 0 computes the segment
-// carries, the two ring positions and candidates; then every round probes
-// 32 * kProbeWarps consecutive blocks on each candidate still running, and
-// the smallest missing block over the warps ends that candidate's run.
+// One CTA of kProbeWarps warps per request.  Warp 0 computes the two ring
+// positions and candidates while warp 1 computes the segment carries; then
+// every round probes 32 * kProbeWarps consecutive blocks on each candidate
+// still running, and the smallest missing block over the warps ends that
+// candidate's run.
 constexpr int kProbeWarps = 8;
 
 __global__ void __launch_bounds__(kProbeWarps * 32, 4) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
@@ -59,11 +60,11 @@ __global__ void __launch_bounds__(kProbeWarps * 32, 4) k_route_probe(DevState d,
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const uint32_t r = blockIdx.x;
-    if (wid == 0) {
-        request_carries(d, r, lane);
-        __syncwarp();
+    if (wid == 1) {
+        request_carries(d, r, lane);   // for the probes below and the commit
+    } else if (wid == 0) {
         uint64_t p1, p2;
-        route_positions(d, r, lane, p1, p2);
+        route_positions_direct(d, r, lane, p1, p2);
         uint32_t lb1, lb2;
         ring_search2(d, p1, p2, lane, lb1, lb2);
         const uint32_t c1 = d.ring[0].owner[lb1];
