@@ -43,8 +43,49 @@
  *     in arrival order within the batch; the request joins the chosen
  *     instance's FIFO queue with work c*(L - h_choice).
  *
+ *   Choice rules.  Between the same two candidates (the ablation of Sec.
+ *     4.3), with the rules of the compared schedulers (Sec. 2.2; Preble's
+ *     and Mooncake's rules as the related-work appendix states them):
+ *       DualMap         the SLO-aware rule above;
+ *       cache affinity  the candidate with more hit tokens; equal hits: the
+ *                       less-loaded by W, tie c1;
+ *       least loaded    smaller W, tie c1 (hits ignored);
+ *       min TTFT        smaller ttft_f = W[c_f] + c*(L - h_f), tie c1 (the
+ *                       appendix prints it as a max of a difference; the
+ *                       minimum of the sum is what the text describes);
+ *       Preble          if the larger hit exceeds half the prompt
+ *                       (2*max(h1,h2) > L): cache affinity, else min TTFT.
+ *     For these, switched = 1 when the hits differ and the candidate with
+ *     fewer of them was chosen.  Over all live instances (the baselines of
+ *     Sec. 2.2 and Sec. 4), h_i probed on every live instance i:
+ *       global cache affinity  c1, the owner on ring 1 (one prompt-aware
+ *                              mapping, Sec. 1);
+ *       global least loaded    smallest W_i, tie lowest id;
+ *       global min TTFT        smallest W_i + c*(L - h_i), tie lowest id;
+ *       global Preble          if 2*max_i h_i > L: among the instances with
+ *                              that hit the smallest W_i, tie lowest id;
+ *                              else global min TTFT;
+ *     switched = 0; ttft1/ttft2 still report the two candidates; the queue
+ *     entry's work is c*(L - h) of the chosen instance.
+ *
  *   Time: batch time = arrival of the batch's last request; before routing,
- *     every instance's queue drains by the elapsed microseconds.
+ *     every instance's queue drains by the elapsed microseconds, starting
+ *     at the previous batch time t0: an entry that finishes after w us of
+ *     that window completes at t0 + w, and its TTFT is that minus the
+ *     batch time it arrived with (kept when rebalancing moves it).
+ *
+ *   Metrics (Sec. 2.2 load-balance CV; Sec. 4.1 cache hit rate, SLO
+ *     attainment, TTFT percentiles): per routed request its L, the hit
+ *     tokens of the chosen candidate, switched, and whether the estimated
+ *     TTFT on the chosen candidate is <= SLO; per completed entry its TTFT
+ *     (sum, max, <= SLO count, and a log-linear histogram: values below 16
+ *     exact, then 16 buckets per power of two); after the choices of a
+ *     non-empty batch one CV sample over the live instances' W,
+ *       CV = sqrt(n*S2 - S1^2) / S1,  S1 = sum W_i, S2 = sum W_i^2
+ *     (the population CV of Sec. 2.2 with the n's cancelled; 0 when S1 = 0),
+ *     with S1, S2 and n*S2 - S1^2 exact 128-bit integers, each turned into
+ *     a double as double(hi)*2^64 + double(lo), every floating step rounded
+ *     to nearest.
  *
  *   Commit (App. A.3.2 "KV cache save"): after route (and rebalance), in
  *     arrival order, each request touches its keys on its final instance,
@@ -67,6 +108,7 @@
  * on every membership change, an LRU as hash map + recency list, queues as
  * plain arrays.
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -135,7 +177,16 @@ typedef struct {
     uint32_t max_batch;
     uint64_t max_batch_tokens;
     uint64_t seed;
+    uint32_t choice_rule;   /* OR_RULE_* */
 } or_config;
+
+enum { OR_RULE_DUALMAP = 0, OR_RULE_CACHE_AFFINITY = 1, OR_RULE_LEAST_LOADED = 2,
+       OR_RULE_MIN_TTFT = 3, OR_RULE_PREBLE = 4, OR_RULE_GLOBAL_CACHE_AFFINITY = 5,
+       OR_RULE_GLOBAL_LEAST_LOADED = 6, OR_RULE_GLOBAL_MIN_TTFT = 7, OR_RULE_GLOBAL_PREBLE = 8 };
+
+/* TTFT histogram: values 0..15 exact, then 16 buckets per power of two up
+ * to 2^64. */
+#define OR_HIST_BUCKETS 976
 
 typedef struct {
     uint64_t key, stamp;
@@ -157,6 +208,7 @@ typedef struct {
     uint32_t L, c1, c2, h1, h2;
     uint64_t work, remaining;
     uint64_t moved_in_call;  /* rebalance call id that moved it here; 0 = none */
+    uint64_t arrival;        /* batch time the request arrived with */
 } q_entry;
 
 typedef struct {
@@ -190,6 +242,11 @@ typedef struct {
     uint32_t *pend_final, *pend_nblk;
     uint64_t **pend_keys;
     int pending;
+    /* metrics since create / the last reset */
+    uint64_t m_requests, m_prompt_tokens, m_hit_tokens, m_switched, m_est_slo_met;
+    uint64_t m_completed, m_ttft_sum, m_ttft_max, m_slo_met, m_batches;
+    double m_cv_sum, m_cv_last;
+    uint64_t m_hist[OR_HIST_BUCKETS];
 } or_state;
 
 /* ------------------------------------------------------------------ */
@@ -478,18 +535,50 @@ static void q_erase(queue_t *q, uint64_t k)
 }
 
 /* Run `delta` microseconds of prefill work off the head of the queue. */
-static void q_drain(queue_t *q, uint64_t *W, uint64_t delta)
+/* Histogram bucket of a TTFT value: v < 16 is its own bucket; otherwise,
+ * with e = floor(log2 v), bucket 16 + 16(e-4) + (the 4 bits below v's top
+ * bit). */
+uint32_t or_hist_bucket(uint64_t v)
 {
+    if (v < 16) return (uint32_t)v;
+    uint32_t e = 63;
+    while (!((v >> e) & 1)) e--;
+    return 16 + 16 * (e - 4) + (uint32_t)((v >> (e - 4)) & 15);
+}
+
+/* Smallest value of bucket k. */
+uint64_t or_hist_lower(uint32_t k)
+{
+    if (k < 16) return k;
+    uint32_t e = 4 + (k - 16) / 16, sub = (k - 16) % 16;
+    return (uint64_t)(16 + sub) << (e - 4);
+}
+
+static void record_ttft(or_state *s, uint64_t ttft)
+{
+    s->m_completed++;
+    s->m_ttft_sum += ttft;
+    if (ttft > s->m_ttft_max) s->m_ttft_max = ttft;
+    if (ttft <= s->cfg.slo_us) s->m_slo_met++;
+    s->m_hist[or_hist_bucket(ttft)]++;
+}
+
+/* Run `delta` us of instance id's queue, the window starting at t0. */
+static void q_drain(or_state *s, uint32_t id, uint64_t delta, uint64_t t0)
+{
+    queue_t *q = &s->q[id];
+    uint64_t run = 0;   /* work finished since t0 */
     while (q->len > 0) {
         q_entry *h = &q->e[q->head];
-        if (h->remaining <= delta) {
-            delta -= h->remaining;
-            *W -= h->remaining;
+        if (h->remaining <= delta - run) {
+            run += h->remaining;
+            s->W[id] -= h->remaining;
+            record_ttft(s, t0 + run - h->arrival);
             q->head++;
             q->len--;
         } else {
-            h->remaining -= delta;
-            *W -= delta;
+            h->remaining -= delta - run;
+            s->W[id] -= delta - run;
             break;
         }
     }
@@ -534,7 +623,7 @@ int or_create(const or_config *cfg, or_state **out)
 {
     *out = NULL;
     uint32_t B = cfg->block_tokens;
-    if (B < 2 || B > 64 || (B & 1) || cfg->route_prefix_blocks < 1 ||
+    if (B < 2 || B > 64 || (B & 1) || cfg->route_prefix_blocks < 1 || cfg->choice_rule > OR_RULE_GLOBAL_PREBLE ||
         cfg->vnodes_per_instance < 1 || cfg->max_instances < 2 ||
         cfg->cache_capacity_blocks < 1 || cfg->cost_us_per_token < 1 ||
         cfg->hot_den < 1 || cfg->max_batch < 1 || cfg->max_batch_tokens < B)
@@ -581,15 +670,41 @@ int or_remove_instance(or_state *s, uint32_t id)
 /* The routing step                                                     */
 /* ------------------------------------------------------------------ */
 
-/* SLO-aware choice between the two candidates (Sec. 3.2).  Returns the
- * chosen id and sets *switched when the SLO rule overrode cache affinity. */
-uint32_t or_choose(uint32_t c1, uint32_t c2, uint32_t h1, uint32_t h2, uint32_t L,
+/* Cache affinity: more hits; equal hits, the less-loaded (tie c1). */
+static uint32_t choose_affinity(uint32_t c1, uint32_t c2, uint32_t h1, uint32_t h2,
+                                uint64_t W1, uint64_t W2)
+{
+    if (h1 != h2) return h1 > h2 ? c1 : c2;
+    return W2 < W1 ? c2 : c1;
+}
+
+/* The choice between the two candidates under `rule` (Sec. 3.2 for
+ * DualMap's SLO-aware rule; the compared rules as listed in the header).
+ * Returns the chosen id; *switched is set when the SLO rule overrode cache
+ * affinity (DualMap) or when the candidate with fewer hits was chosen
+ * (other rules). */
+uint32_t or_choose(uint32_t rule, uint32_t c1, uint32_t c2, uint32_t h1, uint32_t h2, uint32_t L,
                    uint64_t W1, uint64_t W2, uint64_t slo, uint32_t cost,
                    uint64_t *ttft1, uint64_t *ttft2, uint8_t *switched)
 {
     *ttft1 = W1 + (uint64_t)cost * (L - h1);
     *ttft2 = W2 + (uint64_t)cost * (L - h2);
     *switched = 0;
+    if (rule != OR_RULE_DUALMAP) {
+        uint32_t ch;
+        uint32_t hmax = h1 > h2 ? h1 : h2;
+        if (rule == OR_RULE_GLOBAL_CACHE_AFFINITY) return c1;
+        if (rule == OR_RULE_CACHE_AFFINITY ||
+            (rule == OR_RULE_PREBLE && 2 * (uint64_t)hmax > L))
+            ch = choose_affinity(c1, c2, h1, h2, W1, W2);
+        else if (rule == OR_RULE_LEAST_LOADED)
+            ch = W2 < W1 ? c2 : c1;
+        else   /* min TTFT, and Preble below half the prompt */
+            ch = *ttft2 < *ttft1 ? c2 : c1;
+        uint32_t h_ch = ch == c1 ? h1 : h2, h_other = ch == c1 ? h2 : h1;
+        *switched = h_ch < h_other;
+        return ch;
+    }
     if (h1 == h2) return W2 < W1 ? c2 : c1;
     int a_is_1 = h1 > h2;
     uint64_t ttft_a = a_is_1 ? *ttft1 : *ttft2;
@@ -598,6 +713,53 @@ uint32_t or_choose(uint32_t c1, uint32_t c2, uint32_t h1, uint32_t h2, uint32_t 
     if (ttft_a <= slo) return a;
     *switched = 1;
     return Wb < Wa ? b : a;
+}
+
+static double u128_to_double(unsigned __int128 x)
+{
+    return (double)(uint64_t)(x >> 64) * 18446744073709551616.0 + (double)(uint64_t)x;
+}
+
+/* Coefficient of variation of the live instances' queued work (Sec. 2.2). */
+static double load_cv(const or_state *s)
+{
+    unsigned __int128 S1 = 0, S2 = 0;
+    uint64_t n = 0;
+    for (uint32_t id = 0; id < s->cfg.max_instances; id++)
+        if (s->state[id] == INST_LIVE) {
+            S1 += s->W[id];
+            S2 += (unsigned __int128)s->W[id] * s->W[id];
+            n++;
+        }
+    if (S1 == 0) return 0.0;
+    return sqrt(u128_to_double(n * S2 - S1 * S1)) / u128_to_double(S1);
+}
+
+/* The rules over all live instances (see the header); h[id] = hit tokens
+ * of the request on instance id. */
+static uint32_t choose_global(const or_state *s, uint32_t rule, const uint32_t *h, uint32_t L)
+{
+    const uint64_t cost = s->cfg.cost_us_per_token;
+    uint32_t hmax = 0;
+    for (uint32_t id = 0; id < s->cfg.max_instances; id++)
+        if (s->state[id] == INST_LIVE && h[id] > hmax) hmax = h[id];
+    const int affine = rule == OR_RULE_GLOBAL_PREBLE && 2 * (uint64_t)hmax > L;
+    uint32_t best = UINT32_MAX;
+    uint64_t best_key = 0;
+    for (uint32_t id = 0; id < s->cfg.max_instances; id++) {
+        if (s->state[id] != INST_LIVE) continue;
+        uint64_t key;
+        if (rule == OR_RULE_GLOBAL_LEAST_LOADED) {
+            key = s->W[id];
+        } else if (affine) {
+            if (h[id] != hmax) continue;
+            key = s->W[id];
+        } else {
+            key = s->W[id] + cost * (L - h[id]);
+        }
+        if (best == UINT32_MAX || key < best_key) { best = id; best_key = key; }
+    }
+    return best;
 }
 
 static uint32_t leading_hits(const lru_t *c, const uint64_t *keys, uint32_t nblk)
@@ -626,7 +788,7 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
     /* time advances; every instance's queue runs for the elapsed us */
     uint64_t delta = s->have_time ? t_batch - s->t_prev : 0;
     for (uint32_t id = 0; id < cf->max_instances; id++)
-        if (s->state[id] != INST_ABSENT) q_drain(&s->q[id], &s->W[id], delta);
+        if (s->state[id] != INST_ABSENT) q_drain(s, id, delta, s->t_prev);
     s->t_prev = t_batch;
     s->have_time = 1;
 
@@ -637,6 +799,13 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
     s->pend_nblk = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
     s->pend_keys = (uint64_t **)calloc(n ? n : 1, sizeof(uint64_t *));
     if (!s->pend_final || !s->pend_nblk || !s->pend_keys) return OR_ERR_OOM;
+
+    /* hits on every live instance, for the rules that look at all of them */
+    uint32_t *hall = NULL;
+    if (cf->choice_rule >= OR_RULE_GLOBAL_LEAST_LOADED) {
+        hall = (uint32_t *)malloc(((size_t)n * cf->max_instances + 1) * sizeof(uint32_t));
+        if (!hall) return OR_ERR_OOM;
+    }
 
     /* 1) hash, ring lookup, distinct fix, probes: all against batch-start state */
     for (uint32_t r = 0; r < n; r++) {
@@ -654,23 +823,48 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
         cand2[r] = c2;
         hit1[r] = cf->block_tokens * leading_hits(&s->cache[c1], keys, nblk);
         hit2[r] = cf->block_tokens * leading_hits(&s->cache[c2], keys, nblk);
+        if (hall)
+            for (uint32_t id = 0; id < cf->max_instances; id++)
+                hall[(size_t)r * cf->max_instances + id] =
+                    s->state[id] == INST_LIVE ? cf->block_tokens * leading_hits(&s->cache[id], keys, nblk) : 0;
     }
     /* 2) choices in arrival order; loads update as we go */
     for (uint32_t r = 0; r < n; r++) {
         uint32_t c1 = cand1[r], c2 = cand2[r];
-        uint32_t ch = or_choose(c1, c2, hit1[r], hit2[r], lengths[r], s->W[c1], s->W[c2],
-                                cf->slo_us, cf->cost_us_per_token, &ttft1[r], &ttft2[r],
-                                &switched[r]);
+        uint32_t ch, hch;
+        if (hall) {
+            const uint32_t *h = hall + (size_t)r * cf->max_instances;
+            ch = choose_global(s, cf->choice_rule, h, lengths[r]);
+            ttft1[r] = s->W[c1] + (uint64_t)cf->cost_us_per_token * (lengths[r] - hit1[r]);
+            ttft2[r] = s->W[c2] + (uint64_t)cf->cost_us_per_token * (lengths[r] - hit2[r]);
+            switched[r] = 0;
+            hch = h[ch];
+        } else {
+            ch = or_choose(cf->choice_rule, c1, c2, hit1[r], hit2[r], lengths[r], s->W[c1], s->W[c2],
+                           cf->slo_us, cf->cost_us_per_token, &ttft1[r], &ttft2[r], &switched[r]);
+            hch = ch == c1 ? hit1[r] : hit2[r];
+        }
         chosen[r] = ch;
-        uint32_t hch = ch == c1 ? hit1[r] : hit2[r];
         q_entry e;
         e.seq = s->next_seq++;
         e.L = lengths[r]; e.c1 = c1; e.c2 = c2; e.h1 = hit1[r]; e.h2 = hit2[r];
         e.work = e.remaining = (uint64_t)cf->cost_us_per_token * (lengths[r] - hch);
         e.moved_in_call = 0;
+        e.arrival = t_batch;
         if (q_push(&s->q[ch], &e)) return OR_ERR_OOM;
         s->W[ch] += e.work;
         s->pend_final[r] = ch;
+        s->m_requests++;
+        s->m_prompt_tokens += lengths[r];
+        s->m_hit_tokens += hch;
+        s->m_switched += switched[r];
+        s->m_est_slo_met += s->W[ch] <= cf->slo_us;   /* the load including this request */
+    }
+    free(hall);
+    if (n > 0) {
+        s->m_cv_last = load_cv(s);
+        s->m_cv_sum += s->m_cv_last;
+        s->m_batches++;
     }
     s->pending = 1;
     return OR_OK;
@@ -869,7 +1063,7 @@ int or_debug_enqueue(or_state *s, uint32_t id, uint64_t seq, uint32_t L, uint32_
                      uint32_t h1, uint32_t h2, uint64_t work, uint64_t remaining)
 {
     if (id >= s->cfg.max_instances) return OR_ERR_INVALID_ARG;
-    q_entry e = {seq, L, c1, c2, h1, h2, work, remaining, 0};
+    q_entry e = {seq, L, c1, c2, h1, h2, work, remaining, 0, s->t_prev};
     int rc = q_push(&s->q[id], &e);
     if (!rc) s->W[id] += remaining;
     if (seq >= s->next_seq) s->next_seq = seq + 1;
@@ -881,4 +1075,49 @@ int or_debug_touch(or_state *s, uint32_t id, uint64_t key)
 {
     if (id >= s->cfg.max_instances) return OR_ERR_INVALID_ARG;
     return lru_touch(&s->cache[id], key, ++s->clock, s->cfg.cache_capacity_blocks);
+}
+
+/* ------------------------------------------------------------------ */
+/* Metrics                                                             */
+/* ------------------------------------------------------------------ */
+
+/* Lower edge of the bucket holding the ceil(pnum/pden * count)-th smallest
+ * value (rank at least 1); 0 when the histogram is empty. */
+static uint64_t hist_percentile(const uint64_t *hist, uint64_t count, uint64_t pnum, uint64_t pden)
+{
+    if (count == 0) return 0;
+    uint64_t rank = (pnum * count + pden - 1) / pden;
+    if (rank == 0) rank = 1;
+    uint64_t cum = 0;
+    for (uint32_t k = 0; k < OR_HIST_BUCKETS; k++) {
+        cum += hist[k];
+        if (cum >= rank) return or_hist_lower(k);
+    }
+    return or_hist_lower(OR_HIST_BUCKETS - 1);
+}
+
+/* Metrics since create or the last reset.  u[0..12]: requests routed,
+ * prompt tokens, hit tokens on the chosen candidates, switched, estimated
+ * TTFT <= SLO, completed, TTFT sum, TTFT max, completed with TTFT <= SLO,
+ * TTFT p50, p90, p99 (histogram lower edges), CV samples.  d[0..1]: sum of
+ * the CV samples, the last one.  hist: OR_HIST_BUCKETS counts, or NULL. */
+void or_get_metrics(or_state *s, uint64_t *u, double *d, uint64_t *hist, int reset)
+{
+    u[0] = s->m_requests; u[1] = s->m_prompt_tokens; u[2] = s->m_hit_tokens;
+    u[3] = s->m_switched; u[4] = s->m_est_slo_met; u[5] = s->m_completed;
+    u[6] = s->m_ttft_sum; u[7] = s->m_ttft_max; u[8] = s->m_slo_met;
+    u[9] = hist_percentile(s->m_hist, s->m_completed, 50, 100);
+    u[10] = hist_percentile(s->m_hist, s->m_completed, 90, 100);
+    u[11] = hist_percentile(s->m_hist, s->m_completed, 99, 100);
+    u[12] = s->m_batches;
+    d[0] = s->m_cv_sum;
+    d[1] = s->m_cv_last;
+    if (hist) memcpy(hist, s->m_hist, sizeof s->m_hist);
+    if (reset) {
+        s->m_requests = s->m_prompt_tokens = s->m_hit_tokens = s->m_switched = 0;
+        s->m_est_slo_met = s->m_completed = s->m_ttft_sum = s->m_ttft_max = 0;
+        s->m_slo_met = s->m_batches = 0;
+        s->m_cv_sum = s->m_cv_last = 0.0;
+        memset(s->m_hist, 0, sizeof s->m_hist);
+    }
 }

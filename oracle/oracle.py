@@ -24,7 +24,7 @@ def build(force=False):
         return LIB
     tmp = LIB + f".tmp{os.getpid()}"
     subprocess.check_call(["gcc", "-O2", "-std=gnu11", "-shared", "-fPIC", "-Wall", "-Wextra",
-                           "-Wno-unused-parameter", SRC, "-o", tmp])
+                           "-Wno-unused-parameter", SRC, "-o", tmp, "-lm"])
     os.replace(tmp, LIB)
     return LIB
 
@@ -43,7 +43,16 @@ class or_config(C.Structure):
         ("max_batch", C.c_uint32),
         ("max_batch_tokens", C.c_uint64),
         ("seed", C.c_uint64),
+        ("choice_rule", C.c_uint32),
     ]
+
+
+RULE_DUALMAP, RULE_CACHE_AFFINITY, RULE_LEAST_LOADED, RULE_MIN_TTFT, RULE_PREBLE = 0, 1, 2, 3, 4
+RULE_GLOBAL_CACHE_AFFINITY, RULE_GLOBAL_LEAST_LOADED, RULE_GLOBAL_MIN_TTFT, RULE_GLOBAL_PREBLE = 5, 6, 7, 8
+HIST_BUCKETS = 976
+METRIC_KEYS = ["requests", "prompt_tokens", "hit_tokens", "switched", "est_slo_met", "completed",
+               "ttft_sum_us", "ttft_max_us", "slo_met", "ttft_p50_us", "ttft_p90_us", "ttft_p99_us",
+               "cv_samples"]
 
 
 _lib = None
@@ -70,7 +79,7 @@ def lib():
             "or_destroy": (None, [V]),
             "or_add_instance": (C.c_int, [V, C.c_uint32]),
             "or_remove_instance": (C.c_int, [V, C.c_uint32]),
-            "or_choose": (C.c_uint32, [C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32,
+            "or_choose": (C.c_uint32, [C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32,
                                        C.c_uint64, C.c_uint64, C.c_uint64, C.c_uint32,
                                        P(C.c_uint64), P(C.c_uint64), P(C.c_uint8)]),
             "or_route_batch": (C.c_int, [V, u32p, u64p, u32p, C.c_uint32, C.c_uint64,
@@ -91,6 +100,9 @@ def lib():
                                            C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint64,
                                            C.c_uint64]),
             "or_debug_touch": (C.c_int, [V, C.c_uint32, C.c_uint64]),
+            "or_hist_bucket": (C.c_uint32, [C.c_uint64]),
+            "or_hist_lower": (C.c_uint64, [C.c_uint32]),
+            "or_get_metrics": (None, [V, u64p, P(C.c_double), V, C.c_int]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -138,10 +150,19 @@ def ring_successor(vpos, p):
     return lib().or_ring_successor(vp, len(vp), p)
 
 
-def choose(c1, c2, h1, h2, L, W1, W2, slo, cost=1):
+def choose(c1, c2, h1, h2, L, W1, W2, slo, cost=1, rule=RULE_DUALMAP):
     t1, t2, sw = C.c_uint64(), C.c_uint64(), C.c_uint8()
-    ch = lib().or_choose(c1, c2, h1, h2, L, W1, W2, slo, cost, C.byref(t1), C.byref(t2), C.byref(sw))
+    ch = lib().or_choose(rule, c1, c2, h1, h2, L, W1, W2, slo, cost, C.byref(t1), C.byref(t2),
+                         C.byref(sw))
     return ch, t1.value, t2.value, sw.value
+
+
+def hist_bucket(v):
+    return lib().or_hist_bucket(v)
+
+
+def hist_lower(k):
+    return lib().or_hist_lower(k)
 
 
 def config_from_workload(w, **kw):
@@ -196,6 +217,16 @@ class Oracle:
 
     def commit(self):
         return lib().or_commit(self.h)
+
+    def metrics(self, reset=False):
+        """Counters (METRIC_KEYS), cv_sum, cv_last and the TTFT histogram."""
+        u = np.zeros(len(METRIC_KEYS), np.uint64)
+        d = (C.c_double * 2)()
+        hist = np.zeros(HIST_BUCKETS, np.uint64)
+        lib().or_get_metrics(self.h, u, d, hist.ctypes.data, 1 if reset else 0)
+        m = {k: int(v) for k, v in zip(METRIC_KEYS, u)}
+        m["cv_sum"], m["cv_last"] = d[0], d[1]
+        return m, hist
 
     def rebalance(self, cap=1 << 16):
         seq = np.zeros(cap, np.uint64)
