@@ -231,6 +231,8 @@ def main():
                     help="override a workload field (small cases for profiling)")
     ap.add_argument("--max-touch", type=int, default=0, help="override max_touch_per_instance")
     ap.add_argument("--index-slots-log2", type=int, default=0, help="override the index size (log2 slots)")
+    ap.add_argument("--rule", default="dualmap",
+                    help="choice rule (dualmap, pair_*, cache_affinity, least_loaded, min_ttft, preble)")
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":
@@ -256,6 +258,8 @@ def main():
         kw["max_touch_per_instance"] = args.max_touch
     if args.index_slots_log2:
         kw["index_slots_log2"] = args.index_slots_log2
+    rule = D.RULE_NAMES.index(args.rule)
+    kw["choice_rule"] = rule
 
     # all batches' tokens resident in HBM (a pass longer than the trace replays it cyclically)
     used = min(nb, W + K)
@@ -396,12 +400,14 @@ def main():
     st_all = D.dm_get_stage_times(g.h, reset=True)
     D.dm_set_profiling(g.h, False)
     assert g.last_error() == 0
+    met, _ = D.dm_get_metrics(g.h)
     stage_ms = {k: v[0] / max(v[1], 1) for k, v in st_all.items()}
     prompt_gbps = bytes_per_launch / ((stage_ms["hash"] + stage_ms["probe"]) / 1e3) / 1e9
     # route: setup (with the queue drain), segmap, hash, probe, choice (5); commit:
     # maint_plan, maint_a, compact_scan, maint_c, commit_prep, commit_touch,
     # touch_deferred, req_counts, evict (9); rebalance (1)
-    launches_per_step = 5 + 9 + (1 if w.get("rebalance") else 0)
+    # (the cluster-wide rules add the all-instance probe kernel)
+    launches_per_step = 5 + 9 + (1 if w.get("rebalance") else 0) + (1 if rule >= D.DM_RULE_LEAST_LOADED else 0)
     clocks = sampler.summary(wall0, wall1)
     g.close()
     del g
@@ -430,6 +436,7 @@ def main():
                                    f"batches of {w['batch']} prompts of {describe_lengths(w)} tokens "
                                    f"(~{bytes_per_launch / 1e6:.0f} MB per batch)",
                        "global_batch": w["batch"], "parallelism": f"replicas x{world}",
+                       "choice_rule": args.rule,
                        "l2": ("inputs larger than L2 (each batch > 129 MB, distinct per step)"
                               if bytes_per_launch > 129e6 else
                               "batches smaller than L2, L2 not flushed between steps"),
@@ -439,6 +446,12 @@ def main():
                          "traffic": traffic_per_launch(bytes_per_launch), "bytes_per_launch": bytes_per_launch,
                          "avg_launch_ms": hash_avg_s * 1e3},
             "stage_ms_per_step": stage_ms,
+            "serving": {"hit_rate": met["hit_tokens"] / max(met["prompt_tokens"], 1),
+                        "cv_mean": met["cv_sum"] / max(met["cv_samples"], 1),
+                        "slo_attainment": met["slo_met"] / max(met["completed"], 1),
+                        "ttft_p50_us": met["ttft_p50_us"], "ttft_p90_us": met["ttft_p90_us"],
+                        "completed": met["completed"], "requests": met["requests"],
+                        "note": "scheduler time model over the stage-breakdown replay"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches_per_step * K, "clocks": clocks,
         }
         print(json.dumps(line), flush=True)

@@ -58,6 +58,43 @@ typedef enum {
     DM_ERR_OOM = 9            /* device or host allocation failed */
 } dm_status;
 
+/* Choice rules of dm_route_batch's last step.
+ *
+ * DualMap's own rule (Sec. 3.2): ttft_f = W[c_f] + cost * (L - hit_f); the
+ * candidate with more hit tokens unless its ttft exceeds the SLO, then the
+ * less-loaded (by W) of the two, tie: the higher-hit one ("switched");
+ * equal hits take the less-loaded, tie c1.
+ *
+ * Between the same two candidates (the ablation variants of Sec. 4.3):
+ *   PAIR_CACHE_AFFINITY  more hit tokens; equal hits: less loaded, tie c1.
+ *   PAIR_LEAST_LOADED    smaller W, tie c1.
+ *   PAIR_MIN_TTFT        smaller ttft_f, tie c1.
+ *   PAIR_PREBLE          2 * max(hit1, hit2) > L ? PAIR_CACHE_AFFINITY
+ *                        : PAIR_MIN_TTFT (Preble's 50% rule, Sec. 2.2).
+ *   switched = the hits differ and the candidate with fewer was chosen.
+ * Over every live instance (the cluster-wide baselines of Sec. 2.2 and
+ * Sec. 4; hit_i is probed on every live instance, an extra kernel whose
+ * cost grows with the instance count):
+ *   CACHE_AFFINITY  always c1, the ring-1 owner (one prompt-aware mapping).
+ *   LEAST_LOADED    smallest W_i, tie lowest id.
+ *   MIN_TTFT        smallest W_i + cost * (L - hit_i), tie lowest id
+ *                   (Mooncake's rule as Sec. 2.2 describes it).
+ *   PREBLE          2 * max_i hit_i > L ? among the instances with that hit
+ *                   the smallest W_i, tie lowest id : MIN_TTFT.
+ *   switched = 0; ttft1/ttft2 still describe the two candidates, and the
+ *   queued work is cost * (L - hit) of the chosen instance. */
+typedef enum {
+    DM_RULE_DUALMAP = 0,
+    DM_RULE_PAIR_CACHE_AFFINITY = 1,
+    DM_RULE_PAIR_LEAST_LOADED = 2,
+    DM_RULE_PAIR_MIN_TTFT = 3,
+    DM_RULE_PAIR_PREBLE = 4,
+    DM_RULE_CACHE_AFFINITY = 5,
+    DM_RULE_LEAST_LOADED = 6,
+    DM_RULE_MIN_TTFT = 7,
+    DM_RULE_PREBLE = 8
+} dm_choice_rule;
+
 /* Scheduler configuration (copied at dm_create). */
 typedef struct {
     /* Tokens per block, B.  One of 4, 8, 16, 32, 64.  Blocks are the unit of
@@ -98,6 +135,12 @@ typedef struct {
      * 64; <= 32.  dm_create returns DM_ERR_INVALID_ARG when the resulting
      * index would exceed 2^32 slots (it records slot numbers as 32 bits). */
     uint32_t index_slots_log2;
+    /* The choice rule of dm_route_batch (dm_choice_rule); 0 = DualMap's
+     * SLO-aware rule.  The others are the rules DualMap is compared with,
+     * for experiments; DM_ERR_INVALID_ARG for an unknown value. */
+    uint32_t choice_rule;
+    /* Must be 0. */
+    uint32_t reserved1;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */
@@ -146,7 +189,8 @@ enum {
                               stage's kernel, so it is timed there; 0 calls) */
     DM_STAGE_HASH = 2,     /* token hashing into chained block prefix values */
     DM_STAGE_PROBE = 3,    /* ring lookup, distinct fix, cache probes */
-    DM_STAGE_CHOICE = 4,   /* sequential SLO-aware choice */
+    DM_STAGE_CHOICE = 4,   /* sequential choice (with the all-instance probes of the
+                              cluster-wide rules) */
     DM_STAGE_COMMIT = 5,   /* cache commit with LRU eviction */
     DM_STAGE_REBALANCE = 6,/* hotspot-aware rebalancing */
     DM_STAGE_COUNT = 7
@@ -182,7 +226,8 @@ DM_API dm_status dm_remove_instance(dm_handle *h, uint32_t id);
  *      block keys (index state as of the start of the batch);
  *   5. in arrival order: TTFT_f = W[c_f] + cost * (L - hit_f); the higher-hit
  *      candidate unless its TTFT exceeds the SLO, then the less-loaded one;
- *      equal hits take the less-loaded one; the request is queued there.
+ *      equal hits take the less-loaded one; the request is queued there
+ *      (or the configured dm_choice_rule decides).
  * The batch is kept for dm_commit_cache.  Asynchronous. */
 DM_API dm_status dm_route_batch(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
 
@@ -290,6 +335,43 @@ DM_API dm_status dm_get_clock(dm_handle *h, uint64_t *clock_host);
  * any routing result.  For tests and monitoring; read-only, synchronous,
  * works after a sticky error. */
 DM_API dm_status dm_get_maint_counts(dm_handle *h, uint64_t *rebuilds_host, uint64_t *compactions_host);
+
+/* Serving metrics kept on the device since dm_create or the last reset
+ * (Sec. 2.2: load-balance CV; Sec. 4.1: cache hit rate, SLO attainment,
+ * TTFT percentiles).  The time model is the scheduler's own: each queue
+ * runs its work at one microsecond per microsecond from the batch times
+ * on, so a request completes when the work ahead of it and its own is
+ * done, and its TTFT is that moment minus its batch time (kept across
+ * migrations).  Requests still queued are not counted as completed. */
+#define DM_HIST_BUCKETS 976u   /* TTFT histogram: 0..15 exact, then 16 per power of two */
+typedef struct {
+    uint64_t requests;        /* routed requests */
+    uint64_t prompt_tokens;   /* sum of their lengths */
+    uint64_t hit_tokens;      /* sum of the cached-prefix tokens on the chosen instance at routing */
+    uint64_t switched;        /* requests routed with switched = 1 */
+    uint64_t est_slo_met;     /* requests whose estimated TTFT on the chosen instance
+                                 (its load including the request) was <= SLO when routed */
+    uint64_t completed;       /* requests whose prefill completed in a drain */
+    uint64_t ttft_sum_us;     /* sum of their TTFTs */
+    uint64_t ttft_max_us;
+    uint64_t slo_met;         /* completed with TTFT <= SLO */
+    uint64_t ttft_p50_us;     /* the lower edge of the histogram bucket holding the */
+    uint64_t ttft_p90_us;     /* ceil(p * completed)-th smallest TTFT (0 if none); the */
+    uint64_t ttft_p99_us;     /* bucket is at most 1/16 of its lower edge wide */
+    uint64_t cv_samples;      /* batches with at least one request */
+    double cv_sum;            /* sum over those batches of the CV of the live instances' W
+                                 after the batch's choices: sqrt(n*S2 - S1^2) / S1 with
+                                 S1 = sum W_i, S2 = sum W_i^2 (0 if S1 = 0) */
+    double cv_last;           /* the last sample */
+} dm_metrics;
+
+/* Copy the metrics into *out_host and, if hist_host is not NULL, the first
+ * min(hist_cap, DM_HIST_BUCKETS) TTFT histogram counts; bucket k holds
+ * values v with v = k for k < 16, else e = floor(log2 v), k = 16 + 16(e-4) +
+ * ((v >> (e-4)) & 15).  reset = 1 then clears them.  Synchronous; works
+ * after a sticky error. */
+DM_API dm_status dm_get_metrics(dm_handle *h, dm_metrics *out_host, uint64_t *hist_host, uint32_t hist_cap,
+                                int reset);
 
 /* Synchronise the stream and return the sticky error (DM_OK if none). */
 DM_API dm_status dm_last_error(dm_handle *h);

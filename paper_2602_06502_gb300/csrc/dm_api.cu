@@ -202,6 +202,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.max_batch < 1 || c.max_batch > (1u << 24) || c.max_batch_tokens < B) return DM_ERR_INVALID_ARG;
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
     if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
+    if (c.choice_rule > DM_RULE_PREBLE || c.reserved1 != 0) return DM_ERR_INVALID_ARG;
 
     dm_handle *h = new dm_handle();
     h->cfg = c;
@@ -217,6 +218,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.hot_num = c.hot_num;
     d.hot_den = c.hot_den;
     d.max_batch = c.max_batch;
+    d.rule = c.choice_rule;
     d.max_blocks = c.max_batch_tokens / B;
     d.max_segs = d.max_blocks / dm::kSegBlocks + c.max_batch;
     d.T = c.max_touch_per_instance ? c.max_touch_per_instance : d.max_blocks;
@@ -290,6 +292,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.maint_count, 2));
     A(dalloc(h, &d.err, 1));
     A(dalloc(h, &d.seq_next, 1));
+    A(dalloc(h, &d.metrics, 1));
+    if (c.choice_rule >= DM_RULE_LEAST_LOADED) A(dalloc(h, &d.h_all, uint64_t(c.max_batch) * M));
     A(dalloc(h, &d.rb_key, d.rb_cap));
     A(dalloc(h, &d.rb_seq, d.rb_cap));
     A(dalloc(h, &d.rb_ttft, d.rb_cap));
@@ -335,6 +339,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     set_levels(d, 0);
     A(cudaMemsetAsync(d.inst_state, 0, M, h->st));
     A(cudaMemsetAsync(d.W, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.metrics, 0, sizeof(dm::DevMetrics), h->st));
     A(cudaMemsetAsync(d.q_head, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.q_tail, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.table, 0, M * 8, h->st));
@@ -521,16 +526,17 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
     if (h->n_live < 2) return DM_ERR_NO_INSTANCES;
     if (h->have_time && b->batch_time_us < h->t_prev) return DM_ERR_ORDER;
     const uint64_t delta = h->have_time ? b->batch_time_us - h->t_prev : 0;
+    const uint64_t t0 = h->have_time ? h->t_prev : b->batch_time_us;   // start of the drain window
     h->t_prev = b->batch_time_us;
     h->have_time = true;
     const DevState &d = h->d;
     cudaError_t e;
-    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_drain(d, *b, delta, h->st); }   // drain included
+    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_drain(d, *b, delta, t0, h->st); }   // drain included
     if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_HASH); e = dm::launch_hash(d, *b, h->hash_grid, h->st); }
     if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_PROBE); e = dm::launch_route_probe(d, *b, *o, h->st); }
     if (e == cudaSuccess && b->n) {
         Stage st(h, DM_STAGE_CHOICE);
-        e = dm::launch_choice(d, *o, b->n, h->seq_next, h->st);
+        e = dm::launch_choice(d, *o, b->n, h->seq_next, b->batch_time_us, h->st);
     }
     if (e != cudaSuccess) return map_cuda(h, e);
     h->pending = true;
@@ -753,6 +759,52 @@ dm_status dm_get_maint_counts(dm_handle *h, uint64_t *rebuilds_host, uint64_t *c
     if (e != cudaSuccess) return map_cuda(h, e);
     *rebuilds_host = c[0];
     *compactions_host = c[1];
+    return DM_OK;
+}
+
+// Lower edge of the histogram bucket holding the ceil(pnum/pden * count)-th
+// smallest value (0 for an empty histogram).
+static uint64_t hist_quantile(const unsigned long long *hist, uint64_t count, uint64_t pnum, uint64_t pden) {
+    if (count == 0) return 0;
+    uint64_t rank = (pnum * count + pden - 1) / pden;
+    if (rank == 0) rank = 1;
+    uint64_t cum = 0;
+    uint32_t k = 0;
+    for (; k + 1 < dm::kHistBuckets; ++k) {
+        cum += hist[k];
+        if (cum >= rank) break;
+    }
+    if (k < 16) return k;
+    const uint32_t e = 4 + (k - 16) / 16, sub = (k - 16) % 16;
+    return uint64_t(16 + sub) << (e - 4);
+}
+
+dm_status dm_get_metrics(dm_handle *h, dm_metrics *out, uint64_t *hist_host, uint32_t hist_cap, int reset) {
+    dm_status s = check_handle(h);
+    if (s) return s;
+    if (!out || (hist_cap && !hist_host)) return DM_ERR_INVALID_ARG;
+    dm::DevMetrics m;
+    cudaError_t e = cudaMemcpyAsync(&m, h->d.metrics, sizeof m, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess && reset) e = cudaMemsetAsync(h->d.metrics, 0, sizeof m, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    dm::fold_cv(&m);   // the last batch's sample (the device folds it at the next batch)
+    out->requests = m.requests;
+    out->prompt_tokens = m.prompt_tokens;
+    out->hit_tokens = m.hit_tokens;
+    out->switched = m.switched;
+    out->est_slo_met = m.est_slo_met;
+    out->completed = m.completed;
+    out->ttft_sum_us = m.ttft_sum;
+    out->ttft_max_us = m.ttft_max;
+    out->slo_met = m.slo_met;
+    out->ttft_p50_us = hist_quantile(m.hist, m.completed, 50, 100);
+    out->ttft_p90_us = hist_quantile(m.hist, m.completed, 90, 100);
+    out->ttft_p99_us = hist_quantile(m.hist, m.completed, 99, 100);
+    out->cv_samples = m.cv_samples;
+    out->cv_sum = m.cv_sum;
+    out->cv_last = m.cv_last;
+    for (uint32_t k = 0; k < hist_cap && k < dm::kHistBuckets; ++k) hist_host[k] = m.hist[k];
     return DM_OK;
 }
 

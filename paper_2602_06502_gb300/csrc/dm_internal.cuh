@@ -20,12 +20,66 @@ constexpr uint32_t kRbChunk = 4096;      // index slots per rebuild chunk
 constexpr uint64_t kSpinLimit = 1ull << 26; // bound of every data-dependent device loop
 constexpr uint32_t kGroup = 8;           // consecutive blocks of a prompt homed in one 128-byte index line
 
-// One queued request (48 bytes).
+// One queued request (56 bytes).
 struct QEntry {
     uint64_t seq, work, remaining;
     uint32_t L, c1, c2, h1, h2;
     uint32_t moved;   // 0, or the rebalance call that moved it here, or kTomb
+    uint64_t arrival; // batch time the request arrived with
 };
+
+// Serving metrics (dm_metrics before the percentiles), updated by the
+// choice kernels and the drain.  A choice kernel leaves its batch's load
+// sums (S1 = sum W, S2 = sum W^2 over the live instances, n of them; exact
+// 128-bit integers) pending; the next setup kernel, or dm_get_metrics,
+// turns them into the batch's CV sample, so the floating-point steps stay
+// off the choice kernel's tail.
+constexpr uint32_t kHistBuckets = DM_HIST_BUCKETS;
+struct DevMetrics {
+    unsigned long long requests, prompt_tokens, hit_tokens, switched, est_slo_met;
+    unsigned long long completed, ttft_sum, ttft_max, slo_met, cv_samples;
+    double cv_sum, cv_last;
+    unsigned long long pend, pend_n, pend_s1[2], pend_s2[2];   // [lo, hi]
+    unsigned long long hist[kHistBuckets];
+};
+
+// Population CV of Sec. 2.2 from the exact sums: sqrt(n*S2 - S1^2) / S1
+// (0 when S1 = 0); each 128-bit integer becomes double(hi) * 2^64 +
+// double(lo), every step rounded to nearest.
+__host__ __device__ inline double u128_as_double(unsigned __int128 x) {
+#ifdef __CUDA_ARCH__
+    return __dadd_rn(__dmul_rn(__ull2double_rn((uint64_t)(x >> 64)), 18446744073709551616.0),
+                     __ull2double_rn((uint64_t)x));
+#else
+    const double hi = (double)(uint64_t)(x >> 64) * 18446744073709551616.0;   // exact
+    return hi + (double)(uint64_t)x;
+#endif
+}
+
+__host__ __device__ inline double load_cv(uint64_t n, unsigned __int128 S1, unsigned __int128 S2) {
+    if (S1 == 0) return 0.0;
+#ifdef __CUDA_ARCH__
+    return __ddiv_rn(__dsqrt_rn(u128_as_double((unsigned __int128)n * S2 - S1 * S1)), u128_as_double(S1));
+#else
+    return __builtin_sqrt(u128_as_double((unsigned __int128)n * S2 - S1 * S1)) / u128_as_double(S1);
+#endif
+}
+
+// Fold a pending CV sample into the running sum.  One thread.
+__host__ __device__ inline void fold_cv(DevMetrics *m) {
+    if (!m->pend) return;
+    const unsigned __int128 S1 = ((unsigned __int128)m->pend_s1[1] << 64) | m->pend_s1[0];
+    const unsigned __int128 S2 = ((unsigned __int128)m->pend_s2[1] << 64) | m->pend_s2[0];
+    const double cv = load_cv(m->pend_n, S1, S2);
+#ifdef __CUDA_ARCH__
+    m->cv_sum = __dadd_rn(m->cv_sum, cv);
+#else
+    m->cv_sum = m->cv_sum + cv;
+#endif
+    m->cv_last = cv;
+    m->cv_samples += 1;
+    m->pend = 0;
+}
 
 // One index slot (16 bytes): a block key and 1 + the position of its latest
 // record in the instance's recency log; key 0 marks an empty slot.  A key is
@@ -93,6 +147,7 @@ struct DevState {
     uint32_t B, Kroute, V, M;
     uint64_t C, slo;
     uint32_t cost, hot_num, hot_den, max_batch;
+    uint32_t rule;                  // dm_choice_rule
     uint64_t max_blocks, max_segs, T, S, logcap;
     uint32_t Q;
     // key material
@@ -143,6 +198,8 @@ struct DevState {
     uint64_t *maint_count;          // index rebuilds and log compactions so far (2 counters)
     uint32_t *err;
     uint64_t *seq_next;
+    DevMetrics *metrics;
+    uint32_t *h_all;                // max_batch x M hit tokens (cluster-wide rules only)
     // rebalance scratch
     uint64_t *rb_key;               // sort keys (benefit, biased) per candidate
     uint64_t *rb_seq;
@@ -353,9 +410,51 @@ __device__ __forceinline__ void route_positions(const DevState &d, uint32_t r, i
     pos2 = fmix64(p2 ^ d.Sr2);
 }
 
+// ---------------------------------------------------------------------------
+// Metrics helpers.
+
+// TTFT histogram bucket: v < 16 exact; else e = floor(log2 v) and the four
+// bits below the top one select one of 16 buckets of [2^e, 2^(e+1)).
+__device__ __forceinline__ uint32_t hist_bucket(uint64_t v) {
+    if (v < 16) return (uint32_t)v;
+    const uint32_t e = 63 - __clzll((long long)v);
+    return 16 + 16 * (e - 4) + (uint32_t)((v >> (e - 4)) & 15);
+}
+
+__device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) v += shfl_xor_u64(v, o);
+    return v;
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) v = max(v, shfl_xor_u64(v, o));
+    return v;
+}
+
+// Completed requests of one warp step: lanes with fin set finished with
+// TTFT ttft.  Whole warp.
+__device__ __forceinline__ void record_completions(DevMetrics *m, bool fin, uint64_t ttft, uint64_t slo,
+                                                   int lane) {
+    const uint32_t fm = __ballot_sync(0xffffffffu, fin);
+    if (!fm) return;
+    if (fin) atomicAdd(&m->hist[hist_bucket(ttft)], 1ull);
+    const uint64_t sum = warp_sum_u64(fin ? ttft : 0);
+    const uint64_t mx = warp_max_u64(fin ? ttft : 0);
+    const uint32_t met = __popc(__ballot_sync(0xffffffffu, fin && ttft <= slo));
+    if (lane == 0) {
+        atomicAdd(&m->completed, (unsigned long long)__popc(fm));
+        atomicAdd(&m->ttft_sum, (unsigned long long)sum);
+        atomicMax(&m->ttft_max, (unsigned long long)mx);
+        if (met) atomicAdd(&m->slo_met, (unsigned long long)met);
+    }
+}
+
 // Run `delta` us of prefill work off the head of instance i's queue (Sec.
 // 3.2: an instance's load is its pending prefill work).  Whole warp.
-__device__ __forceinline__ void drain_queue(const DevState &d, uint32_t i, uint64_t delta, int lane) {
+__device__ __forceinline__ void drain_queue(const DevState &d, uint32_t i, uint64_t delta, uint64_t t0,
+                                            int lane) {
     uint32_t head = d.q_head[i];
     const uint32_t tail = d.q_tail[i];
     if (head == tail) return;
@@ -364,10 +463,17 @@ __device__ __forceinline__ void drain_queue(const DevState &d, uint32_t i, uint6
     while (head != tail) {
         const uint32_t cnt = min(32u, tail - head);
         const uint32_t idx = (head + lane) & (d.Q - 1);
-        const uint64_t rem = (uint32_t)lane < cnt ? qb[idx].remaining : 0;
+        const bool valid = (uint32_t)lane < cnt;
+        const uint64_t rem = valid ? qb[idx].remaining : 0;
+        const uint32_t moved = valid ? qb[idx].moved : 0;
+        const uint64_t arrival = valid ? qb[idx].arrival : 0;
         const uint64_t inc = warp_incl_scan(rem, lane);
-        const uint32_t done = __ballot_sync(0xffffffffu, (uint32_t)lane < cnt && inc <= left);
+        const uint32_t done = __ballot_sync(0xffffffffu, valid && inc <= left);
         const uint32_t ndone = __popc(done);   // a prefix of the lanes
+        // Entry `lane` completes `used + inc` us into the window that starts
+        // at t0; migrated-away entries (no work left here) are not requests.
+        const bool fin = ((done >> lane) & 1u) && moved != kTomb;
+        record_completions(d.metrics, fin, fin ? t0 + used + inc - arrival : 0, d.slo, lane);
         if (ndone == cnt) {                    // whole chunk drained
             const uint64_t tot = shfl_u64(inc, 31);
             left -= tot;
@@ -425,13 +531,14 @@ inline int full_grid(K kernel, int block) {
 // ---------------------------------------------------------------------------
 // Host-side launchers (one translation unit each).
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st);
-cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, cudaStream_t st);
+cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, uint64_t t0,
+                               cudaStream_t st);
 cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st);
 int hash_grid_size();
 cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
                                cudaStream_t st);
 cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, uint64_t seq0,
-                          cudaStream_t st);
+                          uint64_t t_batch, cudaStream_t st);
 cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st);
 cudaError_t launch_rebalance(const DevState &d, uint32_t n, uint64_t seq0, uint32_t call,
                              dm_migration *out, uint32_t cap, uint32_t *n_out, cudaStream_t st);

@@ -316,6 +316,7 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
                 e.h1 = Ch.h1[k];
                 e.h2 = Ch.h2[k];
                 e.moved = call;
+                e.arrival = src->arrival;   // TTFT still counts from the original arrival
                 d.q[uint64_t(j) * d.Q + (Ch.mv_slot[t] & (d.Q - 1))] = e;
                 if (e.seq >= seq0 && e.seq < seq0 + n) {
                     d.r_final[e.seq - seq0] = j;

@@ -43,17 +43,22 @@ __device__ __forceinline__ void block_scan2(uint64_t a, uint32_t b, uint64_t &ea
 }
 
 // CTA 0: validate the batch and lay out per-request block / segment
-// offsets.  CTAs 1.. (routing only): drain the queues by `delta` us, a warp
-// per instance (independent of the batch layout).
+// offsets.  Routing only: CTA 1 folds the previous batch's pending CV
+// sample into the metrics; CTAs 2.. drain the queues by `delta` us from
+// time t0 on, a warp per instance (independent of the batch layout).
 __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off, const uint32_t *len,
-                                                uint32_t n, uint64_t total_tokens, uint64_t delta) {
+                                                uint32_t n, uint64_t total_tokens, uint64_t delta, uint64_t t0) {
     pdl_enter();
     __shared__ uint64_t sa[32];
     __shared__ uint32_t sb[32];
     if (has_err(d.err)) return;
-    if (blockIdx.x > 0) {
-        const uint32_t i = (blockIdx.x - 1) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-        if (i < d.M) drain_queue(d, i, delta, threadIdx.x & 31);
+    if (blockIdx.x == 1) {   // the previous batch's CV sample (beside the layout)
+        if (threadIdx.x == 0) fold_cv(d.metrics);
+        return;
+    }
+    if (blockIdx.x > 1) {
+        const uint32_t i = (blockIdx.x - 2) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+        if (i < d.M) drain_queue(d, i, delta, t0, threadIdx.x & 31);
         return;
     }
     uint64_t carry_blk = 0;
@@ -108,14 +113,17 @@ __global__ void k_segmap(DevState d, uint32_t n) {
 }
 
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st) {
-    DM_TRY(launch_pdl(k_setup, 1, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens, uint64_t(0)));
+    DM_TRY(launch_pdl(k_setup, 1, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens, uint64_t(0),
+                      uint64_t(0)));
     if (b.n) DM_TRY(launch_pdl(k_segmap, (b.n + 7) / 8, 256, 0, st, d, b.n));
     return cudaGetLastError();
 }
 
-cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, cudaStream_t st) {
+cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, uint64_t t0,
+                               cudaStream_t st) {
     const unsigned drain_ctas = (d.M + 31) / 32;
-    DM_TRY(launch_pdl(k_setup, 1 + drain_ctas, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens, delta));
+    DM_TRY(launch_pdl(k_setup, 2 + drain_ctas, 1024, 0, st, d, b.offsets, b.lengths, b.n, b.total_tokens, delta,
+                      t0));
     if (b.n) DM_TRY(launch_pdl(k_segmap, (b.n + 7) / 8, 256, 0, st, d, b.n));
     return cudaGetLastError();
 }

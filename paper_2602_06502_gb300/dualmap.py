@@ -19,6 +19,14 @@ DM_ERR_DUPLICATE_ID, DM_ERR_UNKNOWN_ID, DM_ERR_ORDER, DM_ERR_CUDA = 4, 5, 6, 7
 DM_ERR_TIMEOUT, DM_ERR_OOM = 8, 9
 STAGES = ["setup", "drain", "hash", "probe", "choice", "commit", "rebalance"]
 
+# dm_choice_rule
+DM_RULE_DUALMAP, DM_RULE_PAIR_CACHE_AFFINITY, DM_RULE_PAIR_LEAST_LOADED = 0, 1, 2
+DM_RULE_PAIR_MIN_TTFT, DM_RULE_PAIR_PREBLE = 3, 4
+DM_RULE_CACHE_AFFINITY, DM_RULE_LEAST_LOADED, DM_RULE_MIN_TTFT, DM_RULE_PREBLE = 5, 6, 7, 8
+RULE_NAMES = ["dualmap", "pair_cache_affinity", "pair_least_loaded", "pair_min_ttft", "pair_preble",
+              "cache_affinity", "least_loaded", "min_ttft", "preble"]
+DM_HIST_BUCKETS = 976
+
 
 class dm_config(C.Structure):
     _fields_ = [
@@ -36,6 +44,8 @@ class dm_config(C.Structure):
         ("max_touch_per_instance", C.c_uint64),
         ("max_queue", C.c_uint32),
         ("index_slots_log2", C.c_uint32),
+        ("choice_rule", C.c_uint32),
+        ("reserved1", C.c_uint32),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]
@@ -56,6 +66,13 @@ class dm_batch(C.Structure):
 class dm_route_out(C.Structure):
     _fields_ = [(name, C.c_void_p) for name in
                 ("cand1", "cand2", "hit1", "hit2", "ttft1", "ttft2", "chosen", "switched")]
+
+
+class dm_metrics(C.Structure):
+    _fields_ = [(name, C.c_uint64) for name in
+                ("requests", "prompt_tokens", "hit_tokens", "switched", "est_slo_met", "completed", "ttft_sum_us",
+                 "ttft_max_us", "slo_met", "ttft_p50_us", "ttft_p90_us", "ttft_p99_us", "cv_samples")] + \
+               [("cv_sum", C.c_double), ("cv_last", C.c_double)]
 
 
 class dm_migration(C.Structure):
@@ -94,6 +111,7 @@ SIGNATURES = {
                                  C.POINTER(C.c_uint32)]),
     "dm_get_clock": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64)]),
     "dm_get_maint_counts": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
+    "dm_get_metrics": (C.c_int, [C.c_void_p, C.POINTER(dm_metrics), C.c_void_p, C.c_uint32, C.c_int]),
     "dm_last_error": (C.c_int, [C.c_void_p]),
     "dm_set_profiling": (C.c_int, [C.c_void_p, C.c_int]),
     "dm_get_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int]),
@@ -243,6 +261,15 @@ def dm_get_maint_counts(h):
     a, b = C.c_uint64(), C.c_uint64()
     _check(lib().dm_get_maint_counts(h, C.byref(a), C.byref(b)), "dm_get_maint_counts")
     return a.value, b.value
+
+
+def dm_get_metrics(h, reset=False):
+    """(dict of dm_metrics fields, TTFT histogram counts)."""
+    m = dm_metrics()
+    hist = np.zeros(DM_HIST_BUCKETS, np.uint64)
+    _check(lib().dm_get_metrics(h, C.byref(m), hist.ctypes.data, DM_HIST_BUCKETS, 1 if reset else 0),
+           "dm_get_metrics")
+    return {name: getattr(m, name) for name, _ in dm_metrics._fields_}, hist
 
 
 def dm_last_error(h):

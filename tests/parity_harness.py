@@ -17,7 +17,7 @@ class Pair:
     """An oracle and a GPU scheduler built from the same workload dict."""
 
     def __init__(self, w, max_instances=None, max_batch_tokens=None, max_touch=0, max_queue=0, capacity=None,
-                 index_slots_log2=0):
+                 index_slots_log2=0, choice_rule=0):
         import torch
         from paper_2602_06502_gb300.scheduler import Scheduler
         self.torch = torch
@@ -27,12 +27,13 @@ class Pair:
         w = self.w
         self.M = max_instances or (w["n_instances"] + 8)
         mbt = max_batch_tokens or (1 << 24)
-        self.ora = O.Oracle(**O.config_from_workload(w, max_instances=self.M, max_batch_tokens=mbt))
+        self.ora = O.Oracle(**O.config_from_workload(w, max_instances=self.M, max_batch_tokens=mbt),
+                            choice_rule=choice_rule)
         self.gpu = Scheduler(block_tokens=w["block_tokens"], route_prefix_blocks=w["route_prefix_blocks"],
                              vnodes=w["vnodes"], max_instances=self.M, capacity=w["capacity"], slo_us=w["slo_us"],
                              cost_us=w["cost_us"], max_batch=w["batch"], max_batch_tokens=mbt,
                              max_touch_per_instance=max_touch, max_queue=max_queue,
-                             index_slots_log2=index_slots_log2, seed=w["seed"])
+                             index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule)
         self.dev = torch.device("cuda:0")
         self.n_migrations = 0
         self.n_switched = 0
@@ -91,6 +92,19 @@ class Pair:
         assert self.gpu.last_error() == 0, tag
         assert np.array_equal(self.gpu.loads(), self.ora.loads()), tag
 
+    def check_metrics(self, tag=""):
+        """Serving metrics: every counter, the TTFT histogram and the CV
+        samples (floating point, bit for bit)."""
+        from paper_2602_06502_gb300 import dualmap as D
+        gm, gh = D.dm_get_metrics(self.gpu.h)
+        om, oh = self.ora.metrics()
+        assert np.array_equal(gh, oh), f"{tag}: TTFT histogram"
+        for k in O.METRIC_KEYS:
+            assert gm[k] == om[k], f"{tag}: {k} gpu {gm[k]} vs oracle {om[k]}"
+        for k in ("cv_sum", "cv_last"):
+            assert gm[k] == om[k], f"{tag}: {k} gpu {gm[k]!r} vs oracle {om[k]!r}"
+        return om
+
     def check_state(self, ids=None, tag=""):
         """Loads, queues (seq, work, remaining), resident (key, stamp) sets, clock."""
         from paper_2602_06502_gb300 import dualmap as D
@@ -130,5 +144,7 @@ def run_trace(pair, tr, batches=None, rebalance=None, state_every=0, check_state
         pair.check_loads(tag=f"batch {b}")
         if state_every and (b + 1) % state_every == 0:
             pair.check_state(tag=f"batch {b}")
+            pair.check_metrics(tag=f"batch {b}")
     if check_state_end:
         pair.check_state(tag="end")
+    return pair.check_metrics(tag="end")

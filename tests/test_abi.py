@@ -54,15 +54,18 @@ def test_status_strings_without_gpu(built):
 def test_create_rejects_bad_config_without_touching_gpu(built):
     """Synchronous argument checks run before any CUDA call."""
     D = built
-    bad = D.dm_config(17, 16, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)   # B = 17
-    bad4 = D.dm_config(16, 16, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 41, 1, None)  # index > 2^40
+
+    def cfg(**kw):
+        base = dict(block_tokens=16, route_prefix_blocks=16, vnodes_per_instance=8, max_instances=8,
+                    cache_capacity_blocks=1024, slo_us=1, cost_us_per_token=1, hot_num=3, hot_den=2, max_batch=16,
+                    max_batch_tokens=1 << 20, seed=1)
+        base.update(kw)
+        return D.dm_config(**base)
+
     h = C.c_void_p()
-    assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
-    bad2 = D.dm_config(16, 0, 8, 8, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)   # K_route = 0
-    assert D.lib().dm_create(C.byref(bad2), C.byref(h)) == D.DM_ERR_INVALID_ARG
-    bad3 = D.dm_config(16, 16, 8, 1, 1024, 1, 1, 3, 2, 16, 1 << 20, 0, 0, 0, 1, None)  # one instance
-    assert D.lib().dm_create(C.byref(bad3), C.byref(h)) == D.DM_ERR_INVALID_ARG
-    assert D.lib().dm_create(C.byref(bad4), C.byref(h)) == D.DM_ERR_INVALID_ARG
+    for bad in (cfg(block_tokens=17), cfg(index_slots_log2=41), cfg(route_prefix_blocks=0),
+                cfg(max_instances=1), cfg(choice_rule=D.DM_RULE_PREBLE + 1), cfg(reserved1=1)):
+        assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
     assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
 
 
@@ -74,20 +77,26 @@ def test_struct_layouts_match_header(built, tmp_path):
         "dm_batch": [f for f, _ in D.dm_batch._fields_],
         "dm_route_out": [f for f, _ in D.dm_route_out._fields_],
         "dm_migration": ["req_seq", "from", "to"],
+        "dm_metrics": [f for f, _ in D.dm_metrics._fields_],
     }
     lines = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HDR}"', "int main(void) {"]
     for st, fs in fields.items():
         lines.append(f'printf("{st} %zu\\n", sizeof({st}));')
         for f in fs:
             lines.append(f'printf("{st}.{f} %zu\\n", offsetof({st}, {f}));')
+    consts = ["DM_HIST_BUCKETS"] + [f"DM_RULE_{n.upper()}" for n in D.RULE_NAMES]
+    for c in consts:
+        lines.append(f'printf("{c} %u\\n", (unsigned){c});')
     lines.append("return 0; }")
     prog.write_text("\n".join(lines))
     exe = tmp_path / "layout"
     subprocess.run(["gcc", str(prog), "-o", str(exe)], check=True)
     out = dict(l.rsplit(" ", 1) for l in subprocess.run([str(exe)], capture_output=True, text=True,
                                                         check=True).stdout.split("\n") if l)
+    for c in consts:
+        assert int(out[c]) == getattr(D, c), c
     for st, cls in (("dm_config", D.dm_config), ("dm_batch", D.dm_batch), ("dm_route_out", D.dm_route_out),
-                    ("dm_migration", D.dm_migration)):
+                    ("dm_migration", D.dm_migration), ("dm_metrics", D.dm_metrics)):
         assert int(out[st]) == C.sizeof(cls), st
         for (py, _), cn in zip(cls._fields_, fields[st]):
             assert int(out[f"{st}.{cn}"]) == getattr(cls, py).offset, (st, cn)

@@ -172,6 +172,56 @@ def test_scaling_parity_with_events():
     run_trace(p, tr, rebalance=True)
 
 
+# -- choice rules and serving metrics -------------------------------------------------
+
+RULES = list(range(9))   # dm_choice_rule: DualMap, four pair variants, four cluster-wide rules
+
+
+@pytest.mark.parametrize("rule", RULES)
+def test_choice_rules_tiny(rule):
+    """Every rule, bit for bit, with the metrics (completion TTFTs, CV)."""
+    w = workload("tiny", n_requests=2000, batch=100, zipf_s=1.2, rho=0.9, slo_us=20_000)
+    tr = Trace(w)
+    m = run_trace(Pair(w, choice_rule=rule), tr, state_every=5)
+    assert m["requests"] == 2000 and m["completed"] > 0 and m["cv_samples"] == 20
+
+
+@pytest.mark.parametrize("rule", [0, 3, 7, 8])
+def test_choice_rules_agent(rule):
+    """Tight load (the SLO switch fires), 64 instances, 4,096-request batches."""
+    tr = Trace(workload("agent", n_requests=2 * 4096))
+    p = Pair(tr.cfg, max_batch_tokens=40_000_000, max_touch=1 << 20, choice_rule=rule)
+    run_trace(p, tr)
+
+
+@pytest.mark.parametrize("rule", [0, 6, 8])
+def test_choice_rules_with_scaling_and_rebalance(rule):
+    """Instances added and removed between batches (the cluster-wide rules
+    skip removed ones), rebalancing after every batch (migrated requests
+    keep their arrival time for the TTFT)."""
+    w = workload("scaling", n_requests=4 * 2048, batch=2048, scale_every=2048, n_instances=48, vnodes=64,
+                 capacity=20_000)
+    tr = Trace(w)
+    assert len(tr.events) >= 3
+    p = Pair(tr.cfg, max_instances=w["n_instances"] + 4, max_batch_tokens=20_000_000, max_touch=1 << 20,
+             choice_rule=rule)
+    run_trace(p, tr, rebalance=True)
+
+
+def test_metrics_reset_and_rebalanced_ttft():
+    """Completion TTFTs after migrations, then a reset clears every metric."""
+    from paper_2602_06502_gb300 import dualmap as D
+    w = workload("tiny", n_requests=1500, batch=100, capacity=700, zipf_s=1.3, rho=1.2)
+    tr = Trace(w)
+    p = Pair(w, max_touch=2600)
+    run_trace(p, tr, rebalance=True)
+    assert p.n_migrations > 0
+    gm, gh = D.dm_get_metrics(p.gpu.h, reset=True)
+    assert gm["completed"] > 0
+    gm, gh = D.dm_get_metrics(p.gpu.h)
+    assert all(v == 0 for v in gm.values()) and gh.sum() == 0
+
+
 # -- edge cases ---------------------------------------------------------------------
 
 def _mk(**kw):
