@@ -178,6 +178,9 @@ typedef struct {
     uint64_t max_batch_tokens;
     uint64_t seed;
     uint32_t choice_rule;   /* OR_RULE_* */
+    uint32_t adapt_step_blocks;   /* adaptive prefix: blocks per extension; 0 = fixed K_route */
+    uint32_t adapt_max_blocks;    /* longest hash prefix, in blocks */
+    uint32_t adapt_window;        /* non-empty batches per hotness window */
 } or_config;
 
 enum { OR_RULE_DUALMAP = 0, OR_RULE_CACHE_AFFINITY = 1, OR_RULE_LEAST_LOADED = 2,
@@ -242,6 +245,17 @@ typedef struct {
     uint32_t *pend_final, *pend_nblk;
     uint64_t **pend_keys;
     int pending;
+    /* adaptive prefix: expanded nodes (sorted keys), this window's path
+     * records (node key, depth), its requests and non-empty batches, and
+     * the hash prefix length of each request of the last batch */
+    uint64_t *ad_set;
+    uint64_t ad_set_n;
+    uint64_t *ad_rec_key;
+    uint32_t *ad_rec_depth;
+    uint64_t ad_rec_n, ad_rec_cap;
+    uint64_t ad_requests, ad_batches;
+    uint32_t *last_K;
+    uint32_t last_n;
     /* metrics since create / the last reset */
     uint64_t m_requests, m_prompt_tokens, m_hit_tokens, m_switched, m_est_slo_met;
     uint64_t m_completed, m_ttft_sum, m_ttft_max, m_slo_met, m_batches;
@@ -616,6 +630,10 @@ void or_destroy(or_state *s)
     free(s->state);
     free(s->ring[0]);
     free(s->ring[1]);
+    free(s->ad_set);
+    free(s->ad_rec_key);
+    free(s->ad_rec_depth);
+    free(s->last_K);
     free(s);
 }
 
@@ -627,6 +645,10 @@ int or_create(const or_config *cfg, or_state **out)
         cfg->vnodes_per_instance < 1 || cfg->max_instances < 2 ||
         cfg->cache_capacity_blocks < 1 || cfg->cost_us_per_token < 1 ||
         cfg->hot_den < 1 || cfg->max_batch < 1 || cfg->max_batch_tokens < B)
+        return OR_ERR_INVALID_ARG;
+    if (cfg->adapt_step_blocks &&
+        (cfg->adapt_max_blocks <= cfg->route_prefix_blocks || cfg->adapt_max_blocks > 2048 ||
+         cfg->adapt_window < 1))
         return OR_ERR_INVALID_ARG;
     or_state *s = (or_state *)calloc(1, sizeof(or_state));
     if (!s) return OR_ERR_OOM;
@@ -762,6 +784,121 @@ static uint32_t choose_global(const or_state *s, uint32_t rule, const uint32_t *
     return best;
 }
 
+/* ------------------------------------------------------------------ */
+/* Adaptive hash-prefix length (Sec. 3.2, "how long prefix")            */
+/* ------------------------------------------------------------------ */
+
+/* Ring positions of a prompt hashed over its first K blocks. */
+static void positions_for(const or_state *s, const uint32_t *tok, uint32_t K, uint64_t *pos)
+{
+    const uint32_t B = s->cfg.block_tokens;
+    uint64_t P1 = 0, P2 = 0;
+    for (uint32_t k = 0; k < K; k++) {
+        const uint32_t *t = tok + (uint64_t)k * B;
+        P1 += or_fmix64(or_nh(t, s->K1, B) + (uint64_t)(k + 1) * s->G1);
+        P2 += or_fmix64(or_nh(t, s->K2, B) + (uint64_t)(k + 1) * s->G2);
+    }
+    pos[0] = or_fmix64(P1 ^ s->Sr1);
+    pos[1] = or_fmix64(P2 ^ s->Sr2);
+}
+
+static int cmp_u64(const void *a, const void *b)
+{
+    uint64_t x = *(const uint64_t *)a, y = *(const uint64_t *)b;
+    return x < y ? -1 : x > y;
+}
+
+static int expanded(const or_state *s, uint64_t key)
+{
+    return s->ad_set_n && bsearch(&key, s->ad_set, s->ad_set_n, sizeof(uint64_t), cmp_u64) != NULL;
+}
+
+static int path_push(or_state *s, uint64_t key, uint32_t depth)
+{
+    if (s->ad_rec_n == s->ad_rec_cap) {
+        uint64_t nc = s->ad_rec_cap ? 2 * s->ad_rec_cap : 1024;
+        uint64_t *k = (uint64_t *)realloc(s->ad_rec_key, nc * sizeof(uint64_t));
+        if (!k) return OR_ERR_OOM;
+        s->ad_rec_key = k;
+        uint32_t *d = (uint32_t *)realloc(s->ad_rec_depth, nc * sizeof(uint32_t));
+        if (!d) return OR_ERR_OOM;
+        s->ad_rec_depth = d;
+        s->ad_rec_cap = nc;
+    }
+    s->ad_rec_key[s->ad_rec_n] = key;
+    s->ad_rec_depth[s->ad_rec_n] = depth;
+    s->ad_rec_n++;
+    return OR_OK;
+}
+
+/* The request's hash prefix length: start at min(K_route, n_blk) blocks;
+ * while the node of the current prefix (the key of its last block) is
+ * expanded and the prompt and the cap allow, extend by one step.  Every
+ * node on the way is recorded for this window's hotness counts. */
+static int adapt_walk(or_state *s, const uint64_t *keys, uint32_t nblk, uint32_t *K)
+{
+    const or_config *c = &s->cfg;
+    uint32_t d = c->route_prefix_blocks < nblk ? c->route_prefix_blocks : nblk;
+    int rc = path_push(s, keys[d - 1], d);
+    while (!rc && d < nblk && d < c->adapt_max_blocks && expanded(s, keys[d - 1])) {
+        d += c->adapt_step_blocks;
+        if (d > nblk) d = nblk;
+        if (d > c->adapt_max_blocks) d = c->adapt_max_blocks;
+        rc = path_push(s, keys[d - 1], d);
+    }
+    *K = d;
+    return rc;
+}
+
+static int cmp_rec(const void *a, const void *b)
+{
+    const uint64_t *x = (const uint64_t *)a, *y = (const uint64_t *)b;
+    return x[0] < y[0] ? -1 : x[0] > y[0];
+}
+
+/* End of a window: with n live instances and T requests in the window, a
+ * node not expanded becomes expanded when its share count/T > 2/n and it
+ * lies above the cap; an expanded node stays expanded unless count/T < 1/n
+ * (so nodes no request reached are dropped).  Counts then restart. */
+static int adapt_window_end(or_state *s)
+{
+    const uint64_t n = n_live(s), T = s->ad_requests;
+    uint64_t m = s->ad_rec_n;
+    uint64_t *rec = (uint64_t *)malloc((m ? m : 1) * 2 * sizeof(uint64_t));
+    uint64_t *next = (uint64_t *)malloc((s->ad_set_n + m + 1) * sizeof(uint64_t));
+    if (!rec || !next) { free(rec); free(next); return OR_ERR_OOM; }
+    for (uint64_t i = 0; i < m; i++) {
+        rec[2 * i] = s->ad_rec_key[i];
+        rec[2 * i + 1] = s->ad_rec_depth[i];
+    }
+    qsort(rec, m, 2 * sizeof(uint64_t), cmp_rec);
+    uint64_t nn = 0;
+    /* expanded nodes: kept unless cold */
+    for (uint64_t j = 0; j < s->ad_set_n; j++) {
+        uint64_t key = s->ad_set[j], count = 0;
+        for (uint64_t i = 0; i < m; i++)
+            if (rec[2 * i] == key) count++;
+        if (!(count * n < T)) next[nn++] = key;
+    }
+    /* nodes reached this window: expanded when hot */
+    for (uint64_t i = 0; i < m;) {
+        uint64_t e = i;
+        while (e < m && rec[2 * e] == rec[2 * i]) e++;
+        const uint64_t key = rec[2 * i], depth = rec[2 * i + 1], count = e - i;
+        if (!expanded(s, key) && depth < s->cfg.adapt_max_blocks && count * n > 2 * T) next[nn++] = key;
+        i = e;
+    }
+    qsort(next, nn, sizeof(uint64_t), cmp_u64);
+    free(rec);
+    free(s->ad_set);
+    s->ad_set = next;
+    s->ad_set_n = nn;
+    s->ad_rec_n = 0;
+    s->ad_requests = 0;
+    s->ad_batches = 0;
+    return OR_OK;
+}
+
 static uint32_t leading_hits(const lru_t *c, const uint64_t *keys, uint32_t nblk)
 {
     uint32_t m = 0;
@@ -798,6 +935,10 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
     s->pend_final = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
     s->pend_nblk = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
     s->pend_keys = (uint64_t **)calloc(n ? n : 1, sizeof(uint64_t *));
+    uint32_t *lk = (uint32_t *)realloc(s->last_K, (n ? n : 1) * sizeof(uint32_t));
+    if (!lk) return OR_ERR_OOM;
+    s->last_K = lk;
+    s->last_n = n;
     if (!s->pend_final || !s->pend_nblk || !s->pend_keys) return OR_ERR_OOM;
 
     /* hits on every live instance, for the rules that look at all of them */
@@ -814,6 +955,14 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
         if (!keys) return OR_ERR_OOM;
         uint64_t pos[2];
         uint32_t nblk = prompt_keys(s, tokens + offsets[r], L, keys, pos);
+        uint32_t K = cf->route_prefix_blocks < nblk ? cf->route_prefix_blocks : nblk;
+        if (cf->adapt_step_blocks) {
+            int rc = adapt_walk(s, keys, nblk, &K);
+            if (rc) return rc;
+            if (K != (cf->route_prefix_blocks < nblk ? cf->route_prefix_blocks : nblk))
+                positions_for(s, tokens + offsets[r], K, pos);
+        }
+        s->last_K[r] = K;
         s->pend_keys[r] = keys;
         s->pend_nblk[r] = nblk;
         uint32_t c1 = ring_owner(s, 0, pos[0]);
@@ -865,6 +1014,13 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
         s->m_cv_last = load_cv(s);
         s->m_cv_sum += s->m_cv_last;
         s->m_batches++;
+    }
+    if (cf->adapt_step_blocks && n > 0) {
+        s->ad_requests += n;
+        if (++s->ad_batches == cf->adapt_window) {
+            int rc = adapt_window_end(s);
+            if (rc) return rc;
+        }
     }
     s->pending = 1;
     return OR_OK;
@@ -1120,4 +1276,20 @@ void or_get_metrics(or_state *s, uint64_t *u, double *d, uint64_t *hist, int res
         s->m_cv_sum = s->m_cv_last = 0.0;
         memset(s->m_hist, 0, sizeof s->m_hist);
     }
+}
+
+/* Hash prefix length (blocks) of each request of the last routed batch;
+ * returns the batch size. */
+uint32_t or_last_route_blocks(const or_state *s, uint32_t *K)
+{
+    if (K && s->last_n) memcpy(K, s->last_K, s->last_n * sizeof(uint32_t));
+    return s->last_n;
+}
+
+/* Expanded nodes of the prefix hotness tree (sorted keys); returns their
+ * number (entries beyond cap are not written). */
+uint64_t or_prefix_tree(const or_state *s, uint64_t *keys, uint64_t cap)
+{
+    for (uint64_t i = 0; i < s->ad_set_n && i < cap; i++) keys[i] = s->ad_set[i];
+    return s->ad_set_n;
 }

@@ -44,6 +44,9 @@ class or_config(C.Structure):
         ("max_batch_tokens", C.c_uint64),
         ("seed", C.c_uint64),
         ("choice_rule", C.c_uint32),
+        ("adapt_step_blocks", C.c_uint32),
+        ("adapt_max_blocks", C.c_uint32),
+        ("adapt_window", C.c_uint32),
     ]
 
 
@@ -103,6 +106,8 @@ def lib():
             "or_hist_bucket": (C.c_uint32, [C.c_uint64]),
             "or_hist_lower": (C.c_uint64, [C.c_uint32]),
             "or_get_metrics": (None, [V, u64p, P(C.c_double), V, C.c_int]),
+            "or_last_route_blocks": (C.c_uint32, [V, V]),
+            "or_prefix_tree": (C.c_uint64, [V, V, C.c_uint64]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -217,6 +222,20 @@ class Oracle:
 
     def commit(self):
         return lib().or_commit(self.h)
+
+    def route_blocks(self):
+        """Hash prefix length (blocks) of each request of the last batch."""
+        n = lib().or_last_route_blocks(self.h, None)
+        K = np.zeros(max(n, 1), np.uint32)
+        lib().or_last_route_blocks(self.h, K.ctypes.data)
+        return K[:n]
+
+    def prefix_tree(self):
+        """Sorted keys of the expanded nodes of the prefix hotness tree."""
+        n = lib().or_prefix_tree(self.h, None, 0)
+        k = np.zeros(max(n, 1), np.uint64)
+        lib().or_prefix_tree(self.h, k.ctypes.data, n)
+        return k[:n]
 
     def metrics(self, reset=False):
         """Counters (METRIC_KEYS), cv_sum, cv_last and the TTFT histogram."""
