@@ -231,6 +231,8 @@ def main():
                     help="override a workload field (small cases for profiling)")
     ap.add_argument("--max-touch", type=int, default=0, help="override max_touch_per_instance")
     ap.add_argument("--index-slots-log2", type=int, default=0, help="override the index size (log2 slots)")
+    ap.add_argument("--adapt", default="", metavar="STEP,MAX[,WINDOW]",
+                    help="adaptive hash-prefix length: blocks per step, longest prefix, batches per window")
     ap.add_argument("--rule", default="dualmap",
                     help="choice rule (dualmap, pair_*, cache_affinity, least_loaded, min_ttft, preble)")
     args = ap.parse_args()
@@ -260,6 +262,9 @@ def main():
         kw["index_slots_log2"] = args.index_slots_log2
     rule = D.RULE_NAMES.index(args.rule)
     kw["choice_rule"] = rule
+    if args.adapt:
+        a = [int(x) for x in args.adapt.split(",")]
+        kw.update(adapt_step_blocks=a[0], adapt_max_blocks=a[1], adapt_window=a[2] if len(a) > 2 else 1)
 
     # all batches' tokens resident in HBM (a pass longer than the trace replays it cyclically)
     used = min(nb, W + K)
@@ -408,6 +413,8 @@ def main():
     # touch_deferred, req_counts, evict (9); rebalance (1)
     # (the cluster-wide rules add the all-instance probe kernel)
     launches_per_step = 5 + 9 + (1 if w.get("rebalance") else 0) + (1 if rule >= D.DM_RULE_LEAST_LOADED else 0)
+    if args.adapt:   # window end: the update kernel, once per window
+        launches_per_step += 1.0 / kw["adapt_window"]
     clocks = sampler.summary(wall0, wall1)
     g.close()
     del g
@@ -437,6 +444,9 @@ def main():
                                    f"(~{bytes_per_launch / 1e6:.0f} MB per batch)",
                        "global_batch": w["batch"], "parallelism": f"replicas x{world}",
                        "choice_rule": args.rule,
+                       "hash_prefix": (f"adaptive: base {w['route_prefix_blocks']} blocks, step {kw['adapt_step_blocks']}, "
+                                       f"max {kw['adapt_max_blocks']}, window {kw['adapt_window']} batch(es)"
+                                       if args.adapt else f"fixed {w['route_prefix_blocks']} blocks"),
                        "l2": ("inputs larger than L2 (each batch > 129 MB, distinct per step)"
                               if bytes_per_launch > 129e6 else
                               "batches smaller than L2, L2 not flushed between steps"),
@@ -452,7 +462,7 @@ def main():
                         "ttft_p50_us": met["ttft_p50_us"], "ttft_p90_us": met["ttft_p90_us"],
                         "completed": met["completed"], "requests": met["requests"],
                         "note": "scheduler time model over the stage-breakdown replay"},
-            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches_per_step * K, "clocks": clocks,
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": int(round(launches_per_step * K)), "clocks": clocks,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -139,8 +139,22 @@ typedef struct {
      * SLO-aware rule.  The others are the rules DualMap is compared with,
      * for experiments; DM_ERR_INVALID_ARG for an unknown value. */
     uint32_t choice_rule;
-    /* Must be 0. */
-    uint32_t reserved1;
+    /* Adaptive hash-prefix length (Sec. 3.2, "how long prefix is
+     * appropriate"); adapt_step_blocks = 0 keeps every request at
+     * min(K_route, n_blk).  Otherwise a prefix hotness tree decides each
+     * request's length: a node is a prefix, named by its last block's key;
+     * a request starts at min(K_route, n_blk) blocks and, while its node is
+     * expanded and its prompt and adapt_max_blocks allow, goes
+     * adapt_step_blocks deeper (capped by n_blk and adapt_max_blocks).  Every
+     * adapt_window routed non-empty batches form a window; at its end, with
+     * n live instances and T requests in the window, a node reached by more
+     * than 2T/n of them (and shorter than adapt_max_blocks) is expanded and
+     * an expanded node reached by fewer than T/n is dropped; the new tree
+     * applies from the next batch.  K_route < adapt_max_blocks <= 2048,
+     * adapt_window >= 1. */
+    uint32_t adapt_step_blocks;
+    uint32_t adapt_max_blocks;
+    uint32_t adapt_window;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */
@@ -266,8 +280,9 @@ DM_API dm_status dm_commit_cache(dm_handle *h);
  * cache keys at positions key_off[r] .. key_off[r] + n_blk(r), where
  * key_off (device, n+1 entries, written by the call) is the exclusive prefix
  * sum of n_blk; pos_dev (device, 2n entries) receives (pos1, pos2) per
- * request.  keys_dev must hold sum(n_blk) entries (at most
- * total_tokens / B).  Asynchronous. */
+ * request, hashed over min(K_route, n_blk) blocks (the fixed length, also
+ * with the adaptive length on).  keys_dev must hold sum(n_blk) entries (at
+ * most total_tokens / B).  Asynchronous. */
 DM_API dm_status dm_hash_prompts(dm_handle *h, const dm_batch *batch, uint64_t *keys_dev,
                           uint64_t *key_off_dev, uint64_t *pos_dev);
 
@@ -372,6 +387,16 @@ typedef struct {
  * after a sticky error. */
 DM_API dm_status dm_get_metrics(dm_handle *h, dm_metrics *out_host, uint64_t *hist_host, uint32_t hist_cap,
                                 int reset);
+
+/* Hash prefix length (blocks) each request of the last routed batch was
+ * mapped with: min(K_route, n_blk), or the adaptive length.  Copies n
+ * (<= that batch's size) values to out_dev (device).  Asynchronous. */
+DM_API dm_status dm_get_route_blocks(dm_handle *h, uint32_t *out_dev, uint32_t n);
+
+/* Expanded nodes of the adaptive prefix hotness tree (their keys, in
+ * unspecified order); *n_out = their number (entries beyond cap are not
+ * written).  0 nodes when the length is fixed.  Synchronous. */
+DM_API dm_status dm_export_prefix_tree(dm_handle *h, uint64_t *keys_host, uint64_t cap, uint64_t *n_out);
 
 /* Synchronise the stream and return the sticky error (DM_OK if none). */
 DM_API dm_status dm_last_error(dm_handle *h);

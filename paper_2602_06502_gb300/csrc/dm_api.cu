@@ -3,6 +3,7 @@
 // Every computation of the routing path runs in the kernels of the other
 // translation units; this file only validates, allocates and enqueues.
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <utility>
 #include <vector>
@@ -33,6 +34,11 @@ struct dm_handle {
     uint64_t pending_seq0 = 0;
     uint32_t rebalance_calls = 0;
     int hash_grid = 0;
+    // adaptive prefix length: the second expanded-node table (the next
+    // window's target), requests and non-empty batches in the current window
+    uint64_t *ad_alt = nullptr;
+    uint64_t ad_T = 0;
+    uint32_t ad_batches = 0;
     uint64_t *vpos_buf[2][2] = {};
     uint32_t *owner_buf[2][2] = {}, *vidx_buf[2][2] = {};
     int cur[2] = {0, 0};
@@ -202,7 +208,10 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.max_batch < 1 || c.max_batch > (1u << 24) || c.max_batch_tokens < B) return DM_ERR_INVALID_ARG;
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
     if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
-    if (c.choice_rule > DM_RULE_PREBLE || c.reserved1 != 0) return DM_ERR_INVALID_ARG;
+    if (c.choice_rule > DM_RULE_PREBLE) return DM_ERR_INVALID_ARG;
+    if (c.adapt_step_blocks &&
+        (c.adapt_max_blocks <= c.route_prefix_blocks || c.adapt_max_blocks > 2048 || c.adapt_window < 1))
+        return DM_ERR_INVALID_ARG;
 
     dm_handle *h = new dm_handle();
     h->cfg = c;
@@ -219,6 +228,9 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.hot_den = c.hot_den;
     d.max_batch = c.max_batch;
     d.rule = c.choice_rule;
+    d.ad_step = c.adapt_step_blocks;
+    d.ad_max = c.adapt_step_blocks ? c.adapt_max_blocks : c.route_prefix_blocks;
+    d.Kf2 = d.ad_max;
     d.max_blocks = c.max_batch_tokens / B;
     d.max_segs = d.max_blocks / dm::kSegBlocks + c.max_batch;
     d.T = c.max_touch_per_instance ? c.max_touch_per_instance : d.max_blocks;
@@ -293,6 +305,20 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.err, 1));
     A(dalloc(h, &d.seq_next, 1));
     A(dalloc(h, &d.metrics, 1));
+    uint64_t ad_levels = 0;
+    if (c.adapt_step_blocks) {
+        // at most n expanded nodes per level (each holds >= 1/n of a window's requests)
+        ad_levels = (d.ad_max - c.route_prefix_blocks + d.ad_step - 1) / d.ad_step + 1;
+        d.ad_set_mask = pow2_at_least(std::max<uint64_t>(1024, 4 * M * ad_levels)) - 1;
+        d.ad_cnt_mask = pow2_at_least(std::max<uint64_t>(1024, 2ull * c.max_batch * c.adapt_window * ad_levels)) - 1;
+        if (d.ad_cnt_mask >= (1ull << 26)) {
+            dm_destroy(h);
+            return DM_ERR_INVALID_ARG;
+        }
+        A(dalloc(h, &d.ad_set, d.ad_set_mask + 1));
+        A(dalloc(h, &h->ad_alt, d.ad_set_mask + 1));
+        A(dalloc(h, &d.ad_cnt, d.ad_cnt_mask + 1));
+    }
     if (c.choice_rule >= DM_RULE_LEAST_LOADED) A(dalloc(h, &d.h_all, uint64_t(c.max_batch) * M));
     A(dalloc(h, &d.rb_key, d.rb_cap));
     A(dalloc(h, &d.rb_seq, d.rb_cap));
@@ -318,6 +344,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         A(dalloc(h, &x->seg_newly, d.max_segs));
         A(dalloc(h, &x->seg_claims, d.max_segs));
         A(dalloc(h, &x->plocal, d.max_blocks));
+        if (x == &h->d && c.adapt_step_blocks) A(dalloc(h, &x->p2local, d.max_blocks));
+        A(dalloc(h, &x->r_K, c.max_batch));
         A(dalloc(h, &x->r_c1, c.max_batch));
         A(dalloc(h, &x->r_c2, c.max_batch));
         A(dalloc(h, &x->r_h1, c.max_batch));
@@ -330,6 +358,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         dm_destroy(h);
         return e == cudaErrorMemoryAllocation ? DM_ERR_OOM : DM_ERR_CUDA;
     }
+    h->dh.ad_step = 0;   // dm_hash_prompts hashes the fixed length
+    h->dh.Kf2 = c.route_prefix_blocks;
     for (int f = 0; f < 2; ++f) {
         d.ring[f].vpos = h->vpos_buf[f][0];
         d.ring[f].owner = h->owner_buf[f][0];
@@ -340,6 +370,10 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(cudaMemsetAsync(d.inst_state, 0, M, h->st));
     A(cudaMemsetAsync(d.W, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.metrics, 0, sizeof(dm::DevMetrics), h->st));
+    if (c.adapt_step_blocks) {
+        A(cudaMemsetAsync(d.ad_set, 0, (d.ad_set_mask + 1) * 8, h->st));
+        A(cudaMemsetAsync(d.ad_cnt, 0, (d.ad_cnt_mask + 1) * sizeof(dm::AdCount), h->st));
+    }
     A(cudaMemsetAsync(d.q_head, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.q_tail, 0, M * 4, h->st));
     A(cudaMemsetAsync(d.table, 0, M * 8, h->st));
@@ -537,6 +571,20 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
     if (e == cudaSuccess && b->n) {
         Stage st(h, DM_STAGE_CHOICE);
         e = dm::launch_choice(d, *o, b->n, h->seq_next, b->batch_time_us, h->st);
+    }
+    if (e == cudaSuccess && b->n && d.ad_step) {
+        // end of an adaptive window: rebuild the expanded nodes into the
+        // other table, restart the counts; the next batch walks the new tree
+        h->ad_T += b->n;
+        if (++h->ad_batches == h->cfg.adapt_window) {
+            e = cudaMemsetAsync(h->ad_alt, 0, (d.ad_set_mask + 1) * 8, h->st);
+            if (e == cudaSuccess) e = dm::launch_adapt_update(d, h->ad_alt, h->n_live, h->ad_T, h->st);
+            if (e == cudaSuccess)
+                e = cudaMemsetAsync(d.ad_cnt, 0, (d.ad_cnt_mask + 1) * sizeof(dm::AdCount), h->st);
+            std::swap(h->d.ad_set, h->ad_alt);
+            h->ad_T = 0;
+            h->ad_batches = 0;
+        }
     }
     if (e != cudaSuccess) return map_cuda(h, e);
     h->pending = true;
@@ -759,6 +807,35 @@ dm_status dm_get_maint_counts(dm_handle *h, uint64_t *rebuilds_host, uint64_t *c
     if (e != cudaSuccess) return map_cuda(h, e);
     *rebuilds_host = c[0];
     *compactions_host = c[1];
+    return DM_OK;
+}
+
+dm_status dm_get_route_blocks(dm_handle *h, uint32_t *out_dev, uint32_t n) {
+    dm_status s = check_handle(h);
+    if (s) return s;
+    if (n > h->pending_n || (n && !out_dev)) return DM_ERR_INVALID_ARG;
+    if (n == 0) return DM_OK;
+    cudaError_t e = cudaMemcpyAsync(out_dev, h->d.r_K, n * sizeof(uint32_t), cudaMemcpyDeviceToDevice, h->st);
+    return e == cudaSuccess ? DM_OK : map_cuda(h, e);
+}
+
+dm_status dm_export_prefix_tree(dm_handle *h, uint64_t *keys_host, uint64_t cap, uint64_t *n_out) {
+    dm_status s = check_handle(h);
+    if (s) return s;
+    if (!n_out || (cap && !keys_host)) return DM_ERR_INVALID_ARG;
+    *n_out = 0;
+    if (!h->d.ad_step) return DM_OK;
+    std::vector<uint64_t> t(h->d.ad_set_mask + 1);
+    cudaError_t e = cudaMemcpyAsync(t.data(), h->d.ad_set, t.size() * 8, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    uint64_t k = 0;
+    for (uint64_t x : t)
+        if (x) {
+            if (k < cap) keys_host[k] = x;
+            ++k;
+        }
+    *n_out = k;
     return DM_OK;
 }
 

@@ -9,8 +9,10 @@
 // Because the chain is a plain prefix sum, every 64-block segment of every
 // prompt is hashed independently (one warp each); a segment writes its local
 // prefix values and its totals, and the probe kernel adds the carry of the
-// earlier segments.  f2 only runs over the first K = min(K_route, n_blk)
-// blocks: segments below K write the sum of their f2 digests.
+// earlier segments.  f2 only runs over the first K = min(Kf2, n_blk) blocks
+// (Kf2 = K_route, or the longest adaptive prefix): segments below K write the
+// sum of their f2 digests and, with the adaptive length, each block's
+// in-segment f2 prefix value.
 #include "dm_internal.cuh"
 
 namespace dm {
@@ -53,8 +55,9 @@ __device__ __forceinline__ uint64_t reduce_scatter(uint64_t (&p)[U], int q) {
 // j*(32/U)+l/U.  Both iterations' loads are issued before any arithmetic
 // (4 KB in flight per warp at B = 16).  After the reduce-scatter lane l
 // holds block (l%U)*(32/U) + l/U; one shuffle puts block m on lane m for the
-// scan.  Segments below K also sum their f2 digests (blocks < K).
-template <int U>
+// scan.  Segments below K also sum their f2 digests (blocks < K); kP2 adds
+// their per-block prefix values (the adaptive length picks its K later).
+template <int U, bool kP2>
 __global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__restrict__ tokens) {
     pdl_enter();
     constexpr int IT = kSegBlocks / 32;
@@ -80,7 +83,7 @@ __global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__r
         const uint32_t nb = min(kSegBlocks, nblk - b0);
         const uint4 *src4 = reinterpret_cast<const uint4 *>(tokens + d.r_tokoff[r] + uint64_t(b0) * d.B);
         uint64_t *out = d.plocal + d.r_blkoff[r] + b0;
-        const uint32_t K = min(d.Kroute, nblk);
+        const uint32_t K = min(d.Kf2, nblk);
         uint4 v[IT][U];
 #pragma unroll
         for (int it = 0; it < IT; ++it)
@@ -90,7 +93,7 @@ __global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__r
                 v[it][jj] = blk < nb ? ld_stream(src4 + uint64_t(it) * 32 * U + jj * 32 + lane)
                                      : make_uint4(0, 0, 0, 0);
             }
-        uint64_t carry1 = 0, sum2 = 0;
+        uint64_t carry1 = 0, sum2 = 0;   // kP2: sum2 is the running f2 prefix (uniform)
 #pragma unroll
         for (int it = 0; it < IT; ++it) {
             if ((uint32_t)it * 32 >= nb) break;
@@ -110,11 +113,21 @@ __global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__r
 #pragma unroll
                 for (int jj = 0; jj < U; ++jj) p2[jj] = nh4(v[it][jj], k2);
                 const uint64_t s2 = reduce_scatter<U>(p2, q);
-                sum2 += ((uint32_t)bq < nvalid && kb < K) ? fmix64(s2 + uint64_t(kb + 1) * G2) : 0;
+                const uint64_t dg2 = ((uint32_t)bq < nvalid && kb < K) ? fmix64(s2 + uint64_t(kb + 1) * G2) : 0;
+                if constexpr (kP2) {
+                    const uint64_t P2 = warp_incl_scan(shfl_u64(dg2, src), lane) + sum2;
+                    if ((uint32_t)lane < nvalid && b0 + it * 32 + lane < K)
+                        d.p2local[d.r_blkoff[r] + b0 + it * 32 + lane] = P2;
+                    sum2 = shfl_u64(P2, 31);
+                } else {
+                    sum2 += dg2;
+                }
             }
         }
+        if constexpr (!kP2) {
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) sum2 += shfl_xor_u64(sum2, o);
+            for (int o = 16; o >= 1; o >>= 1) sum2 += shfl_xor_u64(sum2, o);
+        }
         if (lane == 0) {
             d.seg_total[seg] = carry1;
             d.seg_total2[seg] = sum2;
@@ -128,22 +141,27 @@ int hash_grid_size() {
         int dev = 0, sms = 0, per = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_hash<4>, 256, 0);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_hash<4, false>, 256, 0);
         grid = sms * (per > 0 ? per : 1);
     }
     return grid;
 }
 
-cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st) {
+template <bool kP2>
+static cudaError_t launch_hash_t(const DevState &d, const dm_batch &b, int grid, cudaStream_t st) {
     switch (d.B) {
-        case 4: DM_TRY(launch_pdl(k_hash<1>, grid, 256, 0, st, d, b.tokens)); break;
-        case 8: DM_TRY(launch_pdl(k_hash<2>, grid, 256, 0, st, d, b.tokens)); break;
-        case 16: DM_TRY(launch_pdl(k_hash<4>, grid, 256, 0, st, d, b.tokens)); break;
-        case 32: DM_TRY(launch_pdl(k_hash<8>, grid, 256, 0, st, d, b.tokens)); break;
-        case 64: DM_TRY(launch_pdl(k_hash<16>, grid, 256, 0, st, d, b.tokens)); break;
+        case 4: DM_TRY(launch_pdl(k_hash<1, kP2>, grid, 256, 0, st, d, b.tokens)); break;
+        case 8: DM_TRY(launch_pdl(k_hash<2, kP2>, grid, 256, 0, st, d, b.tokens)); break;
+        case 16: DM_TRY(launch_pdl(k_hash<4, kP2>, grid, 256, 0, st, d, b.tokens)); break;
+        case 32: DM_TRY(launch_pdl(k_hash<8, kP2>, grid, 256, 0, st, d, b.tokens)); break;
+        case 64: DM_TRY(launch_pdl(k_hash<16, kP2>, grid, 256, 0, st, d, b.tokens)); break;
         default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();
+}
+
+cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st) {
+    return d.ad_step ? launch_hash_t<true>(d, b, grid, st) : launch_hash_t<false>(d, b, grid, st);
 }
 
 // ---------------------------------------------------------------------------

@@ -123,6 +123,13 @@ struct Deferred {
     uint32_t home, f, found, bucket;
 };
 
+// One node count of the adaptive prefix tree's current window (16 bytes):
+// key 0 marks an empty slot.
+struct AdCount {
+    uint64_t key;
+    uint32_t count, depth;   // requests that reached the node; its length in blocks
+};
+
 // Per-batch values produced on the device.
 struct BatchInfo {
     uint64_t total_blocks;
@@ -148,6 +155,13 @@ struct DevState {
     uint64_t C, slo;
     uint32_t cost, hot_num, hot_den, max_batch;
     uint32_t rule;                  // dm_choice_rule
+    // adaptive prefix length (ad_step = 0: every request hashes min(Kroute, n_blk) blocks)
+    uint32_t Kf2;                   // the f2 digests are hashed over blocks < min(Kf2, n_blk)
+    uint32_t ad_step, ad_max;
+    uint64_t *ad_set;               // expanded nodes: open addressing on the key, 0 = empty
+    uint64_t ad_set_mask;
+    AdCount *ad_cnt;                // node counts of the current window
+    uint64_t ad_cnt_mask;
     uint64_t max_blocks, max_segs, T, S, logcap;
     uint32_t Q;
     // key material
@@ -185,6 +199,8 @@ struct DevState {
     uint64_t *r_tokoff, *r_blkoff;
     uint32_t *seg_req;
     uint64_t *seg_total, *seg_carry, *plocal;
+    uint64_t *p2local;              // adaptive only: per block < Kf2, in-segment prefix of its f2 digests
+    uint32_t *r_K;                  // per request: the hash prefix length it was routed with
     uint64_t *seg_total2;           // per segment: f2 digest sum over its blocks < K
     uint32_t *seg_newly, *seg_claims;   // per segment: keys made resident / index slots taken by the commit
     Deferred *defer;                // kSegBlocks per segment: touches left to the commit's second pass
@@ -411,6 +427,61 @@ __device__ __forceinline__ void route_positions(const DevState &d, uint32_t r, i
 }
 
 // ---------------------------------------------------------------------------
+// Adaptive prefix tree tables (open addressing, linear probing, bounded).
+
+__device__ __forceinline__ uint64_t ad_slot(uint64_t key, uint64_t mask) {
+    return fmix64(key ^ 0x2545F4914F6CDD1Dull) & mask;
+}
+
+__device__ __forceinline__ bool ad_set_contains(const uint64_t *set, uint64_t mask, uint64_t key, uint32_t *err) {
+    uint64_t x = ad_slot(key, mask);
+    for (uint64_t i = 0; i <= mask; ++i, x = (x + 1) & mask) {
+        const uint64_t k = set[x];
+        if (k == key) return true;
+        if (k == 0) return false;
+    }
+    set_err(err, DM_ERR_CAPACITY);
+    return false;
+}
+
+__device__ __forceinline__ void ad_set_insert(uint64_t *set, uint64_t mask, uint64_t key, uint32_t *err) {
+    uint64_t x = ad_slot(key, mask);
+    for (uint64_t i = 0; i <= mask; ++i, x = (x + 1) & mask) {
+        const unsigned long long k = atomicCAS(reinterpret_cast<unsigned long long *>(set + x), 0ull,
+                                               (unsigned long long)key);
+        if (k == 0 || k == key) return;
+    }
+    set_err(err, DM_ERR_CAPACITY);
+}
+
+// One more request reached node `key` (length `depth` blocks).
+__device__ __forceinline__ void ad_count_add(AdCount *cnt, uint64_t mask, uint64_t key, uint32_t depth,
+                                             uint32_t *err) {
+    uint64_t x = ad_slot(key, mask);
+    for (uint64_t i = 0; i <= mask; ++i, x = (x + 1) & mask) {
+        const unsigned long long k = atomicCAS(reinterpret_cast<unsigned long long *>(&cnt[x].key), 0ull,
+                                               (unsigned long long)key);
+        if (k == 0 || k == key) {
+            if (k == 0) cnt[x].depth = depth;
+            atomicAdd(&cnt[x].count, 1u);
+            return;
+        }
+    }
+    set_err(err, DM_ERR_CAPACITY);
+}
+
+__device__ __forceinline__ uint32_t ad_count_get(const AdCount *cnt, uint64_t mask, uint64_t key, uint32_t *err) {
+    uint64_t x = ad_slot(key, mask);
+    for (uint64_t i = 0; i <= mask; ++i, x = (x + 1) & mask) {
+        const uint64_t k = cnt[x].key;
+        if (k == key) return cnt[x].count;
+        if (k == 0) return 0;
+    }
+    set_err(err, DM_ERR_CAPACITY);
+    return 0;
+}
+
+// ---------------------------------------------------------------------------
 // Metrics helpers.
 
 // TTFT histogram bucket: v < 16 exact; else e = floor(log2 v) and the four
@@ -537,6 +608,7 @@ cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStre
 int hash_grid_size();
 cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
                                cudaStream_t st);
+cudaError_t launch_adapt_update(const DevState &d, uint64_t *new_set, uint64_t n_live, uint64_t T, cudaStream_t st);
 cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, uint64_t seq0,
                           uint64_t t_batch, cudaStream_t st);
 cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st);

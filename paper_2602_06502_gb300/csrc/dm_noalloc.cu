@@ -111,6 +111,8 @@ extern "C" DM_API dm_status dm_hash_prompts_noalloc(uint32_t block_tokens, uint3
     DevState d{};
     d.B = B;
     d.Kroute = route_prefix_blocks;
+    d.Kf2 = route_prefix_blocks;   // fixed hash length: f2 over the first K_route blocks
+    d.ad_step = 0;
     d.max_batch = kNaReq;
     d.max_blocks = kNaBlocks;
     d.max_segs = kNaSegs;

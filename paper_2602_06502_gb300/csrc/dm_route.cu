@@ -46,6 +46,47 @@ __device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uin
     lb2 = (uint32_t)(i2 + 1 == (int64_t)d.R ? 0 : i2 + 1);
 }
 
+// Adaptive hash-prefix length (Sec. 3.2): the walk from min(K_route, n_blk)
+// blocks, one step deeper while the node (the key of the prefix's last
+// block) is expanded.  Level j sits at depth min(d0 + j * step, cap), so
+// lane j evaluates level j of each 32-level round at once: the request's
+// length is the first level that cannot extend.  Every level passed and the
+// final one count toward the window's hotness.  Then the two positions of
+// that length.  Whole warp; needs ad_max <= 2048 (segment carries in one
+// warp scan).
+__device__ __forceinline__ void adaptive_positions(const DevState &d, uint32_t r, int lane, uint64_t &pos1,
+                                                   uint64_t &pos2) {
+    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
+    const uint64_t bo = d.r_blkoff[r];
+    const uint32_t d0 = min(d.Kroute, nblk), cap = min(d.ad_max, nblk);
+    const uint32_t nseg = (cap - 1) / kSegBlocks + 1;   // <= 32
+    const uint64_t t1 = (uint32_t)lane < nseg ? d.seg_total[s0 + lane] : 0;
+    const uint64_t t2 = (uint32_t)lane < nseg ? d.seg_total2[s0 + lane] : 0;
+    const uint64_t c1 = warp_incl_scan(t1, lane) - t1, c2 = warp_incl_scan(t2, lane) - t2;   // exclusive
+    uint32_t K = d0;
+    uint64_t P1K = 0;
+    for (uint32_t j0 = 0;; j0 += 32) {
+        const uint64_t want = uint64_t(d0) + uint64_t(j0 + lane) * d.ad_step;
+        const uint32_t dj = want < cap ? (uint32_t)want : cap;
+        const uint32_t b = dj - 1;
+        const uint64_t P1 = d.plocal[bo + b] + shfl_u64(c1, b / kSegBlocks);
+        const uint64_t key = cache_key(P1, d.Sc);
+        const bool ext = dj < cap && ad_set_contains(d.ad_set, d.ad_set_mask, key, d.err);
+        const uint32_t stop = __ballot_sync(0xffffffffu, !ext);
+        const int last = stop ? __ffs(stop) - 1 : 31;   // levels of this round that count
+        if (lane <= last) ad_count_add(d.ad_cnt, d.ad_cnt_mask, key, dj, d.err);
+        if (stop) {
+            K = __shfl_sync(0xffffffffu, dj, last);
+            P1K = shfl_u64(P1, last);
+            break;
+        }
+    }
+    const uint64_t P2K = d.p2local[bo + K - 1] + shfl_u64(c2, (K - 1) / kSegBlocks);
+    pos1 = fmix64(P1K ^ d.Sr1);
+    pos2 = fmix64(P2K ^ d.Sr2);
+    if (lane == 0) d.r_K[r] = K;
+}
+
 // One CTA of kProbeWarps warps per request.  Warp 0 computes the two ring
 // positions and candidates while warp 1 computes the segment carries; then
 // every round probes 32 * kProbeWarps consecutive blocks on each candidate
@@ -53,6 +94,7 @@ __device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uin
 // candidate's run.
 constexpr int kProbeWarps = 8;
 
+template <bool kAdapt>
 __global__ void __launch_bounds__(kProbeWarps * 32, 4) k_route_probe(DevState d, dm_route_out o, uint32_t n) {
     pdl_enter();
     __shared__ uint32_t s_c[2];
@@ -64,7 +106,12 @@ __global__ void __launch_bounds__(kProbeWarps * 32, 4) k_route_probe(DevState d,
         request_carries(d, r, lane);   // for the probes below and the commit
     } else if (wid == 0) {
         uint64_t p1, p2;
-        route_positions_direct(d, r, lane, p1, p2);
+        if constexpr (kAdapt) {
+            adaptive_positions(d, r, lane, p1, p2);
+        } else {
+            route_positions_direct(d, r, lane, p1, p2);
+            if (lane == 0) d.r_K[r] = min(d.Kroute, d.r_nblk[r]);
+        }
         uint32_t lb1, lb2;
         ring_search2(d, p1, p2, lane, lb1, lb2);
         const uint32_t c1 = d.ring[0].owner[lb1];
@@ -128,7 +175,10 @@ __global__ void __launch_bounds__(kProbeWarps * 32, 4) k_route_probe(DevState d,
 cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
                                cudaStream_t st) {
     if (b.n == 0) return cudaSuccess;
-    DM_TRY(launch_pdl(k_route_probe, b.n, kProbeWarps * 32, 0, st, d, o, b.n));
+    if (d.ad_step)
+        DM_TRY(launch_pdl(k_route_probe<true>, b.n, kProbeWarps * 32, 0, st, d, o, b.n));
+    else
+        DM_TRY(launch_pdl(k_route_probe<false>, b.n, kProbeWarps * 32, 0, st, d, o, b.n));
     return cudaGetLastError();
 }
 
@@ -150,6 +200,43 @@ cudaError_t launch_ring_lookup(const DevState &d, const uint64_t *pos, uint32_t 
                                uint32_t *o2, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
     k_ring_lookup<<<(n + 7) / 8, 256, 0, st>>>(d, pos, n, o1, o2);
+    return cudaGetLastError();
+}
+
+}  // namespace dm
+
+namespace dm {
+
+// End of an adaptive window: new_set (cleared) receives the expanded nodes
+// that stay (reached by at least T/n requests) and the nodes that become
+// expanded (reached by more than 2T/n, shorter than the cap).  Grid-stride
+// over both tables.
+__global__ void k_adapt_update(DevState d, uint64_t *new_set, uint64_t n_live, uint64_t T) {
+    pdl_enter();
+    if (has_err(d.err)) return;
+    const uint64_t ns = d.ad_set_mask + 1, nc = d.ad_cnt_mask + 1, tot = ns > nc ? ns : nc;
+    const uint64_t stride = uint64_t(gridDim.x) * blockDim.x;
+    for (uint64_t x = uint64_t(blockIdx.x) * blockDim.x + threadIdx.x; x < tot; x += stride) {
+        if (x < ns) {
+            const uint64_t key = d.ad_set[x];
+            if (key) {
+                const uint64_t c = ad_count_get(d.ad_cnt, d.ad_cnt_mask, key, d.err);
+                if (!(c * n_live < T)) ad_set_insert(new_set, d.ad_set_mask, key, d.err);
+            }
+        }
+        if (x < nc) {
+            const AdCount e = d.ad_cnt[x];
+            if (e.key && e.depth < d.ad_max && uint64_t(e.count) * n_live > 2 * T &&
+                !ad_set_contains(d.ad_set, d.ad_set_mask, e.key, d.err))
+                ad_set_insert(new_set, d.ad_set_mask, e.key, d.err);
+        }
+    }
+}
+
+cudaError_t launch_adapt_update(const DevState &d, uint64_t *new_set, uint64_t n_live, uint64_t T, cudaStream_t st) {
+    const uint64_t tot = (d.ad_set_mask > d.ad_cnt_mask ? d.ad_set_mask : d.ad_cnt_mask) + 1;
+    const unsigned grid = (unsigned)((tot + 255) / 256 < 4096 ? (tot + 255) / 256 : 4096);
+    DM_TRY(launch_pdl(k_adapt_update, grid, 256, 0, st, d, new_set, n_live, T));
     return cudaGetLastError();
 }
 

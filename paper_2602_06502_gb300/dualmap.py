@@ -45,7 +45,9 @@ class dm_config(C.Structure):
         ("max_queue", C.c_uint32),
         ("index_slots_log2", C.c_uint32),
         ("choice_rule", C.c_uint32),
-        ("reserved1", C.c_uint32),
+        ("adapt_step_blocks", C.c_uint32),
+        ("adapt_max_blocks", C.c_uint32),
+        ("adapt_window", C.c_uint32),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]
@@ -112,6 +114,8 @@ SIGNATURES = {
     "dm_get_clock": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64)]),
     "dm_get_maint_counts": (C.c_int, [C.c_void_p, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
     "dm_get_metrics": (C.c_int, [C.c_void_p, C.POINTER(dm_metrics), C.c_void_p, C.c_uint32, C.c_int]),
+    "dm_get_route_blocks": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32]),
+    "dm_export_prefix_tree": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint64, C.POINTER(C.c_uint64)]),
     "dm_last_error": (C.c_int, [C.c_void_p]),
     "dm_set_profiling": (C.c_int, [C.c_void_p, C.c_int]),
     "dm_get_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int]),
@@ -270,6 +274,19 @@ def dm_get_metrics(h, reset=False):
     _check(lib().dm_get_metrics(h, C.byref(m), hist.ctypes.data, DM_HIST_BUCKETS, 1 if reset else 0),
            "dm_get_metrics")
     return {name: getattr(m, name) for name, _ in dm_metrics._fields_}, hist
+
+
+def dm_get_route_blocks(h, out_dev, n):
+    return lib().dm_get_route_blocks(h, _ptr(out_dev), n)
+
+
+def dm_export_prefix_tree(h):
+    """Keys of the expanded nodes of the adaptive prefix tree (sorted)."""
+    n = C.c_uint64()
+    _check(lib().dm_export_prefix_tree(h, None, 0, C.byref(n)), "dm_export_prefix_tree")
+    k = np.zeros(max(n.value, 1), np.uint64)
+    _check(lib().dm_export_prefix_tree(h, k.ctypes.data, n.value, C.byref(n)), "dm_export_prefix_tree")
+    return np.sort(k[:n.value])
 
 
 def dm_last_error(h):

@@ -23,7 +23,7 @@ import sys
 import numpy as np
 
 
-def simulate(workload_name, rules, overrides=None, rebalance=None, batches=None, device="cuda:0"):
+def simulate(workload_name, rules, overrides=None, rebalance=None, batches=None, device="cuda:0", adapt=None):
     """Replay the trace once per rule; returns one dict per rule."""
     import torch
 
@@ -54,10 +54,11 @@ def simulate(workload_name, rules, overrides=None, rebalance=None, batches=None,
         g = Scheduler(block_tokens=w["block_tokens"], route_prefix_blocks=w["route_prefix_blocks"],
                       vnodes=w["vnodes"], max_instances=max_id + 1, capacity=w["capacity"], slo_us=w["slo_us"],
                       cost_us=w["cost_us"], max_batch=w["batch"], max_batch_tokens=max(max_len, 1 << 16),
-                      seed=w["seed"], choice_rule=rule, device=device)
+                      seed=w["seed"], choice_rule=rule, device=device, **(adapt or {}))
         for i in range(w["n_instances"]):
             assert g.add_instance(i) == 0
         D.dm_set_profiling(g.h, True, stages=["choice"])
+        ksum = kmax = 0
         for b in range(nb):
             for kind, i in events.get(b, []):
                 assert (g.add_instance(i) if kind == "add" else g.remove_instance(i)) == 0
@@ -65,6 +66,9 @@ def simulate(workload_name, rules, overrides=None, rebalance=None, batches=None,
             t0 = int(tr.req_off[s])
             g.route(tokens[t0:t0 + nt + 4], torch.from_numpy(off.view(np.int64)).to(dev),
                     torch.from_numpy(lens.view(np.int32)).to(dev), e - s, nt, tr.batch_time(b))
+            K = g.route_blocks(e - s)
+            ksum += int(K.sum())
+            kmax = max(kmax, int(K.max()))
             if rebalance:
                 g.rebalance()
             g.commit()
@@ -72,6 +76,7 @@ def simulate(workload_name, rules, overrides=None, rebalance=None, batches=None,
         if err:
             raise D.DualMapError(err, f"rule {name}")
         m, _ = D.dm_get_metrics(g.h)
+        tree = D.dm_export_prefix_tree(g.h)
         st = D.dm_get_stage_times(g.h)
         g.close()
         ms, calls = st["choice"]
@@ -84,6 +89,8 @@ def simulate(workload_name, rules, overrides=None, rebalance=None, batches=None,
             "completed": m["completed"], "ttft_mean_us": m["ttft_sum_us"] / max(m["completed"], 1),
             "ttft_p50_us": m["ttft_p50_us"], "ttft_p90_us": m["ttft_p90_us"], "ttft_p99_us": m["ttft_p99_us"],
             "switched": m["switched"], "choice_ms_per_batch": ms / max(calls, 1),
+            "hash_blocks_mean": ksum / max(m["requests"], 1), "hash_blocks_max": kmax,
+            "prefix_tree_nodes": None if not adapt else len(tree),
         })
     return out
 
@@ -96,6 +103,8 @@ def main():
     ap.add_argument("--set", action="append", default=[], metavar="KEY=VALUE", help="override a workload field")
     ap.add_argument("--rebalance", choices=["auto", "on", "off"], default="auto")
     ap.add_argument("--batches", type=int, default=None)
+    ap.add_argument("--adapt", default="", metavar="STEP,MAX[,WINDOW]",
+                    help="adaptive hash-prefix length (blocks per step, longest prefix, batches per window)")
     args = ap.parse_args()
     rules = D.RULE_NAMES if args.rules == "all" else args.rules.split(",")
     over = {}
@@ -103,7 +112,11 @@ def main():
         k, v = kv.split("=", 1)
         over[k] = float(v) if "." in v else int(v)
     rb = None if args.rebalance == "auto" else args.rebalance == "on"
-    for r in simulate(args.workload, rules, over, rb, args.batches):
+    ad = None
+    if args.adapt:
+        a = [int(x) for x in args.adapt.split(",")]
+        ad = dict(adapt_step_blocks=a[0], adapt_max_blocks=a[1], adapt_window=a[2] if len(a) > 2 else 1)
+    for r in simulate(args.workload, rules, over, rb, args.batches, adapt=ad):
         print(json.dumps(r), flush=True)
 
 

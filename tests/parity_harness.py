@@ -17,7 +17,7 @@ class Pair:
     """An oracle and a GPU scheduler built from the same workload dict."""
 
     def __init__(self, w, max_instances=None, max_batch_tokens=None, max_touch=0, max_queue=0, capacity=None,
-                 index_slots_log2=0, choice_rule=0):
+                 index_slots_log2=0, choice_rule=0, adapt=None):
         import torch
         from paper_2602_06502_gb300.scheduler import Scheduler
         self.torch = torch
@@ -27,13 +27,15 @@ class Pair:
         w = self.w
         self.M = max_instances or (w["n_instances"] + 8)
         mbt = max_batch_tokens or (1 << 24)
+        ad = dict(adapt_step_blocks=0, adapt_max_blocks=0, adapt_window=1) if adapt is None else dict(adapt)
+        self.adaptive = bool(ad["adapt_step_blocks"])
         self.ora = O.Oracle(**O.config_from_workload(w, max_instances=self.M, max_batch_tokens=mbt),
-                            choice_rule=choice_rule)
+                            choice_rule=choice_rule, **ad)
         self.gpu = Scheduler(block_tokens=w["block_tokens"], route_prefix_blocks=w["route_prefix_blocks"],
                              vnodes=w["vnodes"], max_instances=self.M, capacity=w["capacity"], slo_us=w["slo_us"],
                              cost_us=w["cost_us"], max_batch=w["batch"], max_batch_tokens=mbt,
                              max_touch_per_instance=max_touch, max_queue=max_queue,
-                             index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule)
+                             index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule, **ad)
         self.dev = torch.device("cuda:0")
         self.n_migrations = 0
         self.n_switched = 0
@@ -70,6 +72,14 @@ class Pair:
                 bad = np.nonzero(g != want[k])[0]
                 raise AssertionError(f"{tag}: {k} differs at {bad[:8].tolist()} "
                                      f"(gpu {g[bad[:4]].tolist()} vs oracle {want[k][bad[:4]].tolist()})")
+        gk, ok = self.gpu.route_blocks(n), self.ora.route_blocks()
+        if not np.array_equal(gk, ok):
+            bad = np.nonzero(gk != ok)[0]
+            raise AssertionError(f"{tag}: route blocks differ at {bad[:8].tolist()} "
+                                 f"(gpu {gk[bad[:4]].tolist()} vs oracle {ok[bad[:4]].tolist()})")
+        if self.adaptive:
+            from paper_2602_06502_gb300 import dualmap as D
+            assert np.array_equal(D.dm_export_prefix_tree(self.gpu.h), self.ora.prefix_tree()), f"{tag}: tree"
         self.n_switched += int(want["switched"].sum())
         self.hit_tokens += int(np.where(want["chosen"] == want["cand1"], want["hit1"], want["hit2"]).sum())
         return want

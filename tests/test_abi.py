@@ -64,7 +64,10 @@ def test_create_rejects_bad_config_without_touching_gpu(built):
 
     h = C.c_void_p()
     for bad in (cfg(block_tokens=17), cfg(index_slots_log2=41), cfg(route_prefix_blocks=0),
-                cfg(max_instances=1), cfg(choice_rule=D.DM_RULE_PREBLE + 1), cfg(reserved1=1)):
+                cfg(max_instances=1), cfg(choice_rule=D.DM_RULE_PREBLE + 1),
+                cfg(adapt_step_blocks=4, adapt_max_blocks=16, adapt_window=1),    # cap not above K_route
+                cfg(adapt_step_blocks=4, adapt_max_blocks=4096, adapt_window=1),  # cap above 2048
+                cfg(adapt_step_blocks=4, adapt_max_blocks=64, adapt_window=0)):
         assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
     assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
 

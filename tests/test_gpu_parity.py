@@ -222,6 +222,49 @@ def test_metrics_reset_and_rebalanced_ttft():
     assert all(v == 0 for v in gm.values()) and gh.sum() == 0
 
 
+# -- adaptive hash-prefix length --------------------------------------------------------
+
+def _ad(step, kmax, window=1):
+    return dict(adapt_step_blocks=step, adapt_max_blocks=kmax, adapt_window=window)
+
+
+@pytest.mark.parametrize("window", [1, 2])
+def test_adaptive_prefix_tiny(window):
+    """Zipf-1.2 prefixes over 8 instances: the top prefixes pass 2/n and
+    deepen 8 blocks per window up to their shared length; every request's
+    length and the expanded nodes match the oracle after every batch."""
+    w = workload("tiny", n_requests=2000, batch=100, zipf_s=1.2, rho=0.9)
+    tr = Trace(w)
+    p = Pair(w, adapt=_ad(8, 128, window))
+    run_trace(p, tr, state_every=5)
+    from paper_2602_06502_gb300 import dualmap as D
+    assert len(D.dm_export_prefix_tree(p.gpu.h)) > 0
+
+
+def test_adaptive_prefix_agent():
+    tr = Trace(workload("agent", n_requests=3 * 4096))
+    p = Pair(tr.cfg, max_batch_tokens=40_000_000, max_touch=1 << 20, adapt=_ad(32, 1024))
+    run_trace(p, tr)
+
+
+def test_adaptive_prefix_longctx_deepens_past_shared_prefix():
+    """16k-token shared prefixes (1,024 blocks), 128 instances: hot prefixes
+    deepen 128 blocks per batch; the longest lengths grow batch by batch."""
+    tr = Trace(workload("longctx", n_requests=6 * 512))
+    p = Pair(tr.cfg, max_batch_tokens=70_000_000, max_touch=1 << 20, capacity=200_000, adapt=_ad(128, 2048))
+    run_trace(p, tr)
+    assert int(p.ora.route_blocks().max()) > 16 + 3 * 128
+
+
+def test_adaptive_prefix_with_scaling_and_rebalance():
+    w = workload("scaling", n_requests=4 * 2048, batch=2048, scale_every=2048, n_instances=48, vnodes=64,
+                 capacity=20_000)
+    tr = Trace(w)
+    p = Pair(tr.cfg, max_instances=w["n_instances"] + 4, max_batch_tokens=20_000_000, max_touch=1 << 20,
+             adapt=_ad(16, 256))
+    run_trace(p, tr, rebalance=True)
+
+
 # -- edge cases ---------------------------------------------------------------------
 
 def _mk(**kw):
