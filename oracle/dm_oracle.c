@@ -101,6 +101,8 @@
  *     and TTFT_{r,j} < SLO and j is live; stop once i is no longer a
  *     hotspot.  Single round; a request moves at most once per call.
  *
+ *   Rebalancing variants (rebalance_flags): see OR_RB_* below.
+ *
  *   Scaling (Sec. 3.4; App. A.1.3): add inserts V nodes per ring; remove
  *     deletes them, the instance keeps draining and takes no new work.
  *
@@ -181,7 +183,18 @@ typedef struct {
     uint32_t adapt_step_blocks;   /* adaptive prefix: blocks per extension; 0 = fixed K_route */
     uint32_t adapt_max_blocks;    /* longest hash prefix, in blocks */
     uint32_t adapt_window;        /* non-empty batches per hotness window */
+    uint32_t rebalance_flags;     /* OR_RB_* */
 } or_config;
+
+/* Rebalancing variants (the paper's own wording of Sec. 3.3 / App. A.1.2):
+ * OR_RB_SLO_TARGET: an instance is overloaded when its queued work exceeds
+ *   the SLO, and migration from it stops once its queued work is within the
+ *   SLO ("until all requests in the overloaded instance's queue are
+ *   expected to meet the TTFT SLO");
+ * OR_RB_DOUBLE_OVERLOAD: a call migrates only after a routed batch in which
+ *   some request's estimated TTFT exceeded the SLO on both candidates (the
+ *   trigger "both candidate instances ... identified as overloaded"). */
+enum { OR_RB_SLO_TARGET = 1, OR_RB_DOUBLE_OVERLOAD = 2 };
 
 enum { OR_RULE_DUALMAP = 0, OR_RULE_CACHE_AFFINITY = 1, OR_RULE_LEAST_LOADED = 2,
        OR_RULE_MIN_TTFT = 3, OR_RULE_PREBLE = 4, OR_RULE_GLOBAL_CACHE_AFFINITY = 5,
@@ -239,6 +252,7 @@ typedef struct {
     uint64_t clock, next_seq, t_prev;
     int have_time;
     uint64_t rebalance_calls;
+    int both_over;      /* the last routed batch had a request over the SLO on both candidates */
     /* the last routed batch, kept for commit */
     uint32_t pend_n;
     uint64_t pend_seq0;
@@ -978,6 +992,7 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
                     s->state[id] == INST_LIVE ? cf->block_tokens * leading_hits(&s->cache[id], keys, nblk) : 0;
     }
     /* 2) choices in arrival order; loads update as we go */
+    s->both_over = 0;
     for (uint32_t r = 0; r < n; r++) {
         uint32_t c1 = cand1[r], c2 = cand2[r];
         uint32_t ch, hch;
@@ -994,6 +1009,7 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
             hch = ch == c1 ? hit1[r] : hit2[r];
         }
         chosen[r] = ch;
+        if (ttft1[r] > cf->slo_us && ttft2[r] > cf->slo_us) s->both_over = 1;
         q_entry e;
         e.seq = s->next_seq++;
         e.L = lengths[r]; e.c1 = c1; e.c2 = c2; e.h1 = hit1[r]; e.h2 = hit2[r];
@@ -1077,13 +1093,17 @@ int or_rebalance(or_state *s, uint64_t *mig_seq, uint32_t *mig_from, uint32_t *m
     uint32_t N = n_live(s);
     uint64_t sumW = 0;
     for (uint32_t i = 0; i < M; i++) if (s->state[i] == INST_LIVE) sumW += s->W[i];
+    const int slo_target = (cf->rebalance_flags & OR_RB_SLO_TARGET) != 0;
+    *n_out = 0;
+    if ((cf->rebalance_flags & OR_RB_DOUBLE_OVERLOAD) && !s->both_over) return OR_OK;
 
     /* hotspots at the start of the call, by W descending, then id */
     uint32_t *hot = (uint32_t *)malloc(M * sizeof(uint32_t));
     if (!hot) return OR_ERR_OOM;
     uint32_t nh = 0;
     for (uint32_t i = 0; i < M; i++)
-        if (s->state[i] == INST_LIVE && is_hot(s, i, sumW, N)) hot[nh++] = i;
+        if (s->state[i] == INST_LIVE && (slo_target ? s->W[i] > cf->slo_us : is_hot(s, i, sumW, N)))
+            hot[nh++] = i;
     for (uint32_t a = 1; a < nh; a++) {      /* insertion sort, stable by id */
         uint32_t x = hot[a], b = a;
         while (b > 0 && s->W[hot[b - 1]] < s->W[x]) { hot[b] = hot[b - 1]; b--; }
@@ -1112,7 +1132,7 @@ int or_rebalance(or_state *s, uint64_t *mig_seq, uint32_t *mig_from, uint32_t *m
         }
         qsort(cand, nc, sizeof(mig_cand), mig_cmp);
         for (uint32_t a = 0; a < nc; a++) {
-            if (!is_hot(s, i, sumW, N)) break;
+            if (slo_target ? !(s->W[i] > cf->slo_us) : !is_hot(s, i, sumW, N)) break;
             /* find the entry again (its position may have shifted) */
             uint64_t k = 0;
             while (k < q->len && q->e[q->head + k].seq != cand[a].seq) k++;
