@@ -155,6 +155,11 @@ typedef struct {
     uint32_t adapt_step_blocks;
     uint32_t adapt_max_blocks;
     uint32_t adapt_window;
+    /* Variants of dm_rebalance (DM_REBALANCE_* bits); 0 = the rule described
+     * at dm_rebalance. */
+    uint32_t rebalance_flags;
+    /* Must be 0. */
+    uint32_t reserved2;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */
@@ -210,6 +215,18 @@ enum {
     DM_STAGE_COUNT = 7
 };
 
+/* dm_config.rebalance_flags.  DM_REBALANCE_SLO_TARGET: an instance is
+ * overloaded when its queued work exceeds the SLO, and migration from it
+ * stops once its queued work is within the SLO (Sec. 3.3: "until all
+ * requests in the overloaded instance's queue are expected to meet the
+ * TTFT SLO"), instead of the 1.5x-mean hotspot rule.
+ * DM_REBALANCE_DOUBLE_OVERLOAD: dm_rebalance migrates only if, in the last
+ * routed batch, some request's estimated TTFT exceeded the SLO on both of
+ * its candidates (App. A.1.2: rebalancing starts "whenever both candidate
+ * instances of a request are identified as overloaded"). */
+#define DM_REBALANCE_SLO_TARGET 1u
+#define DM_REBALANCE_DOUBLE_OVERLOAD 2u
+
 /* Create a scheduler with no instances.  Allocates all device state except
  * the per-instance indices (allocated on first dm_add_instance of an id).
  * Derives the hash key material from cfg->seed.  Synchronous. */
@@ -261,6 +278,7 @@ DM_API dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *batch, 
 
 /* Hotspot-aware rebalancing (Sec. 3.3, Eq. "rebalance"; App. A.1.2), to be
  * called after dm_route_batch and before dm_commit_cache.  Hot instances
+ * (hot_den * N * W_i > hot_num * sum W, or see DM_REBALANCE_SLO_TARGET)
  * are visited in descending W; their queued, not-started requests are
  * ranked by migration benefit B = TTFT_{r,i} - TTFT_{r,j} (j the request's
  * other candidate) and moved to j while i stays hot, B > 0 and

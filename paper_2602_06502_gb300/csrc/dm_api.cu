@@ -209,6 +209,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
     if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
     if (c.choice_rule > DM_RULE_PREBLE) return DM_ERR_INVALID_ARG;
+    if (c.rebalance_flags > (DM_REBALANCE_SLO_TARGET | DM_REBALANCE_DOUBLE_OVERLOAD) || c.reserved2 != 0)
+        return DM_ERR_INVALID_ARG;
     if (c.adapt_step_blocks &&
         (c.adapt_max_blocks <= c.route_prefix_blocks || c.adapt_max_blocks > 2048 || c.adapt_window < 1))
         return DM_ERR_INVALID_ARG;
@@ -228,6 +230,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.hot_den = c.hot_den;
     d.max_batch = c.max_batch;
     d.rule = c.choice_rule;
+    d.rb_flags = c.rebalance_flags;
     d.ad_step = c.adapt_step_blocks;
     d.ad_max = c.adapt_step_blocks ? c.adapt_max_blocks : c.route_prefix_blocks;
     d.Kf2 = d.ad_max;

@@ -240,6 +240,7 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
             ms.hits += (ch == (a_is_c2 ? b : a)) ? h1 : h2;
             ms.sw += sw;
             ms.est += (pb ? tb : ta) <= slo;
+            if (ta > slo && tb > slo) d.info->both_over = 1;
             d.r_touchoff[r] = S.pt[k] >> 32;          // offset among this batch's records of ch
             const uint32_t slot = (uint32_t)S.pt[k];
             if (slot - d.q_head[ch] >= d.Q) {
@@ -467,6 +468,7 @@ __global__ void __launch_bounds__(1024) k_choice_global(DevState d, dm_route_out
             ms.tokens += L;
             ms.hits += h;
             ms.est += s_wa[rr] <= slo;
+            if (s_t1[rr] > slo && s_t2[rr] > slo) d.info->both_over = 1;
             const uint32_t slot = (uint32_t)Pold;
             if (slot - d.q_head[ch] >= d.Q) {
                 set_err(d.err, DM_ERR_CAPACITY);

@@ -139,7 +139,7 @@ struct BatchInfo {
     uint32_t final_dirty;   // a rebalance moved a request of this batch
     uint32_t mc_chunks;     // log-compaction chunks of this commit
     uint32_t mr_chunks;     // index-rebuild chunks of this commit
-    uint32_t pad;
+    uint32_t both_over;     // a request of this batch estimated TTFT > SLO on both candidates
 };
 
 struct Ring {
@@ -155,6 +155,7 @@ struct DevState {
     uint64_t C, slo;
     uint32_t cost, hot_num, hot_den, max_batch;
     uint32_t rule;                  // dm_choice_rule
+    uint32_t rb_flags;              // DM_REBALANCE_*
     // adaptive prefix length (ad_step = 0: every request hashes min(Kroute, n_blk) blocks)
     uint32_t Kf2;                   // the f2 digests are hashed over blocks < min(Kf2, n_blk)
     uint32_t ad_step, ad_max;

@@ -151,11 +151,15 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
     }
     const uint64_t sumW0 = block_sum_u64(myW, s_u);
     const uint32_t N = (uint32_t)block_sum_u64(myN, s_u);
-    // hot list (ids in ascending order), then ranks by (W desc, id asc)
+    // hot list (ids in ascending order), then ranks by (W desc, id asc);
+    // none when the double-overload trigger did not fire
+    const bool slo_target = (d.rb_flags & DM_REBALANCE_SLO_TARGET) != 0;
+    const bool armed = !(d.rb_flags & DM_REBALANCE_DOUBLE_OVERLOAD) || d.info->both_over;
     uint32_t nhot = 0;
     for (uint32_t base = 0; base < M; base += blockDim.x) {
         const uint32_t i = base + threadIdx.x;
-        const bool h = i < M && st[i] == 1 && hot(W[i], sumW0, N, d.hot_num, d.hot_den);
+        const bool h = armed && i < M && st[i] == 1 &&
+                       (slo_target ? W[i] > d.slo : hot(W[i], sumW0, N, d.hot_num, d.hot_den));
         uint32_t tot;
         const uint32_t rk = rank_in_block(h, s_w, tot);
         if (h) d.rb_pos[nhot + rk] = i;   // scratch: unsorted hot ids
@@ -277,7 +281,10 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
                 uint64_t sumW = s_sumW;
                 uint32_t nmv = 0, stop = 0;
                 for (uint32_t k = 0; k < m; ++k) {
-                    if (!hot(W[i], sumW, N, d.hot_num, d.hot_den)) { stop = 1; break; }
+                    if (slo_target ? !(W[i] > d.slo) : !hot(W[i], sumW, N, d.hot_num, d.hot_den)) {
+                        stop = 1;
+                        break;
+                    }
                     const uint32_t j = Ch.j[k];
                     if (st[j] != 1) continue;
                     const uint64_t nw = Ch.new_work[k];

@@ -96,6 +96,7 @@ __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off,
         d.info->total_blocks = carry_blk;
         d.info->total_segs = carry_seg;
         d.info->n = n;
+        d.info->both_over = 0;
         if (carry_blk > d.max_blocks || carry_seg > d.max_segs) set_err(d.err, DM_ERR_CAPACITY);
     }
 }

@@ -26,6 +26,7 @@ DM_RULE_CACHE_AFFINITY, DM_RULE_LEAST_LOADED, DM_RULE_MIN_TTFT, DM_RULE_PREBLE =
 RULE_NAMES = ["dualmap", "pair_cache_affinity", "pair_least_loaded", "pair_min_ttft", "pair_preble",
               "cache_affinity", "least_loaded", "min_ttft", "preble"]
 DM_HIST_BUCKETS = 976
+DM_REBALANCE_SLO_TARGET, DM_REBALANCE_DOUBLE_OVERLOAD = 1, 2
 
 
 class dm_config(C.Structure):
@@ -48,6 +49,8 @@ class dm_config(C.Structure):
         ("adapt_step_blocks", C.c_uint32),
         ("adapt_max_blocks", C.c_uint32),
         ("adapt_window", C.c_uint32),
+        ("rebalance_flags", C.c_uint32),
+        ("reserved2", C.c_uint32),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]

@@ -17,7 +17,7 @@ class Pair:
     """An oracle and a GPU scheduler built from the same workload dict."""
 
     def __init__(self, w, max_instances=None, max_batch_tokens=None, max_touch=0, max_queue=0, capacity=None,
-                 index_slots_log2=0, choice_rule=0, adapt=None):
+                 index_slots_log2=0, choice_rule=0, adapt=None, rebalance_flags=0):
         import torch
         from paper_2602_06502_gb300.scheduler import Scheduler
         self.torch = torch
@@ -30,12 +30,13 @@ class Pair:
         ad = dict(adapt_step_blocks=0, adapt_max_blocks=0, adapt_window=1) if adapt is None else dict(adapt)
         self.adaptive = bool(ad["adapt_step_blocks"])
         self.ora = O.Oracle(**O.config_from_workload(w, max_instances=self.M, max_batch_tokens=mbt),
-                            choice_rule=choice_rule, **ad)
+                            choice_rule=choice_rule, rebalance_flags=rebalance_flags, **ad)
         self.gpu = Scheduler(block_tokens=w["block_tokens"], route_prefix_blocks=w["route_prefix_blocks"],
                              vnodes=w["vnodes"], max_instances=self.M, capacity=w["capacity"], slo_us=w["slo_us"],
                              cost_us=w["cost_us"], max_batch=w["batch"], max_batch_tokens=mbt,
                              max_touch_per_instance=max_touch, max_queue=max_queue,
-                             index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule, **ad)
+                             index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule,
+                             rebalance_flags=rebalance_flags, **ad)
         self.dev = torch.device("cuda:0")
         self.n_migrations = 0
         self.n_switched = 0

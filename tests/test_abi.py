@@ -67,7 +67,8 @@ def test_create_rejects_bad_config_without_touching_gpu(built):
                 cfg(max_instances=1), cfg(choice_rule=D.DM_RULE_PREBLE + 1),
                 cfg(adapt_step_blocks=4, adapt_max_blocks=16, adapt_window=1),    # cap not above K_route
                 cfg(adapt_step_blocks=4, adapt_max_blocks=4096, adapt_window=1),  # cap above 2048
-                cfg(adapt_step_blocks=4, adapt_max_blocks=64, adapt_window=0)):
+                cfg(adapt_step_blocks=4, adapt_max_blocks=64, adapt_window=0),
+                cfg(rebalance_flags=4), cfg(reserved2=1)):
         assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
     assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
 
@@ -87,7 +88,8 @@ def test_struct_layouts_match_header(built, tmp_path):
         lines.append(f'printf("{st} %zu\\n", sizeof({st}));')
         for f in fs:
             lines.append(f'printf("{st}.{f} %zu\\n", offsetof({st}, {f}));')
-    consts = ["DM_HIST_BUCKETS"] + [f"DM_RULE_{n.upper()}" for n in D.RULE_NAMES]
+    consts = ["DM_HIST_BUCKETS", "DM_REBALANCE_SLO_TARGET", "DM_REBALANCE_DOUBLE_OVERLOAD"] + \
+        [f"DM_RULE_{n.upper()}" for n in D.RULE_NAMES]
     for c in consts:
         lines.append(f'printf("{c} %u\\n", (unsigned){c});')
     lines.append("return 0; }")

@@ -265,6 +265,30 @@ def test_adaptive_prefix_with_scaling_and_rebalance():
     run_trace(p, tr, rebalance=True)
 
 
+# -- rebalancing variants -------------------------------------------------------------
+
+@pytest.mark.parametrize("flags", [0, 1, 2, 3])
+def test_rebalance_variants_skewed(flags):
+    """A skewed 16-instance workload with a 5 ms SLO, rebalancing after every
+    batch: the 1.5x-mean rule, the SLO target, the double-overload trigger
+    and both (DM_REBALANCE_* bits); migrations bit for bit."""
+    w = workload("scaling", n_requests=3000, batch=50, n_instances=16, vnodes=32, n_prefix=100, zipf_s=1.2,
+                 len_lo=400, len_hi=512, prefix_lo=384, prefix_hi=384, scale_every=0, rho=1.0, slo_us=5000)
+    tr = Trace(w)
+    p = Pair(w, max_instances=16, rebalance_flags=flags)
+    run_trace(p, tr, rebalance=True, state_every=10)
+    assert p.n_migrations > 0
+
+
+@pytest.mark.parametrize("flags", [1, 3])
+def test_rebalance_variants_tiny(flags):
+    w = workload("tiny", n_requests=2000, batch=100, capacity=700, zipf_s=1.3, rho=1.2, slo_us=20_000)
+    tr = Trace(w)
+    p = Pair(w, max_touch=2600, rebalance_flags=flags)
+    run_trace(p, tr, rebalance=True, state_every=5)
+    assert p.n_migrations > 0
+
+
 # -- edge cases ---------------------------------------------------------------------
 
 def _mk(**kw):
