@@ -1313,3 +1313,57 @@ uint64_t or_prefix_tree(const or_state *s, uint64_t *keys, uint64_t cap)
     for (uint64_t i = 0; i < s->ad_set_n && i < cap; i++) keys[i] = s->ad_set[i];
     return s->ad_set_n;
 }
+
+/* ------------------------------------------------------------------ */
+/* Power of d choices (App. A.8, "Optimal Candidate Set Size")          */
+/* ------------------------------------------------------------------ */
+
+/* Choice k of ball t in trial s: with c = (s * m + t) * d + k, the value
+ * x_c = the (c+1)-th output of SplitMix64 seeded with `seed`, and the bin
+ * floor(x_c * n / 2^64). */
+uint32_t or_potc_choice(uint64_t seed, uint64_t c, uint32_t n)
+{
+    uint64_t state = seed + c * 0x9E3779B97F4A7C15ULL;   /* the state before output c+1 */
+    uint64_t x = or_splitmix64_next(&state);
+    return (uint32_t)(((unsigned __int128)x * n) >> 64);
+}
+
+/* Place one ball: the least loaded of its d choices, ties to the earlier
+ * choice. */
+static uint32_t potc_place(uint32_t *load, const uint32_t *choice, uint32_t d)
+{
+    uint32_t best = choice[0];
+    for (uint32_t k = 1; k < d; k++)
+        if (load[choice[k]] < load[best]) best = choice[k];
+    load[best]++;
+    return best;
+}
+
+/* Hand-given choices (tests): choices[t*d + k]; fills load[n]. */
+void or_potc_place_all(const uint32_t *choices, uint64_t m, uint32_t d, uint32_t n, uint32_t *load)
+{
+    memset(load, 0, n * sizeof(uint32_t));
+    for (uint64_t t = 0; t < m; t++) potc_place(load, choices + t * d, d);
+}
+
+/* Maximum bin load of each of `trials` trials of m balls into n bins with
+ * d choices each. */
+int or_potc_max_loads(uint32_t n, uint64_t m, uint32_t d, uint32_t trials, uint64_t seed, uint32_t *max_load)
+{
+    if (n < 1 || d < 1 || d > 64) return OR_ERR_INVALID_ARG;
+    uint32_t *load = (uint32_t *)malloc(n * sizeof(uint32_t));
+    if (!load) return OR_ERR_OOM;
+    uint32_t choice[64];
+    for (uint32_t s = 0; s < trials; s++) {
+        memset(load, 0, n * sizeof(uint32_t));
+        for (uint64_t t = 0; t < m; t++) {
+            for (uint32_t k = 0; k < d; k++) choice[k] = or_potc_choice(seed, ((uint64_t)s * m + t) * d + k, n);
+            potc_place(load, choice, d);
+        }
+        uint32_t mx = 0;
+        for (uint32_t i = 0; i < n; i++) if (load[i] > mx) mx = load[i];
+        max_load[s] = mx;
+    }
+    free(load);
+    return OR_OK;
+}

@@ -109,6 +109,9 @@ def lib():
             "or_hist_lower": (C.c_uint64, [C.c_uint32]),
             "or_get_metrics": (None, [V, u64p, P(C.c_double), V, C.c_int]),
             "or_last_route_blocks": (C.c_uint32, [V, V]),
+            "or_potc_choice": (C.c_uint32, [C.c_uint64, C.c_uint64, C.c_uint32]),
+            "or_potc_place_all": (None, [u32p, C.c_uint64, C.c_uint32, C.c_uint32, u32p]),
+            "or_potc_max_loads": (C.c_int, [C.c_uint32, C.c_uint64, C.c_uint32, C.c_uint32, C.c_uint64, u32p]),
             "or_prefix_tree": (C.c_uint64, [V, V, C.c_uint64]),
         }
         for name, (res, args) in sig.items():
@@ -162,6 +165,25 @@ def choose(c1, c2, h1, h2, L, W1, W2, slo, cost=1, rule=RULE_DUALMAP):
     ch = lib().or_choose(rule, c1, c2, h1, h2, L, W1, W2, slo, cost, C.byref(t1), C.byref(t2),
                          C.byref(sw))
     return ch, t1.value, t2.value, sw.value
+
+
+def potc_choice(seed, c, n):
+    return lib().or_potc_choice(seed, c, n)
+
+
+def potc_place_all(choices, n):
+    ch = np.ascontiguousarray(choices, dtype=np.uint32)
+    load = np.zeros(n, np.uint32)
+    lib().or_potc_place_all(ch.reshape(-1), ch.shape[0], ch.shape[1], n, load)
+    return load
+
+
+def potc_max_loads(n, m, d, trials, seed):
+    out = np.zeros(max(trials, 1), np.uint32)
+    rc = lib().or_potc_max_loads(n, m, d, trials, seed, out)
+    if rc:
+        raise ValueError(f"or_potc_max_loads: {rc}")
+    return out[:trials]
 
 
 def hist_bucket(v):
