@@ -416,6 +416,19 @@ DM_API dm_status dm_get_route_blocks(dm_handle *h, uint32_t *out_dev, uint32_t n
  * written).  0 nodes when the length is fixed.  Synchronous. */
 DM_API dm_status dm_export_prefix_tree(dm_handle *h, uint64_t *keys_host, uint64_t cap, uint64_t *n_out);
 
+/* The power-of-d-choices experiment behind DualMap's two candidates (App.
+ * A.8): `trials` independent trials of m_balls balls into n_bins bins, each
+ * ball placed in the least loaded of d uniformly random bins (ties to the
+ * earlier choice); max_load_dev (device, `trials` entries) receives each
+ * trial's maximum bin load (the deviation is that minus m/n).  Ball t's
+ * choice k in trial s is floor(x * n_bins / 2^64) for x the (c+1)-th output
+ * of SplitMix64(seed), c = (s * m_balls + t) * d + k.  No handle; work is
+ * enqueued on `stream` (a cudaStream_t, NULL = legacy default stream).
+ * 1 <= n_bins <= 256, 1 <= d <= 64, m_balls < 2^32; DM_ERR_INVALID_ARG
+ * otherwise, DM_ERR_CUDA if the launch fails. */
+DM_API dm_status dm_potc_max_loads(uint32_t n_bins, uint64_t m_balls, uint32_t d, uint32_t trials, uint64_t seed,
+                                   uint32_t *max_load_dev, void *stream);
+
 /* Synchronise the stream and return the sticky error (DM_OK if none). */
 DM_API dm_status dm_last_error(dm_handle *h);
 

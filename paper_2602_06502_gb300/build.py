@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(ROOT, "_build", "dualmap")
 LIB = os.path.join(HERE, "libdualmap.so")
 SOURCES = ["dm_api.cu", "dm_setup.cu", "dm_hash.cu", "dm_route.cu", "dm_choice.cu", "dm_commit.cu",
-           "dm_rebalance.cu", "dm_ring.cu", "dm_noalloc.cu"]
+           "dm_rebalance.cu", "dm_ring.cu", "dm_noalloc.cu", "dm_potc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

@@ -119,6 +119,8 @@ SIGNATURES = {
     "dm_get_metrics": (C.c_int, [C.c_void_p, C.POINTER(dm_metrics), C.c_void_p, C.c_uint32, C.c_int]),
     "dm_get_route_blocks": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32]),
     "dm_export_prefix_tree": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint64, C.POINTER(C.c_uint64)]),
+    "dm_potc_max_loads": (C.c_int, [C.c_uint32, C.c_uint64, C.c_uint32, C.c_uint32, C.c_uint64, C.c_void_p,
+                                    C.c_void_p]),
     "dm_last_error": (C.c_int, [C.c_void_p]),
     "dm_set_profiling": (C.c_int, [C.c_void_p, C.c_int]),
     "dm_get_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int]),
@@ -290,6 +292,10 @@ def dm_export_prefix_tree(h):
     k = np.zeros(max(n.value, 1), np.uint64)
     _check(lib().dm_export_prefix_tree(h, k.ctypes.data, n.value, C.byref(n)), "dm_export_prefix_tree")
     return np.sort(k[:n.value])
+
+
+def dm_potc_max_loads(n_bins, m_balls, d, trials, seed, max_load_dev, stream=None):
+    return lib().dm_potc_max_loads(n_bins, m_balls, d, trials, seed, _ptr(max_load_dev), stream)
 
 
 def dm_last_error(h):
