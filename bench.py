@@ -38,7 +38,7 @@ def longctx_handle_kwargs(w):
     """Handle sizes used for the long-context workload (bench and its parity test)."""
     return dict(max_instances=w["n_instances"] + 8, max_batch=w["batch"],
                 max_batch_tokens=w["batch"] * w["len_hi"] + 4 * w["batch"],
-                max_touch_per_instance=1 << 20, index_slots_log2=24)
+                max_touch_per_instance=1 << 20, index_slots_log2=25, rebuild_pool=16)
 
 
 def handle_kwargs(w, max_id):

@@ -158,8 +158,13 @@ typedef struct {
     /* Variants of dm_rebalance (DM_REBALANCE_* bits); 0 = the rule described
      * at dm_rebalance. */
     uint32_t rebalance_flags;
-    /* Must be 0. */
-    uint32_t reserved2;
+    /* Spare index buffers shared by all instances as rebuild targets (a
+     * rebuild builds the new index in a spare and returns the old one to the
+     * pool); 0 = one per instance.  Fewer than max_instances halves the
+     * index memory; rebuilds beyond the pool then wait their turn (round
+     * robin), so dm_create requires index_slots / 2 >= ceil(max_instances /
+     * rebuild_pool) * max_touch_per_instance (DM_ERR_INVALID_ARG otherwise). */
+    uint32_t rebuild_pool;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */

@@ -44,7 +44,8 @@ struct dm_handle {
     int cur[2] = {0, 0};
     uint64_t *ring_spos = nullptr;
     uint32_t *ring_svidx = nullptr;
-    std::vector<Slot *> tables, tables2;   // both index buffers of each id (host copies)
+    std::vector<Slot *> tables;   // the index buffer first allocated for each id (null: never added)
+    uint32_t pool_target = 0;     // spare index buffers wanted (one per allocated id, up to rebuild_pool)
     std::vector<Rec *> logs, logs2;        // both log buffers
     std::vector<uint8_t *> stales, stales2;
     std::vector<uint32_t *> homes, homes2;  // both index-home logs
@@ -209,8 +210,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
     if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
     if (c.choice_rule > DM_RULE_PREBLE) return DM_ERR_INVALID_ARG;
-    if (c.rebalance_flags > (DM_REBALANCE_SLO_TARGET | DM_REBALANCE_DOUBLE_OVERLOAD) || c.reserved2 != 0)
-        return DM_ERR_INVALID_ARG;
+    if (c.rebalance_flags > (DM_REBALANCE_SLO_TARGET | DM_REBALANCE_DOUBLE_OVERLOAD)) return DM_ERR_INVALID_ARG;
     if (c.adapt_step_blocks &&
         (c.adapt_max_blocks <= c.route_prefix_blocks || c.adapt_max_blocks > 2048 || c.adapt_window < 1))
         return DM_ERR_INVALID_ARG;
@@ -241,6 +241,15 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.index_slots_log2 && (1ull << c.index_slots_log2) > d.S) d.S = 1ull << c.index_slots_log2;
     if (d.S < 64) d.S = 64;   // at least a few whole groups
     if (d.S > (1ull << 32)) {
+        delete h;
+        return DM_ERR_INVALID_ARG;
+    }
+    // a pool smaller than the instance count makes rebuilds wait up to
+    // ceil(M / pool) commits: the index must hold that many commits' touches
+    // above half full
+    h->pool_target = c.rebuild_pool && c.rebuild_pool < c.max_instances ? c.rebuild_pool : c.max_instances;
+    if (h->pool_target < c.max_instances &&
+        d.S / 2 < uint64_t((c.max_instances + h->pool_target - 1) / h->pool_target) * d.T) {
         delete h;
         return DM_ERR_INVALID_ARG;
     }
@@ -285,6 +294,9 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.table, M));
     A(dalloc(h, &d.logbuf, M));
     A(dalloc(h, &d.table_alt, M));
+    A(dalloc(h, &d.pool, h->pool_target));
+    A(dalloc(h, &d.rb_slot, M));
+    A(dalloc(h, &d.rb_rr, 1));
     A(dalloc(h, &d.logbuf_alt, M));
     A(dalloc(h, &d.stale, M));
     A(dalloc(h, &d.stale_alt, M));
@@ -382,6 +394,8 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(cudaMemsetAsync(d.table, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.logbuf, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.table_alt, 0, M * 8, h->st));
+    A(cudaMemsetAsync(d.pool, 0, uint64_t(h->pool_target) * 8, h->st));
+    A(cudaMemsetAsync(d.rb_rr, 0, 4, h->st));
     A(cudaMemsetAsync(d.logbuf_alt, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.stale, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.stale_alt, 0, M * 8, h->st));
@@ -406,7 +420,7 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     h->state.assign(M, 0);
     h->tables.assign(M, nullptr);
     h->logs.assign(M, nullptr);
-    h->tables2.assign(M, nullptr);
+
     h->logs2.assign(M, nullptr);
     h->stales.assign(M, nullptr);
     h->stales2.assign(M, nullptr);
@@ -475,13 +489,15 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         if (e != cudaSuccess) return map_cuda(h, e);
         if (ht[0] != ht[1]) return DM_ERR_DUPLICATE_ID;
     }
-    if (!h->tables[id]) {
-        Slot *t = nullptr, *t2 = nullptr;
+    Slot *cur = h->tables[id];   // the index this id uses now (rebuilds trade buffers with the pool)
+    const bool first = cur == nullptr;
+    if (first) {
+        Slot *t = nullptr, *spare = nullptr;
         Rec *lg = nullptr, *lg2 = nullptr;
         uint8_t *sf = nullptr, *sf2 = nullptr;
         uint32_t *hm = nullptr, *hm2 = nullptr;
         e = dalloc(h, &t, d.S);
-        if (e == cudaSuccess) e = dalloc(h, &t2, d.S);
+        if (e == cudaSuccess && d.pool_n < h->pool_target) e = dalloc(h, &spare, d.S);
         if (e == cudaSuccess) e = dalloc(h, &lg, d.logcap);
         if (e == cudaSuccess) e = dalloc(h, &lg2, d.logcap);
         if (e == cudaSuccess) e = dalloc(h, &sf, d.logcap);
@@ -489,8 +505,14 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         if (e == cudaSuccess) e = dalloc(h, &hm, d.logcap);
         if (e == cudaSuccess) e = dalloc(h, &hm2, d.logcap);
         if (e != cudaSuccess) { cudaGetLastError(); return DM_ERR_OOM; }
+        if (spare) {
+            e = cudaMemcpyAsync(d.pool + d.pool_n, &spare, sizeof(Slot *), cudaMemcpyHostToDevice, h->st);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+            if (e != cudaSuccess) return map_cuda(h, e);
+            ++h->d.pool_n;
+        }
         h->tables[id] = t;
-        h->tables2[id] = t2;
+        cur = t;
         h->logs[id] = lg;
         h->logs2[id] = lg2;
         h->stales[id] = sf;
@@ -498,9 +520,14 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         h->homes[id] = hm;
         h->homes2[id] = hm2;
     }
-    // a (re-)added instance starts empty, both buffers of each
+    if (!first) {   // a re-added id keeps whichever index buffer it holds now
+        e = cudaMemcpyAsync(&cur, d.table + id, sizeof(Slot *), cudaMemcpyDeviceToHost, h->st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+        if (e != cudaSuccess) return map_cuda(h, e);
+    }
+    // a (re-)added instance starts empty, both buffers of each log
     struct { void *dst; const void *src; } ptrs[] = {
-        {d.table + id, &h->tables[id]}, {d.table_alt + id, &h->tables2[id]},
+        {d.table + id, &cur},
         {d.logbuf + id, &h->logs[id]}, {d.logbuf_alt + id, &h->logs2[id]},
         {d.stale + id, &h->stales[id]}, {d.stale_alt + id, &h->stales2[id]},
         {d.loghome + id, &h->homes[id]}, {d.loghome_alt + id, &h->homes2[id]}};
@@ -508,8 +535,7 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
         if (e == cudaSuccess) e = cudaMemcpyAsync(pp.dst, pp.src, sizeof(void *), cudaMemcpyHostToDevice, h->st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
     if (e != cudaSuccess) return map_cuda(h, e);
-    e = cudaMemsetAsync(h->tables[id], 0, d.S * sizeof(Slot), h->st);
-    if (e == cudaSuccess) e = cudaMemsetAsync(h->tables2[id], 0, d.S * sizeof(Slot), h->st);
+    e = cudaMemsetAsync(cur, 0, d.S * sizeof(Slot), h->st);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->stales[id], 0, d.logcap, h->st);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->stales2[id], 0, d.logcap, h->st);
     if (e == cudaSuccess) e = cudaMemsetAsync(d.log_front + id, 0, 8, h->st);

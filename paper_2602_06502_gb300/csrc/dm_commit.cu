@@ -33,6 +33,12 @@ constexpr uint32_t kZeroChunk = 4096;   // slots or flag bytes cleared per chunk
 // contents.  Every slot update of the touch passes goes through this, so key
 // and position change together and never tear (whole-bucket reads are plain
 // 16-byte loads used only to pick the next slot to try).
+// Raise the position word of a slot whose key is set (keys never change once
+// set, and positions only grow): returns the value it had before.
+__device__ __forceinline__ uint64_t pos_max(Slot *s, uint64_t p1) {
+    return atomicMax(reinterpret_cast<unsigned long long *>(&s->pos1), (unsigned long long)p1);
+}
+
 __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
     Slot old;
     asm volatile(
@@ -71,12 +77,9 @@ __device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64
     const uint64_t limit = mask + 1 + (1ull << 20);
     for (uint64_t it = 0; it < limit; ++it) {
         if (old.key == 0) { *claimed = true; return 0; }   // a CAS from {0,0} that failed returns a key
-        if (old.key == key) {
+        if (old.key == key) {   // the slot's key never changes: raise its position word alone
             if (old.pos1 >= p1) return old.pos1;
-            const Slot now = slot_cas(&t[i], old, Slot{key, p1});
-            if (now.pos1 == old.pos1) return old.pos1;      // keys never change once set
-            old = now;
-            continue;
+            return pos_max(&t[i], p1);
         }
         Slot sn[kGroup];
 #pragma unroll
@@ -185,24 +188,60 @@ __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
     for (uint32_t r = threadIdx.x; r < n; r += blockDim.x)
         atomicAdd(&cntv[d.r_final[r]], (unsigned long long)d.r_nblk[r]);
     __syncthreads();
+    // 1) what each instance needs: compaction if its log would overflow,
+    //    a rebuild if its index would pass half full
+    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
+        uint32_t fl = 0;
+        if (d.table[i]) {
+            const uint64_t cnt = cntv[i];
+            if (cnt > d.T) set_err(d.err, DM_ERR_CAPACITY);
+            if (d.log_tail[i] - d.log_front[i] + cnt > d.logcap) fl |= kFlagCompact;
+            if (d.used[i] + cnt > d.S / 2) fl |= kFlagRebuild;
+            d.touch_cnt[i] = cnt;
+        }
+        d.mt_flags[i] = fl;
+    }
+    __syncthreads();
+    // 2) rebuilds take spare buffers from the pool, in id order from a
+    //    rotating start; those beyond the pool wait for a later commit (each
+    //    waits at most ceil(M / pool) commits; dm_create checks the index
+    //    has that much headroom above half full)
+    __shared__ uint32_t s_served, s_last;
+    if (threadIdx.x == 0) { s_served = 0; s_last = 0; }
+    __syncthreads();
+    const uint32_t rr = *d.rb_rr;
+    for (uint32_t base = 0; base < d.M; base += blockDim.x) {
+        const uint32_t k = base + threadIdx.x;
+        const uint32_t i = k < d.M ? (rr + k) % d.M : 0;
+        const bool want = k < d.M && (d.mt_flags[i] & kFlagRebuild);
+        uint32_t tot;
+        const uint32_t rank = s_served + block_excl_u32(want ? 1u : 0u, s_w, tot);
+        if (want) {
+            if (rank < d.pool_n) {
+                d.rb_slot[i] = rank;
+                d.table_alt[i] = d.pool[rank];
+                atomicMax(&s_last, k);   // the last position served
+            } else {
+                d.mt_flags[i] &= ~kFlagRebuild;
+            }
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) s_served += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0 && s_served) *d.rb_rr = (rr + s_last + 1) % d.M;
+    __syncthreads();
+    // 3) chunk offsets of the work the final flags ask for
     uint32_t cw = 0, cz = 0;
     for (uint32_t base = 0; base < d.M; base += blockDim.x) {
         const uint32_t i = base + threadIdx.x;
         uint32_t nw = 0, nz = 0, fl = 0;
         if (i < d.M && d.table[i]) {
-            const uint64_t cnt = cntv[i];
-            if (cnt > d.T) set_err(d.err, DM_ERR_CAPACITY);
+            fl = d.mt_flags[i];
             const uint64_t len = d.log_tail[i] - d.log_front[i];
-            if (len + cnt > d.logcap) {
-                fl |= kFlagCompact;
-                nz += (uint32_t)((d.logcap + kZeroChunk - 1) / kZeroChunk);
-            }
-            if (d.used[i] + cnt > d.S / 2) {
-                fl |= kFlagRebuild;
-                nz += (uint32_t)((d.S + kZeroChunk - 1) / kZeroChunk);
-            }
+            if (fl & kFlagCompact) nz += (uint32_t)((d.logcap + kZeroChunk - 1) / kZeroChunk);
+            if (fl & kFlagRebuild) nz += (uint32_t)((d.S + kZeroChunk - 1) / kZeroChunk);
             if (fl) nw = (uint32_t)((len + kEvChunk - 1) / kEvChunk);
-            d.touch_cnt[i] = cnt;
         }
         uint32_t tw, tz;
         const uint32_t ew = block_excl_u32(nw, s_w, tw);
@@ -370,10 +409,10 @@ __global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
             d.log_tail[i] = d.mt_newtail[i];
             atomicAdd(reinterpret_cast<unsigned long long *>(&d.maint_count[1]), 1ull);
         }
-        if (fl & kFlagRebuild) {
-            Slot *a = d.table[i];
+        if (fl & kFlagRebuild) {   // the old index goes back to the pool
+            d.pool[d.rb_slot[i]] = d.table[i];
             d.table[i] = d.table_alt[i];
-            d.table_alt[i] = a;
+            d.table_alt[i] = nullptr;
             d.used[i] = d.live[i];
             atomicAdd(reinterpret_cast<unsigned long long *>(&d.maint_count[0]), 1ull);
         }
@@ -513,8 +552,10 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
                 x0 = lane < (int)cn ? d.plocal[pi + lane] : 0;
                 x1 = lane + 32 < (int)cn ? d.plocal[pi + lane + 32] : 0;
             }
-            // a key found at its home with an older position: one attempt to
-            // raise it here.  A key whose home slot holds another key, in a
+            // a key found at its home with an older position: raised here by
+            // an atomic max on its position word, which always settles the
+            // touch (the value it returns orders it against every other
+            // touch of the key).  A key whose home slot holds another key, in a
             // group whose 8 lanes found every slot of the home bucket taken
             // and none holding the key, continues its probe order in the
             // next bucket: one attempt there.  (Slots never empty again, so
@@ -541,9 +582,9 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             }
             const uint64_t n0 = probe_bucket(1, h0 & ~uint64_t(kGroup - 1), k0, mask) | (h0 & (kGroup - 1));
             const uint64_t n1 = probe_bucket(1, h1 & ~uint64_t(kGroup - 1), k1, mask) | (h1 & (kGroup - 1));
-            if (up0) r0 = slot_cas(&g.t[h0], c0s, Slot{k0, p0 + 1});
+            if (up0) r0 = Slot{k0, pos_max(&g.t[h0], p0 + 1)};
             else if (mv0) r0 = slot_cas(&g.t[n0], Slot{0, 0}, Slot{k0, p0 + 1});
-            if (up1) r1 = slot_cas(&g.t[h1], c1s, Slot{k1, p1 + 1});
+            if (up1) r1 = Slot{k1, pos_max(&g.t[h1], p1 + 1)};
             else if (mv1) r1 = slot_cas(&g.t[n1], Slot{0, 0}, Slot{k1, p1 + 1});
             // settled here: a claim of an empty home slot, a raise that went
             // through, or the key found with a later position already; the
@@ -555,19 +596,17 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
                 if (c0s.key == 0 || (mv0 && r0.key == 0)) { ++newly; ++claims; }
                 else if (mv0 && r0.key == k0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
                 else if (mv0) { need0 = true; x0 = r0.pos1; }
-                else if (up0 && r0.pos1 == c0s.pos1) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
-                else if (up0 && r0.pos1 > p0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);
+                else if (up0) touch_outcome(r0.pos1, p0, g.front, g.st, lmask, newly);   // the max settles it
                 else if (!up0 && c0s.key == k0) touch_outcome(c0s.pos1, p0, g.front, g.st, lmask, newly);
-                else { need0 = true; x0 = up0 ? r0.pos1 : c0s.pos1; }
+                else { need0 = true; x0 = c0s.pos1; }
             }
             if (v1) {
                 if (c1s.key == 0 || (mv1 && r1.key == 0)) { ++newly; ++claims; }
                 else if (mv1 && r1.key == k1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
                 else if (mv1) { need1 = true; x1 = r1.pos1; }
-                else if (up1 && r1.pos1 == c1s.pos1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
-                else if (up1 && r1.pos1 > p1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
+                else if (up1) touch_outcome(r1.pos1, p1, g.front, g.st, lmask, newly);
                 else if (!up1 && c1s.key == k1) touch_outcome(c1s.pos1, p1, g.front, g.st, lmask, newly);
-                else { need1 = true; x1 = up1 ? r1.pos1 : c1s.pos1; }
+                else { need1 = true; x1 = c1s.pos1; }
             }
             // deferred touches go to the segment's own slice of the queue
             const uint32_t m0 = __ballot_sync(0xffffffffu, need0), m1 = __ballot_sync(0xffffffffu, need1);
@@ -594,12 +633,12 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
 }
 
 // Second pass over the deferred touches, a warp per segment: raise the
-// position of a found key (CAS loop), or walk the probe order of a key whose
-// home slot holds another key.  Every record still ends up marked stale
-// exactly once unless it is its key's latest: the first pass settled only
-// touches whose outcome its own CAS fixed (a claim of an empty slot, a raise
-// that went through, a later position already there), and the maxima taken
-// here order the rest.
+// position of a found key (atomic max), or walk the probe order of a key
+// whose home slot holds another key.  Every record still ends up marked
+// stale exactly once unless it is its key's latest: the first pass settled
+// only touches whose outcome its own atomic fixed (a claim of an empty slot,
+// a raise, a later position already there), and the maxima taken here order
+// the rest.
 __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
     pdl_enter();
     if (has_err(d.err)) return;

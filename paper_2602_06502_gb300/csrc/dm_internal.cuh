@@ -183,7 +183,11 @@ struct DevState {
     Rec **logbuf;                   // per id: logcap records
     uint8_t **stale;                // per id: logcap flags, 1 = record superseded by a later touch
     uint32_t **loghome;             // per id: logcap index home slots, one per record
-    Slot **table_alt;               // per id: second index buffer (rebuild target)
+    Slot **table_alt;               // per id: its rebuild target during a commit that rebuilds it, else null
+    Slot **pool;                    // spare index buffers shared by all ids (pool_n of them)
+    uint32_t pool_n;
+    uint32_t *rb_slot;              // per id: the pool entry its rebuild took this commit
+    uint32_t *rb_rr;                // round-robin start of the rebuild order (1 entry)
     Rec **logbuf_alt;               // per id: second log buffer (compaction target)
     uint8_t **stale_alt;
     uint32_t **loghome_alt;

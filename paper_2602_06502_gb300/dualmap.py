@@ -50,7 +50,7 @@ class dm_config(C.Structure):
         ("adapt_max_blocks", C.c_uint32),
         ("adapt_window", C.c_uint32),
         ("rebalance_flags", C.c_uint32),
-        ("reserved2", C.c_uint32),
+        ("rebuild_pool", C.c_uint32),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]

@@ -17,7 +17,7 @@ class Pair:
     """An oracle and a GPU scheduler built from the same workload dict."""
 
     def __init__(self, w, max_instances=None, max_batch_tokens=None, max_touch=0, max_queue=0, capacity=None,
-                 index_slots_log2=0, choice_rule=0, adapt=None, rebalance_flags=0):
+                 index_slots_log2=0, choice_rule=0, adapt=None, rebalance_flags=0, rebuild_pool=0):
         import torch
         from paper_2602_06502_gb300.scheduler import Scheduler
         self.torch = torch
@@ -36,7 +36,7 @@ class Pair:
                              cost_us=w["cost_us"], max_batch=w["batch"], max_batch_tokens=mbt,
                              max_touch_per_instance=max_touch, max_queue=max_queue,
                              index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule,
-                             rebalance_flags=rebalance_flags, **ad)
+                             rebalance_flags=rebalance_flags, rebuild_pool=rebuild_pool, **ad)
         self.dev = torch.device("cuda:0")
         self.n_migrations = 0
         self.n_switched = 0

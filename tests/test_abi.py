@@ -68,7 +68,8 @@ def test_create_rejects_bad_config_without_touching_gpu(built):
                 cfg(adapt_step_blocks=4, adapt_max_blocks=16, adapt_window=1),    # cap not above K_route
                 cfg(adapt_step_blocks=4, adapt_max_blocks=4096, adapt_window=1),  # cap above 2048
                 cfg(adapt_step_blocks=4, adapt_max_blocks=64, adapt_window=0),
-                cfg(rebalance_flags=4), cfg(reserved2=1)):
+                cfg(rebalance_flags=4),
+                cfg(rebuild_pool=1, index_slots_log2=12, max_touch_per_instance=1024)):   # 4 waits x 1024 > 2^11
         assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
     assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
 

@@ -527,6 +527,27 @@ def test_index_rebuild_and_log_compaction():
     assert rebuilds > rebuilds0, (rebuilds, compactions2)
 
 
+def test_rebuilds_share_a_one_buffer_pool():
+    """One spare index buffer for all instances: two instances filling their
+    indices at the same rate cross half full together, so one rebuild waits
+    a commit for the buffer the other returns; results stay bit-exact and
+    the rebuild counter keeps rising."""
+    from paper_2602_06502_gb300 import dualmap as D
+    rng = np.random.default_rng(24)
+    w = _mk(n_instances=3, vnodes=16, capacity=1000, batch=64)
+    p = Pair(w, max_instances=3, max_touch=4096, index_slots_log2=15, rebuild_pool=1)
+    for i in range(3):
+        assert p.add(i) == 0
+    uniq = [[rng.integers(0, 32000, size=16 * 64, dtype=np.uint32) for _ in range(64)] for _ in range(30)]
+    t = _run_prompts(p, uniq[:24], state_every=3)
+    rebuilds, _ = D.dm_get_maint_counts(p.gpu.h)
+    assert rebuilds >= 3, rebuilds
+    assert p.remove(1) == 0
+    t = _run_prompts(p, uniq[24:26], t0=t + 10**9, state_every=1)   # instance 1's queue drains
+    assert p.add(1) == 0                   # a re-added id keeps whichever buffer it holds now
+    _run_prompts(p, uniq[26:], t0=t, state_every=1)
+
+
 def test_eviction_of_more_than_one_round():
     """Each commit evicts about 327k records per instance, more than one
     eviction round (4 CTAs x 65,536 records) covers."""
