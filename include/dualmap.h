@@ -130,8 +130,9 @@ typedef struct {
     uint32_t max_queue;
     /* log2 of the index slots per instance; 0 = automatic, the smallest
      * power of two >= 2 x (C + max_touch_per_instance).  A larger index is
-     * rebuilt less often (it is rebuilt when half full, counting the slots
-     * evicted keys keep).  Never smaller than the automatic size, nor than
+     * rebuilt less often (it is rebuilt when a quarter full if a quarter
+     * still holds C + max_touch_per_instance keys, else when half full,
+     * counting the slots evicted keys keep).  Never smaller than the automatic size, nor than
      * 64; <= 32.  dm_create returns DM_ERR_INVALID_ARG when the resulting
      * index would exceed 2^32 slots (it records slot numbers as 32 bits). */
     uint32_t index_slots_log2;

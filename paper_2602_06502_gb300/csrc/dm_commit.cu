@@ -189,14 +189,14 @@ __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
         atomicAdd(&cntv[d.r_final[r]], (unsigned long long)d.r_nblk[r]);
     __syncthreads();
     // 1) what each instance needs: compaction if its log would overflow,
-    //    a rebuild if its index would pass half full
+    //    a rebuild if its index would pass rb_thr taken slots
     for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
         uint32_t fl = 0;
         if (d.table[i]) {
             const uint64_t cnt = cntv[i];
             if (cnt > d.T) set_err(d.err, DM_ERR_CAPACITY);
             if (d.log_tail[i] - d.log_front[i] + cnt > d.logcap) fl |= kFlagCompact;
-            if (d.used[i] + cnt > d.S / 2) fl |= kFlagRebuild;
+            if (d.used[i] + cnt > d.rb_thr) fl |= kFlagRebuild;
             d.touch_cnt[i] = cnt;
         }
         d.mt_flags[i] = fl;

@@ -164,6 +164,7 @@ struct DevState {
     AdCount *ad_cnt;                // node counts of the current window
     uint64_t ad_cnt_mask;
     uint64_t max_blocks, max_segs, T, S, logcap;
+    uint64_t rb_thr;                // an index is rebuilt when its taken slots would pass this
     uint32_t Q;
     // key material
     uint32_t K1[64], K2[64];
