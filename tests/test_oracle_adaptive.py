@@ -197,8 +197,8 @@ def test_no_hot_prefix_is_fixed_length_routing():
 
 def test_identical_prefixes_share_length_and_candidates():
     """Requests with the same first K blocks walk the same nodes, so they get
-    the same length and the same candidate pair (the spec invariant
-    still holds with adaptive lengths)."""
+    the same length and the same candidate pair: identical prefixes still map
+    to one candidate pair with adaptive lengths."""
     r = Run(mk())
     for _ in range(3):
         K, out = r.batch(mixed(6, 4))
