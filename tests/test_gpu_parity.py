@@ -289,6 +289,21 @@ def test_rebalance_variants_tiny(flags):
     assert p.n_migrations > 0
 
 
+# -- features combined ------------------------------------------------------------------
+
+@pytest.mark.parametrize("rule,flags", [(7, 3), (3, 1)])
+def test_rule_adaptive_and_rebalance_together(rule, flags):
+    """A compared rule, the adaptive hash length and a rebalancing variant in
+    one run: they share the route, choice and rebalance kernels' state."""
+    w = workload("scaling", n_requests=3000, batch=50, n_instances=16, vnodes=32, n_prefix=100, zipf_s=1.2,
+                 len_lo=400, len_hi=512, prefix_lo=384, prefix_hi=384, scale_every=0, rho=1.0, slo_us=5000)
+    tr = Trace(w)
+    p = Pair(w, max_instances=16, choice_rule=rule, rebalance_flags=flags, adapt=_ad(4, 32))
+    run_trace(p, tr, rebalance=True, state_every=10)
+    from paper_2602_06502_gb300 import dualmap as D
+    assert len(D.dm_export_prefix_tree(p.gpu.h)) > 0
+
+
 # -- edge cases ---------------------------------------------------------------------
 
 def _mk(**kw):

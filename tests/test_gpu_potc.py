@@ -19,7 +19,8 @@ def _built():
 
 @pytest.mark.parametrize("n,m,d,trials", [(8, 8000, 1, 64), (8, 8000, 2, 100), (16, 16000, 2, 64),
                                           (24, 24000, 3, 33), (32, 32000, 4, 64), (1, 500, 2, 5),
-                                          (256, 4000, 2, 70), (7, 3000, 64, 9), (32, 10, 2, 300)])
+                                          (256, 4000, 2, 70), (7, 3000, 64, 9), (32, 10, 2, 300),
+                                          (4, 0, 2, 8)])
 def test_potc_matches_oracle(n, m, d, trials):
     import torch
     from paper_2602_06502_gb300 import dualmap as D
