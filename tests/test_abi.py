@@ -74,6 +74,29 @@ def test_create_rejects_bad_config_without_touching_gpu(built):
     assert D.lib().dm_route_batch(None, None, None) == D.DM_ERR_INVALID_ARG
 
 
+def test_potc_rejects_bad_arguments_without_touching_gpu(built):
+    """dm_potc_max_loads checks its arguments before any CUDA call, and zero
+    trials is a no-op."""
+    D = built
+    buf = C.c_void_p(16)   # never dereferenced: every call below returns before launching
+    assert D.lib().dm_potc_max_loads(0, 10, 2, 4, 1, buf, None) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_potc_max_loads(257, 10, 2, 4, 1, buf, None) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_potc_max_loads(8, 10, 0, 4, 1, buf, None) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_potc_max_loads(8, 10, 65, 4, 1, buf, None) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_potc_max_loads(8, 1 << 32, 2, 4, 1, buf, None) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_potc_max_loads(8, 10, 2, 4, 1, None, None) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_potc_max_loads(8, 10, 2, 0, 1, buf, None) == D.DM_OK
+
+
+def test_read_back_calls_reject_a_null_handle_without_touching_gpu(built):
+    D = built
+    m = D.dm_metrics()
+    n = C.c_uint64()
+    assert D.lib().dm_get_metrics(None, C.byref(m), None, 0, 0) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_export_prefix_tree(None, None, 0, C.byref(n)) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_get_route_blocks(None, None, 0) == D.DM_ERR_INVALID_ARG
+
+
 def test_struct_layouts_match_header(built, tmp_path):
     D = built
     prog = tmp_path / "layout.c"
