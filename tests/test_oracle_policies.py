@@ -290,3 +290,55 @@ def test_rule_ordering_of_sec_2_2():
         assert hit[GLL] < hit[r] < hit[GAFF]
         assert cv[GLL] < cv[r] < cv[GAFF]
     assert hit[DM] >= 0.97 * hit[GAFF] and cv[DM] < cv[GAFF]
+
+
+def test_completion_metrics_match_an_independent_queue_model():
+    """Re-run the time model in plain Python from the oracle's routing
+    decisions: one FIFO per instance, served at 1 us per us from each batch
+    time; a request completes when the work ahead of it and its own is done.
+    Its TTFT count, sum, max, SLO count, histogram and the estimated-SLO
+    count must equal the oracle's metrics."""
+    w = workload("tiny", n_requests=1500, batch=100, zipf_s=1.2, rho=1.1, slo_us=6000)
+    tr = Trace(w)
+    o = O.Oracle(**O.config_from_workload(w, max_instances=w["n_instances"]))
+    for i in range(w["n_instances"]):
+        assert o.add_instance(i) == 0
+    cost, slo = w["cost_us"], w["slo_us"]
+    queues = {i: [] for i in range(w["n_instances"])}   # [remaining, arrival]
+    ttfts, est = [], 0
+    t_prev = None
+    for b in range(len(tr.batches)):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        t = tr.batch_time(b)
+        if t_prev is not None:                       # drain the window [t_prev, t)
+            for q in queues.values():
+                left, run = t - t_prev, 0
+                while q and q[0][0] <= left - run:
+                    rem, arr = q.pop(0)
+                    run += rem
+                    ttfts.append(t_prev + run - arr)
+                if q:
+                    q[0][0] -= left - run
+        t_prev = t
+        rc, out = o.route_batch(tr.batch_tokens(b), off, lens, t)
+        assert rc == 0
+        assert o.commit() == 0
+        for r in range(len(lens)):
+            ch = int(out["chosen"][r])
+            h = int(out["hit1"][r] if ch == out["cand1"][r] else out["hit2"][r])
+            queues[ch].append([cost * (int(lens[r]) - h), t])
+            est += sum(x[0] for x in queues[ch]) <= slo
+    m, hist = o.metrics()
+    assert m["completed"] == len(ttfts) > 0
+    assert m["ttft_sum_us"] == sum(ttfts) and m["ttft_max_us"] == max(ttfts)
+    assert m["slo_met"] == sum(x <= slo for x in ttfts)
+    assert m["est_slo_met"] == est
+    want = np.zeros(O.HIST_BUCKETS, np.uint64)
+    for x in ttfts:
+        want[O.hist_bucket(x)] += 1
+    assert np.array_equal(hist, want)
+    srt = sorted(ttfts)
+    for key, p in (("ttft_p50_us", 50), ("ttft_p90_us", 90), ("ttft_p99_us", 99)):
+        exact = srt[max(1, -(-p * len(srt) // 100)) - 1]   # the ceil(p n)-th smallest
+        assert m[key] == O.hist_lower(O.hist_bucket(exact))
+        assert m[key] <= exact and (exact - m[key]) * 16 <= max(m[key], 16)
