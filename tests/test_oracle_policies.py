@@ -342,3 +342,118 @@ def test_completion_metrics_match_an_independent_queue_model():
         exact = srt[max(1, -(-p * len(srt) // 100)) - 1]   # the ceil(p n)-th smallest
         assert m[key] == O.hist_lower(O.hist_bucket(exact))
         assert m[key] <= exact and (exact - m[key]) * 16 <= max(m[key], 16)
+
+
+@pytest.mark.parametrize("rule", [GLL, GMT, GPRE])
+def test_cluster_wide_rules_match_an_independent_model(rule):
+    """Each request's choice under a cluster-wide rule, recomputed in plain
+    Python: hits from the resident key sets as of the batch start (leading
+    run of the prompt's block keys), loads from an independent FIFO model,
+    then the rule's argmin in arrival order."""
+    w = workload("tiny", n_requests=600, batch=100, zipf_s=1.2, rho=1.0)
+    tr = Trace(w)
+    n_inst, B, cost = w["n_instances"], w["block_tokens"], w["cost_us"]
+    o = O.Oracle(**O.config_from_workload(w, max_instances=n_inst), choice_rule=rule)
+    for i in range(n_inst):
+        assert o.add_instance(i) == 0
+    queues = {i: [] for i in range(n_inst)}
+    t_prev = None
+    for b in range(len(tr.batches)):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        t = tr.batch_time(b)
+        if t_prev is not None:
+            for q in queues.values():
+                left = t - t_prev
+                while q and q[0] <= left:
+                    left -= q.pop(0)
+                if q:
+                    q[0] -= left
+        t_prev = t
+        resident = {i: set(o.cache(i)[0].tolist()) for i in range(n_inst)}
+        W = {i: sum(queues[i]) for i in range(n_inst)}
+        tok = tr.batch_tokens(b)
+        rc, out = o.route_batch(tok, off, lens, t)
+        assert rc == 0
+        for r in range(len(lens)):
+            L = int(lens[r])
+            keys = o.prompt_keys(tok[int(off[r]):int(off[r]) + L])[0].tolist()
+            hits = {}
+            for i in range(n_inst):
+                m = 0
+                while m < len(keys) and keys[m] in resident[i]:
+                    m += 1
+                hits[i] = B * m
+            hmax = max(hits.values())
+            if rule == GLL:
+                key = {i: (W[i], i) for i in range(n_inst)}
+            elif rule == GPRE and 2 * hmax > L:
+                key = {i: (W[i], i) for i in range(n_inst) if hits[i] == hmax}
+            else:
+                key = {i: (W[i] + cost * (L - hits[i]), i) for i in range(n_inst)}
+            ch = min(key, key=lambda i: key[i])
+            assert int(out["chosen"][r]) == ch, (b, r)
+            work = cost * (L - hits[ch])
+            queues[ch].append(work)
+            W[ch] += work
+        assert o.commit() == 0
+
+
+def _pair_choice(rule, c1, c2, h1, h2, L, W1, W2, slo, cost):
+    """The two-candidate rules written out again in Python."""
+    t1, t2 = W1 + cost * (L - h1), W2 + cost * (L - h2)
+    if rule == DM:
+        if h1 == h2:
+            return c2 if W2 < W1 else c1
+        a, b, Wa, Wb, ta = (c1, c2, W1, W2, t1) if h1 > h2 else (c2, c1, W2, W1, t2)
+        if ta <= slo:
+            return a
+        return b if Wb < Wa else a
+    if rule == AFF or (rule == PRE and 2 * max(h1, h2) > L):
+        if h1 != h2:
+            return c1 if h1 > h2 else c2
+        return c2 if W2 < W1 else c1
+    if rule == LL:
+        return c2 if W2 < W1 else c1
+    return c2 if t2 < t1 else c1                       # min TTFT, and Preble below half
+
+
+@pytest.mark.parametrize("rule", [DM, AFF, LL, MT, PRE])
+def test_pair_rules_match_an_independent_model_on_a_trace(rule):
+    """DualMap's rule and the pair variants on a trace under load (the SLO
+    switch fires): loads from an independent FIFO model, the reported
+    candidates and hits, each choice recomputed in arrival order."""
+    w = workload("tiny", n_requests=1000, batch=100, zipf_s=1.2, rho=1.2, slo_us=3000)
+    tr = Trace(w)
+    n_inst, cost, slo = w["n_instances"], w["cost_us"], w["slo_us"]
+    o = O.Oracle(**O.config_from_workload(w, max_instances=n_inst), choice_rule=rule)
+    for i in range(n_inst):
+        assert o.add_instance(i) == 0
+    queues = {i: [] for i in range(n_inst)}
+    t_prev, switched = None, 0
+    for b in range(len(tr.batches)):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        t = tr.batch_time(b)
+        if t_prev is not None:
+            for q in queues.values():
+                left = t - t_prev
+                while q and q[0] <= left:
+                    left -= q.pop(0)
+                if q:
+                    q[0] -= left
+        t_prev = t
+        W = {i: sum(queues[i]) for i in range(n_inst)}
+        rc, out = o.route_batch(tr.batch_tokens(b), off, lens, t)
+        assert rc == 0
+        for r in range(len(lens)):
+            c1, c2 = int(out["cand1"][r]), int(out["cand2"][r])
+            h1, h2, L = int(out["hit1"][r]), int(out["hit2"][r]), int(lens[r])
+            ch = _pair_choice(rule, c1, c2, h1, h2, L, W[c1], W[c2], slo, cost)
+            assert int(out["chosen"][r]) == ch, (b, r)
+            assert int(out["ttft1"][r]) == W[c1] + cost * (L - h1)
+            work = cost * (L - (h1 if ch == c1 else h2))
+            queues[ch].append(work)
+            W[ch] += work
+        switched += int(out["switched"].sum())
+        assert o.commit() == 0
+    if rule == DM:
+        assert switched > 0
