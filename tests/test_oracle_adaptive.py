@@ -213,3 +213,49 @@ def test_bad_adaptive_config_rejected():
         mk(kmax=4096)                            # above 2048
     with pytest.raises(ValueError):
         mk(window=0)
+
+
+@pytest.mark.parametrize("window", [1, 3])
+def test_matches_an_independent_tree_model_on_a_trace(window):
+    """The hotness tree re-implemented in plain Python (walk, per-window node
+    counts, expand above 2T/n, drop below T/n) on a Zipf-skewed trace: every
+    request's length and the expanded set after every batch agree."""
+    from tracegen import Trace, workload
+    w = workload("tiny", n_requests=1500, batch=100, zipf_s=1.2)
+    tr = Trace(w)
+    kr, step, kmax, n = w["route_prefix_blocks"], 8, 96, w["n_instances"]
+    o = O.Oracle(**O.config_from_workload(w, max_instances=n), adapt_step_blocks=step, adapt_max_blocks=kmax,
+                 adapt_window=window)
+    for i in range(n):
+        assert o.add_instance(i) == 0
+    expanded, counts, T, nb = set(), {}, 0, 0
+    deepest = 0
+    for b in range(len(tr.batches)):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        tok = tr.batch_tokens(b)
+        want = []
+        for r in range(len(lens)):
+            keys = o.prompt_keys(tok[int(off[r]):int(off[r]) + int(lens[r])])[0].tolist()
+            nblk = len(keys)
+            d = min(kr, nblk)
+            path = [(keys[d - 1], d)]
+            while d < nblk and d < kmax and keys[d - 1] in expanded:
+                d = min(d + step, nblk, kmax)
+                path.append((keys[d - 1], d))
+            want.append(d)
+            for k, dep in path:
+                c, _ = counts.get(k, (0, dep))
+                counts[k] = (c + 1, dep)
+        rc, out = o.route_batch(tok, off, lens, tr.batch_time(b))
+        assert rc == 0
+        assert o.route_blocks().tolist() == want, b
+        T += len(lens)
+        nb += 1
+        if nb == window:
+            keep = {k for k in expanded if not counts.get(k, (0, 0))[0] * n < T}
+            new = {k for k, (c, dep) in counts.items() if k not in expanded and dep < kmax and c * n > 2 * T}
+            expanded, counts, T, nb = keep | new, {}, 0, 0
+        assert sorted(expanded) == o.prefix_tree().tolist(), b
+        deepest = max(deepest, max(want))
+        assert o.commit() == 0
+    assert deepest > kr                          # the trace does make prefixes hot
