@@ -6,6 +6,7 @@ both candidate instances of a request are identified as overloaded".
 Expected values are worked out by hand."""
 
 import numpy as np
+import pytest
 
 from oracle import oracle as O
 
@@ -99,3 +100,95 @@ def test_double_overload_trigger_gates_the_rule():
     assert results["quiet", 0][0]                       # the untriggered rule moves
     assert results["loud", O.RB_DOUBLE_OVERLOAD] == results["loud", 0]
     assert results["loud", 0][0]
+
+
+def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
+    """Hotspot-aware rebalancing written out again in plain Python."""
+    W = {i: sum(e["rem"] for e in q) for i, q in queues.items()}
+    if flags & O.RB_DOUBLE_OVERLOAD and not both_over:
+        return []
+    N = len(live)
+    sumW = sum(W[i] for i in live)
+
+    def over(i):
+        return W[i] > slo if flags & O.RB_SLO_TARGET else 2 * N * W[i] > 3 * sumW
+
+    hot = sorted((i for i in live if over(i)), key=lambda i: (-W[i], i))
+    moves = []
+    for i in hot:
+        ahead, cands = 0, []
+        for e in queues[i]:
+            ttft_i = ahead + e["rem"]
+            ahead += e["rem"]
+            if e["rem"] != e["work"] or e["moved"] == call:
+                continue
+            j = e["c2"] if e["c1"] == i else e["c1"]
+            hj = e["h1"] if j == e["c1"] else e["h2"]
+            cands.append((-(ttft_i - (W[j] + cost * (e["L"] - hj))), e["seq"], ttft_i))
+        for _, seq, ttft_i in sorted(cands):
+            if not over(i):
+                break
+            e = next(x for x in queues[i] if x["seq"] == seq)
+            j = e["c2"] if e["c1"] == i else e["c1"]
+            if j not in live:
+                continue
+            hj = e["h1"] if j == e["c1"] else e["h2"]
+            nw = cost * (e["L"] - hj)
+            if not (ttft_i > W[j] + nw and W[j] + nw < slo):
+                continue
+            queues[i].remove(e)
+            W[i] -= e["work"]
+            sumW -= e["work"]
+            e.update(work=nw, rem=nw, moved=call)
+            queues[j].append(e)
+            W[j] += nw
+            sumW += nw
+            moves.append((seq, i, j))
+    return moves
+
+
+@pytest.mark.parametrize("flags", [0, O.RB_SLO_TARGET, O.RB_DOUBLE_OVERLOAD, 3])
+def test_variants_match_an_independent_model_on_a_trace(flags):
+    """A skewed 16-instance workload with a 5 ms SLO, rebalancing after
+    every batch: the migrations of every call and the loads after it equal
+    an independent model of the queues and of the rule."""
+    from tracegen import Trace, workload
+    w = workload("scaling", n_requests=3000, batch=50, n_instances=16, vnodes=32, n_prefix=100, zipf_s=1.2,
+                 len_lo=400, len_hi=512, prefix_lo=384, prefix_hi=384, scale_every=0, rho=1.0, slo_us=5000)
+    tr = Trace(w)
+    n, cost, slo = 16, w["cost_us"], w["slo_us"]
+    o = O.Oracle(**O.config_from_workload(w, max_instances=n), rebalance_flags=flags)
+    for i in range(n):
+        assert o.add_instance(i) == 0
+    queues = {i: [] for i in range(n)}
+    live = set(range(n))
+    t_prev, seq, total = None, 0, 0
+    for b in range(len(tr.batches)):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        t = tr.batch_time(b)
+        if t_prev is not None:
+            for q in queues.values():
+                left = t - t_prev
+                while q and q[0]["rem"] <= left:
+                    left -= q.pop(0)["rem"]
+                if q:
+                    q[0]["rem"] -= left
+        t_prev = t
+        rc, out = o.route_batch(tr.batch_tokens(b), off, lens, t)
+        assert rc == 0
+        both = False
+        for r in range(len(lens)):
+            c1, c2, ch = int(out["cand1"][r]), int(out["cand2"][r]), int(out["chosen"][r])
+            h1, h2, L = int(out["hit1"][r]), int(out["hit2"][r]), int(lens[r])
+            wk = cost * (L - (h1 if ch == c1 else h2))
+            queues[ch].append(dict(seq=seq, L=L, c1=c1, c2=c2, h1=h1, h2=h2, work=wk, rem=wk, moved=0))
+            both |= int(out["ttft1"][r]) > slo and int(out["ttft2"][r]) > slo
+            seq += 1
+        want = _model_rebalance(queues, live, flags, both, slo, cost, b + 1)
+        rc, nm, (mseq, mfr, mto) = o.rebalance()
+        assert rc == 0
+        assert list(zip(mseq.tolist(), mfr.tolist(), mto.tolist())) == want, b
+        assert o.loads()[:n].tolist() == [sum(x["rem"] for x in queues[i]) for i in range(n)], b
+        total += len(want)
+        assert o.commit() == 0
+    assert total > 0
