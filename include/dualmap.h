@@ -132,8 +132,8 @@ typedef struct {
      * power of two >= 2 x (C + max_touch_per_instance).  A larger index is
      * rebuilt less often (it is rebuilt when a quarter full if a quarter
      * still holds C + max_touch_per_instance keys, else when half full,
-     * counting the slots evicted keys keep).  Never smaller than the automatic size, nor than
-     * 64; <= 32.  dm_create returns DM_ERR_INVALID_ARG when the resulting
+     * counting the slots evicted keys keep).  Never smaller than the
+     * automatic size, nor than 64; <= 32.  dm_create returns DM_ERR_INVALID_ARG when the resulting
      * index would exceed 2^32 slots (it records slot numbers as 32 bits). */
     uint32_t index_slots_log2;
     /* The choice rule of dm_route_batch (dm_choice_rule); 0 = DualMap's
@@ -161,9 +161,10 @@ typedef struct {
     uint32_t rebalance_flags;
     /* Spare index buffers shared by all instances as rebuild targets (a
      * rebuild builds the new index in a spare and returns the old one to the
-     * pool); 0 = one per instance.  Fewer than max_instances halves the
-     * index memory; rebuilds beyond the pool then wait their turn (round
-     * robin), so dm_create requires index_slots / 2 >= ceil(max_instances /
+     * pool); 0 = one per instance (index memory: two indices per instance).
+     * A pool much smaller than max_instances nearly halves the index memory;
+     * rebuilds beyond the pool then wait their turn (round robin), so
+     * dm_create requires index_slots / 2 >= ceil(max_instances /
      * rebuild_pool) * max_touch_per_instance (DM_ERR_INVALID_ARG otherwise). */
     uint32_t rebuild_pool;
     /* Seed of all hash key material (SplitMix64). */
