@@ -151,7 +151,9 @@ def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
 def test_variants_match_an_independent_model_on_a_trace(flags):
     """A skewed 16-instance workload with a 5 ms SLO, rebalancing after
     every batch: the migrations of every call and the loads after it equal
-    an independent model of the queues and of the rule."""
+    an independent model of the queues and of the rule, and the completion
+    TTFTs (migrated requests keep their arrival) equal the oracle's
+    metrics."""
     from tracegen import Trace, workload
     w = workload("scaling", n_requests=3000, batch=50, n_instances=16, vnodes=32, n_prefix=100, zipf_s=1.2,
                  len_lo=400, len_hi=512, prefix_lo=384, prefix_hi=384, scale_every=0, rho=1.0, slo_us=5000)
@@ -162,17 +164,19 @@ def test_variants_match_an_independent_model_on_a_trace(flags):
         assert o.add_instance(i) == 0
     queues = {i: [] for i in range(n)}
     live = set(range(n))
-    t_prev, seq, total = None, 0, 0
+    t_prev, seq, total, ttfts = None, 0, 0, []
     for b in range(len(tr.batches)):
         s, e, off, lens, nt = tr.batch_layout(b)
         t = tr.batch_time(b)
         if t_prev is not None:
             for q in queues.values():
-                left = t - t_prev
-                while q and q[0]["rem"] <= left:
-                    left -= q.pop(0)["rem"]
+                left, run = t - t_prev, 0
+                while q and q[0]["rem"] <= left - run:
+                    x = q.pop(0)
+                    run += x["rem"]
+                    ttfts.append(t_prev + run - x["arr"])   # a migrated request keeps its arrival
                 if q:
-                    q[0]["rem"] -= left
+                    q[0]["rem"] -= left - run
         t_prev = t
         rc, out = o.route_batch(tr.batch_tokens(b), off, lens, t)
         assert rc == 0
@@ -181,7 +185,7 @@ def test_variants_match_an_independent_model_on_a_trace(flags):
             c1, c2, ch = int(out["cand1"][r]), int(out["cand2"][r]), int(out["chosen"][r])
             h1, h2, L = int(out["hit1"][r]), int(out["hit2"][r]), int(lens[r])
             wk = cost * (L - (h1 if ch == c1 else h2))
-            queues[ch].append(dict(seq=seq, L=L, c1=c1, c2=c2, h1=h1, h2=h2, work=wk, rem=wk, moved=0))
+            queues[ch].append(dict(seq=seq, L=L, c1=c1, c2=c2, h1=h1, h2=h2, work=wk, rem=wk, moved=0, arr=t))
             both |= int(out["ttft1"][r]) > slo and int(out["ttft2"][r]) > slo
             seq += 1
         want = _model_rebalance(queues, live, flags, both, slo, cost, b + 1)
@@ -192,3 +196,6 @@ def test_variants_match_an_independent_model_on_a_trace(flags):
         total += len(want)
         assert o.commit() == 0
     assert total > 0
+    m, _ = o.metrics()
+    assert (m["completed"], m["ttft_sum_us"], m["ttft_max_us"]) == (len(ttfts), sum(ttfts), max(ttfts))
+    assert m["slo_met"] == sum(x <= slo for x in ttfts)
