@@ -138,7 +138,9 @@ typedef struct {
     uint32_t index_slots_log2;
     /* The choice rule of dm_route_batch (dm_choice_rule); 0 = DualMap's
      * SLO-aware rule.  The others are the rules DualMap is compared with,
-     * for experiments; DM_ERR_INVALID_ARG for an unknown value. */
+     * for experiments; DM_ERR_INVALID_ARG for an unknown value.  The
+     * cluster-wide rules allocate max_batch x max_instances u32 hit counts
+     * (DM_ERR_OOM when that does not fit). */
     uint32_t choice_rule;
     /* Adaptive hash-prefix length (Sec. 3.2, "how long prefix is
      * appropriate"); adapt_step_blocks = 0 keeps every request at
@@ -152,7 +154,10 @@ typedef struct {
      * than 2T/n of them (and shorter than adapt_max_blocks) is expanded and
      * an expanded node reached by fewer than T/n is dropped; the new tree
      * applies from the next batch.  K_route < adapt_max_blocks <= 2048,
-     * adapt_window >= 1. */
+     * adapt_window >= 1, and the window's node-count table (2 x max_batch x
+     * adapt_window x levels entries of 16 bytes, levels = ceil((adapt_max_blocks
+     * - K_route) / adapt_step_blocks) + 1) at most 2^26 entries;
+     * DM_ERR_INVALID_ARG otherwise. */
     uint32_t adapt_step_blocks;
     uint32_t adapt_max_blocks;
     uint32_t adapt_window;
