@@ -106,6 +106,12 @@
  *   Scaling (Sec. 3.4; App. A.1.3): add inserts V nodes per ring; remove
  *     deletes them, the instance keeps draining and takes no new work.
  *
+ *   Adaptive hash-prefix length (Sec. 3.2, adapt_step_blocks > 0): see
+ *     adapt_walk and adapt_window_end below (nodes named by the key of a
+ *     prefix's last block; expand above 2T/n, drop below T/n per window).
+ *
+ *   Power of d choices (App. A.8): or_potc_max_loads below.
+ *
  * Data structures are the obvious ones: sorted arrays rebuilt from scratch
  * on every membership change, an LRU as hash map + recency list, queues as
  * plain arrays.
