@@ -457,3 +457,28 @@ def test_pair_rules_match_an_independent_model_on_a_trace(rule):
         assert o.commit() == 0
     if rule == DM:
         assert switched > 0
+
+
+def test_cv_counts_live_instances_only():
+    """A removed instance keeps draining its queue but is not part of the
+    cluster whose balance the CV measures (Sec. 2.2: the instances serving
+    requests): its queued work is left out of the sample."""
+    w = workload("tiny", n_requests=400, batch=100)
+    tr = Trace(w)
+    o = O.Oracle(**O.config_from_workload(w, max_instances=w["n_instances"]))
+    for i in range(w["n_instances"]):
+        assert o.add_instance(i) == 0
+    for b in range(2):
+        s, e, off, lens, nt = tr.batch_layout(b)
+        assert o.route_batch(tr.batch_tokens(b), off, lens, tr.batch_time(b))[0] == 0
+        assert o.commit() == 0
+    gone = int(np.argmax(o.loads()))
+    assert o.loads()[gone] > 0 and o.remove_instance(gone) == 0
+    s, e, off, lens, nt = tr.batch_layout(2)
+    assert o.route_batch(tr.batch_tokens(2), off, lens, tr.batch_time(1))[0] == 0   # no time passes
+    m, _ = o.metrics()
+    W = o.loads().astype(np.float64)
+    live = o.inst_state() == 1
+    assert not live[gone] and W[gone] > 0
+    assert m["cv_last"] == pytest.approx(W[live].std() / W[live].mean(), rel=1e-12)
+    assert m["cv_last"] != pytest.approx(W.std() / W.mean(), rel=1e-6)
