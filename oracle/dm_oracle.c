@@ -110,7 +110,8 @@
  *     adapt_walk and adapt_window_end below (nodes named by the key of a
  *     prefix's last block; expand above 2T/n, drop below T/n per window).
  *
- *   Power of d choices (App. A.8): or_potc_max_loads below.
+ *   Power of d choices (App. A.8): or_potc_max_loads below; routing with d
+ *     candidates instead of two: or_route_batch_d below.
  *
  * Data structures are the obvious ones: sorted arrays rebuilt from scratch
  * on every membership change, an LRU as hash map + recency list, queues as
@@ -190,7 +191,10 @@ typedef struct {
     uint32_t adapt_max_blocks;    /* longest hash prefix, in blocks */
     uint32_t adapt_window;        /* non-empty batches per hotness window */
     uint32_t rebalance_flags;     /* OR_RB_* */
+    uint32_t candidates;          /* rings (hash functions) kept: 0 or 2 = DualMap's two; up to OR_MAX_D */
 } or_config;
+
+#define OR_MAX_D 8
 
 /* Rebalancing variants (the paper's own wording of Sec. 3.3 / App. A.1.2):
  * OR_RB_SLO_TARGET: an instance is overloaded when its queued work exceeds
@@ -249,11 +253,16 @@ typedef struct {
     or_config cfg;
     uint32_t K1[64], K2[64];
     uint64_t G1, G2, Sc, Sr1, Sr2, Sv1, Sv2;
+    /* functions f = 3..d of the d-candidate path: NH keys, salt, ring-position
+     * and vnode seeds (index f - 3) */
+    uint32_t Kx[OR_MAX_D - 2][64];
+    uint64_t Gx[OR_MAX_D - 2], Srx[OR_MAX_D - 2], Svx[OR_MAX_D - 2];
+    uint32_t nrings;    /* rings kept: max(2, candidates) */
     uint8_t *state;     /* per id: absent / live / draining */
     uint64_t *W;        /* queued work per id */
     queue_t *q;
     lru_t *cache;
-    vnode *ring[2];
+    vnode *ring[OR_MAX_D];
     uint32_t ring_len;
     uint64_t clock, next_seq, t_prev;
     int have_time;
@@ -497,11 +506,11 @@ static int rebuild_rings(or_state *s)
     for (uint32_t id = 0; id < s->cfg.max_instances; id++)
         if (s->state[id] == INST_LIVE) n++;
     uint32_t R = n * s->cfg.vnodes_per_instance;
-    for (int f = 0; f < 2; f++) {
+    for (uint32_t f = 0; f < s->nrings; f++) {
         free(s->ring[f]);
         s->ring[f] = (vnode *)malloc((size_t)(R ? R : 1) * sizeof(vnode));
         if (!s->ring[f]) return OR_ERR_OOM;
-        uint64_t Sv = f == 0 ? s->Sv1 : s->Sv2;
+        uint64_t Sv = f == 0 ? s->Sv1 : f == 1 ? s->Sv2 : s->Svx[f - 2];
         uint32_t k = 0;
         for (uint32_t id = 0; id < s->cfg.max_instances; id++) {
             if (s->state[id] != INST_LIVE) continue;
@@ -648,8 +657,7 @@ void or_destroy(or_state *s)
     free(s->q);
     free(s->W);
     free(s->state);
-    free(s->ring[0]);
-    free(s->ring[1]);
+    for (uint32_t f = 0; f < OR_MAX_D; f++) free(s->ring[f]);
     free(s->ad_set);
     free(s->ad_rec_key);
     free(s->ad_rec_depth);
@@ -670,6 +678,7 @@ int or_create(const or_config *cfg, or_state **out)
         (cfg->adapt_max_blocks <= cfg->route_prefix_blocks || cfg->adapt_max_blocks > 2048 ||
          cfg->adapt_window < 1))
         return OR_ERR_INVALID_ARG;
+    if (cfg->candidates > OR_MAX_D) return OR_ERR_INVALID_ARG;
     or_state *s = (or_state *)calloc(1, sizeof(or_state));
     if (!s) return OR_ERR_OOM;
     s->cfg = *cfg;
@@ -677,6 +686,19 @@ int or_create(const or_config *cfg, or_state **out)
     or_derive_keys(cfg->seed, B, s->K1, s->K2, sc);
     s->G1 = sc[0]; s->G2 = sc[1]; s->Sc = sc[2]; s->Sr1 = sc[3]; s->Sr2 = sc[4];
     s->Sv1 = sc[5]; s->Sv2 = sc[6];
+    /* functions 3..d continue the same SplitMix64 stream after DualMap's
+     * nine draws, so two functions keep exactly DualMap's key material */
+    {
+        uint64_t st = cfg->seed;
+        for (uint32_t j = 0; j < 2 * B + 7; j++) or_splitmix64_next(&st);
+        for (uint32_t f = 0; f + 2 < OR_MAX_D; f++) {
+            for (uint32_t j = 0; j < B; j++) s->Kx[f][j] = (uint32_t)or_splitmix64_next(&st);
+            s->Gx[f] = or_splitmix64_next(&st) | 1ULL;
+            s->Srx[f] = or_splitmix64_next(&st);
+            s->Svx[f] = or_splitmix64_next(&st);
+        }
+    }
+    s->nrings = cfg->candidates > 2 ? cfg->candidates : 2;
     uint32_t M = cfg->max_instances;
     s->state = (uint8_t *)calloc(M, 1);
     s->W = (uint64_t *)calloc(M, sizeof(uint64_t));
@@ -1048,6 +1070,147 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
     return OR_OK;
 }
 
+/* ------------------------------------------------------------------ */
+/* d candidates (App. A.8, "Optimal Candidate Set Size")                */
+/* ------------------------------------------------------------------ */
+
+/* The generalisation of the routing step that App. A.8 weighs: d
+ * independent hash functions of the prompt prefix, d rings, d candidates,
+ * d probes, one choice.  Function f's ring position is
+ * fmix64(P^f_{K-1} xor S_rf) with P^f the chained sum of its block digests,
+ * as for f = 1, 2; functions 3..d draw their key material after DualMap's.
+ * Distinct candidates: c_1 = the owner on ring 1; c_f (f >= 2) = the owner on
+ * ring f unless an earlier candidate has it, then the next live id after
+ * that owner, in ascending order, cyclically, that is not yet a candidate
+ * (for d = 2 this is DualMap's rule).  Choice, DualMap's rule over d
+ * candidates (a reading: the paper states it for two): among the
+ * candidates with the most hit tokens, a is the less loaded by W (tie: the
+ * earlier f); a is chosen if every candidate has that many hits or
+ * ttft_a <= SLO; otherwise the least loaded candidate by W (tie: a, then the
+ * earlier f), and the request is flagged "switched" (as DualMap flags it,
+ * even when that candidate is a itself).  d = 2 is DualMap's rule;
+ * d = 1 always takes the ring-1 owner, i.e. cache affinity.  Loads, queues,
+ * metrics and the commit are those of or_route_batch (queue entries keep
+ * the first two candidates; rebalancing is defined for d = 2 only).
+ * cand, hit, ttft hold n*d entries (request-major). */
+static uint64_t ring_pos_f(const or_state *s, const uint32_t *tok, uint32_t K, uint32_t f)
+{
+    const uint32_t B = s->cfg.block_tokens;
+    const uint32_t *Kf = f == 0 ? s->K1 : f == 1 ? s->K2 : s->Kx[f - 2];
+    const uint64_t G = f == 0 ? s->G1 : f == 1 ? s->G2 : s->Gx[f - 2];
+    const uint64_t Sr = f == 0 ? s->Sr1 : f == 1 ? s->Sr2 : s->Srx[f - 2];
+    uint64_t P = 0;
+    for (uint32_t k = 0; k < K; k++) P += or_fmix64(or_nh(tok + (uint64_t)k * B, Kf, B) + (uint64_t)(k + 1) * G);
+    return or_fmix64(P ^ Sr);
+}
+
+int or_route_batch_d(or_state *s, uint32_t d, const uint32_t *tokens, const uint64_t *offsets,
+                     const uint32_t *lengths, uint32_t n, uint64_t t_batch, uint32_t *cand, uint32_t *hit,
+                     uint64_t *ttft, uint32_t *chosen, uint8_t *switched)
+{
+    const or_config *cf = &s->cfg;
+    if (d < 1 || d > s->nrings || cf->adapt_step_blocks || cf->choice_rule != OR_RULE_DUALMAP)
+        return OR_ERR_INVALID_ARG;
+    if (n > cf->max_batch) return OR_ERR_CAPACITY;
+    if (n_live(s) < 2 || n_live(s) < d) return OR_ERR_NO_INSTANCES;
+    if (s->have_time && t_batch < s->t_prev) return OR_ERR_ORDER;
+    uint64_t total = 0;
+    for (uint32_t r = 0; r < n; r++) {
+        if (lengths[r] < cf->block_tokens) return OR_ERR_INVALID_ARG;
+        total += lengths[r];
+    }
+    if (total > cf->max_batch_tokens) return OR_ERR_CAPACITY;
+    uint64_t delta = s->have_time ? t_batch - s->t_prev : 0;
+    for (uint32_t id = 0; id < cf->max_instances; id++)
+        if (s->state[id] != INST_ABSENT) q_drain(s, id, delta, s->t_prev);
+    s->t_prev = t_batch;
+    s->have_time = 1;
+    clear_pending(s);
+    s->pend_n = n;
+    s->pend_seq0 = s->next_seq;
+    s->pend_final = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
+    s->pend_nblk = (uint32_t *)malloc((n ? n : 1) * sizeof(uint32_t));
+    s->pend_keys = (uint64_t **)calloc(n ? n : 1, sizeof(uint64_t *));
+    uint32_t *lk = (uint32_t *)realloc(s->last_K, (n ? n : 1) * sizeof(uint32_t));
+    if (!lk) return OR_ERR_OOM;
+    s->last_K = lk;
+    s->last_n = n;
+    if (!s->pend_final || !s->pend_nblk || !s->pend_keys) return OR_ERR_OOM;
+    /* 1) hash, d ring lookups, distinct fix, d probes (batch-start state) */
+    for (uint32_t r = 0; r < n; r++) {
+        const uint32_t L = lengths[r];
+        const uint32_t *tok = tokens + offsets[r];
+        uint64_t *keys = (uint64_t *)malloc((size_t)(L / cf->block_tokens) * sizeof(uint64_t));
+        if (!keys) return OR_ERR_OOM;
+        uint64_t pos2[2];
+        const uint32_t nblk = prompt_keys(s, tok, L, keys, pos2);
+        const uint32_t K = cf->route_prefix_blocks < nblk ? cf->route_prefix_blocks : nblk;
+        s->last_K[r] = K;
+        s->pend_keys[r] = keys;
+        s->pend_nblk[r] = nblk;
+        uint32_t *c = cand + (size_t)r * d;
+        for (uint32_t f = 0; f < d; f++) {
+            uint32_t x = ring_owner(s, (int)f, ring_pos_f(s, tok, K, f));
+            for (;;) {   /* taken by an earlier candidate: the next live id after it */
+                uint32_t taken = 0;
+                for (uint32_t g = 0; g < f; g++) taken |= c[g] == x;
+                if (!taken) break;
+                x = next_live_after(s, x);
+            }
+            c[f] = x;
+            hit[(size_t)r * d + f] = cf->block_tokens * leading_hits(&s->cache[x], keys, nblk);
+        }
+    }
+    /* 2) choices in arrival order */
+    s->both_over = 0;
+    for (uint32_t r = 0; r < n; r++) {
+        const uint32_t *c = cand + (size_t)r * d, *h = hit + (size_t)r * d;
+        const uint32_t L = lengths[r];
+        uint32_t hmax = 0, nmax = 0;
+        for (uint32_t f = 0; f < d; f++) hmax = h[f] > hmax ? h[f] : hmax;
+        uint32_t a = d;
+        int all_over = 1;
+        for (uint32_t f = 0; f < d; f++) {
+            ttft[(size_t)r * d + f] = s->W[c[f]] + (uint64_t)cf->cost_us_per_token * (L - h[f]);
+            all_over &= ttft[(size_t)r * d + f] > cf->slo_us;
+            if (h[f] == hmax) {
+                nmax++;
+                if (a == d || s->W[c[f]] < s->W[c[a]]) a = f;
+            }
+        }
+        uint32_t pick = a;
+        const int over = nmax < d && ttft[(size_t)r * d + a] > cf->slo_us;
+        if (over)
+            for (uint32_t f = 0; f < d; f++)
+                if (s->W[c[f]] < s->W[c[pick]]) pick = f;
+        switched[r] = (uint8_t)over;
+        const uint32_t ch = c[pick], hch = h[pick];
+        chosen[r] = ch;
+        if (all_over) s->both_over = 1;
+        q_entry e;
+        e.seq = s->next_seq++;
+        e.L = L; e.c1 = c[0]; e.c2 = d > 1 ? c[1] : c[0]; e.h1 = h[0]; e.h2 = d > 1 ? h[1] : h[0];
+        e.work = e.remaining = (uint64_t)cf->cost_us_per_token * (L - hch);
+        e.moved_in_call = 0;
+        e.arrival = t_batch;
+        if (q_push(&s->q[ch], &e)) return OR_ERR_OOM;
+        s->W[ch] += e.work;
+        s->pend_final[r] = ch;
+        s->m_requests++;
+        s->m_prompt_tokens += L;
+        s->m_hit_tokens += hch;
+        s->m_switched += switched[r];
+        s->m_est_slo_met += s->W[ch] <= cf->slo_us;
+    }
+    if (n > 0) {
+        s->m_cv_last = load_cv(s);
+        s->m_cv_sum += s->m_cv_last;
+        s->m_batches++;
+    }
+    s->pending = 1;
+    return OR_OK;
+}
+
 int or_commit(or_state *s)
 {
     if (!s->pending) return OR_OK;
@@ -1202,11 +1365,34 @@ uint32_t or_prompt_keys(const or_state *s, const uint32_t *tok, uint32_t L, uint
 /* Raw ring owners of positions (before the distinct fix). */
 void or_ring_owners(const or_state *s, const uint64_t *pos, uint32_t n, int f, uint32_t *owner)
 {
+    if (f < 0 || (uint32_t)f >= s->nrings) return;
     for (uint32_t i = 0; i < n; i++) owner[i] = ring_owner(s, f, pos[i]);
+}
+
+/* Key material of function f (0-based): its NH keys (B words), and
+ * scalars = {G, S_r, S_v}. */
+void or_key_material_f(const or_state *s, uint32_t f, uint32_t *K, uint64_t *scalars)
+{
+    if (f >= s->nrings) return;
+    const uint32_t *Kf = f == 0 ? s->K1 : f == 1 ? s->K2 : s->Kx[f - 2];
+    memcpy(K, Kf, s->cfg.block_tokens * sizeof(uint32_t));
+    scalars[0] = f == 0 ? s->G1 : f == 1 ? s->G2 : s->Gx[f - 2];
+    scalars[1] = f == 0 ? s->Sr1 : f == 1 ? s->Sr2 : s->Srx[f - 2];
+    scalars[2] = f == 0 ? s->Sv1 : f == 1 ? s->Sv2 : s->Svx[f - 2];
+}
+
+/* Ring position of a prompt under function f (0-based), hashed over its
+ * first min(K_route, n_blk) blocks. */
+uint64_t or_ring_position(const or_state *s, const uint32_t *tok, uint32_t L, uint32_t f)
+{
+    const uint32_t nblk = L / s->cfg.block_tokens;
+    const uint32_t K = s->cfg.route_prefix_blocks < nblk ? s->cfg.route_prefix_blocks : nblk;
+    return f < s->nrings ? ring_pos_f(s, tok, K, f) : 0;
 }
 
 uint32_t or_ring_dump(const or_state *s, int f, uint64_t *vpos, uint32_t *owner, uint32_t *vidx)
 {
+    if (f < 0 || (uint32_t)f >= s->nrings) return 0;
     for (uint32_t k = 0; k < s->ring_len; k++) {
         if (vpos) vpos[k] = s->ring[f][k].pos;
         if (owner) owner[k] = s->ring[f][k].id;

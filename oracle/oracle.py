@@ -48,6 +48,7 @@ class or_config(C.Structure):
         ("adapt_max_blocks", C.c_uint32),
         ("adapt_window", C.c_uint32),
         ("rebalance_flags", C.c_uint32),
+        ("candidates", C.c_uint32),
     ]
 
 
@@ -113,6 +114,10 @@ def lib():
             "or_potc_place_all": (None, [u32p, C.c_uint64, C.c_uint32, C.c_uint32, u32p]),
             "or_potc_max_loads": (C.c_int, [C.c_uint32, C.c_uint64, C.c_uint32, C.c_uint32, C.c_uint64, u32p]),
             "or_prefix_tree": (C.c_uint64, [V, V, C.c_uint64]),
+            "or_route_batch_d": (C.c_int, [V, C.c_uint32, u32p, u64p, u32p, C.c_uint32, C.c_uint64,
+                                           u32p, u32p, u64p, u32p, u8p]),
+            "or_ring_position": (C.c_uint64, [V, u32p, C.c_uint32, C.c_uint32]),
+            "or_key_material_f": (None, [V, C.c_uint32, u32p, u64p]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -243,6 +248,33 @@ class Oracle:
                                   out["cand1"], out["cand2"], out["hit1"], out["hit2"],
                                   out["ttft1"], out["ttft2"], out["chosen"], out["switched"])
         return rc, out
+
+    def route_batch_d(self, d, tokens, offsets, lengths, t_batch):
+        """Routing with d candidates (App. A.8): (status, dict of cand, hit,
+        ttft as n x d arrays, chosen and switched)."""
+        n = len(lengths)
+        cand = np.zeros(n * d, np.uint32)
+        hit = np.zeros(n * d, np.uint32)
+        ttft = np.zeros(n * d, np.uint64)
+        chosen = np.zeros(n, np.uint32)
+        sw = np.zeros(n, np.uint8)
+        tok = np.ascontiguousarray(tokens, dtype=np.uint32)
+        rc = lib().or_route_batch_d(self.h, d, tok if tok.size else np.zeros(1, np.uint32),
+                                    np.ascontiguousarray(offsets, dtype=np.uint64),
+                                    np.ascontiguousarray(lengths, dtype=np.uint32), n, t_batch, cand, hit, ttft,
+                                    chosen, sw)
+        return rc, dict(cand=cand.reshape(n, d), hit=hit.reshape(n, d), ttft=ttft.reshape(n, d), chosen=chosen,
+                        switched=sw)
+
+    def ring_position(self, tokens, f):
+        t = np.ascontiguousarray(tokens, dtype=np.uint32)
+        return lib().or_ring_position(self.h, t, len(t), f)
+
+    def key_material_f(self, f):
+        K = np.zeros(self.B, np.uint32)
+        sc = np.zeros(3, np.uint64)
+        lib().or_key_material_f(self.h, f, K, sc)
+        return K, sc
 
     def commit(self):
         return lib().or_commit(self.h)
