@@ -7,8 +7,9 @@ long-context stress shape (128 instances, 512 prompts of 32,768-131,072
 uint32 tokens per batch, 64 shared 16k-token prefixes, Zipf 0.8), inputs
 resident in HBM (each batch ~168 MB, larger than L2).
 
-Prints one JSON line: routed requests/s (value), prompt GB/s hashed+probed,
-the hashing kernel's HBM roofline, the end-to-end number through the
+Prints one JSON line: routed requests/s (value), prompt GB/s hashed+probed
+(hashing, ring lookup and probes are one kernel, event-timed in the timed
+region) with its HBM roofline, the end-to-end number through the
 host-buffer entry point, the CPU oracle baseline and the SM clocks seen.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl dualmap|reference]
@@ -162,11 +163,13 @@ def dist_setup():
     return world, rank, local
 
 
-def cpu_oracle_run(tr, w, warm, timed, get_tokens, max_id):
+def cpu_oracle_run(tr, w, warm, timed, get_tokens, max_id, keep=None, extra=None):
     """Time the CPU oracle (as it stands, one thread) over the `timed` batches,
-    after routing the `warm` batches untimed on the same state."""
+    after routing the `warm` batches untimed on the same state.  keep: a dict
+    that receives each batch's routing outputs (for the comparison with the
+    GPU's)."""
     from oracle import oracle as O
-    ora = O.Oracle(**O.config_from_workload(w, max_instances=max_id + 9, max_batch_tokens=1 << 40))
+    ora = O.Oracle(**O.config_from_workload(w, max_instances=max_id + 9, max_batch_tokens=1 << 40, **(extra or {})))
     for i in range(w["n_instances"]):
         ora.add_instance(i)
     events = {}
@@ -180,8 +183,10 @@ def cpu_oracle_run(tr, w, warm, timed, get_tokens, max_id):
         t0 = time.perf_counter()
         for kind, i in events.get(b, []):
             (ora.add_instance if kind == "add" else ora.remove_instance)(i)
-        rc, _ = ora.route_batch(tok, off, lens, tr.batch_time(b))
+        rc, out = ora.route_batch(tok, off, lens, tr.batch_time(b))
         assert rc == 0
+        if keep is not None:
+            keep[b] = out
         if w.get("rebalance"):
             ora.rebalance()
         ora.commit()
@@ -346,8 +351,25 @@ def main():
         te = time.perf_counter() - t0
         g.close()
         te = max_over_ranks(te * 1e3, device=dev) / 1e3
-        e2e = {"value": job_throughput(ne, te * 1e3, world), "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
-               "d2h_bytes_per_step": d2h // Ke, "steps": Ke}
+        # pinned host-to-device copy bandwidth of this process, measured on
+        # the same buffers right after: the bound the upload puts on e2e
+        probe_b = need[0]
+        src = host["tok"][probe_b]
+        dst = torch.empty_like(src, device=dev)
+        best = 0.0
+        for _ in range(5):
+            c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            c0.record()
+            dst.copy_(src, non_blocking=True)
+            c1.record()
+            torch.cuda.synchronize()
+            best = max(best, src.numel() * 4 / (c0.elapsed_time(c1) / 1e3) / 1e9)
+        del dst
+        e2e_val = job_throughput(ne, te * 1e3, world)
+        bound = best * 1e9 / (h2d / Ke) * (ne / Ke) * world
+        e2e = {"value": e2e_val, "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
+               "d2h_bytes_per_step": d2h // Ke, "steps": Ke, "h2d_pinned_GBps": best,
+               "h2d_bound_req_s": bound, "frac_of_h2d_bound": e2e_val / bound}
 
     # -- device-resident run -------------------------------------------------
     g = make_sched()
@@ -356,7 +378,7 @@ def main():
     torch.cuda.synchronize()
     assert g.last_error() == 0
     D.dm_get_stage_times(g.h, reset=True)
-    D.dm_set_profiling(g.h, True, stages=["hash"])   # the roofline kernel only: events elsewhere cost time
+    D.dm_set_profiling(g.h, True, stages=["hash"])   # the hash+probe kernel only: events elsewhere cost time
     sampler = ClockSampler(local)
     time.sleep(0.3)
     if world > 1:
@@ -388,7 +410,10 @@ def main():
     hash_avg_s = hash_ms / 1e3 / max(hash_calls, 1)
     bytes_per_launch = prompt_bytes / max(hash_calls, 1)
     peak, peak_kind = peaks()
+    # hashing, ring lookup and probes run in one kernel: its event-timed
+    # duration is the whole hash+probe path of the metric
     achieved = bytes_per_launch / hash_avg_s / 1e9
+    prompt_gbps = achieved
 
     # per-stage breakdown: a fresh handle replays the same steps with every
     # stage timed (events between kernels stop their launch overlap, so this
@@ -396,23 +421,29 @@ def main():
     g.close()
     del g
     g = make_sched()
+    cmp_batches = 0 if (args.no_cpu or rank != 0 or world != 1) else min(args.cpu_batches, used)
+    gpu_out = {}   # the batches the CPU baseline routes: compared decision by decision below
     for j in range(W):
-        step(g, j)
+        n = step(g, j)
+        if j < cmp_batches:
+            gpu_out[j] = g.results(n)
     D.dm_get_stage_times(g.h, reset=True)
     D.dm_set_profiling(g.h, True)
     for j in range(W, W + K):
-        step(g, j)
+        n = step(g, j)
+        if j < cmp_batches:
+            gpu_out[j] = g.results(n)
     st_all = D.dm_get_stage_times(g.h, reset=True)
     D.dm_set_profiling(g.h, False)
     assert g.last_error() == 0
     met, _ = D.dm_get_metrics(g.h)
     stage_ms = {k: v[0] / max(v[1], 1) for k, v in st_all.items()}
-    prompt_gbps = bytes_per_launch / ((stage_ms["hash"] + stage_ms["probe"]) / 1e3) / 1e9
-    # route: setup (with the queue drain), segmap, hash, probe, choice (5); commit:
-    # maint_plan, maint_a, compact_scan, maint_c, commit_prep, commit_touch,
+    # route: setup (with the queue drain), hash + ring lookup + probes (one
+    # kernel), choice (with the segment carries) (3); commit: maint_plan,
+    # maint_a, compact_scan, maint_c, commit_prep, commit_touch,
     # touch_deferred, req_counts, evict (9); rebalance (1)
-    # (the cluster-wide rules add the all-instance probe kernel)
-    launches_per_step = 5 + 9 + (1 if w.get("rebalance") else 0) + (1 if rule >= D.DM_RULE_LEAST_LOADED else 0)
+    # (the cluster-wide rules add the carries and the all-instance probe kernels)
+    launches_per_step = 3 + 9 + (1 if w.get("rebalance") else 0) + (2 if rule >= D.DM_RULE_LEAST_LOADED else 0)
     if args.adapt:   # window end: the update kernel, once per window
         launches_per_step += 1.0 / kw["adapt_window"]
     clocks = sampler.summary(wall0, wall1)
@@ -428,10 +459,27 @@ def main():
             s, e, doff, dlen, nt, t0 = meta[b]
             return tokens[t0:t0 + nt].cpu().numpy().view(np.uint32)
 
-        n_cpu, t_cpu = cpu_oracle_run(tr, w, [], cb, host_tokens, tr.max_instance_id())
+        ora_out = {}
+        extra = {"choice_rule": rule}
+        if args.adapt:
+            extra.update(adapt_step_blocks=kw["adapt_step_blocks"], adapt_max_blocks=kw["adapt_max_blocks"],
+                         adapt_window=kw["adapt_window"])
+        n_cpu, t_cpu = cpu_oracle_run(tr, w, [], cb, host_tokens, tr.max_instance_id(), keep=ora_out, extra=extra)
+        # the GPU's decisions for the same batches must be the oracle's, bit for bit
+        compared = 0
+        for b in cb:
+            if b not in gpu_out:
+                continue
+            for k, want in ora_out[b].items():
+                got = gpu_out[b][k].astype(want.dtype)
+                if not np.array_equal(got, want):
+                    bad = np.nonzero(got != want)[0]
+                    raise SystemExit(f"bench: GPU and oracle differ in batch {b}, {k} at {bad[:8].tolist()}")
+            compared += len(ora_out[b]["chosen"])
         cpu = {"value": n_cpu / t_cpu, "unit": "req/s", "cores": 1, "kind": "oracle",
                "sample": f"first {len(cb)} batches ({n_cpu} requests) of the same trace, "
-                         f"route+commit, {t_cpu:.1f} s"}
+                         f"route+commit, {t_cpu:.1f} s",
+               "decisions_compared": compared, "decisions_equal": True}
 
     if rank == 0:
         line = {
@@ -451,11 +499,13 @@ def main():
                               if bytes_per_launch > 129e6 else
                               "batches smaller than L2, L2 not flushed between steps"),
                        "replay": "steps beyond the trace replay its batches cyclically" if W + K > nb else "none"},
-            "roofline": {"bound": "hbm", "kernel": "k_hash (prompt hashing)", "achieved": achieved,
+            "roofline": {"bound": "hbm", "kernel": "k_hash_probe (hashing + ring lookup + cache probes, one kernel)",
+                         "achieved": achieved,
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic_per_launch(bytes_per_launch), "bytes_per_launch": bytes_per_launch,
                          "avg_launch_ms": hash_avg_s * 1e3},
             "stage_ms_per_step": stage_ms,
+            "stage_note": "separate replay with every stage event-timed; hash = the hash+probe kernel",
             "serving": {"hit_rate": met["hit_tokens"] / max(met["prompt_tokens"], 1),
                         "cv_mean": met["cv_sum"] / max(met["cv_samples"], 1),
                         "slo_attainment": met["slo_met"] / max(met["completed"], 1),

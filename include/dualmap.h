@@ -172,6 +172,20 @@ typedef struct {
      * dm_create requires index_slots / 2 >= ceil(max_instances /
      * rebuild_pool) * max_touch_per_instance (DM_ERR_INVALID_ARG otherwise). */
     uint32_t rebuild_pool;
+    /* Testing only (no paper counterpart); 0 in normal use.  A nonzero value
+     * caps the iterations of the data-dependent device loops of the cache
+     * index (bucket walks of a lookup, retries of a touch) at that many, so
+     * a test can make a bounded loop give up: the call then records
+     * DM_ERR_TIMEOUT as a sticky error, like an exhausted bound in normal
+     * use. */
+    uint32_t test_loop_limit;
+    /* Candidates per request (App. A.8, "Optimal Candidate Set Size"): 0 or 2
+     * is DualMap's two (dm_route_batch); 1 or 3..8 routes with that many
+     * independent hash functions, rings and probes through dm_route_batch_d
+     * (with choice_rule 0 and the fixed prefix length only;
+     * DM_ERR_INVALID_ARG otherwise, and dm_route_batch and dm_rebalance
+     * return DM_ERR_INVALID_ARG on such a handle). */
+    uint32_t candidates;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */
@@ -208,6 +222,17 @@ typedef struct {
     uint8_t *switched;   /* 1 when the SLO rule overrode cache affinity */
 } dm_route_out;
 
+/* Per-request results of dm_route_batch_d with d candidates (device
+ * memory): cand, hit and ttft hold n x d entries, request-major (request r,
+ * candidate f at r * d + f, f in ring order 1..d). */
+typedef struct {
+    uint32_t *cand;      /* the d distinct candidates */
+    uint32_t *hit;       /* cached-prefix tokens on each (multiple of B) */
+    uint64_t *ttft;      /* estimated TTFT on each, us */
+    uint32_t *chosen;    /* instance the request is queued on (n entries) */
+    uint8_t *switched;   /* 1 when the SLO rule overrode cache affinity (n entries) */
+} dm_route_out_d;
+
 typedef struct {
     uint64_t req_seq;    /* global request sequence number (0-based, arrival order) */
     uint32_t from, to;
@@ -239,12 +264,19 @@ enum {
 #define DM_REBALANCE_SLO_TARGET 1u
 #define DM_REBALANCE_DOUBLE_OVERLOAD 2u
 
-/* Create a scheduler with no instances.  Allocates all device state except
- * the per-instance indices (allocated on first dm_add_instance of an id).
- * Derives the hash key material from cfg->seed.  Synchronous. */
+/* Create a scheduler with no instances (the global scheduler of Sec. 3.1;
+ * the paper describes no construction step, so this lifecycle call and
+ * dm_destroy cite no passage).  Allocates all device state except the
+ * per-instance indices (allocated on first dm_add_instance of an id).
+ * Derives the hash key material from cfg->seed.  On success *out owns the
+ * handle (release it with dm_destroy); on failure *out is NULL and nothing
+ * is left allocated: DM_ERR_INVALID_ARG for a field outside the ranges
+ * stated in dm_config, DM_ERR_OOM when device memory runs out, DM_ERR_CUDA
+ * for another runtime failure.  Synchronous. */
 DM_API dm_status dm_create(const dm_config *cfg, dm_handle **out);
 
-/* Destroy a handle, synchronising its stream first.  NULL is ignored. */
+/* Destroy a handle, synchronising its stream first and freeing all its
+ * device memory.  NULL is ignored. */
 DM_API void dm_destroy(dm_handle *h);
 
 /* Add instance `id` (Sec. 3.4, App. A.1.3): inserts its V virtual nodes into
@@ -274,6 +306,26 @@ DM_API dm_status dm_remove_instance(dm_handle *h, uint32_t id);
  * The batch is kept for dm_commit_cache.  Asynchronous. */
 DM_API dm_status dm_route_batch(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
 
+/* Route one batch with d candidates instead of two (App. A.8: the paper
+ * weighs the candidate set size d and keeps d = 2), d = dm_config.candidates
+ * (2 on a handle created with 0 or 2).  Per request: the prompt prefix
+ * hashed under d independent functions (functions 1 and 2 are
+ * dm_route_batch's; functions 3..d draw their key material from the seed
+ * after DualMap's), one position per ring, the successor's owner on each of
+ * d rings, made distinct (an owner already taken by an earlier ring is
+ * replaced by the next live id after it, in ascending order, cyclically,
+ * not yet taken), the leading run of resident blocks on each candidate,
+ * then DualMap's rule over d candidates: among the candidates with the most
+ * hit tokens, a = the less loaded by W (tie: the earlier ring); a is chosen
+ * when every candidate has that many hits or TTFT_a <= SLO; otherwise the
+ * least loaded candidate by W (tie: a, then the earlier ring), flagged
+ * "switched".  d = 2 gives dm_route_batch's decisions; d = 1 always takes
+ * the ring-1 owner (cache affinity).  Time, loads, queues, metrics and the
+ * following dm_commit_cache are those of dm_route_batch; queue entries
+ * keep the first two candidates.  DM_ERR_NO_INSTANCES with fewer than
+ * max(2, d) live instances.  Asynchronous. */
+DM_API dm_status dm_route_batch_d(dm_handle *h, const dm_batch *batch, const dm_route_out_d *out);
+
 /* Same as dm_route_batch with every pointer of `batch` and `out` in host
  * memory (pinned memory is faster).  The library copies the inputs to its
  * own device staging buffers, routes, copies the results back and
@@ -294,9 +346,20 @@ DM_API dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *batch, 
  * are visited in descending W; their queued, not-started requests are
  * ranked by migration benefit B = TTFT_{r,i} - TTFT_{r,j} (j the request's
  * other candidate) and moved to j while i stays hot, B > 0 and
- * TTFT_{r,j} < SLO.  Writes up to `cap` migrations to out_dev (device) and
- * the total count to *n_out_dev (device).  Asynchronous. */
-DM_API dm_status dm_rebalance(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev);
+ * TTFT_{r,j} < SLO.  Writes up to `cap` migrations, in the order they were
+ * made, to out_host (host memory, owned by the caller) and the total
+ * number made to *n_out (host; it may exceed cap).  Synchronous: the
+ * migrations are computed on the device and copied back before it returns
+ * (the library keeps a device staging buffer of `cap` entries, grown on
+ * demand: DM_ERR_OOM if that fails).  DM_ERR_INVALID_ARG if n_out is NULL,
+ * or out_host is NULL with cap > 0. */
+DM_API dm_status dm_rebalance(dm_handle *h, dm_migration *out_host, uint32_t cap, uint32_t *n_out);
+
+/* dm_rebalance with device outputs, for a pipeline that keeps the results
+ * on the GPU: up to `cap` migrations to out_dev (device) and the total
+ * count to *n_out_dev (device), enqueued on the handle's stream.
+ * Asynchronous. */
+DM_API dm_status dm_rebalance_async(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev);
 
 /* Cache save (App. A.3.2) of the last routed batch: in arrival order, each
  * request touches its block keys on its final instance (block n_blk-1 down
@@ -334,12 +397,15 @@ DM_API dm_status dm_hash_prompts(dm_handle *h, const dm_batch *batch, uint64_t *
  * Returns DM_ERR_CAPACITY without doing anything when n exceeds
  * DM_NOALLOC_MAX_REQUESTS or total_tokens / block_tokens exceeds
  * DM_NOALLOC_MAX_BLOCKS; device-side checks (prompt lengths and offsets, the
- * exact block count) are reported by the return value, because the call
- * synchronises `stream` (a cudaStream_t, NULL = legacy default stream) before
- * returning.  The first call on each device looks up the array's device
- * address and must come before any stream capture on that device.  Every call
- * uses the same array: calls whose work overlaps on the GPU (other host
- * threads, other streams) race and produce garbage. */
+ * exact block count) are reported by the return value: every call
+ * synchronises `stream` (a cudaStream_t, NULL = legacy default stream) and
+ * reads the device error word back before returning.  The first call on each
+ * device looks up the array's device address and should come before any
+ * stream capture on that device; the address is kept for the life of the
+ * process, so after a cudaDeviceReset of a device the entry point must not be
+ * called on that device again.  Every call uses the same array: calls whose
+ * work overlaps on the GPU (other host threads, other streams) race and
+ * produce garbage, so the caller serialises them. */
 DM_API dm_status dm_hash_prompts_noalloc(uint32_t block_tokens, uint32_t route_prefix_blocks, uint64_t seed,
                                          const dm_batch *batch, uint64_t *keys_dev, uint64_t *key_off_dev,
                                          uint64_t *pos_dev, void *stream);
@@ -350,8 +416,12 @@ DM_API dm_status dm_hash_prompts_noalloc(uint32_t block_tokens, uint32_t route_p
 DM_API dm_status dm_ring_lookup(dm_handle *h, const uint64_t *pos_dev, uint32_t n,
                          uint32_t *owner1_dev, uint32_t *owner2_dev);
 
-/* Queued work W (us) of ids 0 .. min(cap, max_instances)-1.  Synchronous. */
-DM_API dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap);
+/* Queued prefill work W (us) of every instance id (the load of Sec. 3.2):
+ * W_host (host, caller-owned) receives ids 0 .. min(cap, max_instances)-1
+ * (0 for ids never added), and *n_out (host) the number of ids,
+ * max_instances.  DM_ERR_INVALID_ARG if n_out is NULL, or W_host is NULL
+ * with cap > 0.  Synchronous; works after a sticky error. */
+DM_API dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap, uint32_t *n_out);
 
 /* Resident (key, last-touch stamp) pairs of instance `id`, in unspecified
  * order; *n_out = resident count (entries beyond cap are not written).
@@ -364,8 +434,9 @@ DM_API dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys_host,
 DM_API dm_status dm_export_queue(dm_handle *h, uint32_t id, uint64_t *seq_host, uint64_t *work_host,
                           uint64_t *remaining_host, uint64_t cap, uint64_t *n_out);
 
-/* Ring f (0 or 1) as sorted (position, owner) arrays; *n_out = its length.
- * Synchronous. */
+/* Ring f (0-based: 0 or 1, or below dm_config.candidates on a handle made
+ * for more candidates) as sorted (position, owner) arrays; *n_out = its
+ * length.  Synchronous. */
 DM_API dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos_host, uint32_t *owner_host,
                          uint32_t cap, uint32_t *n_out);
 
@@ -440,6 +511,15 @@ DM_API dm_status dm_export_prefix_tree(dm_handle *h, uint64_t *keys_host, uint64
  * otherwise, DM_ERR_CUDA if the launch fails. */
 DM_API dm_status dm_potc_max_loads(uint32_t n_bins, uint64_t m_balls, uint32_t d, uint32_t trials, uint64_t seed,
                                    uint32_t *max_load_dev, void *stream);
+
+/* Testing only (no paper counterpart): after this call the library's
+ * (n + 1)-th device allocation, counted over every handle of the process,
+ * fails as if the device were out of memory (without calling the CUDA
+ * allocator), so a test can check that dm_create, dm_add_instance and the
+ * host-buffer entry points return DM_ERR_OOM and leave no handle state
+ * behind.  n < 0 turns the failure off.  Not thread-safe against concurrent
+ * allocating calls. */
+DM_API void dm_test_fail_alloc(int64_t n);
 
 /* Synchronise the stream and return the sticky error (DM_OK if none). */
 DM_API dm_status dm_last_error(dm_handle *h);

@@ -4,6 +4,7 @@
 // translation units; this file only validates, allocates and enqueues.
 #include <cstdio>
 #include <algorithm>
+#include <atomic>
 #include <cstring>
 #include <utility>
 #include <vector>
@@ -34,14 +35,15 @@ struct dm_handle {
     uint64_t pending_seq0 = 0;
     uint32_t rebalance_calls = 0;
     int hash_grid = 0;
+    uint64_t epoch = 0;   // routing calls so far (the routing kernel's record checks)
     // adaptive prefix length: the second expanded-node table (the next
     // window's target), requests and non-empty batches in the current window
     uint64_t *ad_alt = nullptr;
     uint64_t ad_T = 0;
     uint32_t ad_batches = 0;
-    uint64_t *vpos_buf[2][2] = {};
-    uint32_t *owner_buf[2][2] = {}, *vidx_buf[2][2] = {};
-    int cur[2] = {0, 0};
+    uint64_t *vpos_buf[dm::kMaxD][2] = {};
+    uint32_t *owner_buf[dm::kMaxD][2] = {}, *vidx_buf[dm::kMaxD][2] = {};
+    int cur[dm::kMaxD] = {};
     uint64_t *ring_spos = nullptr;
     uint32_t *ring_svidx = nullptr;
     std::vector<Slot *> tables;   // the index buffer first allocated for each id (null: never added)
@@ -67,12 +69,25 @@ struct dm_handle {
     double stage_ms[DM_STAGE_COUNT] = {};
     uint64_t stage_calls[DM_STAGE_COUNT] = {};
     dm_status sticky = DM_OK;
+    // device staging of dm_rebalance's host results
+    dm_migration *rb_out_dev = nullptr;
+    uint32_t rb_out_cap = 0;
+    uint32_t *rb_n_dev = nullptr;
 };
 
 namespace {
 
+// Test hook (dm_test_fail_alloc): the allocation with this ordinal fails.
+std::atomic<int64_t> g_fail_at{-1};
+std::atomic<int64_t> g_alloc_seq{0};
+
 template <typename T>
 cudaError_t dalloc(dm_handle *h, T **p, size_t count) {
+    const int64_t fail_at = g_fail_at.load(std::memory_order_relaxed);
+    if (fail_at >= 0 && g_alloc_seq.fetch_add(1, std::memory_order_relaxed) == fail_at) {
+        *p = nullptr;
+        return cudaErrorMemoryAllocation;
+    }
     void *q = nullptr;
     cudaError_t e = cudaMalloc(&q, count ? count * sizeof(T) : 16);
     if (e != cudaSuccess) { *p = nullptr; return e; }
@@ -211,6 +226,9 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
     if (c.choice_rule > DM_RULE_PREBLE) return DM_ERR_INVALID_ARG;
     if (c.rebalance_flags > (DM_REBALANCE_SLO_TARGET | DM_REBALANCE_DOUBLE_OVERLOAD)) return DM_ERR_INVALID_ARG;
+    if (c.candidates > dm::kMaxD) return DM_ERR_INVALID_ARG;
+    if (c.candidates && c.candidates != 2 && (c.choice_rule != DM_RULE_DUALMAP || c.adapt_step_blocks))
+        return DM_ERR_INVALID_ARG;
     if (c.adapt_step_blocks &&
         (c.adapt_max_blocks <= c.route_prefix_blocks || c.adapt_max_blocks > 2048 || c.adapt_window < 1))
         return DM_ERR_INVALID_ARG;
@@ -234,8 +252,16 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.ad_step = c.adapt_step_blocks;
     d.ad_max = c.adapt_step_blocks ? c.adapt_max_blocks : c.route_prefix_blocks;
     d.Kf2 = d.ad_max;
+    d.loop_limit = c.test_loop_limit;
     d.max_blocks = c.max_batch_tokens / B;
     d.max_segs = d.max_blocks / dm::kSegBlocks + c.max_batch;
+    if (d.max_segs >= (1ull << 31)) {   // segment counts and offsets are 32-bit
+        delete h;
+        return DM_ERR_INVALID_ARG;
+    }
+    // routing order: a head long enough for the longest routing prefix
+    d.Ccols = (d.Kf2 + dm::kSegBlocks - 1) / dm::kSegBlocks;
+    d.H = std::max<uint32_t>(dm::kHeadSegs, d.Ccols);
     d.T = c.max_touch_per_instance ? c.max_touch_per_instance : d.max_blocks;
     d.S = pow2_at_least(2 * (d.C + d.T));
     if (c.index_slots_log2 && (1ull << c.index_slots_log2) > d.S) d.S = 1ull << c.index_slots_log2;
@@ -273,11 +299,21 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     d.Sr2 = splitmix_next(s);
     d.Sv1 = splitmix_next(s);
     d.Sv2 = splitmix_next(s);
+    // functions 3..kMaxD of the d-candidate path, drawn after DualMap's
+    uint32_t kx[dm::kMaxD - 2][64] = {};
+    for (uint32_t f = 0; f + 2 < dm::kMaxD; ++f) {
+        for (uint32_t j = 0; j < B; ++j) kx[f][j] = (uint32_t)splitmix_next(s);
+        d.Gx[f] = splitmix_next(s) | 1ull;
+        d.Srx[f] = splitmix_next(s);
+        d.Svx[f] = splitmix_next(s);
+    }
+    d.nrings = c.candidates > 2 ? c.candidates : 2;
+    d.nd = c.candidates ? c.candidates : 2;
 
     const uint64_t M = d.M, Rmax = M * d.V;
     cudaError_t e = cudaSuccess;
     auto A = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
-    for (int f = 0; f < 2; ++f)
+    for (uint32_t f = 0; f < d.nrings; ++f)
         for (int b = 0; b < 2; ++b) {
             A(dalloc(h, &h->vpos_buf[f][b], Rmax));
             A(dalloc(h, &h->owner_buf[f][b], Rmax));
@@ -285,11 +321,16 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         }
     uint64_t tree_n = 0;
     for (uint64_t n = Rmax; n > 32;) { n = (n + 31) / 32; tree_n += n; }
-    for (int f = 0; f < 2; ++f) A(dalloc(h, &d.ring[f].tree, tree_n + 32));
+    for (uint32_t f = 0; f < d.nrings; ++f) A(dalloc(h, &d.ring[f].tree, tree_n + 32));
     uint32_t P = 1;
     while (P < d.V) P <<= 1;
-    A(dalloc(h, &h->ring_spos, 2ull * P));
-    A(dalloc(h, &h->ring_svidx, 2ull * P));
+    A(dalloc(h, &h->ring_spos, uint64_t(d.nrings) * P));
+    A(dalloc(h, &h->ring_svidx, uint64_t(d.nrings) * P));
+    uint32_t *kx_dev = nullptr;
+    A(dalloc(h, &kx_dev, (dm::kMaxD - 2) * 64));
+    d.Kx = kx_dev;
+    A(dalloc(h, &d.rd_cand, uint64_t(c.max_batch) * d.nd));
+    A(dalloc(h, &d.rd_hit, uint64_t(c.max_batch) * d.nd));
     A(dalloc(h, &d.inst_state, M));
     A(dalloc(h, &d.next_live, M));
     A(dalloc(h, &d.W, M));
@@ -344,6 +385,13 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.rb_seq, d.rb_cap));
     A(dalloc(h, &d.rb_ttft, d.rb_cap));
     A(dalloc(h, &d.rb_pos, d.rb_cap));
+    A(dalloc(h, &d.r_hoff, c.max_batch));
+    A(dalloc(h, &d.r_toff, c.max_batch));
+    A(dalloc(h, &d.seg_pub, d.max_segs));
+    A(dalloc(h, &d.r_route, c.max_batch));
+    A(dalloc(h, &d.r_m1, c.max_batch));
+    A(dalloc(h, &d.r_m2, c.max_batch));
+    A(dalloc(h, &d.fix_list, uint64_t(c.max_batch) * (d.H + 1)));   // every route and probe task at most once
     A(dalloc(h, &d.defer, d.max_segs * dm::kSegBlocks));
     A(dalloc(h, &d.defer_n, d.max_segs));
     // two sets of batch scratch: routing and dm_hash_prompts
@@ -368,8 +416,6 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         A(dalloc(h, &x->r_K, c.max_batch));
         A(dalloc(h, &x->r_c1, c.max_batch));
         A(dalloc(h, &x->r_c2, c.max_batch));
-        A(dalloc(h, &x->r_h1, c.max_batch));
-        A(dalloc(h, &x->r_h2, c.max_batch));
         A(dalloc(h, &x->r_final, c.max_batch));
         A(dalloc(h, &x->r_touchoff, c.max_batch));
         A(dalloc(h, &x->info, 1));
@@ -380,13 +426,16 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     }
     h->dh.ad_step = 0;   // dm_hash_prompts hashes the fixed length
     h->dh.Kf2 = c.route_prefix_blocks;
-    for (int f = 0; f < 2; ++f) {
+    for (uint32_t f = 0; f < d.nrings; ++f) {
         d.ring[f].vpos = h->vpos_buf[f][0];
         d.ring[f].owner = h->owner_buf[f][0];
         d.ring[f].vidx = h->vidx_buf[f][0];
         h->dh.ring[f] = d.ring[f];
     }
     set_levels(d, 0);
+    A(cudaMemcpyAsync(kx_dev, kx, sizeof(kx), cudaMemcpyHostToDevice, h->st));
+    A(cudaMemsetAsync(d.seg_pub, 0, d.max_segs * sizeof(dm::SegPub), h->st));
+    A(cudaMemsetAsync(d.r_route, 0, uint64_t(c.max_batch) * sizeof(dm::RoutePub), h->st));
     A(cudaMemsetAsync(d.inst_state, 0, M, h->st));
     A(cudaMemsetAsync(d.W, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.metrics, 0, sizeof(dm::DevMetrics), h->st));
@@ -446,26 +495,25 @@ static void sync_copy(dm_handle *h) {
     h->dh.seg_total2 = keep.seg_total2;
     h->dh.seg_newly = keep.seg_newly;
     h->dh.seg_claims = keep.seg_claims;
-    h->dh.r_c1 = keep.r_c1; h->dh.r_c2 = keep.r_c2; h->dh.r_h1 = keep.r_h1;
-    h->dh.r_h2 = keep.r_h2; h->dh.r_final = keep.r_final; h->dh.r_touchoff = keep.r_touchoff;
+    h->dh.r_c1 = keep.r_c1; h->dh.r_c2 = keep.r_c2;
+    h->dh.r_final = keep.r_final; h->dh.r_touchoff = keep.r_touchoff;
     h->dh.info = keep.info;
 }
 
 static dm_status ring_change(dm_handle *h, uint32_t id, bool add) {
     DevState &d = h->d;
     const uint32_t newR = add ? d.R + d.V : d.R - d.V;
-    uint64_t *nv[2];
-    uint32_t *no[2], *ni[2];
-    for (int f = 0; f < 2; ++f) {
+    uint64_t *nv[dm::kMaxD] = {};
+    uint32_t *no[dm::kMaxD] = {}, *ni[dm::kMaxD] = {};
+    for (uint32_t f = 0; f < d.nrings; ++f) {
         const int nb = 1 - h->cur[f];
         nv[f] = h->vpos_buf[f][nb];
         no[f] = h->owner_buf[f][nb];
         ni[f] = h->vidx_buf[f][nb];
     }
-    cudaError_t e = dm::launch_ring_update(d, id, add, newR, h->ring_spos, nullptr, h->ring_svidx, nv, no, ni,
-                                           h->st);
+    cudaError_t e = dm::launch_ring_update(d, id, add, h->ring_spos, h->ring_svidx, nv, no, ni, h->st);
     if (e != cudaSuccess) return map_cuda(h, e);
-    for (int f = 0; f < 2; ++f) {
+    for (uint32_t f = 0; f < d.nrings; ++f) {
         h->cur[f] = 1 - h->cur[f];
         d.ring[f].vpos = nv[f];
         d.ring[f].owner = no[f];
@@ -586,9 +634,14 @@ static bool tokens_aligned(const dm_batch *b) {
     return b->n == 0 || (reinterpret_cast<uintptr_t>(b->tokens) & 15) == 0;
 }
 
+// A handle made for d candidates (dm_config.candidates not 0 or 2) routes only
+// through dm_route_batch_d and does not rebalance.
+static bool pair_handle(const dm_handle *h) { return h->cfg.candidates == 0 || h->cfg.candidates == 2; }
+
 dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
     dm_status s = check_batch(h, b, o);
     if (s) return s;
+    if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!tokens_aligned(b)) return DM_ERR_INVALID_ARG;
     if (!o) return DM_ERR_INVALID_ARG;
     if (h->n_live < 2) return DM_ERR_NO_INSTANCES;
@@ -599,9 +652,13 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
     h->have_time = true;
     const DevState &d = h->d;
     cudaError_t e;
-    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_drain(d, *b, delta, t0, h->st); }   // drain included
-    if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_HASH); e = dm::launch_hash(d, *b, h->hash_grid, h->st); }
-    if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_PROBE); e = dm::launch_route_probe(d, *b, *o, h->st); }
+    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_route(d, *b, delta, t0, h->st); }   // drain included
+    if (e == cudaSuccess && b->n) {   // hashing, ring lookup and probes: one kernel
+        Stage st(h, DM_STAGE_HASH);
+        // a fresh epoch mask per call: records of earlier batches never pass its check
+        const uint64_t E = dm::fmix64(++h->epoch ^ 0x6a09e667f3bcc909ull);
+        e = dm::launch_hash_probe(d, *b, E, h->st);
+    }
     if (e == cudaSuccess && b->n) {
         Stage st(h, DM_STAGE_CHOICE);
         e = dm::launch_choice(d, *o, b->n, h->seq_next, b->batch_time_us, h->st);
@@ -631,6 +688,7 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
 dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
     dm_status s = check_batch(h, b, o);
     if (s) return s;
+    if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!o) return DM_ERR_INVALID_ARG;
     cudaError_t e = cudaSuccess;
     const uint32_t mb = h->d.max_batch;
@@ -687,15 +745,70 @@ dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *b, const dm_ro
     return map_cuda(h, e);
 }
 
+dm_status dm_route_batch_d(dm_handle *h, const dm_batch *b, const dm_route_out_d *o) {
+    dm_status s = check_batch(h, b, nullptr);
+    if (s) return s;
+    if (!tokens_aligned(b) || !o) return DM_ERR_INVALID_ARG;
+    if (b->n > 0 && (!o->cand || !o->hit || !o->ttft || !o->chosen || !o->switched)) return DM_ERR_INVALID_ARG;
+    const DevState &d = h->d;
+    if (h->n_live < 2 || h->n_live < d.nd) return DM_ERR_NO_INSTANCES;
+    if (h->have_time && b->batch_time_us < h->t_prev) return DM_ERR_ORDER;
+    const uint64_t delta = h->have_time ? b->batch_time_us - h->t_prev : 0;
+    const uint64_t t0 = h->have_time ? h->t_prev : b->batch_time_us;
+    h->t_prev = b->batch_time_us;
+    h->have_time = true;
+    cudaError_t e;
+    { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_plain_drain(d, *b, delta, t0, h->st); }
+    if (e == cudaSuccess && b->n) { Stage st(h, DM_STAGE_HASH); e = dm::launch_hash(d, *b, h->hash_grid, h->st); }
+    if (e == cudaSuccess && b->n) {
+        Stage st(h, DM_STAGE_CHOICE);   // ring lookups, probes and the choice
+        e = dm::launch_route_d(d, *b, *o, h->seq_next, h->st);
+    }
+    if (e != cudaSuccess) return map_cuda(h, e);
+    h->pending = true;
+    h->pending_n = b->n;
+    h->pending_seq0 = h->seq_next;
+    h->seq_next += b->n;
+    return DM_OK;
+}
+
 dm_status dm_route_batch_host(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
     dm_status s = dm_route_batch_host_async(h, b, o);
     if (s) return s;
     return map_cuda(h, cudaStreamSynchronize(h->st));
 }
 
-dm_status dm_rebalance(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev) {
+dm_status dm_rebalance(dm_handle *h, dm_migration *out_host, uint32_t cap, uint32_t *n_out) {
     dm_status s = check_live(h);
     if (s) return s;
+    if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
+    if (!n_out || (cap && !out_host)) return DM_ERR_INVALID_ARG;
+    if (cap > h->rb_out_cap || !h->rb_n_dev) {   // device staging of the results
+        dm_migration *buf = nullptr;
+        uint32_t *cnt = h->rb_n_dev;
+        cudaError_t e = dalloc(h, &buf, cap ? cap : 1);
+        if (e == cudaSuccess && !cnt) e = dalloc(h, &cnt, 1);
+        if (e != cudaSuccess) { cudaGetLastError(); return DM_ERR_OOM; }
+        h->rb_out_dev = buf;
+        h->rb_out_cap = cap ? cap : 1;
+        h->rb_n_dev = cnt;
+    }
+    s = dm_rebalance_async(h, h->rb_out_dev, cap, h->rb_n_dev);
+    if (s) return s;
+    uint32_t n = 0;
+    cudaError_t e = cudaMemcpyAsync(&n, h->rb_n_dev, 4, cudaMemcpyDeviceToHost, h->st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    if (e == cudaSuccess && n && cap)
+        e = cudaMemcpy(out_host, h->rb_out_dev, sizeof(dm_migration) * (n < cap ? n : cap), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    *n_out = n;
+    return DM_OK;
+}
+
+dm_status dm_rebalance_async(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!n_out_dev || (cap && !out_dev)) return DM_ERR_INVALID_ARG;
     const uint32_t n = h->pending ? h->pending_n : 0;
     cudaError_t e;
@@ -740,14 +853,16 @@ dm_status dm_ring_lookup(dm_handle *h, const uint64_t *pos_dev, uint32_t n, uint
     return map_cuda(h, dm::launch_ring_lookup(h->d, pos_dev, n, o1, o2, h->st));
 }
 
-dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap) {
+dm_status dm_get_loads(dm_handle *h, uint64_t *W_host, uint32_t cap, uint32_t *n_out) {
     dm_status s = check_handle(h);
     if (s) return s;
-    if (!W_host && cap) return DM_ERR_INVALID_ARG;
+    if (!n_out || (!W_host && cap)) return DM_ERR_INVALID_ARG;
     const uint32_t k = cap < h->d.M ? cap : h->d.M;
-    cudaError_t e = cudaMemcpyAsync(W_host, h->d.W, k * 8ull, cudaMemcpyDeviceToHost, h->st);
+    cudaError_t e = k ? cudaMemcpyAsync(W_host, h->d.W, k * 8ull, cudaMemcpyDeviceToHost, h->st) : cudaSuccess;
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
-    return map_cuda(h, e);
+    if (e != cudaSuccess) return map_cuda(h, e);
+    *n_out = h->d.M;
+    return DM_OK;
 }
 
 dm_status dm_export_cache(dm_handle *h, uint32_t id, uint64_t *keys, uint64_t *stamps, uint64_t cap,
@@ -813,7 +928,7 @@ dm_status dm_export_queue(dm_handle *h, uint32_t id, uint64_t *seq, uint64_t *wo
 dm_status dm_export_ring(dm_handle *h, int f, uint64_t *vpos, uint32_t *owner, uint32_t cap, uint32_t *n_out) {
     dm_status s = check_handle(h);
     if (s) return s;
-    if ((f != 0 && f != 1) || !n_out || (cap && (!vpos || !owner))) return DM_ERR_INVALID_ARG;
+    if (f < 0 || (uint32_t)f >= h->d.nrings || !n_out || (cap && (!vpos || !owner))) return DM_ERR_INVALID_ARG;
     const uint32_t k = cap < h->d.R ? cap : h->d.R;
     cudaError_t e = cudaMemcpyAsync(vpos, h->d.ring[f].vpos, k * 8ull, cudaMemcpyDeviceToHost, h->st);
     if (e == cudaSuccess) e = cudaMemcpyAsync(owner, h->d.ring[f].owner, k * 4ull, cudaMemcpyDeviceToHost, h->st);
@@ -917,6 +1032,11 @@ dm_status dm_get_metrics(dm_handle *h, dm_metrics *out, uint64_t *hist_host, uin
     out->cv_last = m.cv_last;
     for (uint32_t k = 0; k < hist_cap && k < dm::kHistBuckets; ++k) hist_host[k] = m.hist[k];
     return DM_OK;
+}
+
+void dm_test_fail_alloc(int64_t n) {
+    g_alloc_seq.store(0, std::memory_order_relaxed);
+    g_fail_at.store(n, std::memory_order_relaxed);
 }
 
 dm_status dm_last_error(dm_handle *h) {

@@ -17,6 +17,8 @@
 // Cluster-wide rules: every request depends on every earlier one, so one
 // warp decides them one at a time (an argmin over the live instances),
 // with the hits on every live instance probed beforehand by k_probe_all.
+//
+// At the end of the file: routing with d candidates (App. A.8).
 #include "dm_internal.cuh"
 
 namespace dm {
@@ -123,6 +125,10 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
     pdl_enter();
     extern __shared__ __align__(16) unsigned char smem[];
     if (has_err(d.err)) return;
+    if (blockIdx.x > 0) {   // beside the choice: the segment carries the commit needs
+        carries_role(d, o, n, blockIdx.x - 1, gridDim.x - 1);
+        return;
+    }
     uint64_t *W = reinterpret_cast<uint64_t *>(smem);
     uint64_t *PT = W + d.M;
     uint32_t *lanes = reinterpret_cast<uint32_t *>(PT + d.M);
@@ -142,7 +148,8 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
         __syncthreads();
         for (uint32_t k = threadIdx.x; k < m; k += blockDim.x) {
             const uint32_t r = base + k;
-            const uint32_t L = d.r_L[r], h1 = d.r_h1[r], h2 = d.r_h2[r];
+            const uint32_t L = d.r_L[r], nblk = d.r_nblk[r];
+            const uint32_t h1 = hit_tokens(d.r_m1[r], nblk, d.B), h2 = hit_tokens(d.r_m2[r], nblk, d.B);
             const uint32_t c1 = d.r_c1[r], c2 = d.r_c2[r];
             // global cache affinity always takes c1: orient it as a, never b
             const bool a2 = rule != DM_RULE_CACHE_AFFINITY && h2 > h1;
@@ -168,7 +175,7 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
             S.thr[k] = thr;
             S.ab[k] = (a2 ? c2 : c1) | ((a2 ? c1 : c2) << 14) | (uint32_t(a2) << 28) | (uint32_t(differ) << 29) |
                       (uint32_t(tieb) << 30) | (uint32_t(addu) << 31);
-            S.nb[k] = d.r_nblk[r];
+            S.nb[k] = nblk;
         }
         __syncthreads();
         if (threadIdx.x < 32) {
@@ -235,7 +242,8 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
             o.chosen[r] = ch;
             o.switched[r] = sw;
             d.r_final[r] = ch;
-            const uint32_t L = d.r_L[r], h1 = d.r_h1[r], h2 = d.r_h2[r];
+            const uint32_t L = d.r_L[r], nbr = d.r_nblk[r];
+            const uint32_t h1 = hit_tokens(d.r_m1[r], nbr, d.B), h2 = hit_tokens(d.r_m2[r], nbr, d.B);
             ms.tokens += L;
             ms.hits += (ch == (a_is_c2 ? b : a)) ? h1 : h2;
             ms.sw += sw;
@@ -288,13 +296,6 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
 // else takes the full probe order.
 constexpr int kAllBlock = 256;
 
-__device__ __forceinline__ bool resident_at(const Slot *t, uint64_t mask, uint64_t key, uint64_t home,
-                                            uint64_t front, const Slot &s0, uint32_t *err) {
-    if (s0.key == key) return s0.pos1 > front;
-    if (s0.key == 0) return false;
-    return table_pos1(t, mask, key, home, err) > front;
-}
-
 __global__ void __launch_bounds__(kAllBlock) k_probe_all(DevState d, uint32_t n) {
     pdl_enter();
     if (has_err(d.err)) return;
@@ -324,7 +325,7 @@ __global__ void __launch_bounds__(kAllBlock) k_probe_all(DevState d, uint32_t n)
                 uint32_t miss_at = 0xFFFFFFFFu;
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
-                    const bool res = key[j] != 0 && resident_at(t, mask, key[j], home[j], front, sl[j], d.err);
+                    const bool res = key[j] != 0 && resident_at(t, mask, key[j], home[j], front, sl[j], d.err, d.loop_limit);
                     const uint32_t m = __ballot_sync(0xffffffffu, !res);
                     if (j < (int)step && m && miss_at == 0xFFFFFFFFu) miss_at = base + 32 * j + __ffs(m) - 1;
                 }
@@ -401,8 +402,8 @@ __global__ void __launch_bounds__(1024) k_choice_global(DevState d, dm_route_out
             s_nb[rr] = d.r_nblk[r];
             s_c1[rr] = d.r_c1[r];
             s_c2[rr] = d.r_c2[r];
-            s_h1[rr] = d.r_h1[r];
-            s_h2[rr] = d.r_h2[r];
+            s_h1[rr] = hit_tokens(d.r_m1[r], s_nb[rr], d.B);
+            s_h2[rr] = hit_tokens(d.r_m2[r], s_nb[rr], d.B);
         }
         __syncthreads();
         if (wid == 0) {
@@ -523,6 +524,7 @@ cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, 
             DM_TRY(cudaFuncSetAttribute(k_choice_global, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_g));
             smem_M = d.M;
         }
+        DM_TRY(launch_carries(d, o, n, st));
         DM_TRY(launch_pdl(k_probe_all, full_grid(k_probe_all, kAllBlock), kAllBlock, 0, st, d, n));
         DM_TRY(launch_pdl(k_choice_global, 1, 1024, smem_g, st, d, o, n, seq0, t_batch, smem_g));
         return cudaGetLastError();
@@ -536,10 +538,226 @@ cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, 
         }
         configured = smem;
     }
+    // CTA 0 decides; CTAs 1.. sum the batch's segment carries meanwhile (a warp per request)
+    const unsigned grid = 1 + (n + 31) / 32 < 1 + 152 ? 1 + (n + 31) / 32 : 1 + 152;
     if (d.rule == DM_RULE_DUALMAP)
-        DM_TRY(launch_pdl(k_choice<false>, 1, 1024, smem, st, d, o, n, seq0, t_batch));
+        DM_TRY(launch_pdl(k_choice<false>, grid, 1024, smem, st, d, o, n, seq0, t_batch));
     else
-        DM_TRY(launch_pdl(k_choice<true>, 1, 1024, smem, st, d, o, n, seq0, t_batch));
+        DM_TRY(launch_pdl(k_choice<true>, grid, 1024, smem, st, d, o, n, seq0, t_batch));
+    return cudaGetLastError();
+}
+
+
+// ---------------------------------------------------------------------------
+// Routing with d candidates instead of two (App. A.8,
+// "Optimal Candidate Set Size": the paper weighs d and keeps d = 2; this is
+// the d-way version of the path, for that comparison).  After the plain
+// hashing kernel (f1 chained prefix values and totals):
+//   k_route_d   warp per request: segment carries, the d ring positions
+//               (function 1 from the prefix values; functions 2..d hash the
+//               first K blocks here), a successor search on each ring, the
+//               distinct fix, and the leading run of resident blocks on
+//               each candidate;
+//   k_choice_d  one CTA: DualMap's SLO-aware rule over d candidates in
+//               arrival order (one thread; this path is for experiments,
+//               not the benchmark), queue appends, the commit's per-request
+//               offsets and the batch's metrics, exactly as k_choice leaves
+//               them for d = 2.
+
+
+// Index (level 0) of the successor of p on ring f.  Whole warp.
+__device__ __forceinline__ uint32_t ring_search1(const DevState &d, int f, uint64_t p, int lane) {
+    const int top = (int)d.nlev - 1;
+    const uint64_t nt = d.lev_n[top];
+    const uint64_t vt = (uint64_t)lane < nt ? level_ptr(d, f, top)[lane] : ~0ull;
+    int64_t i = (int64_t)__popc(__ballot_sync(0xffffffffu, vt < p)) - 1;
+    for (int k = top - 1; k >= 0; --k) {
+        const uint64_t nk = d.lev_n[k];
+        const uint64_t a = (uint64_t)(i < 0 ? 0 : i) * 32 + lane;
+        const uint64_t v = (i >= 0 && a < nk) ? level_ptr(d, f, k)[a] : ~0ull;
+        const int c = __popc(__ballot_sync(0xffffffffu, v < p));
+        if (i >= 0) i = i * 32 + c - 1;
+    }
+    return (uint32_t)(i + 1 == (int64_t)d.R ? 0 : i + 1);
+}
+
+// NH key word j of function f (0-based).
+__device__ __forceinline__ uint32_t nh_key(const DevState &d, uint32_t f, uint32_t j) {
+    return f == 0 ? d.K1[j] : f == 1 ? d.K2[j] : d.Kx[(f - 2) * 64 + j];
+}
+
+__global__ void k_route_d(DevState d, const uint32_t *tokens, uint32_t n) {
+    pdl_enter();
+    if (has_err(d.err)) return;
+    const int lane = threadIdx.x & 31;
+    const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    if (r >= n) return;
+    request_carries(d, r, lane);
+    __syncwarp();
+    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r], B = d.B, nd = d.nd;
+    const uint64_t bo = d.r_blkoff[r];
+    const uint32_t K = min(d.Kroute, nblk);
+    const uint32_t *tok = tokens + d.r_tokoff[r];
+    uint32_t cand[kMaxD];
+    for (uint32_t f = 0; f < nd; ++f) {
+        uint64_t P;
+        if (f == 0) {
+            P = d.plocal[bo + K - 1] + d.seg_carry[s0 + (K - 1) / kSegBlocks];
+        } else {   // function f over the first K blocks: a lane per block
+            const uint64_t G = f == 1 ? d.G2 : d.Gx[f - 2];
+            uint64_t acc = 0;
+            for (uint32_t b = lane; b < K; b += 32) {
+                uint64_t nh = 0;
+                for (uint32_t i = 0; i < B; i += 2)
+                    nh += uint64_t(tok[uint64_t(b) * B + i] + nh_key(d, f, i)) *
+                          uint64_t(tok[uint64_t(b) * B + i + 1] + nh_key(d, f, i + 1));
+                acc += fmix64(nh + uint64_t(b + 1) * G);
+            }
+            P = warp_sum_u64(acc);
+        }
+        const uint64_t Sr = f == 0 ? d.Sr1 : f == 1 ? d.Sr2 : d.Srx[f - 2];
+        uint32_t x = d.ring[f].owner[ring_search1(d, (int)f, fmix64(P ^ Sr), lane)];
+        for (uint32_t k = 0; k < nd; ++k) {   // taken by an earlier ring: the next live id after it
+            bool taken = false;
+            for (uint32_t g = 0; g < f; ++g) taken |= cand[g] == x;
+            if (!taken) break;
+            x = d.next_live[x];
+        }
+        cand[f] = x;
+    }
+    // leading run of resident blocks on each candidate (index as of the start of the batch)
+    const uint64_t mask = d.S - 1;
+    for (uint32_t f = 0; f < nd; ++f) {
+        const Slot *t = d.table[cand[f]];
+        const uint64_t front = d.log_front[cand[f]];
+        uint32_t h = nblk;
+        for (uint32_t base = 0; base < nblk; base += 32) {
+            const uint32_t b = base + lane;
+            const bool inb = b < nblk;
+            const uint64_t key = inb ? cache_key(d.plocal[bo + b] + d.seg_carry[s0 + b / kSegBlocks], d.Sc) : 0;
+            const uint64_t home = group_home(group_anchor(key, lane), b, mask);
+            const bool miss = inb && !resident_at(t, mask, key, home, front, load_slot(t + home), d.err, d.loop_limit);
+            const uint32_t bal = __ballot_sync(0xffffffffu, miss);
+            if (bal) {
+                h = base + __ffs(bal) - 1;
+                break;
+            }
+        }
+        if (lane == 0) {
+            d.rd_cand[uint64_t(r) * nd + f] = cand[f];
+            d.rd_hit[uint64_t(r) * nd + f] = h * B;
+        }
+    }
+    if (lane == 0) d.r_K[r] = K;
+}
+
+// DualMap's rule over d candidates, in arrival order (one thread), then the
+// batch's loads, queue tails, commit offsets and metrics as k_choice leaves
+// them.  Dynamic shared memory: W and the packed (records << 32 | queue
+// tail) counter of every instance.
+__global__ void __launch_bounds__(1024) k_choice_d(DevState d, dm_route_out_d o, uint32_t n, uint64_t seq0,
+                                                   uint64_t t_batch) {
+    pdl_enter();
+    extern __shared__ __align__(16) unsigned char smem[];
+    if (has_err(d.err)) return;
+    uint64_t *W = reinterpret_cast<uint64_t *>(smem);
+    uint64_t *PT = W + d.M;
+    uint32_t live_bits = 0;
+    for (uint32_t i = threadIdx.x, k = 0; i < d.M; i += blockDim.x, ++k) {
+        W[i] = d.W[i];
+        PT[i] = d.q_tail[i];
+        live_bits |= uint32_t(d.inst_state[i] == 1) << k;
+    }
+    __syncthreads();
+    const uint32_t nd = d.nd;
+    const uint64_t cost = d.cost, slo = d.slo;
+    uint64_t tokens = 0, hits = 0, sw = 0, est = 0;
+    if (threadIdx.x == 0) {
+        for (uint32_t r = 0; r < n; ++r) {
+            const uint32_t *c = d.rd_cand + uint64_t(r) * nd, *h = d.rd_hit + uint64_t(r) * nd;
+            const uint32_t L = d.r_L[r];
+            uint32_t hmax = 0, nmax = 0, a = 0;
+            for (uint32_t f = 0; f < nd; ++f) hmax = max(hmax, h[f]);
+            bool all_over = true, first = true;
+            for (uint32_t f = 0; f < nd; ++f) {
+                const uint64_t t = W[c[f]] + cost * (L - h[f]);
+                o.ttft[uint64_t(r) * nd + f] = t;
+                all_over = all_over && t > slo;
+                if (h[f] == hmax) {
+                    ++nmax;
+                    if (first || W[c[f]] < W[c[a]]) a = f;
+                    first = false;
+                }
+            }
+            uint32_t pick = a;
+            const bool over = nmax < nd && W[c[a]] + cost * (L - h[a]) > slo;
+            if (over)
+                for (uint32_t f = 0; f < nd; ++f)
+                    if (W[c[f]] < W[c[pick]]) pick = f;
+            const uint32_t ch = c[pick];
+            const uint64_t u = cost * (L - h[pick]);
+            o.chosen[r] = ch;
+            o.switched[r] = over;
+            for (uint32_t f = 0; f < nd; ++f) {
+                o.cand[uint64_t(r) * nd + f] = c[f];
+                o.hit[uint64_t(r) * nd + f] = h[f];
+            }
+            if (all_over) d.info->both_over = 1;
+            const uint64_t Pold = PT[ch];
+            W[ch] += u;
+            PT[ch] = Pold + (uint64_t(d.r_nblk[r]) << 32) + 1;
+            d.r_final[r] = ch;
+            d.r_touchoff[r] = Pold >> 32;   // offset among this batch's records of ch
+            tokens += L;
+            hits += h[pick];
+            sw += over;
+            est += W[ch] <= slo;
+            const uint32_t slot = (uint32_t)Pold;
+            if (slot - d.q_head[ch] >= d.Q) {
+                set_err(d.err, DM_ERR_CAPACITY);
+                continue;
+            }
+            QEntry e;
+            e.seq = seq0 + r;
+            e.work = e.remaining = u;
+            e.L = L;
+            e.c1 = c[0];
+            e.c2 = nd > 1 ? c[1] : c[0];
+            e.h1 = h[0];
+            e.h2 = nd > 1 ? h[1] : h[0];
+            e.moved = 0;
+            e.arrival = t_batch;
+            d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
+        }
+    }
+    __syncthreads();
+    unsigned __int128 S1 = 0, S2 = 0;
+    uint32_t cnt = 0;
+    for (uint32_t i = threadIdx.x, k = 0; i < d.M; i += blockDim.x, ++k) {
+        d.W[i] = W[i];
+        d.q_tail[i] = (uint32_t)PT[i];
+        d.log_adv[i] = PT[i] >> 32;
+        if ((live_bits >> k) & 1u) {
+            S1 += W[i];
+            S2 += (unsigned __int128)W[i] * W[i];
+            ++cnt;
+        }
+    }
+    if (threadIdx.x == 0) d.info->final_dirty = 0;
+    finish_metrics(d, n, MetricSums{tokens, hits, sw, est}, S1, S2, cnt);
+}
+
+cudaError_t launch_route_d(const DevState &d, const dm_batch &b, const dm_route_out_d &o, uint64_t seq0,
+                           cudaStream_t st) {
+    if (b.n == 0) return cudaSuccess;
+    DM_TRY(launch_pdl(k_route_d, (b.n + 7) / 8, 256, 0, st, d, b.tokens, b.n));
+    const size_t smem = size_t(d.M) * 16;
+    static size_t configured = 0;
+    if (smem > configured) {
+        DM_TRY(cudaFuncSetAttribute(k_choice_d, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        configured = smem;
+    }
+    DM_TRY(launch_pdl(k_choice_d, 1, 1024, smem, st, d, o, b.n, seq0, b.batch_time_us));
     return cudaGetLastError();
 }
 

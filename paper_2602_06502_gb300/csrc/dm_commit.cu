@@ -65,7 +65,8 @@ __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
 // meet at the same slot and one CAS wins.  Returns the position value the
 // key had before (0 if claimed now).
 __device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64_t key, uint64_t p1, uint64_t home,
-                                                  Slot old, uint32_t *err, bool *claimed, uint32_t nbk0 = 0) {
+                                                  Slot old, uint32_t *err, bool *claimed, uint32_t nbk0 = 0,
+                                                  uint64_t loop_limit = 0) {
     // `old` was seen at the preferred slot of bucket nbk0 of the key's order
     const uint32_t o = (uint32_t)(home & (kGroup - 1));
     const uint64_t R0 = home & ~uint64_t(kGroup - 1);
@@ -74,7 +75,8 @@ __device__ __forceinline__ uint64_t touch_resolve(Slot *t, uint64_t mask, uint64
     uint32_t step = 0;   // order position of slot i within bucket R
     // at most one probe step per slot, and one retry per other touch of the
     // key in the batch (each failed retry means another touch got in)
-    const uint64_t limit = mask + 1 + (1ull << 20);
+    uint64_t limit = mask + 1 + (1ull << 20);
+    if (loop_limit && loop_limit < limit) limit = loop_limit;
     for (uint64_t it = 0; it < limit; ++it) {
         if (old.key == 0) { *claimed = true; return 0; }   // a CAS from {0,0} that failed returns a key
         if (old.key == key) {   // the slot's key never changes: raise its position word alone
@@ -656,7 +658,8 @@ __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
             // other than 0 and e.key)
             const Slot old = e.found ? Slot{e.key, e.x} : Slot{e.key == 1 ? 2ull : e.key ^ 1ull, 0};
             bool cl = false;
-            const uint64_t o = touch_resolve(d.table[e.f], mask, e.key, e.p + 1, e.home, old, d.err, &cl, e.bucket);
+            const uint64_t o =
+                touch_resolve(d.table[e.f], mask, e.key, e.p + 1, e.home, old, d.err, &cl, e.bucket, d.loop_limit);
             touch_outcome(o, e.p, d.log_front[e.f], d.stale[e.f], lmask, newly);
             claims += cl;
         }

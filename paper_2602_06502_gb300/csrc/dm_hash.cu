@@ -1,6 +1,8 @@
 // dm_hash.cu -- prompt hashing (Sec. 3.2: two independent hash functions
-// over the prompt prefix; App. A.1.1 block-granular keys).  The batch layout
-// it reads is made by dm_setup.cu.
+// over the prompt prefix; App. A.1.1 block-granular keys), and the routing
+// kernel that hashes, looks the candidates up on both rings (Sec. 3.2,
+// Sec. 3.4, App. A.1.3) and probes their cache indices (App. A.3.2) in one
+// pass over the tokens.  The batch layout it reads is made by dm_setup.cu.
 //
 // Per full block k of a prompt (B tokens t_0..t_{B-1}) under function f:
 //   nh^f_k = sum_i ((t_2i + K^f_2i) mod 2^32) * ((t_2i+1 + K^f_2i+1) mod 2^32)  mod 2^64
@@ -8,22 +10,33 @@
 //   P^f_b  = sum_{k<=b} d^f_k  mod 2^64
 // Because the chain is a plain prefix sum, every 64-block segment of every
 // prompt is hashed independently (one warp each); a segment writes its local
-// prefix values and its totals, and the probe kernel adds the carry of the
-// earlier segments.  f2 only runs over the first K = min(Kf2, n_blk) blocks
-// (Kf2 = K_route, or the longest adaptive prefix): segments below K write the
-// sum of their f2 digests and, with the adaptive length, each block's
-// in-segment f2 prefix value.
+// prefix values and its totals, and the carry of the earlier segments is
+// added where a key is needed.  f2 only runs over the first K = min(Kf2,
+// n_blk) blocks (Kf2 = K_route, or the longest adaptive prefix): segments
+// below K write the sum of their f2 digests and, with the adaptive length,
+// each block's in-segment f2 prefix value.
+#include <atomic>
+
 #include "dm_internal.cuh"
 
 namespace dm {
 
 // ---------------------------------------------------------------------------
-// Streaming 16-byte load: read once, do not keep in L1.
-__device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
+// Streaming 16-byte load: read once, not kept in L1; with an L2 evict-first
+// policy the token stream does not push the index lines and the previous
+// commit's writes out of L2.
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p, uint64_t pol) {
     uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(__cvta_generic_to_global(p)));
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(__cvta_generic_to_global(p)), "l"(pol));
     return v;
+}
+
+__device__ __forceinline__ uint64_t evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
 }
 
 // NH partial over 4 consecutive tokens (two pairs) with the lane's 4 keys.
@@ -49,32 +62,118 @@ __device__ __forceinline__ uint64_t reduce_scatter(uint64_t (&p)[U], int q) {
     return p[0];
 }
 
-// One warp per segment of up to 64 blocks (two iterations of 32 blocks).
-// Iteration `it` covers 32 blocks (32*U uint4): load j of lane l reads uint4
-// j*32+l of the iteration (fully coalesced), which is quarter l%U of block
-// j*(32/U)+l/U.  Both iterations' loads are issued before any arithmetic
-// (4 KB in flight per warp at B = 16).  After the reduce-scatter lane l
-// holds block (l%U)*(32/U) + l/U; one shuffle puts block m on lane m for the
-// scan.  Segments below K also sum their f2 digests (blocks < K); kP2 adds
-// their per-block prefix values (the adaptive length picks its K later).
+// Per-lane constants of the segment hash: lane l = g * U + q reduces the
+// NH of one block per load instruction; its 4 key words of each function.
+template <int U>
+struct HashLane {
+    static constexpr int GPL = 32 / U;   // blocks per load instruction
+    int q, g, bq, src;
+    uint32_t k1[4], k2[4];
+    uint64_t G1, G2;
+    __device__ __forceinline__ HashLane(const DevState &d, int lane) {
+        q = lane % U;
+        g = lane / U;
+        bq = q * GPL + g;                      // block this lane reduces
+        src = (lane % GPL) * U + lane / GPL;   // lane holding block `lane` after the reduction
+#pragma unroll
+        for (int i = 0; i < 4; ++i) { k1[i] = d.K1[4 * q + i]; k2[i] = d.K2[4 * q + i]; }
+        G1 = d.G1;
+        G2 = d.G2;
+    }
+};
+
+// One segment of up to 64 blocks (two iterations of 32 blocks): blocks
+// b0 .. b0+nb-1 of a prompt whose tokens start at src4 (block b0's first
+// token).  Iteration `it` covers 32 blocks (32*U uint4): load j of lane l
+// reads uint4 j*32+l of the iteration (fully coalesced), which is quarter
+// l%U of block j*(32/U)+l/U.  Both iterations' loads are issued before any
+// arithmetic (4 KB in flight per warp at B = 16); load_segment issues them
+// and hash_loaded consumes them, so a caller can do other work in between.
+template <int U>
+__device__ __forceinline__ void load_segment(const HashLane<U> &hl, const uint4 *src4, uint32_t nb, int lane,
+                                             uint64_t pol, uint4 (&v)[2][U]) {
+    constexpr int GPL = HashLane<U>::GPL;
+#pragma unroll
+    for (int it = 0; it < 2; ++it)
+#pragma unroll
+        for (int jj = 0; jj < U; ++jj) {
+            const uint32_t blk = it * 32 + jj * GPL + hl.g;
+            v[it][jj] = blk < nb ? ld_stream(src4 + uint64_t(it) * 32 * U + jj * 32 + lane, pol)
+                                 : make_uint4(0, 0, 0, 0);
+        }
+}
+
+// After the reduce-scatter lane l holds block (l%U)*(32/U) + l/U; one
+// shuffle puts block m on lane m for the scan.  Lane l returns P[it] = the
+// local f1 prefix value of block b0 + 32 it + l (0 past the segment) and
+// every lane the f1 total; blocks below K also take f2: kF2 sums their
+// digests into sum2 (kP2: also each block's in-segment f2 prefix value into
+// p2out, indexed from b0).
+template <int U, bool kF2, bool kP2>
+__device__ __forceinline__ void hash_loaded(const HashLane<U> &hl, const uint4 (&v)[2][U], uint32_t b0, uint32_t nb,
+                                            uint32_t K, int lane, uint64_t (&P)[2], uint64_t &tot1, uint64_t &sum2,
+                                            uint64_t *p2out) {
+    uint64_t carry1 = 0, s2 = 0;   // kP2: s2 is the running f2 prefix (uniform)
+#pragma unroll
+    for (int it = 0; it < 2; ++it) {
+        P[it] = 0;
+        if ((uint32_t)it * 32 >= nb) continue;
+        const uint32_t nvalid = min(32u, nb - it * 32);
+        uint64_t p1[U];
+#pragma unroll
+        for (int jj = 0; jj < U; ++jj) p1[jj] = nh4(v[it][jj], hl.k1);
+        const uint64_t a1 = reduce_scatter<U>(p1, hl.q);
+        const uint32_t kb = b0 + it * 32 + hl.bq;   // block index within the prompt
+        uint64_t dg1 = (uint32_t)hl.bq < nvalid ? fmix64(a1 + uint64_t(kb + 1) * hl.G1) : 0;
+        dg1 = shfl_u64(dg1, hl.src);
+        const uint64_t P1 = warp_incl_scan(dg1, lane) + carry1;
+        P[it] = (uint32_t)lane < nvalid ? P1 : 0;
+        carry1 = shfl_u64(P1, 31);
+        if constexpr (kF2) {
+            if (b0 + it * 32 < K) {                   // second function, blocks < K
+                uint64_t p2[U];
+#pragma unroll
+                for (int jj = 0; jj < U; ++jj) p2[jj] = nh4(v[it][jj], hl.k2);
+                const uint64_t a2 = reduce_scatter<U>(p2, hl.q);
+                const uint64_t dg2 =
+                    ((uint32_t)hl.bq < nvalid && kb < K) ? fmix64(a2 + uint64_t(kb + 1) * hl.G2) : 0;
+                if constexpr (kP2) {
+                    const uint64_t P2 = warp_incl_scan(shfl_u64(dg2, hl.src), lane) + s2;
+                    if ((uint32_t)lane < nvalid && b0 + it * 32 + lane < K) p2out[it * 32 + lane] = P2;
+                    s2 = shfl_u64(P2, 31);
+                } else {
+                    s2 += dg2;
+                }
+            }
+        }
+    }
+    if constexpr (kF2 && !kP2) s2 = warp_sum_u64(s2);
+    tot1 = carry1;
+    sum2 = s2;
+}
+
+template <int U, bool kF2, bool kP2>
+__device__ __forceinline__ void hash_segment(const HashLane<U> &hl, const uint4 *src4, uint32_t b0, uint32_t nb,
+                                             uint32_t K, int lane, uint64_t pol, uint64_t (&P)[2], uint64_t &tot1,
+                                             uint64_t &sum2, uint64_t *p2out) {
+    uint4 v[2][U];
+    load_segment<U>(hl, src4, nb, lane, pol, v);
+    hash_loaded<U, kF2, kP2>(hl, v, b0, nb, K, lane, P, tot1, sum2, p2out);
+}
+
+// Hashing only (dm_hash_prompts and the allocation-free variant): one warp
+// per segment in segment order; writes every block's local prefix value and
+// each segment's totals.
 template <int U, bool kP2>
 __global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__restrict__ tokens) {
     pdl_enter();
-    constexpr int IT = kSegBlocks / 32;
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
     const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t total_segs = d.info->total_segs;
-    constexpr int GPL = 32 / U;  // blocks per load instruction
-    const int q = lane % U, g = lane / U;
-    const int bq = q * GPL + g;                    // block this lane reduces
-    const int src = (lane % GPL) * U + lane / GPL; // lane holding block `lane`
-    uint32_t k1[4], k2[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) { k1[i] = d.K1[4 * q + i]; k2[i] = d.K2[4 * q + i]; }
-    const uint64_t G1 = d.G1, G2 = d.G2;
-
+    const HashLane<U> hl(d, lane);
+    const uint64_t pol = evict_first_policy();
     for (uint32_t seg = gw; seg < total_segs; seg += nwarps) {
         const uint32_t r = d.seg_req[seg];
         const uint32_t j = seg - d.r_segoff[r];
@@ -82,70 +181,39 @@ __global__ void __launch_bounds__(256, 4) k_hash(DevState d, const uint32_t *__r
         const uint32_t b0 = j * kSegBlocks;
         const uint32_t nb = min(kSegBlocks, nblk - b0);
         const uint4 *src4 = reinterpret_cast<const uint4 *>(tokens + d.r_tokoff[r] + uint64_t(b0) * d.B);
-        uint64_t *out = d.plocal + d.r_blkoff[r] + b0;
-        const uint32_t K = min(d.Kf2, nblk);
-        uint4 v[IT][U];
-#pragma unroll
-        for (int it = 0; it < IT; ++it)
-#pragma unroll
-            for (int jj = 0; jj < U; ++jj) {
-                const uint32_t blk = it * 32 + jj * GPL + g;
-                v[it][jj] = blk < nb ? ld_stream(src4 + uint64_t(it) * 32 * U + jj * 32 + lane)
-                                     : make_uint4(0, 0, 0, 0);
-            }
-        uint64_t carry1 = 0, sum2 = 0;   // kP2: sum2 is the running f2 prefix (uniform)
-#pragma unroll
-        for (int it = 0; it < IT; ++it) {
-            if ((uint32_t)it * 32 >= nb) break;
-            const uint32_t nvalid = min(32u, nb - it * 32);
-            uint64_t p1[U];
-#pragma unroll
-            for (int jj = 0; jj < U; ++jj) p1[jj] = nh4(v[it][jj], k1);
-            const uint64_t s1 = reduce_scatter<U>(p1, q);
-            const uint32_t kb = b0 + it * 32 + bq;   // block index within the prompt
-            uint64_t dg1 = (uint32_t)bq < nvalid ? fmix64(s1 + uint64_t(kb + 1) * G1) : 0;
-            dg1 = shfl_u64(dg1, src);
-            const uint64_t P1 = warp_incl_scan(dg1, lane) + carry1;
-            if ((uint32_t)lane < nvalid) out[it * 32 + lane] = P1;
-            carry1 = shfl_u64(P1, 31);
-            if (b0 + it * 32 < K) {                   // second function, blocks < K
-                uint64_t p2[U];
-#pragma unroll
-                for (int jj = 0; jj < U; ++jj) p2[jj] = nh4(v[it][jj], k2);
-                const uint64_t s2 = reduce_scatter<U>(p2, q);
-                const uint64_t dg2 = ((uint32_t)bq < nvalid && kb < K) ? fmix64(s2 + uint64_t(kb + 1) * G2) : 0;
-                if constexpr (kP2) {
-                    const uint64_t P2 = warp_incl_scan(shfl_u64(dg2, src), lane) + sum2;
-                    if ((uint32_t)lane < nvalid && b0 + it * 32 + lane < K)
-                        d.p2local[d.r_blkoff[r] + b0 + it * 32 + lane] = P2;
-                    sum2 = shfl_u64(P2, 31);
-                } else {
-                    sum2 += dg2;
-                }
-            }
-        }
-        if constexpr (!kP2) {
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) sum2 += shfl_xor_u64(sum2, o);
-        }
+        const uint64_t bo = d.r_blkoff[r];
+        uint64_t P[2], tot1, sum2;
+        hash_segment<U, true, kP2>(hl, src4, b0, nb, min(d.Kf2, nblk), lane, pol, P, tot1, sum2,
+                                   kP2 ? d.p2local + bo + b0 : nullptr);
+        uint64_t *out = d.plocal + bo + b0;
+        if ((uint32_t)lane < nb) out[lane] = P[0];
+        if ((uint32_t)lane + 32 < nb) out[lane + 32] = P[1];
         if (lane == 0) {
-            d.seg_total[seg] = carry1;
+            d.seg_total[seg] = tot1;
             d.seg_total2[seg] = sum2;
         }
     }
 }
 
-int hash_grid_size() {
-    static int grid = 0;
-    if (!grid) {
-        int dev = 0, sms = 0, per = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_hash<4, false>, 256, 0);
-        grid = sms * (per > 0 ? per : 1);
+// Grids of the hashing kernels, per device (SM counts may differ).
+namespace {
+constexpr int kGridDevices = 64;
+std::atomic<int> g_grid[kGridDevices][2];
+
+template <typename K>
+int grid_for_device(int which, K kernel) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kGridDevices) return full_grid(kernel, 256);
+    int g = g_grid[dev][which].load(std::memory_order_relaxed);
+    if (!g) {
+        g = full_grid(kernel, 256);
+        g_grid[dev][which].store(g, std::memory_order_relaxed);
     }
-    return grid;
+    return g;
 }
+}  // namespace
+
+int hash_grid_size() { return grid_for_device(0, k_hash<4, false>); }
 
 template <bool kP2>
 static cudaError_t launch_hash_t(const DevState &d, const dm_batch &b, int grid, cudaStream_t st) {
@@ -162,6 +230,624 @@ static cudaError_t launch_hash_t(const DevState &d, const dm_batch &b, int grid,
 
 cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st) {
     return d.ad_step ? launch_hash_t<true>(d, b, grid, st) : launch_hash_t<false>(d, b, grid, st);
+}
+
+// ---------------------------------------------------------------------------
+// Routing: hashing, ring lookup and probes in one kernel.
+//
+// Task order.  A hashing task is one 64-block segment of one prompt.  First
+// come the routing columns: segment j of every request for j < C, column by
+// column, where C covers the longest routing prefix; then the rest of every
+// request's head (its segments below H, which hold the cached run in the
+// workloads here), request after request; then every remaining segment.
+//
+// Warp roles.  In every CTA kHashWarps warps only hash: grid-stride over the
+// tasks, tokens staged through shared memory with cp.async one task ahead,
+// prefix values and totals stored, and, for a head segment, a checked record
+// published for the other warps (SegPub).  The warp that hashes a request's
+// last head segment also puts the request's route task on its CTA's queue.
+// The CTA's kProbeWarps warps work off that queue, so the dependent memory
+// round trips of routing and probing (App. A.3.2's metadata queries) never
+// hold up the token stream:
+//   - A route task, once every head segment of its request is published,
+//     sums their carries, computes the two ring positions, searches both
+//     rings (Sec. 3.4, App. A.1.3), applies the distinct fix (Sec. 3.2) and
+//     tests the first block of every head segment on both candidates.  On a
+//     candidate c_f the first head segment whose first block is missing,
+//     j_f, bounds the leading run: the first miss is that block or lies in
+//     a segment below it.  It publishes the route (RoutePub) and queues a
+//     probe task for each segment below the larger bound.  When every head
+//     segment's first block is resident on c_f, it probes c_f itself from
+//     block 0, hashing the prompt as it goes, until the run ends.
+//   - A probe task probes its segment's 64 blocks on each candidate whose
+//     bound lies beyond it (keys from the stored prefix values, checked
+//     against the segment's record, plus the carry of the segments before
+//     it) and lowers that candidate's first miss (atomic min).  The smallest
+//     first miss over the probed segments is exactly the leading run: every
+//     segment before the true first miss is probed and reports none, the one
+//     holding it reports it.
+// A task whose inputs are not published yet goes back on the queue; after
+// kRetries tries it moves to a list that the kernel's last CTA to finish
+// works off, when everything is published.  Nothing waits on a warp of
+// another CTA.  The segment carries of the whole batch, which the commit
+// needs, and the route outputs are produced by the choice kernel's launch.
+
+// Request holding task x of a part: the largest r < n with off[r] <= x
+// (off: exclusive offsets of that part, nondecreasing).
+__device__ __forceinline__ uint32_t find_req(const uint32_t *off, uint32_t n, uint32_t x) {
+    uint32_t lo = 0, hi = n;   // off[lo] <= x < off[hi] (off[n] taken as infinite)
+    while (hi - lo > 1) {
+        const uint32_t mid = (lo + hi) >> 1;
+        if (__ldg(off + mid) <= x) lo = mid;
+        else hi = mid;
+    }
+    return lo;
+}
+
+// Loads through L2 (data written by other warps during this kernel).
+__device__ __forceinline__ void ld_cg2(const void *p, uint64_t &a, uint64_t &b) {
+    asm volatile("ld.global.cg.v2.u64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(__cvta_generic_to_global(p)));
+}
+__device__ __forceinline__ void st_v2(void *p, uint64_t a, uint64_t b) {
+    asm volatile("st.global.v2.u64 [%0], {%1, %2};" ::"l"(__cvta_generic_to_global(p)), "l"(a), "l"(b) : "memory");
+}
+
+__device__ __forceinline__ bool seg_pub_read(const SegPub *p, uint64_t E, uint64_t &t1, uint64_t &t2, uint64_t &pf,
+                                             uint64_t &pk, uint64_t &px) {
+    uint64_t c;
+    ld_cg2(&p->t1, t1, t2);
+    ld_cg2(&p->pf, pf, pk);
+    ld_cg2(&p->px, px, c);
+    return c == (t1 ^ t2 ^ pf ^ pk ^ px ^ E);
+}
+
+__device__ __forceinline__ void seg_pub_write(SegPub *p, uint64_t E, uint64_t t1, uint64_t t2, uint64_t pf,
+                                              uint64_t pk, uint64_t px) {
+    st_v2(&p->t1, t1, t2);
+    st_v2(&p->pf, pf, pk);
+    st_v2(&p->px, px, t1 ^ t2 ^ pf ^ pk ^ px ^ E);
+}
+
+struct RouteView {
+    const Slot *t1, *t2;
+    uint64_t f1, f2;
+    uint32_t j1, j2;
+};
+
+__device__ __forceinline__ bool route_pub_read(const RoutePub *p, uint64_t E, RouteView &v) {
+    uint64_t cc, t1, t2, f1, f2, js, pad, chk;
+    ld_cg2(&p->cc, cc, t1);
+    ld_cg2(&p->tab2, t2, f1);
+    ld_cg2(&p->fr2, f2, js);
+    ld_cg2(&p->pad, pad, chk);
+    if (chk != (cc ^ t1 ^ t2 ^ f1 ^ f2 ^ js ^ E)) return false;
+    v.t1 = reinterpret_cast<const Slot *>(t1);
+    v.t2 = reinterpret_cast<const Slot *>(t2);
+    v.f1 = f1;
+    v.f2 = f2;
+    v.j1 = (uint32_t)(js & 0xFFFF);
+    v.j2 = (uint32_t)((js >> 16) & 0xFFFF);
+    return true;
+}
+
+constexpr uint32_t kNoMiss = 0xFFFFFFFFu;
+constexpr int kHashWarps = 6, kProbeWarps = 2;   // warp roles of a routing CTA
+constexpr uint32_t kQCap = 512;                  // entries of a CTA's task queue
+constexpr uint32_t kRetries = 1024;              // tries of a task before it goes to the last CTA
+
+// First miss among blocks base + 32 k + lane (k < 2, one segment) below
+// `end` on the candidates flagged (kNoMiss if none).  Whole warp.
+__device__ __forceinline__ void probe_segment(const uint64_t (&key)[2], uint32_t base, uint32_t end, bool do1,
+                                              bool do2, const RouteView &rv, uint64_t mask, uint32_t *err,
+                                              uint64_t lim, int lane, uint32_t &m1, uint32_t &m2) {
+    uint64_t home[2];
+    Slot s1[2], s2[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t b = base + 32 * k + lane;
+        home[k] = group_home(group_anchor(key[k], lane), b, mask);
+        const bool inb = b < end;
+        s1[k] = (inb && do1) ? load_slot(rv.t1 + home[k]) : Slot{0, 0};
+        s2[k] = (inb && do2) ? load_slot(rv.t2 + home[k]) : Slot{0, 0};
+    }
+    m1 = kNoMiss;
+    m2 = kNoMiss;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t b = base + 32 * k + lane;
+        const bool inb = b < end;
+        if (do1) {
+            const bool miss = inb && !resident_at(rv.t1, mask, key[k], home[k], rv.f1, s1[k], err, lim);
+            const uint32_t bal = __ballot_sync(0xffffffffu, miss);
+            if (bal && m1 == kNoMiss) m1 = base + 32 * k + __ffs(bal) - 1;
+        }
+        if (do2) {
+            const bool miss = inb && !resident_at(rv.t2, mask, key[k], home[k], rv.f2, s2[k], err, lim);
+            const uint32_t bal = __ballot_sync(0xffffffffu, miss);
+            if (bal && m2 == kNoMiss) m2 = base + 32 * k + __ffs(bal) - 1;
+        }
+    }
+}
+
+// Probe c_f from block 0 on the candidates flagged, hashing the prompt here
+// segment by segment (f1 only), until each run ends; lowers their first
+// miss.  Whole warp (rare: the run reaches the end of the head).
+template <int U>
+__device__ __noinline__ void probe_from_start(const DevState &d, const uint32_t *tokens, uint64_t pol, uint32_t r,
+                                              uint32_t nblk, bool go1, bool go2, const RouteView &rv, int lane) {
+    const HashLane<U> hl(d, lane);
+    const uint4 *tok4 = reinterpret_cast<const uint4 *>(tokens + d.r_tokoff[r]);
+    const uint32_t nseg = (nblk + kSegBlocks - 1) / kSegBlocks;
+    const uint64_t mask = d.S - 1;
+    uint32_t q1 = go1 ? kNoMiss : 0, q2 = go2 ? kNoMiss : 0;
+    uint64_t run = 0;
+    for (uint32_t j = 0; j < nseg && (q1 == kNoMiss || q2 == kNoMiss); ++j) {
+        const uint32_t c0 = j * kSegBlocks, cn = min(kSegBlocks, nblk - c0);
+        uint64_t P[2], tot, s2u;
+        hash_segment<U, false, false>(hl, tok4 + uint64_t(c0) * d.B / 4, c0, cn, 0, lane, pol, P, tot, s2u,
+                                      nullptr);
+        const uint64_t key[2] = {cache_key(P[0] + run, d.Sc), cache_key(P[1] + run, d.Sc)};
+        uint32_t e1, e2;
+        probe_segment(key, c0, c0 + cn, q1 == kNoMiss, q2 == kNoMiss, rv, mask, d.err, d.loop_limit, lane, e1, e2);
+        if (q1 == kNoMiss && e1 != kNoMiss) q1 = e1;
+        if (q2 == kNoMiss && e2 != kNoMiss) q2 = e2;
+        run += tot;
+    }
+    if (lane == 0) {
+        if (go1 && q1 != kNoMiss) atomicMin(d.r_m1 + r, q1);
+        if (go2 && q2 != kNoMiss) atomicMin(d.r_m2 + r, q2);
+    }
+}
+
+// The route task of request r.  Returns false, changing nothing, when a head
+// segment of r is not published yet; else the number of head segments that
+// still need a probe task (segments 0 .. return-1).  Whole warp; not inlined.
+template <int U, bool kAdapt>
+__device__ __noinline__ int route_task(const DevState &d, const uint32_t *tokens, uint64_t E, uint64_t pol,
+                                       uint32_t r, int lane) {
+    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
+    const uint32_t nseg = (nblk + kSegBlocks - 1) / kSegBlocks, hs = min(nseg, d.H);
+    uint64_t t1 = 0, t2 = 0, pf = 0, pk = 0, px = 0;
+    const bool ok = (uint32_t)lane >= hs || seg_pub_read(d.seg_pub + s0 + lane, E, t1, t2, pf, pk, px);
+    if (!__all_sync(0xffffffffu, ok)) return -1;
+    const uint64_t carry = warp_incl_scan(t1, lane) - t1;   // lane s: f1 carry into head segment s
+    uint64_t pos1, pos2;
+    uint32_t K;
+    if constexpr (kAdapt) {
+        __threadfence();   // the head's prefix values were fenced before their records
+        adaptive_positions(d, r, nblk, d.r_blkoff[r], lane, carry, warp_incl_scan(t2, lane) - t2, pos1, pos2, K);
+    } else {
+        K = min(d.Kroute, nblk);
+        const uint32_t sK = (K - 1) / kSegBlocks;
+        pos1 = fmix64((shfl_u64(carry, sK) + shfl_u64(pk, sK)) ^ d.Sr1);
+        pos2 = fmix64(warp_sum_u64((uint32_t)lane <= sK ? t2 : 0) ^ d.Sr2);
+    }
+    uint32_t lb1, lb2;
+    ring_search2(d, pos1, pos2, lane, lb1, lb2);
+    const uint32_t a = d.ring[0].owner[lb1];
+    const uint32_t raw2 = d.ring[1].owner[lb2];
+    const uint32_t b = raw2 != a ? raw2 : d.next_live[a];
+    RouteView rv;
+    rv.t1 = d.table[a];
+    rv.t2 = d.table[b];
+    rv.f1 = d.log_front[a];   // resident: record at or after the front (as of the batch's start)
+    rv.f2 = d.log_front[b];
+    const uint64_t mask = d.S - 1;
+    // first block of every head segment on both candidates (lane s: segment s)
+    bool miss1 = true, miss2 = true;
+    if ((uint32_t)lane < hs) {
+        const uint64_t key = cache_key(carry + pf, d.Sc);
+        const uint64_t home = group_home(key, 0, mask);   // a segment's first block anchors its own group
+        miss1 = !resident_at(rv.t1, mask, key, home, rv.f1, load_slot(rv.t1 + home), d.err, d.loop_limit);
+        miss2 = !resident_at(rv.t2, mask, key, home, rv.f2, load_slot(rv.t2 + home), d.err, d.loop_limit);
+    }
+    // lanes >= hs count as missing: a bound of hs or more means every head
+    // segment's first block is resident
+    uint32_t j1 = __ffs(__ballot_sync(0xffffffffu, miss1)) - 1, j2 = __ffs(__ballot_sync(0xffffffffu, miss2)) - 1;
+    const bool full1 = j1 >= hs, full2 = j2 >= hs;
+    if (lane == 0) {
+        d.r_K[r] = K;
+        d.r_c1[r] = a;
+        d.r_c2[r] = b;
+        if (!full1) atomicMin(d.r_m1 + r, j1 * kSegBlocks);
+        if (!full2) atomicMin(d.r_m2 + r, j2 * kSegBlocks);
+    }
+    if (full1 || full2) probe_from_start<U>(d, tokens, pol, r, nblk, full1, full2, rv, lane);
+    if (full1) j1 = 0;   // done here: no probe task on that candidate
+    if (full2) j2 = 0;
+    if (lane == 0) {
+        const uint64_t cc = a | uint64_t(b) << 32, js = j1 | uint64_t(j2) << 16 | uint64_t(K) << 32;
+        const uint64_t t1p = reinterpret_cast<uint64_t>(rv.t1), t2p = reinterpret_cast<uint64_t>(rv.t2);
+        RoutePub *p = d.r_route + r;
+        st_v2(&p->cc, cc, t1p);
+        st_v2(&p->tab2, t2p, rv.f1);
+        st_v2(&p->fr2, rv.f2, js);
+        st_v2(&p->pad, 0, cc ^ t1p ^ t2p ^ rv.f1 ^ rv.f2 ^ js ^ E);
+    }
+    return (int)max(j1, j2);
+}
+
+// The probe task of head segment j of request r.  Returns false, changing
+// nothing, when an input is not published (or not visible) yet.  Whole warp.
+__device__ __forceinline__ bool probe_task(const DevState &d, uint64_t E, uint32_t r, uint32_t j, int lane) {
+    RouteView rv;
+    const bool have = route_pub_read(d.r_route + r, E, rv);
+    if (!__all_sync(0xffffffffu, have)) return false;
+    const uint32_t b0 = j * kSegBlocks;
+    const bool do1 = j < rv.j1 && __ldcg(d.r_m1 + r) > b0, do2 = j < rv.j2 && __ldcg(d.r_m2 + r) > b0;
+    if (!do1 && !do2) return true;   // a miss before this segment is known already
+    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
+    const uint32_t nb = min(kSegBlocks, nblk - b0);
+    // carries of the segments before it, its own record, its stored prefix values
+    uint64_t t1 = 0, t2, pf, pk, px = 0;
+    const bool ok = (uint32_t)lane > j || seg_pub_read(d.seg_pub + s0 + lane, E, t1, t2, pf, pk, px);
+    const uint64_t *pl = d.plocal + d.r_blkoff[r] + b0;
+    const uint64_t P0 = (uint32_t)lane < nb ? __ldcg(pl + lane) : 0;
+    const uint64_t P1 = (uint32_t)lane + 32 < nb ? __ldcg(pl + lane + 32) : 0;
+    if (!__all_sync(0xffffffffu, ok)) return false;
+    uint64_t x = P0 ^ P1;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) x ^= shfl_xor_u64(x, o);
+    if (x != shfl_u64(px, j)) return false;   // some prefix value not visible yet
+    const uint64_t carry = warp_sum_u64((uint32_t)lane < j ? t1 : 0);
+    const uint64_t key[2] = {cache_key(P0 + carry, d.Sc), cache_key(P1 + carry, d.Sc)};
+    uint32_t m1, m2;
+    probe_segment(key, b0, b0 + nb, do1, do2, rv, d.S - 1, d.err, d.loop_limit, lane, m1, m2);
+    if (lane == 0) {
+        if (do1 && m1 != kNoMiss) atomicMin(d.r_m1 + r, m1);
+        if (do2 && m2 != kNoMiss) atomicMin(d.r_m2 + r, m2);
+    }
+    return true;
+}
+
+// Token staging: a hashing warp copies its next task's segment into its own
+// shared-memory stage with cp.async while it hashes the current one.  Lane l
+// copies and later reads the same 16-byte pieces as load_segment (coalesced
+// in global memory, conflict-free in shared memory); pieces past the
+// segment are zero-filled.
+template <int U>
+struct HP {
+    static constexpr int kWarps = kHashWarps + kProbeWarps;
+    static constexpr int kThreads = 32 * kWarps;
+    static constexpr uint32_t kStage = 64 * U;   // uint4 per stage: one segment
+    static constexpr size_t kSmem = size_t(kHashWarps) * 2 * kStage * sizeof(uint4);
+};
+
+__device__ __forceinline__ void cp_async16(uint4 *sdst, const uint4 *gsrc, bool valid, uint64_t pol) {
+    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(sdst);
+    asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;" ::"r"(sa),
+                 "l"(__cvta_generic_to_global(gsrc)), "r"(valid ? 16 : 0), "l"(pol)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+template <int U>
+__device__ __forceinline__ void stage_segment(const HashLane<U> &hl, uint4 *stage, const uint4 *src4, uint32_t nb,
+                                              int lane, uint64_t pol) {
+    constexpr int GPL = HashLane<U>::GPL;
+#pragma unroll
+    for (int it = 0; it < 2; ++it)
+#pragma unroll
+        for (int jj = 0; jj < U; ++jj) {
+            const uint32_t blk = it * 32 + jj * GPL + hl.g;
+            const bool valid = blk < nb;
+            const uint4 *g = src4 + uint64_t(it) * 32 * U + jj * 32 + lane;
+            cp_async16(stage + (it * U + jj) * 32 + lane, valid ? g : src4, valid, pol);
+        }
+}
+
+template <int U>
+__device__ __forceinline__ void read_stage(const uint4 *stage, int lane, uint4 (&v)[2][U]) {
+#pragma unroll
+    for (int it = 0; it < 2; ++it)
+#pragma unroll
+        for (int jj = 0; jj < U; ++jj) v[it][jj] = stage[(it * U + jj) * 32 + lane];
+}
+
+// A CTA's task queue in shared memory: a bounded many-producer,
+// many-consumer ring in which every slot carries a sequence number (slot
+// k is free for the producer at position p when its number is p, holds
+// that producer's entry when it is p + 1, and is free again for position
+// p + kQCap once consumed), so neither side ever reads a half-written
+// entry.  An entry is r | j << 32 | route flag << 40 | (tries + 1) << 48,
+// never 0 (what an empty queue returns).
+struct CtaQueue {
+    uint64_t buf[kQCap];
+    uint32_t seq[kQCap];
+    uint32_t head, tail;
+    uint32_t hash_done;   // hashing warps out of tasks
+    uint32_t busy;        // probing warps inside a task
+};
+
+__device__ __forceinline__ uint64_t qentry(uint32_t r, uint32_t j, bool route, uint32_t tries) {
+    return uint64_t(r) | uint64_t(j) << 32 | uint64_t(route) << 40 | uint64_t(tries + 1) << 48;   // never 0
+}
+
+// Push one entry (one thread); a full queue sends it to the last CTA's list.
+__device__ __forceinline__ void q_push(CtaQueue &q, const DevState &d, uint64_t e) {
+    uint32_t pos = *(volatile uint32_t *)&q.tail;
+    for (uint32_t k = 0; k < (1u << 20); ++k) {
+        const uint32_t sq = *(volatile uint32_t *)&q.seq[pos % kQCap];
+        const int32_t dif = (int32_t)(sq - pos);
+        if (dif == 0) {
+            const uint32_t got = atomicCAS(&q.tail, pos, pos + 1);
+            if (got == pos) {
+                *(volatile uint64_t *)&q.buf[pos % kQCap] = e;
+                __threadfence_block();
+                *(volatile uint32_t *)&q.seq[pos % kQCap] = pos + 1;
+                return;
+            }
+            pos = got;
+        } else if (dif < 0) {
+            break;   // full
+        } else {
+            pos = *(volatile uint32_t *)&q.tail;
+        }
+    }
+    d.fix_list[atomicAdd(&d.info->fix_n, 1u)] = e;
+}
+
+// Pop one entry (one thread); 0 when the queue is empty.  A popped entry
+// counts its warp busy until the warp is done with it.
+__device__ __forceinline__ uint64_t q_pop(CtaQueue &q) {
+    uint32_t pos = *(volatile uint32_t *)&q.head;
+    for (uint32_t k = 0; k < (1u << 20); ++k) {
+        const uint32_t sq = *(volatile uint32_t *)&q.seq[pos % kQCap];
+        const int32_t dif = (int32_t)(sq - (pos + 1));
+        if (dif == 0) {
+            atomicAdd(&q.busy, 1u);
+            const uint32_t got = atomicCAS(&q.head, pos, pos + 1);
+            if (got == pos) {
+                __threadfence_block();
+                const uint64_t e = *(volatile uint64_t *)&q.buf[pos % kQCap];
+                __threadfence_block();
+                *(volatile uint32_t *)&q.seq[pos % kQCap] = pos + kQCap;
+                return e;
+            }
+            atomicSub(&q.busy, 1u);
+            pos = got;
+        } else if (dif < 0) {
+            return 0;   // empty
+        } else {
+            pos = *(volatile uint32_t *)&q.head;
+        }
+    }
+    return 0;
+}
+
+template <int U, bool kAdapt>
+__global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_constant__ DevState d,
+                                                                   const uint32_t *__restrict__ tokens, uint64_t E) {
+    pdl_enter();
+    extern __shared__ __align__(16) uint4 s_stage[];
+    __shared__ CtaQueue q;
+    __shared__ uint32_t s_go, s_last;
+    if (threadIdx.x == 0) {
+        s_go = !has_err(d.err);   // one decision per CTA (the CTA meets barriers below)
+        q.head = q.tail = q.hash_done = q.busy = 0;
+    }
+    for (uint32_t i = threadIdx.x; i < kQCap; i += blockDim.x) q.seq[i] = i;
+    __syncthreads();
+    if (!s_go) return;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const uint64_t pol = evict_first_policy();
+    if (wid < kHashWarps) {
+        // ---- hashing warp ----
+        const uint32_t nhw = gridDim.x * kHashWarps;
+        const uint32_t gw = blockIdx.x * kHashWarps + wid;
+        const uint32_t n = d.info->n, ncol = d.info->col_tasks, nhr = d.info->head_segs;
+        const uint32_t total = d.info->tasks;
+        const HashLane<U> hl(d, lane);
+        uint4 *const stage = s_stage + wid * 2 * HP<U>::kStage;
+        // request, segment and layout of the task whose copy is issued next
+        // (nb = 0: a routing column past the end of the prompt, nothing to do)
+        uint32_t r = 0, j = 0, nblk = 0, segoff = 0, nb = 0;
+        uint64_t tokoff = 0, bo = 0;
+        auto issue = [&](uint32_t t, uint4 *st) {
+            if (t < ncol) {
+                j = t / n;
+                r = t - j * n;
+            } else if (t < ncol + nhr) {
+                r = find_req(d.r_hoff, n, t - ncol);
+                j = d.Ccols + (t - ncol - __ldg(d.r_hoff + r));
+            } else {
+                r = find_req(d.r_toff, n, t - ncol - nhr);
+                j = d.H + (t - ncol - nhr - __ldg(d.r_toff + r));
+            }
+            nblk = d.r_nblk[r];
+            segoff = d.r_segoff[r];
+            tokoff = d.r_tokoff[r];
+            bo = d.r_blkoff[r];
+            nb = j * kSegBlocks < nblk ? min(kSegBlocks, nblk - j * kSegBlocks) : 0;
+            if (nb)
+                stage_segment<U>(hl, st,
+                                 reinterpret_cast<const uint4 *>(tokens + tokoff + uint64_t(j) * kSegBlocks * d.B),
+                                 nb, lane, pol);
+        };
+        if (gw < total) issue(gw, stage);
+        cp_async_commit();
+        uint32_t it = 0;
+        for (uint32_t t = gw; t < total; t += nhw, ++it) {
+            const uint32_t rr = r, jj = j, nbk = nblk, seg = segoff + j, cnb = nb;
+            const uint64_t bof = bo;
+            const uint32_t b0 = jj * kSegBlocks;
+            if (t + nhw < total) issue(t + nhw, stage + ((it + 1) & 1) * HP<U>::kStage);
+            cp_async_commit();
+            cp_async_wait<1>();   // this task's copy is complete
+            if (cnb == 0) continue;
+            uint4 v[2][U];
+            read_stage<U>(stage + (it & 1) * HP<U>::kStage, lane, v);
+            uint64_t P[2], tot1, sum2;
+            hash_loaded<U, true, kAdapt>(hl, v, b0, cnb, min(d.Kf2, nbk), lane, P, tot1, sum2,
+                                         kAdapt ? d.p2local + bof + b0 : nullptr);
+            uint64_t *out = d.plocal + bof + b0;
+            if ((uint32_t)lane < cnb) out[lane] = P[0];
+            if ((uint32_t)lane + 32 < cnb) out[lane + 32] = P[1];
+            if (lane == 0) {
+                d.seg_total[seg] = tot1;
+                d.seg_total2[seg] = sum2;
+                d.seg_req[seg] = rr;
+            }
+            const uint32_t hs = min((nbk + kSegBlocks - 1) / kSegBlocks, d.H);
+            if (jj < hs) {
+                // publish the head segment: totals, its first block's and block
+                // K-1's prefix values, and the xor of what it stored in plocal
+                const uint32_t kk = min(d.Kroute, nbk) - 1 - b0;   // block K-1 in this segment, if any
+                const uint64_t pk = shfl_u64(kk < 32 ? P[0] : P[1], kk & 31);
+                const uint64_t pf = shfl_u64(P[0], 0);
+                uint64_t px = P[0] ^ P[1];
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) px ^= shfl_xor_u64(px, o);
+                if constexpr (kAdapt) {
+                    __threadfence();   // the route task reads the head's prefix values (plocal, p2local) directly
+                    __syncwarp();
+                }
+                if (lane == 0) {
+                    seg_pub_write(d.seg_pub + seg, E, tot1, sum2, pf, kk < kSegBlocks ? pk : 0, px);
+                    if (jj + 1 == hs) q_push(q, d, qentry(rr, 0, true, 0));   // the request's route task
+                }
+            }
+        }
+        cp_async_wait<0>();
+        if (lane == 0) atomicAdd(&q.hash_done, 1u);
+    } else {
+        // ---- probing warp: work off the CTA's queue ----
+        // (bounded: kIdleLimit idle polls in a row, a few seconds at most,
+        // then the call ends with DM_ERR_TIMEOUT)
+        constexpr uint32_t kIdleLimit = 1u << 22;
+        for (uint32_t idle = 0;;) {
+            uint64_t e = lane == 0 ? q_pop(q) : 0;
+            e = shfl_u64(e, 0);
+            if (e == 0) {
+                // done once the hashing warps are done, no probing warp holds
+                // a task (it might queue more) and the queue is empty
+                const bool fin = *(volatile uint32_t *)&q.hash_done == kHashWarps &&
+                                 *(volatile uint32_t *)&q.busy == 0 &&
+                                 *(volatile uint32_t *)&q.head == *(volatile uint32_t *)&q.tail;
+                if (__shfl_sync(0xffffffffu, fin, 0)) break;
+                if (++idle >= kIdleLimit) {
+                    if (lane == 0) set_err(d.err, DM_ERR_TIMEOUT);
+                    break;
+                }
+                __nanosleep(idle < 64 ? 64 : 512);
+                continue;
+            }
+            idle = 0;
+            const uint32_t r = (uint32_t)e, j = (uint32_t)(e >> 32) & 0xFF;
+            const bool route = (e >> 40) & 1;
+            const uint32_t tries = (uint32_t)(e >> 48) - 1;
+            bool done;
+            if (route) {
+                const int np = route_task<U, kAdapt>(d, tokens, E, pol, r, lane);
+                done = np >= 0;
+                if (done && lane == 0)
+                    for (int k = 0; k < np; ++k) q_push(q, d, qentry(r, (uint32_t)k, false, 0));
+            } else {
+                done = probe_task(d, E, r, j, lane);
+            }
+            if (lane == 0) {
+                if (!done) {
+                    // inputs of a warp elsewhere not published yet: back on the queue
+                    if (tries + 1 < kRetries) q_push(q, d, qentry(r, j, route, tries + 1));
+                    else d.fix_list[atomicAdd(&d.info->fix_n, 1u)] = qentry(r, j, route, 0);
+                    if (tries > 8) __nanosleep(1000);
+                }
+                atomicSub(&q.busy, 1u);
+            }
+            __syncwarp();
+        }
+    }
+    // the last CTA to finish works off the list: route tasks first (every
+    // head segment is published by then, and each queues its probes here),
+    // then the probes
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        s_last = atomicAdd(&d.info->cta_done, 1u) + 1 == gridDim.x;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    const uint32_t nf = *(volatile uint32_t *)&d.info->fix_n;
+    const uint32_t nw = blockDim.x >> 5;
+    for (uint32_t i = wid; i < nf; i += nw) {
+        const uint64_t e = d.fix_list[i];
+        if (!((e >> 40) & 1)) continue;
+        const uint32_t r = (uint32_t)e;
+        const int np = route_task<U, kAdapt>(d, tokens, E, pol, r, lane);
+        if (np < 0) {
+            if (lane == 0) set_err(d.err, DM_ERR_TIMEOUT);   // cannot happen: everything is published by now
+            continue;
+        }
+        for (int k = 0; k < np; ++k)
+            if (!probe_task(d, E, r, (uint32_t)k, lane) && lane == 0) set_err(d.err, DM_ERR_TIMEOUT);
+    }
+    __syncthreads();
+    for (uint32_t i = wid; i < nf; i += nw) {
+        const uint64_t e = d.fix_list[i];
+        if ((e >> 40) & 1) continue;
+        if (!probe_task(d, E, (uint32_t)e, (uint32_t)(e >> 32) & 0xFF, lane) && lane == 0)
+            set_err(d.err, DM_ERR_TIMEOUT);
+    }
+}
+
+// Launch shape of the routing kernel per device and block size: its
+// shared-memory stages are set up once, the grid fills every SM.
+template <int U, bool kAdapt>
+static cudaError_t launch_hash_probe_u(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st) {
+    static std::atomic<int> grids[kGridDevices];
+    int dev = 0;
+    DM_TRY(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= kGridDevices) return cudaErrorInvalidDevice;
+    int grid = grids[dev].load(std::memory_order_relaxed);
+    if (!grid) {
+        DM_TRY(cudaFuncSetAttribute(k_hash_probe<U, kAdapt>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)HP<U>::kSmem));
+        int sms = 0, per = 0;
+        DM_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+        DM_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_hash_probe<U, kAdapt>, HP<U>::kThreads,
+                                                             HP<U>::kSmem));
+        grid = sms * (per > 0 ? per : 1);
+        grids[dev].store(grid, std::memory_order_relaxed);
+    }
+    DM_TRY(launch_pdl(k_hash_probe<U, kAdapt>, grid, HP<U>::kThreads, HP<U>::kSmem, st, d, b.tokens, E));
+    return cudaGetLastError();
+}
+
+template <bool kAdapt>
+static cudaError_t launch_hash_probe_t(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st) {
+    switch (d.B) {
+        case 4: return launch_hash_probe_u<1, kAdapt>(d, b, E, st);
+        case 8: return launch_hash_probe_u<2, kAdapt>(d, b, E, st);
+        case 16: return launch_hash_probe_u<4, kAdapt>(d, b, E, st);
+        case 32: return launch_hash_probe_u<8, kAdapt>(d, b, E, st);
+        case 64: return launch_hash_probe_u<16, kAdapt>(d, b, E, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_hash_probe(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st) {
+    if (b.n == 0) return cudaSuccess;
+    return d.ad_step ? launch_hash_probe_t<true>(d, b, E, st) : launch_hash_probe_t<false>(d, b, E, st);
+}
+
+// Carries of every segment of the batch and the route outputs (the
+// cluster-wide rules' probes need the carries before their choice kernel;
+// the pair rules' choice kernels do this in their own launch).
+__global__ void k_carries(DevState d, dm_route_out o, uint32_t n) {
+    pdl_enter();
+    if (has_err(d.err)) return;
+    carries_role(d, o, n, blockIdx.x, gridDim.x);
+}
+
+cudaError_t launch_carries(const DevState &d, const dm_route_out &o, uint32_t n, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    DM_TRY(launch_pdl(k_carries, (n + 7) / 8, 256, 0, st, d, o, n));
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------

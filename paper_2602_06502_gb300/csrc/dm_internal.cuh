@@ -19,6 +19,11 @@ constexpr uint32_t kEvChunk = 1024;      // log records per eviction / compactio
 constexpr uint32_t kRbChunk = 4096;      // index slots per rebuild chunk
 constexpr uint64_t kSpinLimit = 1ull << 26; // bound of every data-dependent device loop
 constexpr uint32_t kGroup = 8;           // consecutive blocks of a prompt homed in one 128-byte index line
+constexpr uint32_t kMaxD = 8;            // rings (hash functions) of the d-candidate routing path
+// Head segments per request in the routing kernel's hashing order (the
+// routing prefix and the usual cached run: 24 x 64 blocks = 24,576 tokens at
+// B = 16; at most 32, the carries of a head are one warp scan).
+constexpr uint32_t kHeadSegs = 24;
 
 // One queued request (56 bytes).
 struct QEntry {
@@ -130,16 +135,44 @@ struct AdCount {
     uint32_t count, depth;   // requests that reached the node; its length in blocks
 };
 
+// Values one warp of the routing kernel publishes for the others, without
+// fences: every record ends with chk, the xor of its other words and the
+// batch's epoch mask E (a different value per routing call), so a reader
+// that sees chk match knows every word is this batch's (a torn or stale
+// read fails the check except with probability about 2^-64) and retries.
+// A head segment's record (48 bytes): its f1 total t1, its f2 partial t2,
+// the local f1 prefix value of its first block pf and of block K-1 when that
+// block lies in it (pk), and px, the xor of all its blocks' local f1 prefix
+// values as stored in plocal (a reader of those values checks them
+// against it the same way).
+struct __align__(16) SegPub {
+    uint64_t t1, t2, pf, pk, px, chk;
+};
+// A routed request's record (64 bytes): cc = c1 | c2 << 32, both
+// candidates' index buffers and log fronts, and js = j1 | j2 << 16 | K << 32
+// (j_f: the head segments below it still need a probe on c_f: the first
+// head segment whose first block is not resident on c_f, or 0 when the
+// route task probed c_f itself).
+struct __align__(16) RoutePub {
+    uint64_t cc, tab1, tab2, fr1, fr2, js, pad, chk;
+};
+
 // Per-batch values produced on the device.
 struct BatchInfo {
     uint64_t total_blocks;
     uint32_t total_segs;
     uint32_t n;
+    uint32_t head_segs;     // routing: head segments past the routing columns (the second part)
+    uint32_t col_tasks;     // routing: n x the routing columns (the first part)
+    uint32_t tasks;         // routing: tasks of the routing kernel (all three parts)
+    uint32_t pad0;
     uint64_t clock_base;    // commit clock before this batch's touches
     uint32_t final_dirty;   // a rebalance moved a request of this batch
     uint32_t mc_chunks;     // log-compaction chunks of this commit
     uint32_t mr_chunks;     // index-rebuild chunks of this commit
     uint32_t both_over;     // a request of this batch estimated TTFT > SLO on both candidates
+    uint32_t fix_n;         // routing: entries of the last CTA's list
+    uint32_t cta_done;      // routing: CTAs of the routing kernel that finished
 };
 
 struct Ring {
@@ -164,13 +197,21 @@ struct DevState {
     AdCount *ad_cnt;                // node counts of the current window
     uint64_t ad_cnt_mask;
     uint64_t max_blocks, max_segs, T, S, logcap;
+    uint64_t loop_limit;            // 0, or the test cap of the index's bucket walks and touch retries
     uint64_t rb_thr;                // an index is rebuilt when its taken slots would pass this
     uint32_t Q;
     // key material
     uint32_t K1[64], K2[64];
     uint64_t G1, G2, Sc, Sr1, Sr2, Sv1, Sv2;
-    // rings (both have R entries)
-    Ring ring[2];
+    // functions 3..kMaxD of the d-candidate path: salts and seeds (index f - 2
+    // for 0-based f >= 2), NH keys in device memory (64 words per function)
+    uint64_t Gx[kMaxD - 2], Srx[kMaxD - 2], Svx[kMaxD - 2];
+    const uint32_t *Kx;
+    uint32_t nrings;                // rings kept: 2, or the d-candidate path's d when larger
+    uint32_t nd;                    // candidates of the d-candidate path (0: DualMap's two)
+    uint32_t *rd_cand, *rd_hit;     // d-candidate path: per request, nd candidates and their hit tokens
+    // rings (all have R entries)
+    Ring ring[kMaxD];
     uint32_t R, nlev;
     uint64_t lev_off[kMaxLevels];   // offset of level k (k >= 1) inside tree
     uint64_t lev_n[kMaxLevels];     // entries in level k (lev_n[0] = R)
@@ -204,6 +245,20 @@ struct DevState {
     uint32_t *r_L, *r_nblk, *r_segoff;
     uint64_t *r_tokoff, *r_blkoff;
     uint32_t *seg_req;
+    // routing order of the hashing tasks: the routing columns (segment j < Ccols
+    // of every request), then the rest of each request's head (segments
+    // below H), then the rest; per request the exclusive offsets of the last
+    // two parts
+    uint32_t H, Ccols;              // head segments, routing columns (segments holding any routing prefix)
+    uint32_t *r_hoff, *r_toff;
+    // routing kernel's exchange between warps (see dm_hash.cu): what each
+    // head segment and each routed request publish, the first miss found so
+    // far on each candidate (0xFFFFFFFF: none yet), and the probes left to
+    // the kernel's last CTA
+    SegPub *seg_pub;
+    RoutePub *r_route;
+    uint32_t *r_m1, *r_m2;
+    uint64_t *fix_list;             // entries of the routing kernel's task queues (r, segment, kind)
     uint64_t *seg_total, *seg_carry, *plocal;
     uint64_t *p2local;              // adaptive only: per block < Kf2, in-segment prefix of its f2 digests
     uint32_t *r_K;                  // per request: the hash prefix length it was routed with
@@ -211,7 +266,7 @@ struct DevState {
     uint32_t *seg_newly, *seg_claims;   // per segment: keys made resident / index slots taken by the commit
     Deferred *defer;                // kSegBlocks per segment: touches left to the commit's second pass
     uint32_t *defer_n;              // per segment: deferred touches
-    uint32_t *r_c1, *r_c2, *r_h1, *r_h2, *r_final;
+    uint32_t *r_c1, *r_c2, *r_final;
     uint64_t *r_touchoff;           // per request: offset among its instance's records of the batch
     uint64_t *log_adv;              // per id: log records the pending batch appends
     uint64_t *log_base;             // per id: log tail when the commit starts
@@ -366,13 +421,15 @@ __device__ __forceinline__ uint64_t group_anchor(uint64_t key, int lane) {
 // settles the lookup); otherwise whole buckets are read at once.
 constexpr uint64_t kNoSlot = ~0ull;
 __device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uint64_t key, uint64_t home,
-                                               uint32_t *err, Slot *found) {
+                                               uint32_t *err, Slot *found, uint64_t loop_limit = 0) {
     const Slot h = load_slot(t + home);
     if (h.key == key) { *found = h; return home; }
     if (h.key == 0) return kNoSlot;
     const uint64_t R0 = home & ~uint64_t(kGroup - 1);
     uint64_t R = R0;
-    for (uint64_t nbk = 1; nbk <= (mask >> 3) + kLinearBuckets + 1; ++nbk) {
+    uint64_t walk = (mask >> 3) + kLinearBuckets + 1;
+    if (loop_limit && loop_limit < walk) walk = loop_limit;
+    for (uint64_t nbk = 1; nbk <= walk; ++nbk) {
         Slot sn[kGroup];
 #pragma unroll
         for (int j = 0; j < (int)kGroup; ++j) sn[j] = load_slot(t + R + j);
@@ -394,9 +451,9 @@ __device__ __forceinline__ uint64_t table_find(const Slot *t, uint64_t mask, uin
 
 // 1 + log position of key's latest record (0 if the key has no slot).
 __device__ __forceinline__ uint64_t table_pos1(const Slot *t, uint64_t mask, uint64_t key, uint64_t home,
-                                               uint32_t *err) {
+                                               uint32_t *err, uint64_t loop_limit = 0) {
     Slot s;
-    return table_find(t, mask, key, home, err, &s) == kNoSlot ? 0 : s.pos1;
+    return table_find(t, mask, key, home, err, &s, loop_limit) == kNoSlot ? 0 : s.pos1;
 }
 
 // Carries of one request's segments (exclusive prefix of the segment
@@ -411,6 +468,32 @@ __device__ __forceinline__ void request_carries(const DevState &d, uint32_t r, i
         const uint64_t inc = warp_incl_scan(t, lane);
         if (s < ns) d.seg_carry[s0 + s] = carry + inc - t;
         carry += shfl_u64(inc, 31);
+    }
+}
+
+// Cached-prefix tokens on a candidate: B x the leading run of resident
+// blocks, from the first missing block found by the routing kernel
+// (0xFFFFFFFF: no block of the prompt missed).
+__device__ __forceinline__ uint32_t hit_tokens(uint32_t first_miss, uint32_t nblk, uint32_t B) {
+    return (first_miss < nblk ? first_miss : nblk) * B;
+}
+
+// After the routing kernel, a warp per request, for a kernel whose CTAs
+// cta = 0..nctas-1 take this role: the carries of every segment (the
+// commit needs them) and the request's route outputs.
+__device__ __forceinline__ void carries_role(const DevState &d, const dm_route_out &o, uint32_t n, uint32_t cta,
+                                             uint32_t nctas) {
+    const int lane = threadIdx.x & 31;
+    const uint32_t wpc = blockDim.x >> 5;
+    for (uint32_t r = cta * wpc + (threadIdx.x >> 5); r < n; r += nctas * wpc) {
+        request_carries(d, r, lane);
+        if (lane == 0) {
+            const uint32_t nblk = d.r_nblk[r];
+            o.cand1[r] = d.r_c1[r];
+            o.cand2[r] = d.r_c2[r];
+            o.hit1[r] = hit_tokens(d.r_m1[r], nblk, d.B);
+            o.hit2[r] = hit_tokens(d.r_m2[r], nblk, d.B);
+        }
     }
 }
 
@@ -595,6 +678,94 @@ __device__ __forceinline__ void route_positions_direct(const DevState &d, uint32
     pos2 = fmix64(p2 ^ d.Sr2);
 }
 
+// ---------------------------------------------------------------------------
+// Routing helpers (Sec. 3.2, Sec. 3.4, App. A.1.3, App. A.3.2).
+
+__device__ __forceinline__ const uint64_t *level_ptr(const DevState &d, int f, int k) {
+    return k == 0 ? d.ring[f].vpos : d.ring[f].tree + d.lev_off[k];
+}
+
+// Ring search.  Each ring is a sorted array of virtual-node positions plus a
+// static 32-ary search tree (level k holds every 32^k-th position).  A warp
+// compares one 256-byte row of 32 keys per level and ballots, so a ring of
+// 262,144 nodes takes four coalesced L2 reads.  The successor of p is the
+// first node with position >= p, wrapping to node 0.  Returns the level-0
+// index of the successor of p1 on ring 0 and of p2 on ring 1; whole warp,
+// the two searches interleaved for memory-level parallelism.
+__device__ __forceinline__ void ring_search2(const DevState &d, uint64_t p1, uint64_t p2, int lane,
+                                             uint32_t &lb1, uint32_t &lb2) {
+    const int top = (int)d.nlev - 1;
+    int64_t i1, i2;
+    {
+        const uint64_t nt = d.lev_n[top];
+        const uint64_t v1 = (uint64_t)lane < nt ? level_ptr(d, 0, top)[lane] : ~0ull;
+        const uint64_t v2 = (uint64_t)lane < nt ? level_ptr(d, 1, top)[lane] : ~0ull;
+        i1 = (int64_t)__popc(__ballot_sync(0xffffffffu, v1 < p1)) - 1;
+        i2 = (int64_t)__popc(__ballot_sync(0xffffffffu, v2 < p2)) - 1;
+    }
+    for (int k = top - 1; k >= 0; --k) {
+        const uint64_t nk = d.lev_n[k];
+        const uint64_t a1 = (uint64_t)(i1 < 0 ? 0 : i1) * 32 + lane;
+        const uint64_t a2 = (uint64_t)(i2 < 0 ? 0 : i2) * 32 + lane;
+        const uint64_t v1 = (i1 >= 0 && a1 < nk) ? level_ptr(d, 0, k)[a1] : ~0ull;
+        const uint64_t v2 = (i2 >= 0 && a2 < nk) ? level_ptr(d, 1, k)[a2] : ~0ull;
+        const int c1 = __popc(__ballot_sync(0xffffffffu, v1 < p1));
+        const int c2 = __popc(__ballot_sync(0xffffffffu, v2 < p2));
+        if (i1 >= 0) i1 = i1 * 32 + c1 - 1;
+        if (i2 >= 0) i2 = i2 * 32 + c2 - 1;
+    }
+    lb1 = (uint32_t)(i1 + 1 == (int64_t)d.R ? 0 : i1 + 1);
+    lb2 = (uint32_t)(i2 + 1 == (int64_t)d.R ? 0 : i2 + 1);
+}
+
+// Is key resident on an instance (log front `front`), given s0, the slot
+// already read at its home?  The home slot settles most lookups.
+__device__ __forceinline__ bool resident_at(const Slot *t, uint64_t mask, uint64_t key, uint64_t home,
+                                            uint64_t front, const Slot &s0, uint32_t *err, uint64_t loop_limit = 0) {
+    if (s0.key == key) return s0.pos1 > front;
+    if (s0.key == 0) return false;
+    return table_pos1(t, mask, key, home, err, loop_limit) > front;
+}
+
+// Adaptive hash-prefix length (Sec. 3.2): the walk from min(K_route, n_blk)
+// blocks, one step deeper while the node (the key of the prefix's last
+// block) is expanded.  Level j sits at depth min(d0 + j * step, cap), so
+// lane j evaluates level j of each 32-level round at once: the request's
+// length is the first level that cannot extend.  Every level passed and the
+// final one count toward the window's hotness.  Then the two positions of
+// that length.  c1, c2: lane s holds the carry (exclusive prefix of the
+// segment totals) of segment s of the request under f1 and f2, for every
+// segment below the cap (at most 32: ad_max <= 2048).  Whole warp.  The
+// prefix values are read through L2 (they may have been written by other
+// warps of the calling kernel).
+__device__ __forceinline__ void adaptive_positions(const DevState &d, uint32_t r, uint32_t nblk, uint64_t bo,
+                                                   int lane, uint64_t c1, uint64_t c2, uint64_t &pos1,
+                                                   uint64_t &pos2, uint32_t &Kout) {
+    const uint32_t d0 = min(d.Kroute, nblk), cap = min(d.ad_max, nblk);
+    uint32_t K = d0;
+    uint64_t P1K = 0;
+    for (uint32_t j0 = 0;; j0 += 32) {
+        const uint64_t want = uint64_t(d0) + uint64_t(j0 + lane) * d.ad_step;
+        const uint32_t dj = want < cap ? (uint32_t)want : cap;
+        const uint32_t b = dj - 1;
+        const uint64_t P1 = __ldcg(d.plocal + bo + b) + shfl_u64(c1, b / kSegBlocks);
+        const uint64_t key = cache_key(P1, d.Sc);
+        const bool ext = dj < cap && ad_set_contains(d.ad_set, d.ad_set_mask, key, d.err);
+        const uint32_t stop = __ballot_sync(0xffffffffu, !ext);
+        const int last = stop ? __ffs(stop) - 1 : 31;   // levels of this round that count
+        if (lane <= last) ad_count_add(d.ad_cnt, d.ad_cnt_mask, key, dj, d.err);
+        if (stop) {
+            K = __shfl_sync(0xffffffffu, dj, last);
+            P1K = shfl_u64(P1, last);
+            break;
+        }
+    }
+    const uint64_t P2K = __ldcg(d.p2local + bo + K - 1) + shfl_u64(c2, (K - 1) / kSegBlocks);
+    pos1 = fmix64(P1K ^ d.Sr1);
+    pos2 = fmix64(P2K ^ d.Sr2);
+    Kout = K;
+}
+
 // Grid of a grid-stride kernel: every SM filled to the kernel's occupancy.
 template <typename K>
 inline int full_grid(K kernel, int block) {
@@ -608,12 +779,16 @@ inline int full_grid(K kernel, int block) {
 // ---------------------------------------------------------------------------
 // Host-side launchers (one translation unit each).
 cudaError_t launch_setup(const DevState &d, const dm_batch &b, cudaStream_t st);
-cudaError_t launch_setup_drain(const DevState &d, const dm_batch &b, uint64_t delta, uint64_t t0,
-                               cudaStream_t st);
 cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStream_t st);
 int hash_grid_size();
-cudaError_t launch_route_probe(const DevState &d, const dm_batch &b, const dm_route_out &o,
+cudaError_t launch_setup_route(const DevState &d, const dm_batch &b, uint64_t delta, uint64_t t0,
                                cudaStream_t st);
+cudaError_t launch_setup_plain_drain(const DevState &d, const dm_batch &b, uint64_t delta, uint64_t t0,
+                                     cudaStream_t st);
+cudaError_t launch_route_d(const DevState &d, const dm_batch &b, const dm_route_out_d &o, uint64_t seq0,
+                           cudaStream_t st);
+cudaError_t launch_hash_probe(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st);
+cudaError_t launch_carries(const DevState &d, const dm_route_out &o, uint32_t n, cudaStream_t st);
 cudaError_t launch_adapt_update(const DevState &d, uint64_t *new_set, uint64_t n_live, uint64_t T, cudaStream_t st);
 cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, uint64_t seq0,
                           uint64_t t_batch, cudaStream_t st);
@@ -624,10 +799,9 @@ cudaError_t launch_hash_keys(const DevState &d, uint32_t n, uint64_t *keys, uint
                              uint64_t *pos, cudaStream_t st);
 cudaError_t launch_ring_lookup(const DevState &d, const uint64_t *pos, uint32_t n, uint32_t *o1,
                                uint32_t *o2, cudaStream_t st);
-cudaError_t launch_ring_update(DevState &d, uint32_t id, bool add, uint32_t new_R,
-                               uint64_t *scratch_pos, uint32_t *scratch_owner,
-                               uint32_t *scratch_vidx, uint64_t *new_vpos[2],
-                               uint32_t *new_owner[2], uint32_t *new_vidx[2], cudaStream_t st);
+cudaError_t launch_ring_update(DevState &d, uint32_t id, bool add, uint64_t *scratch_pos, uint32_t *scratch_vidx,
+                               uint64_t *const *new_vpos, uint32_t *const *new_owner, uint32_t *const *new_vidx,
+                               cudaStream_t st);
 cudaError_t launch_tree_build(const DevState &d, cudaStream_t st);
 cudaError_t launch_next_live(const DevState &d, cudaStream_t st);
 cudaError_t launch_set_state(const DevState &d, uint32_t id, uint8_t s, cudaStream_t st);

@@ -1,5 +1,6 @@
 // dm_ring.cu -- dual consistent-hash rings with virtual nodes (Sec. 3.4,
-// App. A.1.3).  Each live id owns V nodes per ring at
+// App. A.1.3; d rings for the d-candidate path of App. A.8).  Each live id
+// owns V nodes per ring at
 //   vpos_f(id, v) = fmix64(splitmix_step((id << 32) | v) ^ S_vf),
 // kept sorted by (position, id, v).  Adding an id inserts its V nodes,
 // removing it deletes them; all other nodes keep their relative order, so
@@ -25,11 +26,16 @@ __device__ __forceinline__ bool vless(uint64_t pa, uint32_t ia, uint32_t va, uin
     return va < vb;
 }
 
-// Generate and sort the V nodes of `id` for both rings (one CTA per ring).
+// Vnode seed of ring f.
+__device__ __forceinline__ uint64_t ring_seed(const DevState &d, int f) {
+    return f == 0 ? d.Sv1 : f == 1 ? d.Sv2 : d.Svx[f - 2];
+}
+
+// Generate and sort the V nodes of `id` for every ring (one CTA per ring).
 __global__ void __launch_bounds__(1024) k_gen_sort(DevState d, uint32_t id, uint64_t *spos, uint32_t *svidx,
                                                    uint32_t P) {
     const int f = blockIdx.x;
-    const uint64_t Sv = f == 0 ? d.Sv1 : d.Sv2;
+    const uint64_t Sv = ring_seed(d, f);
     uint64_t *pos = spos + uint64_t(f) * P;
     uint32_t *vi = svidx + uint64_t(f) * P;
     for (uint32_t v = threadIdx.x; v < P; v += blockDim.x) {
@@ -67,12 +73,17 @@ __device__ __forceinline__ uint32_t count_new_before(const uint64_t *npos, const
     return lo;
 }
 
-// Add: old nodes shift right, new nodes are placed; both rings (blockIdx.y).
+// Destination buffers of every ring.
+struct RingSet {
+    Ring r[kMaxD];
+};
+
+// Add: old nodes shift right, new nodes are placed; every ring (blockIdx.y).
 __global__ void k_merge_add(DevState d, uint32_t id, const uint64_t *spos, const uint32_t *svidx, uint32_t P,
-                            Ring dst0, Ring dst1) {
+                            RingSet dsts) {
     const int f = blockIdx.y;
     const Ring src = d.ring[f];
-    const Ring dst = f == 0 ? dst0 : dst1;
+    const Ring dst = dsts.r[f];
     const uint64_t *npos = spos + uint64_t(f) * P;
     const uint32_t *nvi = svidx + uint64_t(f) * P;
     const uint32_t R = d.R, V = d.V;
@@ -102,10 +113,10 @@ __global__ void k_merge_add(DevState d, uint32_t id, const uint64_t *spos, const
 
 // Remove: surviving nodes shift left by the id nodes that precede them.
 __global__ void k_merge_remove(DevState d, uint32_t id, const uint64_t *spos, const uint32_t *svidx, uint32_t P,
-                               Ring dst0, Ring dst1) {
+                               RingSet dsts) {
     const int f = blockIdx.y;
     const Ring src = d.ring[f];
-    const Ring dst = f == 0 ? dst0 : dst1;
+    const Ring dst = dsts.r[f];
     const uint64_t *npos = spos + uint64_t(f) * P;
     const uint32_t *nvi = svidx + uint64_t(f) * P;
     const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
@@ -120,29 +131,27 @@ __global__ void k_merge_remove(DevState d, uint32_t id, const uint64_t *spos, co
     dst.vidx[k] = v;
 }
 
-cudaError_t launch_ring_update(DevState &d, uint32_t id, bool add, uint32_t new_R, uint64_t *scratch_pos,
-                               uint32_t *scratch_owner, uint32_t *scratch_vidx, uint64_t *new_vpos[2],
-                               uint32_t *new_owner[2], uint32_t *new_vidx[2], cudaStream_t st) {
-    (void)scratch_owner;
+cudaError_t launch_ring_update(DevState &d, uint32_t id, bool add, uint64_t *scratch_pos, uint32_t *scratch_vidx,
+                               uint64_t *const *new_vpos, uint32_t *const *new_owner, uint32_t *const *new_vidx,
+                               cudaStream_t st) {
     uint32_t P = 1;
     while (P < d.V) P <<= 1;
-    k_gen_sort<<<2, 1024, 0, st>>>(d, id, scratch_pos, scratch_vidx, P);
-    Ring dst[2];
-    for (int f = 0; f < 2; ++f) {
-        dst[f].vpos = new_vpos[f];
-        dst[f].owner = new_owner[f];
-        dst[f].vidx = new_vidx[f];
-        dst[f].tree = d.ring[f].tree;
+    k_gen_sort<<<d.nrings, 1024, 0, st>>>(d, id, scratch_pos, scratch_vidx, P);
+    RingSet dst{};
+    for (uint32_t f = 0; f < d.nrings; ++f) {
+        dst.r[f].vpos = new_vpos[f];
+        dst.r[f].owner = new_owner[f];
+        dst.r[f].vidx = new_vidx[f];
+        dst.r[f].tree = d.ring[f].tree;
     }
     const uint32_t work = add ? d.R + d.V : d.R;
     if (work > 0) {
-        dim3 grid((work + 255) / 256, 2);
+        dim3 grid((work + 255) / 256, d.nrings);
         if (add)
-            k_merge_add<<<grid, 256, 0, st>>>(d, id, scratch_pos, scratch_vidx, P, dst[0], dst[1]);
+            k_merge_add<<<grid, 256, 0, st>>>(d, id, scratch_pos, scratch_vidx, P, dst);
         else
-            k_merge_remove<<<grid, 256, 0, st>>>(d, id, scratch_pos, scratch_vidx, P, dst[0], dst[1]);
+            k_merge_remove<<<grid, 256, 0, st>>>(d, id, scratch_pos, scratch_vidx, P, dst);
     }
-    (void)new_R;
     return cudaGetLastError();
 }
 
@@ -158,7 +167,7 @@ __global__ void k_tree(DevState d) {
 
 cudaError_t launch_tree_build(const DevState &d, cudaStream_t st) {
     if (d.nlev <= 1) return cudaSuccess;
-    dim3 grid((uint32_t)((d.lev_n[1] + 255) / 256), 2);
+    dim3 grid((uint32_t)((d.lev_n[1] + 255) / 256), d.nrings);
     k_tree<<<grid, 256, 0, st>>>(d);
     return cudaGetLastError();
 }

@@ -51,6 +51,8 @@ class dm_config(C.Structure):
         ("adapt_window", C.c_uint32),
         ("rebalance_flags", C.c_uint32),
         ("rebuild_pool", C.c_uint32),
+        ("test_loop_limit", C.c_uint32),
+        ("candidates", C.c_uint32),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]
@@ -71,6 +73,10 @@ class dm_batch(C.Structure):
 class dm_route_out(C.Structure):
     _fields_ = [(name, C.c_void_p) for name in
                 ("cand1", "cand2", "hit1", "hit2", "ttft1", "ttft2", "chosen", "switched")]
+
+
+class dm_route_out_d(C.Structure):
+    _fields_ = [(name, C.c_void_p) for name in ("cand", "hit", "ttft", "chosen", "switched")]
 
 
 class dm_metrics(C.Structure):
@@ -100,14 +106,16 @@ SIGNATURES = {
     "dm_remove_instance": (C.c_int, [C.c_void_p, C.c_uint32]),
     "dm_route_batch": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
     "dm_route_batch_host": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
+    "dm_route_batch_d": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out_d)]),
     "dm_route_batch_host_async": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
-    "dm_rebalance": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]),
+    "dm_rebalance": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.POINTER(C.c_uint32)]),
+    "dm_rebalance_async": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]),
     "dm_commit_cache": (C.c_int, [C.c_void_p]),
     "dm_hash_prompts": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.c_void_p, C.c_void_p, C.c_void_p]),
     "dm_hash_prompts_noalloc": (C.c_int, [C.c_uint32, C.c_uint32, C.c_uint64, C.POINTER(dm_batch), C.c_void_p,
                                           C.c_void_p, C.c_void_p, C.c_void_p]),
     "dm_ring_lookup": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p]),
-    "dm_get_loads": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32]),
+    "dm_get_loads": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.POINTER(C.c_uint32)]),
     "dm_export_cache": (C.c_int, [C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p, C.c_uint64,
                                   C.POINTER(C.c_uint64)]),
     "dm_export_queue": (C.c_int, [C.c_void_p, C.c_uint32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_uint64,
@@ -121,6 +129,7 @@ SIGNATURES = {
     "dm_export_prefix_tree": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint64, C.POINTER(C.c_uint64)]),
     "dm_potc_max_loads": (C.c_int, [C.c_uint32, C.c_uint64, C.c_uint32, C.c_uint32, C.c_uint64, C.c_void_p,
                                     C.c_void_p]),
+    "dm_test_fail_alloc": (None, [C.c_int64]),
     "dm_last_error": (C.c_int, [C.c_void_p]),
     "dm_set_profiling": (C.c_int, [C.c_void_p, C.c_int]),
     "dm_get_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int]),
@@ -194,6 +203,10 @@ def dm_route_batch(h, batch, out):
     return lib().dm_route_batch(h, C.byref(batch), C.byref(out))
 
 
+def dm_route_batch_d(h, batch, out):
+    return lib().dm_route_batch_d(h, C.byref(batch), C.byref(out))
+
+
 def dm_route_batch_host(h, batch, out):
     return lib().dm_route_batch_host(h, C.byref(batch), C.byref(out))
 
@@ -202,8 +215,18 @@ def dm_route_batch_host_async(h, batch, out):
     return lib().dm_route_batch_host_async(h, C.byref(batch), C.byref(out))
 
 
-def dm_rebalance(h, out_dev, cap, n_out_dev):
-    return lib().dm_rebalance(h, _ptr(out_dev), cap, _ptr(n_out_dev))
+def dm_rebalance(h, cap):
+    """Synchronous rebalance with host results: (status, count, migrations
+    as a numpy structured array of up to cap entries)."""
+    out = (dm_migration * max(cap, 1))()
+    n = C.c_uint32()
+    rc = lib().dm_rebalance(h, out, cap, C.byref(n))
+    m = np.ctypeslib.as_array(out)[:min(n.value, cap)] if rc == 0 else None
+    return rc, n.value, m
+
+
+def dm_rebalance_async(h, out_dev, cap, n_out_dev):
+    return lib().dm_rebalance_async(h, _ptr(out_dev), cap, _ptr(n_out_dev))
 
 
 def dm_commit_cache(h):
@@ -226,8 +249,9 @@ def dm_ring_lookup(h, pos_dev, n, owner1_dev, owner2_dev):
 
 def dm_get_loads(h, M):
     W = np.zeros(M, np.uint64)
-    _check(lib().dm_get_loads(h, W.ctypes.data, M), "dm_get_loads")
-    return W
+    n = C.c_uint32()
+    _check(lib().dm_get_loads(h, W.ctypes.data, M, C.byref(n)), "dm_get_loads")
+    return W[:min(M, n.value)]
 
 
 def dm_export_cache(h, i):

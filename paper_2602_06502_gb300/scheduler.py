@@ -19,7 +19,7 @@ class Scheduler:
                  capacity=65536, slo_us=2_000_000, cost_us=1, hot_num=3, hot_den=2, max_batch=4096,
                  max_batch_tokens=1 << 24, max_touch_per_instance=0, max_queue=0, index_slots_log2=0, seed=0,
                  choice_rule=0, adapt_step_blocks=0, adapt_max_blocks=0, adapt_window=1, rebalance_flags=0,
-                 rebuild_pool=0, stream=None, device="cuda"):
+                 rebuild_pool=0, test_loop_limit=0, candidates=0, stream=None, device="cuda"):
         self.device = torch.device(device)
         self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
         self.cfg = D.dm_config(block_tokens=block_tokens, route_prefix_blocks=route_prefix_blocks,
@@ -30,7 +30,7 @@ class Scheduler:
                                max_queue=max_queue, index_slots_log2=index_slots_log2, choice_rule=choice_rule,
                                adapt_step_blocks=adapt_step_blocks, adapt_max_blocks=adapt_max_blocks,
                                adapt_window=adapt_window, rebalance_flags=rebalance_flags, rebuild_pool=rebuild_pool,
-                               seed=seed,
+                               test_loop_limit=test_loop_limit, candidates=candidates, seed=seed,
                                stream=C.c_void_p(self.stream.cuda_stream))
         self.h = D.dm_create(self.cfg)
         self.M = max_instances
@@ -65,6 +65,32 @@ class Scheduler:
             raise D.DualMapError(rc, "dm_route_batch")
         return rc
 
+    def route_d(self, tokens, offsets, lengths, n, total_tokens, t_batch, check=True):
+        """Route one batch with d candidates (dm_route_batch_d); returns the
+        status.  results_d(n) reads the outputs."""
+        d = self.cfg.candidates or 2
+        if getattr(self, "out_d", None) is None:
+            self.out_d = {"cand": torch.zeros(self.max_batch * d, dtype=torch.int32, device=self.device),
+                          "hit": torch.zeros(self.max_batch * d, dtype=torch.int32, device=self.device),
+                          "ttft": torch.zeros(self.max_batch * d, dtype=torch.int64, device=self.device),
+                          "chosen": torch.zeros(self.max_batch, dtype=torch.int32, device=self.device),
+                          "switched": torch.zeros(self.max_batch, dtype=torch.uint8, device=self.device)}
+            self.out_d_struct = D.dm_route_out_d(*[self.out_d[k].data_ptr() for k in
+                                                   ("cand", "hit", "ttft", "chosen", "switched")])
+        b = D.make_batch(tokens, offsets, lengths, n, total_tokens, t_batch)
+        rc = D.dm_route_batch_d(self.h, b, self.out_d_struct)
+        if check and rc:
+            raise D.DualMapError(rc, "dm_route_batch_d")
+        return rc
+
+    def results_d(self, n):
+        """Host copies (numpy) of the last dm_route_batch_d outputs (n x d arrays and n vectors)."""
+        torch.cuda.synchronize(self.device)
+        d = self.cfg.candidates or 2
+        out = {k: self.out_d[k][:n * d].cpu().numpy().reshape(n, d) for k in ("cand", "hit", "ttft")}
+        out.update({k: self.out_d[k][:n].cpu().numpy() for k in ("chosen", "switched")})
+        return out
+
     def results(self, n):
         """Host copies (numpy) of the last batch's outputs."""
         torch.cuda.synchronize(self.device)
@@ -80,9 +106,9 @@ class Scheduler:
         return k[:n].cpu().numpy().astype("uint32")
 
     def rebalance(self):
-        rc = D.dm_rebalance(self.h, self.mig, self.mig.shape[0], self.mig_n)
+        rc = D.dm_rebalance_async(self.h, self.mig, self.mig.shape[0], self.mig_n)
         if rc:
-            raise D.DualMapError(rc, "dm_rebalance")
+            raise D.DualMapError(rc, "dm_rebalance_async")
 
     def migrations(self):
         torch.cuda.synchronize(self.device)

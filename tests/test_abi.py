@@ -104,6 +104,7 @@ def test_struct_layouts_match_header(built, tmp_path):
         "dm_config": [f for f, _ in D.dm_config._fields_],
         "dm_batch": [f for f, _ in D.dm_batch._fields_],
         "dm_route_out": [f for f, _ in D.dm_route_out._fields_],
+        "dm_route_out_d": [f for f, _ in D.dm_route_out_d._fields_],
         "dm_migration": ["req_seq", "from", "to"],
         "dm_metrics": [f for f, _ in D.dm_metrics._fields_],
     }
@@ -125,7 +126,64 @@ def test_struct_layouts_match_header(built, tmp_path):
     for c in consts:
         assert int(out[c]) == getattr(D, c), c
     for st, cls in (("dm_config", D.dm_config), ("dm_batch", D.dm_batch), ("dm_route_out", D.dm_route_out),
+                    ("dm_route_out_d", D.dm_route_out_d),
                     ("dm_migration", D.dm_migration), ("dm_metrics", D.dm_metrics)):
         assert int(out[st]) == C.sizeof(cls), st
         for (py, _), cn in zip(cls._fields_, fields[st]):
             assert int(out[f"{st}.{cn}"]) == getattr(cls, py).offset, (st, cn)
+
+
+def test_boundary_signatures_compile_against_the_scope_table(tmp_path):
+    """The calls of the routing boundary keep the signatures of the
+    hot-path scope table (dm_rebalance and dm_get_loads with host results
+    and a count): a C program that binds each to a pointer of exactly that
+    type compiles with incompatible-pointer warnings as errors."""
+    prog = tmp_path / "sig.c"
+    prog.write_text("\n".join([
+        f'#include "{HDR}"',
+        "dm_status (*p_create)(const dm_config *, dm_handle **) = dm_create;",
+        "void (*p_destroy)(dm_handle *) = dm_destroy;",
+        "dm_status (*p_add)(dm_handle *, uint32_t) = dm_add_instance;",
+        "dm_status (*p_remove)(dm_handle *, uint32_t) = dm_remove_instance;",
+        "dm_status (*p_route)(dm_handle *, const dm_batch *, const dm_route_out *) = dm_route_batch;",
+        "dm_status (*p_commit)(dm_handle *) = dm_commit_cache;",
+        "dm_status (*p_rebalance)(dm_handle *, dm_migration *, uint32_t, uint32_t *) = dm_rebalance;",
+        "dm_status (*p_loads)(dm_handle *, uint64_t *, uint32_t, uint32_t *) = dm_get_loads;",
+        "dm_status (*p_err)(dm_handle *) = dm_last_error;",
+        "int main(void) { return 0; }",
+    ]))
+    subprocess.run(["gcc", "-c", "-Werror", "-Wincompatible-pointer-types", str(prog), "-o",
+                    str(tmp_path / "sig.o")], check=True)
+
+
+def test_host_result_calls_check_arguments_without_touching_gpu(built):
+    D = built
+    n = C.c_uint32()
+    w = (C.c_uint64 * 4)()
+    mig = (D.dm_migration * 4)()
+    assert D.lib().dm_get_loads(None, w, 4, C.byref(n)) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_rebalance(None, mig, 4, C.byref(n)) == D.DM_ERR_INVALID_ARG
+    assert D.lib().dm_rebalance_async(None, None, 0, None) == D.DM_ERR_INVALID_ARG
+
+
+def test_allocation_failure_hook_gives_oom_without_a_gpu(built):
+    """dm_test_fail_alloc(0) fails dm_create's first device allocation
+    before any CUDA allocator call: DM_ERR_OOM and no handle, on the CPU;
+    out-of-range candidate counts are refused before any allocation."""
+    D = built
+    cfg = D.dm_config(block_tokens=16, route_prefix_blocks=16, vnodes_per_instance=8, max_instances=8,
+                      cache_capacity_blocks=1024, slo_us=1, cost_us_per_token=1, hot_num=3, hot_den=2, max_batch=16,
+                      max_batch_tokens=1 << 20, seed=1)
+    h = C.c_void_p()
+    D.lib().dm_test_fail_alloc(0)
+    try:
+        assert D.lib().dm_create(C.byref(cfg), C.byref(h)) == D.DM_ERR_OOM
+        assert not h.value
+    finally:
+        D.lib().dm_test_fail_alloc(-1)
+    bad = D.dm_config(block_tokens=16, route_prefix_blocks=16, vnodes_per_instance=8, max_instances=8,
+                      cache_capacity_blocks=1024, slo_us=1, cost_us_per_token=1, hot_num=3, hot_den=2, max_batch=16,
+                      max_batch_tokens=1 << 20, seed=1, candidates=9)
+    assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG
+    bad.candidates, bad.choice_rule = 3, D.DM_RULE_PAIR_MIN_TTFT   # the d-way path takes DualMap's rule only
+    assert D.lib().dm_create(C.byref(bad), C.byref(h)) == D.DM_ERR_INVALID_ARG

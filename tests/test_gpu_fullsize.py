@@ -1,0 +1,70 @@
+"""Parity at the workloads' stated sizes: the long-context workload in the
+benchmark's own handle configuration through the batches where the hot
+instances evict and rebuild their indices, multi-turn over its whole trace
+at a 1M-block capacity, agent batches of 4,096 prompts at 1M blocks, and
+the scaling workload (256 instances x 1,024 virtual nodes, 262,144 blocks)
+across two real add/remove events 100k requests apart, with rebalancing
+after every batch.  Every batch's outputs, loads and metrics are compared
+bit for bit with the CPU oracle."""
+
+import numpy as np
+import pytest
+
+from parity_harness import Pair, lib_ready, run_trace
+from tracegen import Trace, workload
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    lib_ready()
+
+
+def _hottest(pair, k):
+    """Ids of the k instances holding the most resident keys (oracle side)."""
+    sizes = [(len(pair.ora.cache(i)[0]), i) for i in range(pair.M) if pair.ora.inst_state()[i] == 1]
+    return [i for _, i in sorted(sizes, reverse=True)[:k]]
+
+
+def test_longctx_bench_configuration_through_eviction_and_rebuild():
+    from bench import longctx_handle_kwargs
+    from paper_2602_06502_gb300 import dualmap as D
+    tr = Trace(workload("longctx"))
+    kw = longctx_handle_kwargs(tr.cfg)
+    p = Pair(tr.cfg, max_instances=kw["max_instances"], max_batch_tokens=kw["max_batch_tokens"],
+             max_touch=kw["max_touch_per_instance"], index_slots_log2=kw["index_slots_log2"],
+             rebuild_pool=kw["rebuild_pool"])
+    run_trace(p, tr, batches=48, check_state_end=False)
+    rebuilds, _ = D.dm_get_maint_counts(p.gpu.h)
+    assert rebuilds >= 1                      # a pooled index rebuild happened on the way
+    hot = _hottest(p, 2)
+    assert len(p.ora.cache(hot[0])[0]) == tr.cfg["capacity"]   # the hot pair's LRU is full (evicting)
+    p.check_state(ids=hot + [5, 77], tag="after 48 batches")
+
+
+def test_multiturn_whole_trace_at_1m_blocks():
+    tr = Trace(workload("multiturn"))
+    assert tr.cfg["capacity"] == 1 << 20 or tr.cfg["capacity"] >= 1_000_000
+    p = Pair(tr.cfg, max_batch_tokens=1 << 25, max_touch=1 << 20)
+    run_trace(p, tr, state_every=0, check_state_end=False)
+    p.check_state(ids=_hottest(p, 3), tag="end")
+
+
+def test_agent_ten_batches_at_1m_blocks():
+    tr = Trace(workload("agent", n_requests=10 * 4096))
+    p = Pair(tr.cfg, max_batch_tokens=40_000_000, max_touch=1 << 20)
+    run_trace(p, tr, check_state_end=False)
+    assert p.n_switched > 0
+    p.check_state(ids=_hottest(p, 3), tag="end")
+
+
+def test_scaling_across_two_events_at_full_size():
+    w = workload("scaling", n_requests=52 * 4096)
+    tr = Trace(w)
+    assert w["capacity"] == 262_144 and w["vnodes"] == 1024 and w["scale_every"] == 100_000
+    assert [k for _, k, _ in tr.events] == ["add", "remove"]
+    p = Pair(tr.cfg, max_instances=w["n_instances"] + 4, max_batch_tokens=40_000_000, max_touch=1 << 20)
+    run_trace(p, tr, rebalance=True, check_state_end=False)
+    assert p.n_migrations > 0
+    p.check_state(ids=_hottest(p, 3), tag="end")
