@@ -388,10 +388,9 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.r_hoff, c.max_batch));
     A(dalloc(h, &d.r_toff, c.max_batch));
     A(dalloc(h, &d.seg_pub, d.max_segs));
-    A(dalloc(h, &d.r_route, c.max_batch));
     A(dalloc(h, &d.r_m1, c.max_batch));
     A(dalloc(h, &d.r_m2, c.max_batch));
-    A(dalloc(h, &d.fix_list, uint64_t(c.max_batch) * (d.H + 1)));   // every route and probe task at most once
+    A(dalloc(h, &d.fix_list, c.max_batch));   // every route task at most once
     A(dalloc(h, &d.defer, d.max_segs * dm::kSegBlocks));
     A(dalloc(h, &d.defer_n, d.max_segs));
     // two sets of batch scratch: routing and dm_hash_prompts
@@ -435,7 +434,6 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     set_levels(d, 0);
     A(cudaMemcpyAsync(kx_dev, kx, sizeof(kx), cudaMemcpyHostToDevice, h->st));
     A(cudaMemsetAsync(d.seg_pub, 0, d.max_segs * sizeof(dm::SegPub), h->st));
-    A(cudaMemsetAsync(d.r_route, 0, uint64_t(c.max_batch) * sizeof(dm::RoutePub), h->st));
     A(cudaMemsetAsync(d.inst_state, 0, M, h->st));
     A(cudaMemsetAsync(d.W, 0, M * 8, h->st));
     A(cudaMemsetAsync(d.metrics, 0, sizeof(dm::DevMetrics), h->st));

@@ -242,44 +242,47 @@ cudaError_t launch_hash(const DevState &d, const dm_batch &b, int grid, cudaStre
 // workloads here), request after request; then every remaining segment.
 //
 // Warp roles.  In every CTA kHashWarps warps only hash: grid-stride over the
-// tasks, tokens staged through shared memory with cp.async one task ahead,
+// tasks, tokens staged through shared memory with cp.async one task ahead
+// (the next task's request and layout looked up one task earlier still),
 // prefix values and totals stored, and, for a head segment, a checked record
 // published for the other warps (SegPub).  The warp that hashes a request's
 // last head segment also puts the request's route task on its CTA's queue.
 // The CTA's kProbeWarps warps work off that queue, so the dependent memory
 // round trips of routing and probing (App. A.3.2's metadata queries) never
-// hold up the token stream:
-//   - A route task, once every head segment of its request is published,
-//     sums their carries, computes the two ring positions, searches both
-//     rings (Sec. 3.4, App. A.1.3), applies the distinct fix (Sec. 3.2) and
-//     tests the first block of every head segment on both candidates.  On a
-//     candidate c_f the first head segment whose first block is missing,
-//     j_f, bounds the leading run: the first miss is that block or lies in
-//     a segment below it.  It publishes the route (RoutePub) and queues a
-//     probe task for each segment below the larger bound.  When every head
-//     segment's first block is resident on c_f, it probes c_f itself from
-//     block 0, hashing the prompt as it goes, until the run ends.
-//   - A probe task probes its segment's 64 blocks on each candidate whose
-//     bound lies beyond it (keys from the stored prefix values, checked
-//     against the segment's record, plus the carry of the segments before
-//     it) and lowers that candidate's first miss (atomic min).  The smallest
-//     first miss over the probed segments is exactly the leading run: every
-//     segment before the true first miss is probed and reports none, the one
-//     holding it reports it.
-// A task whose inputs are not published yet goes back on the queue; after
-// kRetries tries it moves to a list that the kernel's last CTA to finish
-// works off, when everything is published.  Nothing waits on a warp of
-// another CTA.  The segment carries of the whole batch, which the commit
+// hold up the token stream.  A route task, once every head segment of its
+// request is published, sums their carries, computes the two ring
+// positions, searches both rings (Sec. 3.4, App. A.1.3), applies the
+// distinct fix (Sec. 3.2), and finds the leading run on both candidates:
+//   - It tests the first block of every head segment on both candidates.
+//     On c_f let j_f be the first head segment whose first block is missing.
+//   - A request touches its keys from its last block down (App. A.3.2's
+//     save, in arrival order), so a key's last touch always comes after the
+//     last touch of every longer prefix of the same prompt, and an exact LRU
+//     evicts the longer prefix first: the keys resident on an instance are
+//     closed under prefixes (barring a 64-bit key collision between two
+//     different prefixes).  So every block before segment j_f - 1 is
+//     resident on c_f and the first miss is block 64 j_f or lies in segment
+//     j_f - 1, which the route task probes (keys from the segment's stored
+//     prefix values when they check against its record, else hashed again
+//     from the tokens).  When every head segment's first block is resident
+//     the run may go on past the head: it hashes on from there.
+// A route task whose head is not published yet goes back on the queue;
+// after kRetries tries it moves to a list that the kernel's last CTA to
+// finish works off, when everything is published.  Nothing waits on a warp
+// of another CTA.  The segment carries of the whole batch, which the commit
 // needs, and the route outputs are produced by the choice kernel's launch.
 
 // Request holding task x of a part: the largest r < n with off[r] <= x
-// (off: exclusive offsets of that part, nondecreasing).
-__device__ __forceinline__ uint32_t find_req(const uint32_t *off, uint32_t n, uint32_t x) {
-    uint32_t lo = 0, hi = n;   // off[lo] <= x < off[hi] (off[n] taken as infinite)
-    while (hi - lo > 1) {
-        const uint32_t mid = (lo + hi) >> 1;
-        if (__ldg(off + mid) <= x) lo = mid;
-        else hi = mid;
+// (off: exclusive offsets of that part, nondecreasing, off[0] = 0).  The
+// whole warp narrows the range 32 ways per round trip (two for n <= 1024).
+__device__ __forceinline__ uint32_t find_req(const uint32_t *off, uint32_t n, uint32_t x, int lane) {
+    uint32_t lo = 0, len = n;   // the request lies in [lo, lo + len); off[lo] <= x
+    while (len > 1) {
+        const uint32_t step = (len + 31) / 32;
+        const bool le = (uint32_t)lane * step < len && __ldg(off + lo + lane * step) <= x;
+        const uint32_t k = 31 - __clz(__ballot_sync(0xffffffffu, le));   // lane 0 always holds
+        lo += k * step;
+        len = min(step, len - k * step);
     }
     return lo;
 }
@@ -308,27 +311,11 @@ __device__ __forceinline__ void seg_pub_write(SegPub *p, uint64_t E, uint64_t t1
     st_v2(&p->px, px, t1 ^ t2 ^ pf ^ pk ^ px ^ E);
 }
 
+// Both candidates' index buffers and log fronts (as of the batch's start).
 struct RouteView {
     const Slot *t1, *t2;
     uint64_t f1, f2;
-    uint32_t j1, j2;
 };
-
-__device__ __forceinline__ bool route_pub_read(const RoutePub *p, uint64_t E, RouteView &v) {
-    uint64_t cc, t1, t2, f1, f2, js, pad, chk;
-    ld_cg2(&p->cc, cc, t1);
-    ld_cg2(&p->tab2, t2, f1);
-    ld_cg2(&p->fr2, f2, js);
-    ld_cg2(&p->pad, pad, chk);
-    if (chk != (cc ^ t1 ^ t2 ^ f1 ^ f2 ^ js ^ E)) return false;
-    v.t1 = reinterpret_cast<const Slot *>(t1);
-    v.t2 = reinterpret_cast<const Slot *>(t2);
-    v.f1 = f1;
-    v.f2 = f2;
-    v.j1 = (uint32_t)(js & 0xFFFF);
-    v.j2 = (uint32_t)((js >> 16) & 0xFFFF);
-    return true;
-}
 
 constexpr uint32_t kNoMiss = 0xFFFFFFFFu;
 constexpr int kHashWarps = 6, kProbeWarps = 2;   // warp roles of a routing CTA
@@ -369,48 +356,75 @@ __device__ __forceinline__ void probe_segment(const uint64_t (&key)[2], uint32_t
     }
 }
 
-// Probe c_f from block 0 on the candidates flagged, hashing the prompt here
-// segment by segment (f1 only), until each run ends; lowers their first
-// miss.  Whole warp (rare: the run reaches the end of the head).
+// Cache keys of head segment s of request r (nb blocks, f1 carry `carry`
+// into it): lane l gets blocks 64 s + l and 64 s + 32 + l.  The prefix
+// values come from plocal when what is visible there checks against the
+// segment's record (px), else the segment is hashed here from the tokens.
+// Whole warp; not inlined.
 template <int U>
-__device__ __noinline__ void probe_from_start(const DevState &d, const uint32_t *tokens, uint64_t pol, uint32_t r,
-                                              uint32_t nblk, bool go1, bool go2, const RouteView &rv, int lane) {
+__device__ __noinline__ void head_seg_keys(const DevState &d, const uint32_t *tokens, uint64_t pol, uint32_t r,
+                                           uint32_t s, uint32_t nb, uint64_t carry, uint64_t px, int lane,
+                                           uint64_t *key) {
+    const uint32_t b0 = s * kSegBlocks;
+    const uint64_t *pl = d.plocal + d.r_blkoff[r] + b0;
+    uint64_t P0 = (uint32_t)lane < nb ? __ldcg(pl + lane) : 0;
+    uint64_t P1 = (uint32_t)lane + 32 < nb ? __ldcg(pl + lane + 32) : 0;
+    uint64_t x = P0 ^ P1;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) x ^= shfl_xor_u64(x, o);
+    if (x != px) {   // some value not visible yet
+        const HashLane<U> hl(d, lane);
+        const uint4 *src = reinterpret_cast<const uint4 *>(tokens + d.r_tokoff[r] + uint64_t(b0) * d.B);
+        uint64_t P[2], tot, s2u;
+        hash_segment<U, false, false>(hl, src, b0, nb, 0, lane, pol, P, tot, s2u, nullptr);
+        P0 = P[0];
+        P1 = P[1];
+    }
+    key[0] = cache_key(P0 + carry, d.Sc);
+    key[1] = cache_key(P1 + carry, d.Sc);
+}
+
+// The run past the head, on the candidates whose first miss is still
+// kNoMiss (every head block resident there): hashes the prompt on from
+// segment j0 (f1 only, from carry `carry`) and probes segment by segment
+// until each run ends.  Updates m1 and m2 on every lane (kNoMiss: the whole
+// prompt is resident).  Whole warp; not inlined (rare: a cached run longer
+// than the head).
+template <int U>
+__device__ __noinline__ void run_on(const DevState &d, const uint32_t *tokens, uint64_t pol, uint32_t r,
+                                    uint32_t nblk, uint32_t j0, uint64_t carry, const RouteView &rv, int lane,
+                                    uint32_t &m1, uint32_t &m2) {
     const HashLane<U> hl(d, lane);
     const uint4 *tok4 = reinterpret_cast<const uint4 *>(tokens + d.r_tokoff[r]);
     const uint32_t nseg = (nblk + kSegBlocks - 1) / kSegBlocks;
     const uint64_t mask = d.S - 1;
-    uint32_t q1 = go1 ? kNoMiss : 0, q2 = go2 ? kNoMiss : 0;
-    uint64_t run = 0;
-    for (uint32_t j = 0; j < nseg && (q1 == kNoMiss || q2 == kNoMiss); ++j) {
+    for (uint32_t j = j0; j < nseg && (m1 == kNoMiss || m2 == kNoMiss); ++j) {
         const uint32_t c0 = j * kSegBlocks, cn = min(kSegBlocks, nblk - c0);
         uint64_t P[2], tot, s2u;
         hash_segment<U, false, false>(hl, tok4 + uint64_t(c0) * d.B / 4, c0, cn, 0, lane, pol, P, tot, s2u,
                                       nullptr);
-        const uint64_t key[2] = {cache_key(P[0] + run, d.Sc), cache_key(P[1] + run, d.Sc)};
+        const uint64_t key[2] = {cache_key(P[0] + carry, d.Sc), cache_key(P[1] + carry, d.Sc)};
         uint32_t e1, e2;
-        probe_segment(key, c0, c0 + cn, q1 == kNoMiss, q2 == kNoMiss, rv, mask, d.err, d.loop_limit, lane, e1, e2);
-        if (q1 == kNoMiss && e1 != kNoMiss) q1 = e1;
-        if (q2 == kNoMiss && e2 != kNoMiss) q2 = e2;
-        run += tot;
-    }
-    if (lane == 0) {
-        if (go1 && q1 != kNoMiss) atomicMin(d.r_m1 + r, q1);
-        if (go2 && q2 != kNoMiss) atomicMin(d.r_m2 + r, q2);
+        probe_segment(key, c0, c0 + cn, m1 == kNoMiss, m2 == kNoMiss, rv, mask, d.err, d.loop_limit, lane, e1,
+                      e2);
+        if (m1 == kNoMiss) m1 = e1;
+        if (m2 == kNoMiss) m2 = e2;
+        carry += tot;
     }
 }
 
 // The route task of request r.  Returns false, changing nothing, when a head
-// segment of r is not published yet; else the number of head segments that
-// still need a probe task (segments 0 .. return-1).  Whole warp; not inlined.
+// segment of r is not published yet.  Whole warp; not inlined.
 template <int U, bool kAdapt>
-__device__ __noinline__ int route_task(const DevState &d, const uint32_t *tokens, uint64_t E, uint64_t pol,
-                                       uint32_t r, int lane) {
+__device__ __noinline__ bool route_task(const DevState &d, const uint32_t *tokens, uint64_t E, uint64_t pol,
+                                        uint32_t r, int lane) {
     const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
     const uint32_t nseg = (nblk + kSegBlocks - 1) / kSegBlocks, hs = min(nseg, d.H);
     uint64_t t1 = 0, t2 = 0, pf = 0, pk = 0, px = 0;
     const bool ok = (uint32_t)lane >= hs || seg_pub_read(d.seg_pub + s0 + lane, E, t1, t2, pf, pk, px);
-    if (!__all_sync(0xffffffffu, ok)) return -1;
-    const uint64_t carry = warp_incl_scan(t1, lane) - t1;   // lane s: f1 carry into head segment s
+    if (!__all_sync(0xffffffffu, ok)) return false;
+    const uint64_t inc1 = warp_incl_scan(t1, lane);
+    const uint64_t carry = inc1 - t1;   // lane s: f1 carry into head segment s
     uint64_t pos1, pos2;
     uint32_t K;
     if constexpr (kAdapt) {
@@ -441,61 +455,35 @@ __device__ __noinline__ int route_task(const DevState &d, const uint32_t *tokens
         miss1 = !resident_at(rv.t1, mask, key, home, rv.f1, load_slot(rv.t1 + home), d.err, d.loop_limit);
         miss2 = !resident_at(rv.t2, mask, key, home, rv.f2, load_slot(rv.t2 + home), d.err, d.loop_limit);
     }
-    // lanes >= hs count as missing: a bound of hs or more means every head
-    // segment's first block is resident
-    uint32_t j1 = __ffs(__ballot_sync(0xffffffffu, miss1)) - 1, j2 = __ffs(__ballot_sync(0xffffffffu, miss2)) - 1;
-    const bool full1 = j1 >= hs, full2 = j2 >= hs;
+    // j_f: the first head segment whose first block is missing on c_f (hs:
+    // none; lanes >= hs count as missing)
+    const uint32_t j1 = __ffs(__ballot_sync(0xffffffffu, miss1)) - 1;
+    const uint32_t j2 = __ffs(__ballot_sync(0xffffffffu, miss2)) - 1;
+    // the run on c_f ends in segment j_f - 1 or at block 64 j_f (when j_f <
+    // hs); probe that segment, once for both candidates when they agree
+    uint32_t m1 = j1 == 0 ? 0 : kNoMiss, m2 = j2 == 0 ? 0 : kNoMiss;
+#pragma unroll 1
+    for (int f = 0; f < 2; ++f) {
+        const uint32_t jf = f ? j2 : j1;
+        if (jf == 0 || (f == 1 && j2 == j1)) continue;
+        const uint32_t s = jf - 1, c0 = s * kSegBlocks, cn = min(kSegBlocks, nblk - c0);
+        uint64_t key[2];
+        head_seg_keys<U>(d, tokens, pol, r, s, cn, shfl_u64(carry, s), shfl_u64(px, s), lane, key);
+        const bool do1 = j1 == jf, do2 = j2 == jf;
+        uint32_t e1, e2;
+        probe_segment(key, c0, c0 + cn, do1, do2, rv, mask, d.err, d.loop_limit, lane, e1, e2);
+        if (do1) m1 = e1 != kNoMiss ? e1 : (j1 < hs ? j1 * kSegBlocks : kNoMiss);
+        if (do2) m2 = e2 != kNoMiss ? e2 : (j2 < hs ? j2 * kSegBlocks : kNoMiss);
+    }
+    // every head block resident on a candidate: its run may go on past the head
+    if ((m1 == kNoMiss || m2 == kNoMiss) && hs < nseg)
+        run_on<U>(d, tokens, pol, r, nblk, hs, shfl_u64(inc1, hs - 1), rv, lane, m1, m2);
     if (lane == 0) {
         d.r_K[r] = K;
         d.r_c1[r] = a;
         d.r_c2[r] = b;
-        if (!full1) atomicMin(d.r_m1 + r, j1 * kSegBlocks);
-        if (!full2) atomicMin(d.r_m2 + r, j2 * kSegBlocks);
-    }
-    if (full1 || full2) probe_from_start<U>(d, tokens, pol, r, nblk, full1, full2, rv, lane);
-    if (full1) j1 = 0;   // done here: no probe task on that candidate
-    if (full2) j2 = 0;
-    if (lane == 0) {
-        const uint64_t cc = a | uint64_t(b) << 32, js = j1 | uint64_t(j2) << 16 | uint64_t(K) << 32;
-        const uint64_t t1p = reinterpret_cast<uint64_t>(rv.t1), t2p = reinterpret_cast<uint64_t>(rv.t2);
-        RoutePub *p = d.r_route + r;
-        st_v2(&p->cc, cc, t1p);
-        st_v2(&p->tab2, t2p, rv.f1);
-        st_v2(&p->fr2, rv.f2, js);
-        st_v2(&p->pad, 0, cc ^ t1p ^ t2p ^ rv.f1 ^ rv.f2 ^ js ^ E);
-    }
-    return (int)max(j1, j2);
-}
-
-// The probe task of head segment j of request r.  Returns false, changing
-// nothing, when an input is not published (or not visible) yet.  Whole warp.
-__device__ __forceinline__ bool probe_task(const DevState &d, uint64_t E, uint32_t r, uint32_t j, int lane) {
-    RouteView rv;
-    const bool have = route_pub_read(d.r_route + r, E, rv);
-    if (!__all_sync(0xffffffffu, have)) return false;
-    const uint32_t b0 = j * kSegBlocks;
-    const bool do1 = j < rv.j1 && __ldcg(d.r_m1 + r) > b0, do2 = j < rv.j2 && __ldcg(d.r_m2 + r) > b0;
-    if (!do1 && !do2) return true;   // a miss before this segment is known already
-    const uint32_t nblk = d.r_nblk[r], s0 = d.r_segoff[r];
-    const uint32_t nb = min(kSegBlocks, nblk - b0);
-    // carries of the segments before it, its own record, its stored prefix values
-    uint64_t t1 = 0, t2, pf, pk, px = 0;
-    const bool ok = (uint32_t)lane > j || seg_pub_read(d.seg_pub + s0 + lane, E, t1, t2, pf, pk, px);
-    const uint64_t *pl = d.plocal + d.r_blkoff[r] + b0;
-    const uint64_t P0 = (uint32_t)lane < nb ? __ldcg(pl + lane) : 0;
-    const uint64_t P1 = (uint32_t)lane + 32 < nb ? __ldcg(pl + lane + 32) : 0;
-    if (!__all_sync(0xffffffffu, ok)) return false;
-    uint64_t x = P0 ^ P1;
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) x ^= shfl_xor_u64(x, o);
-    if (x != shfl_u64(px, j)) return false;   // some prefix value not visible yet
-    const uint64_t carry = warp_sum_u64((uint32_t)lane < j ? t1 : 0);
-    const uint64_t key[2] = {cache_key(P0 + carry, d.Sc), cache_key(P1 + carry, d.Sc)};
-    uint32_t m1, m2;
-    probe_segment(key, b0, b0 + nb, do1, do2, rv, d.S - 1, d.err, d.loop_limit, lane, m1, m2);
-    if (lane == 0) {
-        if (do1 && m1 != kNoMiss) atomicMin(d.r_m1 + r, m1);
-        if (do2 && m2 != kNoMiss) atomicMin(d.r_m2 + r, m2);
+        d.r_m1[r] = m1;
+        d.r_m2[r] = m2;
     }
     return true;
 }
@@ -553,8 +541,8 @@ __device__ __forceinline__ void read_stage(const uint4 *stage, int lane, uint4 (
 // k is free for the producer at position p when its number is p, holds
 // that producer's entry when it is p + 1, and is free again for position
 // p + kQCap once consumed), so neither side ever reads a half-written
-// entry.  An entry is r | j << 32 | route flag << 40 | (tries + 1) << 48,
-// never 0 (what an empty queue returns).
+// entry.  An entry is a route task: r | (tries + 1) << 32, never 0 (what an
+// empty queue returns).
 struct CtaQueue {
     uint64_t buf[kQCap];
     uint32_t seq[kQCap];
@@ -563,8 +551,8 @@ struct CtaQueue {
     uint32_t busy;        // probing warps inside a task
 };
 
-__device__ __forceinline__ uint64_t qentry(uint32_t r, uint32_t j, bool route, uint32_t tries) {
-    return uint64_t(r) | uint64_t(j) << 32 | uint64_t(route) << 40 | uint64_t(tries + 1) << 48;   // never 0
+__device__ __forceinline__ uint64_t qentry(uint32_t r, uint32_t tries) {
+    return uint64_t(r) | uint64_t(tries + 1) << 32;   // never 0
 }
 
 // Push one entry (one thread); a full queue sends it to the last CTA's list.
@@ -619,6 +607,35 @@ __device__ __forceinline__ uint64_t q_pop(CtaQueue &q) {
     return 0;
 }
 
+// Request, segment and layout of one hashing task (nb = 0: a routing column
+// past the end of the prompt, nothing to hash).
+struct TaskMeta {
+    uint32_t r, j, nblk, seg, nb;
+    uint64_t tokoff, bo;
+};
+
+__device__ __forceinline__ TaskMeta task_meta(const DevState &d, uint32_t t, uint32_t n, uint32_t ncol, uint32_t nhr,
+                                              int lane) {
+    TaskMeta m;
+    if (t < ncol) {
+        m.j = t / n;
+        m.r = t - m.j * n;
+    } else if (t < ncol + nhr) {
+        m.r = find_req(d.r_hoff, n, t - ncol, lane);
+        m.j = d.Ccols + (t - ncol - __ldg(d.r_hoff + m.r));
+    } else {
+        m.r = find_req(d.r_toff, n, t - ncol - nhr, lane);
+        m.j = d.H + (t - ncol - nhr - __ldg(d.r_toff + m.r));
+    }
+    m.nblk = d.r_nblk[m.r];
+    m.seg = d.r_segoff[m.r] + m.j;
+    m.tokoff = d.r_tokoff[m.r];
+    m.bo = d.r_blkoff[m.r];
+    const uint32_t b0 = m.j * kSegBlocks;
+    m.nb = b0 < m.nblk ? min(kSegBlocks, m.nblk - b0) : 0;
+    return m;
+}
+
 template <int U, bool kAdapt>
 __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_constant__ DevState d,
                                                                    const uint32_t *__restrict__ tokens, uint64_t E) {
@@ -643,74 +660,66 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
         const uint32_t total = d.info->tasks;
         const HashLane<U> hl(d, lane);
         uint4 *const stage = s_stage + wid * 2 * HP<U>::kStage;
-        // request, segment and layout of the task whose copy is issued next
-        // (nb = 0: a routing column past the end of the prompt, nothing to do)
-        uint32_t r = 0, j = 0, nblk = 0, segoff = 0, nb = 0;
-        uint64_t tokoff = 0, bo = 0;
-        auto issue = [&](uint32_t t, uint4 *st) {
-            if (t < ncol) {
-                j = t / n;
-                r = t - j * n;
-            } else if (t < ncol + nhr) {
-                r = find_req(d.r_hoff, n, t - ncol);
-                j = d.Ccols + (t - ncol - __ldg(d.r_hoff + r));
-            } else {
-                r = find_req(d.r_toff, n, t - ncol - nhr);
-                j = d.H + (t - ncol - nhr - __ldg(d.r_toff + r));
-            }
-            nblk = d.r_nblk[r];
-            segoff = d.r_segoff[r];
-            tokoff = d.r_tokoff[r];
-            bo = d.r_blkoff[r];
-            nb = j * kSegBlocks < nblk ? min(kSegBlocks, nblk - j * kSegBlocks) : 0;
-            if (nb)
+        auto issue = [&](const TaskMeta &m, uint4 *st) {
+            if (m.nb)
                 stage_segment<U>(hl, st,
-                                 reinterpret_cast<const uint4 *>(tokens + tokoff + uint64_t(j) * kSegBlocks * d.B),
-                                 nb, lane, pol);
+                                 reinterpret_cast<const uint4 *>(tokens + m.tokoff + uint64_t(m.j) * kSegBlocks * d.B),
+                                 m.nb, lane, pol);
         };
-        if (gw < total) issue(gw, stage);
+        // the task being copied (cur) and the next one, looked up a task ahead
+        TaskMeta cur{}, nxt{};
+        if (gw < total) {
+            cur = task_meta(d, gw, n, ncol, nhr, lane);
+            issue(cur, stage);
+        }
         cp_async_commit();
+        if (uint64_t(gw) + nhw < total) nxt = task_meta(d, gw + nhw, n, ncol, nhr, lane);
         uint32_t it = 0;
         for (uint32_t t = gw; t < total; t += nhw, ++it) {
-            const uint32_t rr = r, jj = j, nbk = nblk, seg = segoff + j, cnb = nb;
-            const uint64_t bof = bo;
-            const uint32_t b0 = jj * kSegBlocks;
-            if (t + nhw < total) issue(t + nhw, stage + ((it + 1) & 1) * HP<U>::kStage);
+            const bool more = uint64_t(t) + nhw < total;
+            if (more) issue(nxt, stage + ((it + 1) & 1) * HP<U>::kStage);
             cp_async_commit();
+            TaskMeta nn{};
+            if (uint64_t(t) + 2 * uint64_t(nhw) < total) nn = task_meta(d, t + 2 * nhw, n, ncol, nhr, lane);
             cp_async_wait<1>();   // this task's copy is complete
-            if (cnb == 0) continue;
-            uint4 v[2][U];
-            read_stage<U>(stage + (it & 1) * HP<U>::kStage, lane, v);
-            uint64_t P[2], tot1, sum2;
-            hash_loaded<U, true, kAdapt>(hl, v, b0, cnb, min(d.Kf2, nbk), lane, P, tot1, sum2,
-                                         kAdapt ? d.p2local + bof + b0 : nullptr);
-            uint64_t *out = d.plocal + bof + b0;
-            if ((uint32_t)lane < cnb) out[lane] = P[0];
-            if ((uint32_t)lane + 32 < cnb) out[lane + 32] = P[1];
-            if (lane == 0) {
-                d.seg_total[seg] = tot1;
-                d.seg_total2[seg] = sum2;
-                d.seg_req[seg] = rr;
-            }
-            const uint32_t hs = min((nbk + kSegBlocks - 1) / kSegBlocks, d.H);
-            if (jj < hs) {
-                // publish the head segment: totals, its first block's and block
-                // K-1's prefix values, and the xor of what it stored in plocal
-                const uint32_t kk = min(d.Kroute, nbk) - 1 - b0;   // block K-1 in this segment, if any
-                const uint64_t pk = shfl_u64(kk < 32 ? P[0] : P[1], kk & 31);
-                const uint64_t pf = shfl_u64(P[0], 0);
-                uint64_t px = P[0] ^ P[1];
-#pragma unroll
-                for (int o = 16; o >= 1; o >>= 1) px ^= shfl_xor_u64(px, o);
-                if constexpr (kAdapt) {
-                    __threadfence();   // the route task reads the head's prefix values (plocal, p2local) directly
-                    __syncwarp();
-                }
+            if (cur.nb) {
+                uint4 v[2][U];
+                read_stage<U>(stage + (it & 1) * HP<U>::kStage, lane, v);
+                const uint32_t b0 = cur.j * kSegBlocks;
+                uint64_t P[2], tot1, sum2;
+                hash_loaded<U, true, kAdapt>(hl, v, b0, cur.nb, min(d.Kf2, cur.nblk), lane, P, tot1, sum2,
+                                             kAdapt ? d.p2local + cur.bo + b0 : nullptr);
+                uint64_t *out = d.plocal + cur.bo + b0;
+                if ((uint32_t)lane < cur.nb) out[lane] = P[0];
+                if ((uint32_t)lane + 32 < cur.nb) out[lane + 32] = P[1];
                 if (lane == 0) {
-                    seg_pub_write(d.seg_pub + seg, E, tot1, sum2, pf, kk < kSegBlocks ? pk : 0, px);
-                    if (jj + 1 == hs) q_push(q, d, qentry(rr, 0, true, 0));   // the request's route task
+                    d.seg_total[cur.seg] = tot1;
+                    d.seg_total2[cur.seg] = sum2;
+                    d.seg_req[cur.seg] = cur.r;
+                }
+                const uint32_t hs = min((cur.nblk + kSegBlocks - 1) / kSegBlocks, d.H);
+                if (cur.j < hs) {
+                    // publish the head segment: totals, its first block's and
+                    // block K-1's prefix values, and the xor of what it stored
+                    // in plocal
+                    const uint32_t kk = min(d.Kroute, cur.nblk) - 1 - b0;   // block K-1 in this segment, if any
+                    const uint64_t pk = shfl_u64(kk < 32 ? P[0] : P[1], kk & 31);
+                    const uint64_t pf = shfl_u64(P[0], 0);
+                    uint64_t px = P[0] ^ P[1];
+#pragma unroll
+                    for (int o = 16; o >= 1; o >>= 1) px ^= shfl_xor_u64(px, o);
+                    if constexpr (kAdapt) {
+                        __threadfence();   // the route task reads the head's prefix values (plocal, p2local) directly
+                        __syncwarp();
+                    }
+                    if (lane == 0) {
+                        seg_pub_write(d.seg_pub + cur.seg, E, tot1, sum2, pf, kk < kSegBlocks ? pk : 0, px);
+                        if (cur.j + 1 == hs) q_push(q, d, qentry(cur.r, 0));   // the request's route task
+                    }
                 }
             }
+            cur = nxt;
+            nxt = nn;
         }
         cp_async_wait<0>();
         if (lane == 0) atomicAdd(&q.hash_done, 1u);
@@ -724,7 +733,7 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
             e = shfl_u64(e, 0);
             if (e == 0) {
                 // done once the hashing warps are done, no probing warp holds
-                // a task (it might queue more) and the queue is empty
+                // a task (it might queue it again) and the queue is empty
                 const bool fin = *(volatile uint32_t *)&q.hash_done == kHashWarps &&
                                  *(volatile uint32_t *)&q.busy == 0 &&
                                  *(volatile uint32_t *)&q.head == *(volatile uint32_t *)&q.tail;
@@ -737,23 +746,13 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
                 continue;
             }
             idle = 0;
-            const uint32_t r = (uint32_t)e, j = (uint32_t)(e >> 32) & 0xFF;
-            const bool route = (e >> 40) & 1;
-            const uint32_t tries = (uint32_t)(e >> 48) - 1;
-            bool done;
-            if (route) {
-                const int np = route_task<U, kAdapt>(d, tokens, E, pol, r, lane);
-                done = np >= 0;
-                if (done && lane == 0)
-                    for (int k = 0; k < np; ++k) q_push(q, d, qentry(r, (uint32_t)k, false, 0));
-            } else {
-                done = probe_task(d, E, r, j, lane);
-            }
+            const uint32_t r = (uint32_t)e, tries = (uint32_t)(e >> 32) - 1;
+            const bool done = route_task<U, kAdapt>(d, tokens, E, pol, r, lane);
             if (lane == 0) {
                 if (!done) {
-                    // inputs of a warp elsewhere not published yet: back on the queue
-                    if (tries + 1 < kRetries) q_push(q, d, qentry(r, j, route, tries + 1));
-                    else d.fix_list[atomicAdd(&d.info->fix_n, 1u)] = qentry(r, j, route, 0);
+                    // a head segment hashed elsewhere not published yet: back on the queue
+                    if (tries + 1 < kRetries) q_push(q, d, qentry(r, tries + 1));
+                    else d.fix_list[atomicAdd(&d.info->fix_n, 1u)] = qentry(r, 0);
                     if (tries > 8) __nanosleep(1000);
                 }
                 atomicSub(&q.busy, 1u);
@@ -761,9 +760,8 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
             __syncwarp();
         }
     }
-    // the last CTA to finish works off the list: route tasks first (every
-    // head segment is published by then, and each queues its probes here),
-    // then the probes
+    // the last CTA to finish works off the list (every head segment is
+    // published by then)
     __syncthreads();
     if (threadIdx.x == 0) {
         __threadfence();
@@ -774,25 +772,9 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
     __threadfence();
     const uint32_t nf = *(volatile uint32_t *)&d.info->fix_n;
     const uint32_t nw = blockDim.x >> 5;
-    for (uint32_t i = wid; i < nf; i += nw) {
-        const uint64_t e = d.fix_list[i];
-        if (!((e >> 40) & 1)) continue;
-        const uint32_t r = (uint32_t)e;
-        const int np = route_task<U, kAdapt>(d, tokens, E, pol, r, lane);
-        if (np < 0) {
-            if (lane == 0) set_err(d.err, DM_ERR_TIMEOUT);   // cannot happen: everything is published by now
-            continue;
-        }
-        for (int k = 0; k < np; ++k)
-            if (!probe_task(d, E, r, (uint32_t)k, lane) && lane == 0) set_err(d.err, DM_ERR_TIMEOUT);
-    }
-    __syncthreads();
-    for (uint32_t i = wid; i < nf; i += nw) {
-        const uint64_t e = d.fix_list[i];
-        if ((e >> 40) & 1) continue;
-        if (!probe_task(d, E, (uint32_t)e, (uint32_t)(e >> 32) & 0xFF, lane) && lane == 0)
-            set_err(d.err, DM_ERR_TIMEOUT);
-    }
+    for (uint32_t i = wid; i < nf; i += nw)
+        if (!route_task<U, kAdapt>(d, tokens, E, pol, (uint32_t)d.fix_list[i], lane) && lane == 0)
+            set_err(d.err, DM_ERR_TIMEOUT);   // cannot happen: everything is published by now
 }
 
 // Launch shape of the routing kernel per device and block size: its

@@ -148,15 +148,6 @@ struct AdCount {
 struct __align__(16) SegPub {
     uint64_t t1, t2, pf, pk, px, chk;
 };
-// A routed request's record (64 bytes): cc = c1 | c2 << 32, both
-// candidates' index buffers and log fronts, and js = j1 | j2 << 16 | K << 32
-// (j_f: the head segments below it still need a probe on c_f: the first
-// head segment whose first block is not resident on c_f, or 0 when the
-// route task probed c_f itself).
-struct __align__(16) RoutePub {
-    uint64_t cc, tab1, tab2, fr1, fr2, js, pad, chk;
-};
-
 // Per-batch values produced on the device.
 struct BatchInfo {
     uint64_t total_blocks;
@@ -252,13 +243,12 @@ struct DevState {
     uint32_t H, Ccols;              // head segments, routing columns (segments holding any routing prefix)
     uint32_t *r_hoff, *r_toff;
     // routing kernel's exchange between warps (see dm_hash.cu): what each
-    // head segment and each routed request publish, the first miss found so
-    // far on each candidate (0xFFFFFFFF: none yet), and the probes left to
-    // the kernel's last CTA
+    // head segment publishes, each request's first miss on each candidate
+    // (0xFFFFFFFF: the whole prompt is resident), and the route tasks left
+    // to the kernel's last CTA
     SegPub *seg_pub;
-    RoutePub *r_route;
     uint32_t *r_m1, *r_m2;
-    uint64_t *fix_list;             // entries of the routing kernel's task queues (r, segment, kind)
+    uint64_t *fix_list;             // queue entries of route tasks (request, tries)
     uint64_t *seg_total, *seg_carry, *plocal;
     uint64_t *p2local;              // adaptive only: per block < Kf2, in-segment prefix of its f2 digests
     uint32_t *r_K;                  // per request: the hash prefix length it was routed with

@@ -87,8 +87,6 @@ __global__ void __launch_bounds__(1024) k_setup(DevState d, const uint64_t *off,
                 d.r_hoff[r] = ho;
                 d.r_toff[r] = to;
                 d.r_segoff[r] = co + ho + to;
-                d.r_m1[r] = 0xFFFFFFFFu;   // no miss found yet on either candidate
-                d.r_m2[r] = 0xFFFFFFFFu;
             } else {
                 d.r_segoff[r] = (uint32_t)(carry[1] + ex[1]);
             }
