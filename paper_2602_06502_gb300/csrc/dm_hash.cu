@@ -318,7 +318,8 @@ struct RouteView {
 };
 
 constexpr uint32_t kNoMiss = 0xFFFFFFFFu;
-constexpr int kHashWarps = 6, kProbeWarps = 2;   // warp roles of a routing CTA
+constexpr int kHashWarps = 7, kProbeWarps = 1;   // warp roles of a routing CTA
+constexpr int kMinBlocks = 2;                    // resident CTAs per SM the registers are sized for
 constexpr uint32_t kQCap = 512;                  // entries of a CTA's task queue
 constexpr uint32_t kRetries = 1024;              // tries of a task before it goes to the last CTA
 
@@ -488,44 +489,55 @@ __device__ __noinline__ bool route_task(const DevState &d, const uint32_t *token
     return true;
 }
 
-// Token staging: a hashing warp copies its next task's segment into its own
-// shared-memory stage with cp.async while it hashes the current one.  Lane l
-// copies and later reads the same 16-byte pieces as load_segment (coalesced
-// in global memory, conflict-free in shared memory); pieces past the
-// segment are zero-filled.
+// Token staging: a hashing warp streams its tasks' segments through a ring
+// of shared-memory stages, kStages - 1 segments ahead of the one it hashes:
+// lane 0 issues one bulk copy per segment (cp.async.bulk, completed on the
+// stage's mbarrier).  A stage holds the segment's tokens as they lie in
+// memory, so lane l reads the same 16-byte pieces as load_segment
+// (conflict-free); blocks past the segment are not copied and the hash
+// masks them out.
 template <int U>
 struct HP {
     static constexpr int kWarps = kHashWarps + kProbeWarps;
     static constexpr int kThreads = 32 * kWarps;
     static constexpr uint32_t kStage = 64 * U;   // uint4 per stage: one segment
-    static constexpr size_t kSmem = size_t(kHashWarps) * 2 * kStage * sizeof(uint4);
+    static constexpr int kStages = U <= 4 ? 3 : (U == 8 ? 2 : 1);
+    static constexpr size_t kSmem = size_t(kHashWarps) * kStages * kStage * sizeof(uint4);
 };
 
-__device__ __forceinline__ void cp_async16(uint4 *sdst, const uint4 *gsrc, bool valid, uint64_t pol) {
-    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(sdst);
-    asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;" ::"r"(sa),
-                 "l"(__cvta_generic_to_global(gsrc)), "r"(valid ? 16 : 0), "l"(pol)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+__device__ __forceinline__ uint32_t smem_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
 }
 
-template <int U>
-__device__ __forceinline__ void stage_segment(const HashLane<U> &hl, uint4 *stage, const uint4 *src4, uint32_t nb,
-                                              int lane, uint64_t pol) {
-    constexpr int GPL = HashLane<U>::GPL;
-#pragma unroll
-    for (int it = 0; it < 2; ++it)
-#pragma unroll
-        for (int jj = 0; jj < U; ++jj) {
-            const uint32_t blk = it * 32 + jj * GPL + hl.g;
-            const bool valid = blk < nb;
-            const uint4 *g = src4 + uint64_t(it) * 32 * U + jj * 32 + lane;
-            cp_async16(stage + (it * U + jj) * 32 + lane, valid ? g : src4, valid, pol);
-        }
+// Lane 0: copy `bytes` (a multiple of 16; both addresses 16-byte aligned)
+// from global memory into a stage; the stage's mbarrier completes its
+// current phase when they have landed.
+__device__ __forceinline__ void bulk_to_stage(uint4 *stage, const uint4 *src, uint32_t bytes, uint64_t *bar,
+                                              uint64_t pol) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+            smem_addr(stage)),
+        "l"(__cvta_generic_to_global(src)), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
+        : "memory");
+}
+
+// Wait (every lane) until the mbarrier's phase with parity `par` completes;
+// false after `lim` polls.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t par, uint64_t lim) {
+    for (uint64_t k = 0; k < lim; ++k) {
+        uint32_t ok;
+        asm volatile(
+            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+            : "=r"(ok)
+            : "r"(smem_addr(bar)), "r"(par)
+            : "memory");
+        if (ok) return true;
+    }
+    return false;
 }
 
 template <int U>
@@ -607,45 +619,106 @@ __device__ __forceinline__ uint64_t q_pop(CtaQueue &q) {
     return 0;
 }
 
-// Request, segment and layout of one hashing task (nb = 0: a routing column
-// past the end of the prompt, nothing to hash).
+// Request, segment and layout of one hashing task (j = kNoTask: past the
+// warp's last task; nb() = 0: nothing to hash, e.g. a routing column past
+// the end of the prompt).
+constexpr uint32_t kNoTask = 0xFFFFFFFFu;
 struct TaskMeta {
-    uint32_t r, j, nblk, seg, nb;
+    uint32_t r, j, nblk, segoff;
     uint64_t tokoff, bo;
+    __device__ __forceinline__ uint32_t nb() const {
+        return j != kNoTask && j * kSegBlocks < nblk ? min(kSegBlocks, nblk - j * kSegBlocks) : 0;
+    }
 };
 
-__device__ __forceinline__ TaskMeta task_meta(const DevState &d, uint32_t t, uint32_t n, uint32_t ncol, uint32_t nhr,
-                                              int lane) {
-    TaskMeta m;
-    if (t < ncol) {
-        m.j = t / n;
-        m.r = t - m.j * n;
-    } else if (t < ncol + nhr) {
-        m.r = find_req(d.r_hoff, n, t - ncol, lane);
-        m.j = d.Ccols + (t - ncol - __ldg(d.r_hoff + m.r));
-    } else {
-        m.r = find_req(d.r_toff, n, t - ncol - nhr, lane);
-        m.j = d.H + (t - ncol - nhr - __ldg(d.r_toff + m.r));
+// A hashing warp's tasks: in each of the three parts (routing columns, head
+// rest, tails) its contiguous share of that part's tasks (the gw-th of nhw
+// equal runs), in order.  The request of a task in the second and third
+// part is found once per part (find_req) and then followed; a request's
+// layout is loaded when the request changes.  Whole warp (uniform).
+struct TaskCursor {
+    uint32_t part, t, hi;     // current part, next task in it, end of this warp's share
+    uint32_t r, rbeg, rend;   // parts 1-2: request of task t and its range in the part (r = kNoTask: not found yet)
+    TaskMeta lay;             // layout of request lay.r (lay.r = kNoTask: none)
+    uint32_t gw, nhw, n, T[3];
+
+    __device__ __forceinline__ void share() {
+        t = uint32_t(uint64_t(T[part]) * gw / nhw);
+        hi = uint32_t(uint64_t(T[part]) * (gw + 1) / nhw);
+        r = kNoTask;
     }
-    m.nblk = d.r_nblk[m.r];
-    m.seg = d.r_segoff[m.r] + m.j;
-    m.tokoff = d.r_tokoff[m.r];
-    m.bo = d.r_blkoff[m.r];
-    const uint32_t b0 = m.j * kSegBlocks;
-    m.nb = b0 < m.nblk ? min(kSegBlocks, m.nblk - b0) : 0;
-    return m;
-}
+    __device__ __forceinline__ void init(uint32_t gw_, uint32_t nhw_, uint32_t n_, uint32_t ncol, uint32_t nhr,
+                                         uint32_t total) {
+        gw = gw_;
+        nhw = nhw_;
+        n = n_;
+        T[0] = ncol;
+        T[1] = nhr;
+        T[2] = total - ncol - nhr;
+        part = 0;
+        lay.r = kNoTask;
+        share();
+    }
+    __device__ __forceinline__ TaskMeta next(const DevState &d, int lane) {
+        while (t >= hi && part < 2) {
+            ++part;
+            share();
+        }
+        TaskMeta m;
+        if (t >= hi) {
+            m.r = 0;
+            m.j = kNoTask;
+            m.nblk = m.segoff = 0;
+            m.tokoff = m.bo = 0;
+            return m;
+        }
+        uint32_t rr, j;
+        if (part == 0) {
+            j = t / n;
+            rr = t - j * n;
+        } else {
+            const uint32_t *off = part == 1 ? d.r_hoff : d.r_toff;
+            if (r == kNoTask) {
+                r = find_req(off, n, t, lane);
+                rbeg = __ldg(off + r);
+                rend = r + 1 < n ? __ldg(off + r + 1) : T[part];
+            }
+            while (t >= rend) {   // ends at the last request, whose range ends at T[part] > t
+                ++r;
+                rbeg = rend;
+                rend = r + 1 < n ? __ldg(off + r + 1) : T[part];
+            }
+            rr = r;
+            j = (part == 1 ? d.Ccols : d.H) + (t - rbeg);
+        }
+        ++t;
+        if (rr != lay.r) {
+            lay.r = rr;
+            lay.nblk = d.r_nblk[rr];
+            lay.segoff = d.r_segoff[rr];
+            lay.tokoff = d.r_tokoff[rr];
+            lay.bo = d.r_blkoff[rr];
+        }
+        m = lay;
+        m.j = j;
+        return m;
+    }
+};
 
 template <int U, bool kAdapt>
-__global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_constant__ DevState d,
+__global__ void __launch_bounds__(HP<U>::kThreads, kMinBlocks) k_hash_probe(const __grid_constant__ DevState d,
                                                                    const uint32_t *__restrict__ tokens, uint64_t E) {
     pdl_enter();
     extern __shared__ __align__(16) uint4 s_stage[];
+    constexpr int S = HP<U>::kStages;
     __shared__ CtaQueue q;
+    __shared__ uint64_t s_bar[kHashWarps * S];   // one mbarrier per stage
     __shared__ uint32_t s_go, s_last;
     if (threadIdx.x == 0) {
         s_go = !has_err(d.err);   // one decision per CTA (the CTA meets barriers below)
         q.head = q.tail = q.hash_done = q.busy = 0;
+        for (int i = 0; i < kHashWarps * S; ++i) mbar_init(s_bar + i);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     for (uint32_t i = threadIdx.x; i < kQCap; i += blockDim.x) q.seq[i] = i;
     __syncthreads();
@@ -659,43 +732,58 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
         const uint32_t n = d.info->n, ncol = d.info->col_tasks, nhr = d.info->head_segs;
         const uint32_t total = d.info->tasks;
         const HashLane<U> hl(d, lane);
-        uint4 *const stage = s_stage + wid * 2 * HP<U>::kStage;
-        auto issue = [&](const TaskMeta &m, uint4 *st) {
-            if (m.nb)
-                stage_segment<U>(hl, st,
-                                 reinterpret_cast<const uint4 *>(tokens + m.tokoff + uint64_t(m.j) * kSegBlocks * d.B),
-                                 m.nb, lane, pol);
+        uint4 *const stage = s_stage + wid * S * HP<U>::kStage;
+        uint64_t *const bar = s_bar + wid * S;
+        constexpr uint64_t kWaitLimit = 1ull << 24;   // polls of a stage's mbarrier (seconds)
+        uint32_t par = 0, pend = 0;                    // per stage: parity of its next phase; copy issued, not waited
+        auto issue = [&](const TaskMeta &m, uint32_t slot) {
+            const uint32_t nb = m.nb();
+            if (nb) {
+                if (lane == 0)
+                    bulk_to_stage(stage + slot * HP<U>::kStage,
+                                  reinterpret_cast<const uint4 *>(tokens + m.tokoff + uint64_t(m.j) * kSegBlocks * d.B),
+                                  nb * d.B * 4, bar + slot, pol);
+                pend |= 1u << slot;
+            }
         };
-        // the task being copied (cur) and the next one, looked up a task ahead
-        TaskMeta cur{}, nxt{};
-        if (gw < total) {
-            cur = task_meta(d, gw, n, ncol, nhr, lane);
-            issue(cur, stage);
+        TaskCursor cur_t;
+        cur_t.init(gw, nhw, n, ncol, nhr, total);
+        // m[s]: the warp's k-th task + s; the copies of m[0 .. S-2] are
+        // issued, m[S-1] is looked up and issued next
+        TaskMeta m[S];
+#pragma unroll
+        for (int s = 0; s < S; ++s) {
+            m[s] = cur_t.next(d, lane);
+            if (s + 1 < S) issue(m[s], s);
         }
-        cp_async_commit();
-        if (uint64_t(gw) + nhw < total) nxt = task_meta(d, gw + nhw, n, ncol, nhr, lane);
-        uint32_t it = 0;
-        for (uint32_t t = gw; t < total; t += nhw, ++it) {
-            const bool more = uint64_t(t) + nhw < total;
-            if (more) issue(nxt, stage + ((it + 1) & 1) * HP<U>::kStage);
-            cp_async_commit();
-            TaskMeta nn{};
-            if (uint64_t(t) + 2 * uint64_t(nhw) < total) nn = task_meta(d, t + 2 * nhw, n, ncol, nhr, lane);
-            cp_async_wait<1>();   // this task's copy is complete
-            if (cur.nb) {
+        for (uint32_t k = 0; m[0].j != kNoTask; ++k) {
+            issue(m[S - 1], (k + S - 1) % S);
+            const TaskMeta mn = cur_t.next(d, lane);
+            const TaskMeta &cur = m[0];
+            const uint32_t cnb = cur.nb(), slot = k % S;
+            if (cnb) {
+                if (!mbar_wait(bar + slot, (par >> slot) & 1, kWaitLimit)) {
+                    if (lane == 0) set_err(d.err, DM_ERR_TIMEOUT);
+                    break;
+                }
+                par ^= 1u << slot;
+                pend &= ~(1u << slot);
                 uint4 v[2][U];
-                read_stage<U>(stage + (it & 1) * HP<U>::kStage, lane, v);
-                const uint32_t b0 = cur.j * kSegBlocks;
+                read_stage<U>(stage + slot * HP<U>::kStage, lane, v);
+                // the stage's next bulk copy (async proxy) comes after these reads
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                const uint32_t b0 = cur.j * kSegBlocks, seg = cur.segoff + cur.j;
                 uint64_t P[2], tot1, sum2;
-                hash_loaded<U, true, kAdapt>(hl, v, b0, cur.nb, min(d.Kf2, cur.nblk), lane, P, tot1, sum2,
+                hash_loaded<U, true, kAdapt>(hl, v, b0, cnb, min(d.Kf2, cur.nblk), lane, P, tot1, sum2,
                                              kAdapt ? d.p2local + cur.bo + b0 : nullptr);
                 uint64_t *out = d.plocal + cur.bo + b0;
-                if ((uint32_t)lane < cur.nb) out[lane] = P[0];
-                if ((uint32_t)lane + 32 < cur.nb) out[lane + 32] = P[1];
+                if ((uint32_t)lane < cnb) out[lane] = P[0];
+                if ((uint32_t)lane + 32 < cnb) out[lane + 32] = P[1];
                 if (lane == 0) {
-                    d.seg_total[cur.seg] = tot1;
-                    d.seg_total2[cur.seg] = sum2;
-                    d.seg_req[cur.seg] = cur.r;
+                    d.seg_total[seg] = tot1;
+                    d.seg_total2[seg] = sum2;
+                    d.seg_req[seg] = cur.r;
                 }
                 const uint32_t hs = min((cur.nblk + kSegBlocks - 1) / kSegBlocks, d.H);
                 if (cur.j < hs) {
@@ -713,15 +801,18 @@ __global__ void __launch_bounds__(HP<U>::kThreads, 3) k_hash_probe(const __grid_
                         __syncwarp();
                     }
                     if (lane == 0) {
-                        seg_pub_write(d.seg_pub + cur.seg, E, tot1, sum2, pf, kk < kSegBlocks ? pk : 0, px);
+                        seg_pub_write(d.seg_pub + seg, E, tot1, sum2, pf, kk < kSegBlocks ? pk : 0, px);
                         if (cur.j + 1 == hs) q_push(q, d, qentry(cur.r, 0));   // the request's route task
                     }
                 }
             }
-            cur = nxt;
-            nxt = nn;
+#pragma unroll
+            for (int s = 0; s + 1 < S; ++s) m[s] = m[s + 1];
+            m[S - 1] = mn;
         }
-        cp_async_wait<0>();
+        // copies still in flight (only after a timeout): let them land
+        for (uint32_t s = 0; s < (uint32_t)S; ++s)
+            if ((pend >> s) & 1) mbar_wait(bar + s, (par >> s) & 1, kWaitLimit);
         if (lane == 0) atomicAdd(&q.hash_done, 1u);
     } else {
         // ---- probing warp: work off the CTA's queue ----
