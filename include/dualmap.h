@@ -55,7 +55,8 @@ typedef enum {
     DM_ERR_ORDER = 6,         /* batch time earlier than the previous batch's */
     DM_ERR_CUDA = 7,          /* a CUDA runtime call failed */
     DM_ERR_TIMEOUT = 8,       /* a bounded device-side loop gave up (state is corrupt) */
-    DM_ERR_OOM = 9            /* device or host allocation failed */
+    DM_ERR_OOM = 9,           /* device or host allocation failed */
+    DM_ERR_BOUNDS = 10        /* debug builds only (libdualmap_debug.so): a device-side index check failed */
 } dm_status;
 
 /* Choice rules of dm_route_batch's last step.
@@ -339,6 +340,38 @@ DM_API dm_status dm_route_batch_host(dm_handle *h, const dm_batch *batch, const 
  * stream has been synchronised (dm_last_error does).  Use pinned host memory
  * for the copies to overlap. */
 DM_API dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
+
+/* Sharded routing (no paper counterpart: the multi-GPU split of the routing
+ * step).  Each of several handles holds the same replicated state (same
+ * config and seed, same instance adds/removes, same batches), typically
+ * one per GPU.  For a batch of n requests each handle calls
+ * dm_route_shard_begin with its own request range [r0, r1) (the ranges
+ * partition [0, n)): it drains the queues and lays the whole batch out
+ * exactly as dm_route_batch does, but hashes, looks up and probes only
+ * requests r0 .. r1-1 (Sec. 3.2, App. A.3.2 for those steps).  It then
+ * exports its results with dm_shard_export, the callers exchange the
+ * buffers (an all-gather), every handle imports the other ranges with
+ * dm_shard_import, and dm_route_shard_finish runs the rest of the step
+ * (choices in arrival order, queues, metrics; the batch becomes the pending
+ * commit) on the whole batch.  Every handle then holds the outputs and state
+ * that dm_route_batch would have produced.  Not with the adaptive prefix
+ * length (DM_ERR_INVALID_ARG).  Between begin and finish every other call
+ * that routes, commits, rebalances, hashes or changes the instances returns
+ * DM_ERR_ORDER.
+ *
+ * Export buffer (device memory, 8-byte aligned, written in stream order):
+ * the local prefix values of the range's blocks (8 bytes each), its
+ * segments' f1 totals (8 bytes), then 4-byte values: its segments' owning
+ * requests, and per request its hash length, both candidates and both first
+ * missing blocks, array by array.  `*bytes_dev` (device, may be null)
+ * receives the size: 8 (blocks + segments) + 4 (segments + 5 requests);
+ * a buffer smaller than that records DM_ERR_CAPACITY (sticky).  Import reads
+ * the same layout for its range from `buf_dev` (`bytes` long). */
+DM_API dm_status dm_route_shard_begin(dm_handle *h, const dm_batch *batch, uint32_t r0, uint32_t r1);
+DM_API dm_status dm_shard_export(dm_handle *h, uint32_t r0, uint32_t r1, void *buf_dev, uint64_t cap,
+                                 uint64_t *bytes_dev);
+DM_API dm_status dm_shard_import(dm_handle *h, uint32_t r0, uint32_t r1, const void *buf_dev, uint64_t bytes);
+DM_API dm_status dm_route_shard_finish(dm_handle *h, const dm_batch *batch, const dm_route_out *out);
 
 /* Hotspot-aware rebalancing (Sec. 3.3, Eq. "rebalance"; App. A.1.2), to be
  * called after dm_route_batch and before dm_commit_cache.  Hot instances

@@ -948,10 +948,10 @@ static uint32_t leading_hits(const lru_t *c, const uint64_t *keys, uint32_t nblk
     return m;
 }
 
-int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
-                   const uint32_t *lengths, uint32_t n, uint64_t t_batch,
-                   uint32_t *cand1, uint32_t *cand2, uint32_t *hit1, uint32_t *hit2,
-                   uint64_t *ttft1, uint64_t *ttft2, uint32_t *chosen, uint8_t *switched)
+/* The start of a routed batch: argument checks, the queues drain for the
+ * elapsed time (Sec. 3.2 load = pending prefill), and the pending-commit
+ * arrays for n requests (keys filled in by the caller). */
+static int route_prologue(or_state *s, const uint32_t *lengths, uint32_t n, uint64_t t_batch)
 {
     const or_config *cf = &s->cfg;
     if (n > cf->max_batch) return OR_ERR_CAPACITY;
@@ -982,6 +982,22 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
     s->last_K = lk;
     s->last_n = n;
     if (!s->pend_final || !s->pend_nblk || !s->pend_keys) return OR_ERR_OOM;
+    return OR_OK;
+}
+
+static int route_choose(or_state *s, const uint32_t *lengths, uint32_t n, uint64_t t_batch,
+                        const uint32_t *cand1, const uint32_t *cand2, const uint32_t *hit1, const uint32_t *hit2,
+                        const uint32_t *hall, uint64_t *ttft1, uint64_t *ttft2, uint32_t *chosen,
+                        uint8_t *switched);
+
+int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
+                   const uint32_t *lengths, uint32_t n, uint64_t t_batch,
+                   uint32_t *cand1, uint32_t *cand2, uint32_t *hit1, uint32_t *hit2,
+                   uint64_t *ttft1, uint64_t *ttft2, uint32_t *chosen, uint8_t *switched)
+{
+    const or_config *cf = &s->cfg;
+    int rc0 = route_prologue(s, lengths, n, t_batch);
+    if (rc0) return rc0;
 
     /* hits on every live instance, for the rules that look at all of them */
     uint32_t *hall = NULL;
@@ -1019,6 +1035,30 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
                 hall[(size_t)r * cf->max_instances + id] =
                     s->state[id] == INST_LIVE ? cf->block_tokens * leading_hits(&s->cache[id], keys, nblk) : 0;
     }
+    int rc2 = route_choose(s, lengths, n, t_batch, cand1, cand2, hit1, hit2, hall, ttft1, ttft2, chosen, switched);
+    free(hall);
+    if (rc2) return rc2;
+    if (cf->adapt_step_blocks && n > 0) {
+        s->ad_requests += n;
+        if (++s->ad_batches == cf->adapt_window) {
+            int rc = adapt_window_end(s);
+            if (rc) return rc;
+        }
+    }
+    s->pending = 1;
+    return OR_OK;
+}
+
+/* The choice half of a routed batch (Sec. 3.2 "SLO-Aware Strategy"): in
+ * arrival order each request's TTFT estimates, its choice (hall: hits on
+ * every instance, for the cluster-wide rules, else NULL), its queue entry
+ * and the loads, the metrics; then the batch's CV sample. */
+static int route_choose(or_state *s, const uint32_t *lengths, uint32_t n, uint64_t t_batch,
+                        const uint32_t *cand1, const uint32_t *cand2, const uint32_t *hit1, const uint32_t *hit2,
+                        const uint32_t *hall, uint64_t *ttft1, uint64_t *ttft2, uint32_t *chosen,
+                        uint8_t *switched)
+{
+    const or_config *cf = &s->cfg;
     /* 2) choices in arrival order; loads update as we go */
     s->both_over = 0;
     for (uint32_t r = 0; r < n; r++) {
@@ -1053,19 +1093,73 @@ int or_route_batch(or_state *s, const uint32_t *tokens, const uint64_t *offsets,
         s->m_switched += switched[r];
         s->m_est_slo_met += s->W[ch] <= cf->slo_us;   /* the load including this request */
     }
-    free(hall);
     if (n > 0) {
         s->m_cv_last = load_cv(s);
         s->m_cv_sum += s->m_cv_last;
         s->m_batches++;
     }
-    if (cf->adapt_step_blocks && n > 0) {
-        s->ad_requests += n;
-        if (++s->ad_batches == cf->adapt_window) {
-            int rc = adapt_window_end(s);
-            if (rc) return rc;
-        }
+    return OR_OK;
+}
+
+/* Sharded routing, the per-rank half (the multi-GPU split of the routing
+ * step; no paper counterpart): for requests r0 .. r1-1 of a batch, their
+ * block keys, hash length, candidates and hits, against the state as it
+ * stands (the batch's start: nothing here changes the state).  keys gets
+ * every request's keys, request after request (at most key_cap).  The
+ * fixed prefix length and the pair rules only. */
+int or_route_part(or_state *s, const uint32_t *tokens, const uint64_t *offsets, const uint32_t *lengths,
+                  uint32_t r0, uint32_t r1, uint32_t *K, uint32_t *cand1, uint32_t *cand2, uint32_t *hit1,
+                  uint32_t *hit2, uint64_t *keys, uint64_t key_cap)
+{
+    const or_config *cf = &s->cfg;
+    if (cf->adapt_step_blocks || cf->choice_rule >= OR_RULE_GLOBAL_LEAST_LOADED || r0 > r1) return OR_ERR_INVALID_ARG;
+    if (n_live(s) < 2) return OR_ERR_NO_INSTANCES;
+    uint64_t used = 0;
+    for (uint32_t r = r0; r < r1; r++) {
+        if (lengths[r] < cf->block_tokens) return OR_ERR_INVALID_ARG;
+        const uint32_t nb = lengths[r] / cf->block_tokens;
+        if (used + nb > key_cap) return OR_ERR_CAPACITY;
+        uint64_t pos[2];
+        uint32_t nblk = prompt_keys(s, tokens + offsets[r], lengths[r], keys + used, pos);
+        const uint32_t k = r - r0;
+        K[k] = cf->route_prefix_blocks < nblk ? cf->route_prefix_blocks : nblk;
+        uint32_t c1 = ring_owner(s, 0, pos[0]);
+        uint32_t c2 = ring_owner(s, 1, pos[1]);
+        if (c2 == c1) c2 = next_live_after(s, c1);
+        cand1[k] = c1;
+        cand2[k] = c2;
+        hit1[k] = cf->block_tokens * leading_hits(&s->cache[c1], keys + used, nblk);
+        hit2[k] = cf->block_tokens * leading_hits(&s->cache[c2], keys + used, nblk);
+        used += nblk;
     }
+    return OR_OK;
+}
+
+/* Sharded routing, the replicated half: the batch routed with every
+ * request's keys, hash length, candidates and hits given (gathered from
+ * the ranks' or_route_part): the same drain, choices, queues, metrics and
+ * pending commit as or_route_batch. */
+int or_route_given(or_state *s, const uint32_t *lengths, uint32_t n, uint64_t t_batch, const uint32_t *K,
+                   const uint32_t *cand1, const uint32_t *cand2, const uint32_t *hit1, const uint32_t *hit2,
+                   const uint64_t *keys, uint64_t *ttft1, uint64_t *ttft2, uint32_t *chosen, uint8_t *switched)
+{
+    const or_config *cf = &s->cfg;
+    if (cf->adapt_step_blocks || cf->choice_rule >= OR_RULE_GLOBAL_LEAST_LOADED) return OR_ERR_INVALID_ARG;
+    int rc = route_prologue(s, lengths, n, t_batch);
+    if (rc) return rc;
+    uint64_t used = 0;
+    for (uint32_t r = 0; r < n; r++) {
+        const uint32_t nb = lengths[r] / cf->block_tokens;
+        uint64_t *k = (uint64_t *)malloc((size_t)(nb ? nb : 1) * sizeof(uint64_t));
+        if (!k) return OR_ERR_OOM;
+        memcpy(k, keys + used, (size_t)nb * sizeof(uint64_t));
+        used += nb;
+        s->pend_keys[r] = k;
+        s->pend_nblk[r] = nb;
+        s->last_K[r] = K[r];
+    }
+    rc = route_choose(s, lengths, n, t_batch, cand1, cand2, hit1, hit2, NULL, ttft1, ttft2, chosen, switched);
+    if (rc) return rc;
     s->pending = 1;
     return OR_OK;
 }

@@ -88,6 +88,10 @@ def lib():
             "or_choose": (C.c_uint32, [C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32, C.c_uint32,
                                        C.c_uint64, C.c_uint64, C.c_uint64, C.c_uint32,
                                        P(C.c_uint64), P(C.c_uint64), P(C.c_uint8)]),
+            "or_route_part": (C.c_int, [V, u32p, u64p, u32p, C.c_uint32, C.c_uint32, u32p, u32p, u32p, u32p,
+                                        u32p, u64p, C.c_uint64]),
+            "or_route_given": (C.c_int, [V, u32p, C.c_uint32, C.c_uint64, u32p, u32p, u32p, u32p, u32p, u64p,
+                                         u64p, u64p, u32p, u8p]),
             "or_route_batch": (C.c_int, [V, u32p, u64p, u32p, C.c_uint32, C.c_uint64,
                                          u32p, u32p, u32p, u32p, u64p, u64p, u32p, u8p]),
             "or_commit": (C.c_int, [V]),
@@ -246,6 +250,40 @@ class Oracle:
         rc = lib().or_route_batch(self.h, tok, np.ascontiguousarray(offsets, dtype=np.uint64),
                                   np.ascontiguousarray(lengths, dtype=np.uint32), n, t_batch,
                                   out["cand1"], out["cand2"], out["hit1"], out["hit2"],
+                                  out["ttft1"], out["ttft2"], out["chosen"], out["switched"])
+        return rc, out
+
+    def route_part(self, tokens, offsets, lengths, r0, r1):
+        """Sharded routing, one rank's half: keys (concatenated), hash length,
+        candidates and hits of requests r0 .. r1-1, the state unchanged."""
+        B = self.B
+        lens = np.ascontiguousarray(lengths, dtype=np.uint32)
+        k = r1 - r0
+        out = dict(K=np.zeros(k, np.uint32), cand1=np.zeros(k, np.uint32), cand2=np.zeros(k, np.uint32),
+                   hit1=np.zeros(k, np.uint32), hit2=np.zeros(k, np.uint32))
+        cap = int((lens[r0:r1] // B).sum())
+        keys = np.zeros(max(cap, 1), np.uint64)
+        tok = np.ascontiguousarray(tokens, dtype=np.uint32)
+        if tok.size == 0:
+            tok = np.zeros(1, np.uint32)
+        rc = lib().or_route_part(self.h, tok, np.ascontiguousarray(offsets, dtype=np.uint64), lens, r0, r1,
+                                 out["K"], out["cand1"], out["cand2"], out["hit1"], out["hit2"], keys, cap)
+        out["keys"] = keys[:cap]
+        return rc, out
+
+    def route_given(self, lengths, t_batch, K, cand1, cand2, hit1, hit2, keys):
+        """Sharded routing, the replicated half: the batch routed with every
+        request's keys, hash length, candidates and hits given."""
+        lens = np.ascontiguousarray(lengths, dtype=np.uint32)
+        n = len(lens)
+        out = dict(ttft1=np.zeros(n, np.uint64), ttft2=np.zeros(n, np.uint64), chosen=np.zeros(n, np.uint32),
+                   switched=np.zeros(n, np.uint8))
+        a = lambda x, t: np.ascontiguousarray(x, dtype=t)
+        kk = a(keys, np.uint64)
+        if kk.size == 0:
+            kk = np.zeros(1, np.uint64)
+        rc = lib().or_route_given(self.h, lens, n, t_batch, a(K, np.uint32), a(cand1, np.uint32),
+                                  a(cand2, np.uint32), a(hit1, np.uint32), a(hit2, np.uint32), kk,
                                   out["ttft1"], out["ttft2"], out["chosen"], out["switched"])
         return rc, out
 

@@ -16,6 +16,10 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(ROOT, "_build", "dualmap")
 LIB = os.path.join(HERE, "libdualmap.so")
+# debug build: the same sources with -DDM_DEBUG (device index checks that
+# record DM_ERR_BOUNDS), its own objects and library
+BUILD_DEBUG = os.path.join(ROOT, "_build", "dualmap_debug")
+LIB_DEBUG = os.path.join(HERE, "libdualmap_debug.so")
 SOURCES = ["dm_api.cu", "dm_setup.cu", "dm_hash.cu", "dm_route.cu", "dm_choice.cu", "dm_commit.cu",
            "dm_rebalance.cu", "dm_ring.cu", "dm_noalloc.cu", "dm_potc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -35,13 +39,16 @@ def _stale(out, deps):
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force=False, verbose=False, extra=()):
-    os.makedirs(BUILD, exist_ok=True)
+def build(force=False, verbose=False, extra=(), debug=False):
+    bdir, lib_path = (BUILD_DEBUG, LIB_DEBUG) if debug else (BUILD, LIB)
+    if debug:
+        extra = ("-DDM_DEBUG",) + tuple(extra)
+    os.makedirs(bdir, exist_ok=True)
     headers = [os.path.join(CSRC, "dm_internal.cuh"), os.path.join(ROOT, "include", "dualmap.h")]
     objs, jobs = [], []
     for s in SOURCES:
         src = os.path.join(CSRC, s)
-        obj = os.path.join(BUILD, s.replace(".cu", ".o"))
+        obj = os.path.join(bdir, s.replace(".cu", ".o"))
         objs.append(obj)
         if force or _stale(obj, [src] + headers):
             jobs.append([nvcc(), *ARCH, *FLAGS, *extra, "-c", src, "-o", obj])
@@ -51,17 +58,16 @@ def build(force=False, verbose=False, extra=()):
                 sys.stderr.write(res.stdout + res.stderr)
             if res.returncode:
                 raise RuntimeError("nvcc failed: " + " ".join(cmd))
-    if force or jobs or _stale(LIB, objs):
-        tmp = LIB + f".tmp{os.getpid()}"
+    if force or jobs or _stale(lib_path, objs):
+        tmp = lib_path + f".tmp{os.getpid()}"
         cmd = [nvcc(), *ARCH, "-shared", "-o", tmp, *objs]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode:
             sys.stderr.write(res.stdout + res.stderr)
             raise RuntimeError("link failed")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
-    build(force="--force" in sys.argv, verbose=True)
-    print(LIB)
+    print(build(force="--force" in sys.argv, verbose=True, debug="--debug" in sys.argv))

@@ -32,6 +32,8 @@ struct dm_handle {
     bool have_time = false;
     bool pending = false;
     uint32_t pending_n = 0;
+    bool shard_open = false;   // between dm_route_shard_begin and dm_route_shard_finish
+    uint32_t shard_n = 0;
     uint64_t pending_seq0 = 0;
     uint32_t rebalance_calls = 0;
     int hash_grid = 0;
@@ -189,6 +191,7 @@ const char *dm_status_string(dm_status s) {
         case DM_ERR_CUDA: return "CUDA runtime error";
         case DM_ERR_TIMEOUT: return "bounded device loop gave up";
         case DM_ERR_OOM: return "out of memory";
+        case DM_ERR_BOUNDS: return "a device index check failed (debug build)";
     }
     return "unknown status";
 }
@@ -528,6 +531,7 @@ static dm_status ring_change(dm_handle *h, uint32_t id, bool add) {
 dm_status dm_add_instance(dm_handle *h, uint32_t id) {
     dm_status s = check_live(h);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     DevState &d = h->d;
     if (id >= d.M) return DM_ERR_INVALID_ARG;
     if (h->state[id] == 1) return DM_ERR_DUPLICATE_ID;
@@ -607,6 +611,7 @@ dm_status dm_add_instance(dm_handle *h, uint32_t id) {
 dm_status dm_remove_instance(dm_handle *h, uint32_t id) {
     dm_status s = check_live(h);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (id >= h->d.M || h->state[id] != 1) return DM_ERR_UNKNOWN_ID;
     s = ring_change(h, id, false);
     if (s) return s;
@@ -636,18 +641,18 @@ static bool tokens_aligned(const dm_batch *b) {
 // through dm_route_batch_d and does not rebalance.
 static bool pair_handle(const dm_handle *h) { return h->cfg.candidates == 0 || h->cfg.candidates == 2; }
 
-dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
-    dm_status s = check_batch(h, b, o);
-    if (s) return s;
+// Routing, first half: time, drain and layout, then the routing kernel for
+// requests r0 .. r1-1 (all of them, or one shard).
+static dm_status route_begin(dm_handle *h, const dm_batch *b, uint32_t r0, uint32_t r1) {
     if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!tokens_aligned(b)) return DM_ERR_INVALID_ARG;
-    if (!o) return DM_ERR_INVALID_ARG;
     if (h->n_live < 2) return DM_ERR_NO_INSTANCES;
     if (h->have_time && b->batch_time_us < h->t_prev) return DM_ERR_ORDER;
     const uint64_t delta = h->have_time ? b->batch_time_us - h->t_prev : 0;
     const uint64_t t0 = h->have_time ? h->t_prev : b->batch_time_us;   // start of the drain window
     h->t_prev = b->batch_time_us;
     h->have_time = true;
+    h->pending = false;   // the batch scratch now holds this batch
     const DevState &d = h->d;
     cudaError_t e;
     { Stage st(h, DM_STAGE_SETUP); e = dm::launch_setup_route(d, *b, delta, t0, h->st); }   // drain included
@@ -655,9 +660,17 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
         Stage st(h, DM_STAGE_HASH);
         // a fresh epoch mask per call: records of earlier batches never pass its check
         const uint64_t E = dm::fmix64(++h->epoch ^ 0x6a09e667f3bcc909ull);
-        e = dm::launch_hash_probe(d, *b, E, h->st);
+        e = dm::launch_hash_probe(d, *b, E, r0, r1, h->st);
     }
-    if (e == cudaSuccess && b->n) {
+    return e == cudaSuccess ? DM_OK : map_cuda(h, e);
+}
+
+// Routing, second half: carries, choices in arrival order, queues,
+// metrics, the adaptive window; the batch becomes the pending commit.
+static dm_status route_finish(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    const DevState &d = h->d;
+    cudaError_t e = cudaSuccess;
+    if (b->n) {
         Stage st(h, DM_STAGE_CHOICE);
         e = dm::launch_choice(d, *o, b->n, h->seq_next, b->batch_time_us, h->st);
     }
@@ -683,9 +696,58 @@ dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o)
     return DM_OK;
 }
 
+dm_status dm_route_batch(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    dm_status s = check_batch(h, b, o);
+    if (s) return s;
+    if (!o) return DM_ERR_INVALID_ARG;
+    if (h->shard_open) return DM_ERR_ORDER;
+    s = route_begin(h, b, 0, b->n);
+    return s ? s : route_finish(h, b, o);
+}
+
+dm_status dm_route_shard_begin(dm_handle *h, const dm_batch *b, uint32_t r0, uint32_t r1) {
+    dm_status s = check_batch(h, b, nullptr);
+    if (s) return s;
+    if (r0 > r1 || r1 > b->n || h->d.ad_step) return DM_ERR_INVALID_ARG;
+    if (h->shard_open) return DM_ERR_ORDER;
+    s = route_begin(h, b, r0, r1);
+    if (s) return s;
+    h->shard_open = true;
+    h->shard_n = b->n;
+    return DM_OK;
+}
+
+dm_status dm_shard_export(dm_handle *h, uint32_t r0, uint32_t r1, void *buf_dev, uint64_t cap, uint64_t *bytes_dev) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!h->shard_open || r0 > r1 || r1 > h->shard_n || (r1 > r0 && !buf_dev)) return DM_ERR_INVALID_ARG;
+    const cudaError_t e = dm::launch_shard_copy(h->d, true, r0, r1, static_cast<uint8_t *>(buf_dev), cap,
+                                                static_cast<uint64_t *>(bytes_dev), h->st);
+    return e == cudaSuccess ? DM_OK : map_cuda(h, e);
+}
+
+dm_status dm_shard_import(dm_handle *h, uint32_t r0, uint32_t r1, const void *buf_dev, uint64_t bytes) {
+    dm_status s = check_live(h);
+    if (s) return s;
+    if (!h->shard_open || r0 > r1 || r1 > h->shard_n || (r1 > r0 && !buf_dev)) return DM_ERR_INVALID_ARG;
+    const cudaError_t e = dm::launch_shard_copy(h->d, false, r0, r1,
+                                                static_cast<uint8_t *>(const_cast<void *>(buf_dev)), bytes, nullptr,
+                                                h->st);
+    return e == cudaSuccess ? DM_OK : map_cuda(h, e);
+}
+
+dm_status dm_route_shard_finish(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
+    dm_status s = check_batch(h, b, o);
+    if (s) return s;
+    if (!o || !h->shard_open || b->n != h->shard_n) return DM_ERR_INVALID_ARG;
+    h->shard_open = false;
+    return route_finish(h, b, o);
+}
+
 dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *b, const dm_route_out *o) {
     dm_status s = check_batch(h, b, o);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!o) return DM_ERR_INVALID_ARG;
     cudaError_t e = cudaSuccess;
@@ -746,6 +808,7 @@ dm_status dm_route_batch_host_async(dm_handle *h, const dm_batch *b, const dm_ro
 dm_status dm_route_batch_d(dm_handle *h, const dm_batch *b, const dm_route_out_d *o) {
     dm_status s = check_batch(h, b, nullptr);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (!tokens_aligned(b) || !o) return DM_ERR_INVALID_ARG;
     if (b->n > 0 && (!o->cand || !o->hit || !o->ttft || !o->chosen || !o->switched)) return DM_ERR_INVALID_ARG;
     const DevState &d = h->d;
@@ -779,6 +842,7 @@ dm_status dm_route_batch_host(dm_handle *h, const dm_batch *b, const dm_route_ou
 dm_status dm_rebalance(dm_handle *h, dm_migration *out_host, uint32_t cap, uint32_t *n_out) {
     dm_status s = check_live(h);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!n_out || (cap && !out_host)) return DM_ERR_INVALID_ARG;
     if (cap > h->rb_out_cap || !h->rb_n_dev) {   // device staging of the results
@@ -806,6 +870,7 @@ dm_status dm_rebalance(dm_handle *h, dm_migration *out_host, uint32_t cap, uint3
 dm_status dm_rebalance_async(dm_handle *h, dm_migration *out_dev, uint32_t cap, uint32_t *n_out_dev) {
     dm_status s = check_live(h);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (!pair_handle(h)) return DM_ERR_INVALID_ARG;
     if (!n_out_dev || (cap && !out_dev)) return DM_ERR_INVALID_ARG;
     const uint32_t n = h->pending ? h->pending_n : 0;
@@ -820,6 +885,7 @@ dm_status dm_rebalance_async(dm_handle *h, dm_migration *out_dev, uint32_t cap, 
 dm_status dm_commit_cache(dm_handle *h) {
     dm_status s = check_live(h);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (!h->pending) return DM_OK;
     cudaError_t e;
     {
@@ -834,6 +900,7 @@ dm_status dm_hash_prompts(dm_handle *h, const dm_batch *b, uint64_t *keys_dev, u
                           uint64_t *pos_dev) {
     dm_status s = check_batch(h, b, nullptr);
     if (s) return s;
+    if (h->shard_open) return DM_ERR_ORDER;   // a sharded batch is between begin and finish
     if (b->n && (!keys_dev || !key_off_dev || !pos_dev)) return DM_ERR_INVALID_ARG;
     if (!tokens_aligned(b)) return DM_ERR_INVALID_ARG;
     if (b->n == 0) return DM_OK;

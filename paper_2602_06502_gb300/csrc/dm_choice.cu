@@ -265,6 +265,7 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
             e.h2 = h2;
             e.moved = 0;
             e.arrival = t_batch;
+            DM_CHECK(ch < d.M, d.err);
             d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
         }
     }
@@ -485,6 +486,7 @@ __global__ void __launch_bounds__(1024) k_choice_global(DevState d, dm_route_out
             e.h2 = s_h2[rr];
             e.moved = 0;
             e.arrival = t_batch;
+            DM_CHECK(ch < d.M, d.err);
             d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
         }
     }
@@ -727,6 +729,7 @@ __global__ void __launch_bounds__(1024) k_choice_d(DevState d, dm_route_out_d o,
             e.h2 = nd > 1 ? h[1] : h[0];
             e.moved = 0;
             e.arrival = t_batch;
+            DM_CHECK(ch < d.M, d.err);
             d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
         }
     }

@@ -501,6 +501,8 @@ __device__ __forceinline__ TouchSeg touch_seg_load(const DevState &d, uint32_t s
     g.lh = d.loghome[f];
     g.cnt = min(nblk - first, kSegBlocks);
     g.f = f;
+    // the segment's records lie inside the instance's log window
+    DM_CHECK(f < d.M && g.p_first + 1 - g.front <= d.logcap && g.pidx + g.cnt <= d.max_blocks, d.err);
     return g;
 }
 

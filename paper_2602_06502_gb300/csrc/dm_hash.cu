@@ -439,9 +439,11 @@ __device__ __noinline__ bool route_task(const DevState &d, const uint32_t *token
     }
     uint32_t lb1, lb2;
     ring_search2(d, pos1, pos2, lane, lb1, lb2);
+    DM_CHECK(lb1 < d.R && lb2 < d.R, d.err);
     const uint32_t a = d.ring[0].owner[lb1];
     const uint32_t raw2 = d.ring[1].owner[lb2];
     const uint32_t b = raw2 != a ? raw2 : d.next_live[a];
+    DM_CHECK(a < d.M && b < d.M && a != b, d.err);
     RouteView rv;
     rv.t1 = d.table[a];
     rv.t2 = d.table[b];
@@ -640,21 +642,39 @@ struct TaskCursor {
     uint32_t part, t, hi;     // current part, next task in it, end of this warp's share
     uint32_t r, rbeg, rend;   // parts 1-2: request of task t and its range in the part (r = kNoTask: not found yet)
     TaskMeta lay;             // layout of request lay.r (lay.r = kNoTask: none)
-    uint32_t gw, nhw, n, T[3];
+    uint32_t gw, nhw, n, r0, nr;
+    uint32_t lo[3], T[3];     // per part: first task of requests r0 .. r0+nr-1 and their task count
+    uint32_t Tall[3];         // per part: tasks of the whole batch
 
     __device__ __forceinline__ void share() {
-        t = uint32_t(uint64_t(T[part]) * gw / nhw);
-        hi = uint32_t(uint64_t(T[part]) * (gw + 1) / nhw);
+        t = lo[part] + uint32_t(uint64_t(T[part]) * gw / nhw);
+        hi = lo[part] + uint32_t(uint64_t(T[part]) * (gw + 1) / nhw);
         r = kNoTask;
     }
-    __device__ __forceinline__ void init(uint32_t gw_, uint32_t nhw_, uint32_t n_, uint32_t ncol, uint32_t nhr,
-                                         uint32_t total) {
+    // The tasks of requests r0_ .. r1_-1 only (a shard of the batch; all of
+    // it when r0_ = 0 and r1_ = n_).
+    __device__ __forceinline__ void init(const DevState &d, uint32_t gw_, uint32_t nhw_, uint32_t n_, uint32_t ncol,
+                                         uint32_t nhr, uint32_t total, uint32_t r0_, uint32_t r1_) {
         gw = gw_;
         nhw = nhw_;
         n = n_;
-        T[0] = ncol;
-        T[1] = nhr;
-        T[2] = total - ncol - nhr;
+        r0 = r0_;
+        nr = r1_ - r0_;
+        Tall[0] = ncol;
+        Tall[1] = nhr;
+        Tall[2] = total - ncol - nhr;
+        lo[0] = 0;
+        T[0] = nr * d.Ccols;
+        if (r0_ == 0 && r1_ == n_) {
+            lo[1] = lo[2] = 0;
+            T[1] = Tall[1];
+            T[2] = Tall[2];
+        } else {
+            lo[1] = __ldg(d.r_hoff + r0_);
+            lo[2] = __ldg(d.r_toff + r0_);
+            T[1] = (r1_ < n_ ? __ldg(d.r_hoff + r1_) : Tall[1]) - lo[1];
+            T[2] = (r1_ < n_ ? __ldg(d.r_toff + r1_) : Tall[2]) - lo[2];
+        }
         part = 0;
         lay.r = kNoTask;
         share();
@@ -673,20 +693,20 @@ struct TaskCursor {
             return m;
         }
         uint32_t rr, j;
-        if (part == 0) {
-            j = t / n;
-            rr = t - j * n;
+        if (part == 0) {   // column-major over the shard's requests
+            j = t / nr;
+            rr = r0 + (t - j * nr);
         } else {
             const uint32_t *off = part == 1 ? d.r_hoff : d.r_toff;
             if (r == kNoTask) {
                 r = find_req(off, n, t, lane);
                 rbeg = __ldg(off + r);
-                rend = r + 1 < n ? __ldg(off + r + 1) : T[part];
+                rend = r + 1 < n ? __ldg(off + r + 1) : Tall[part];
             }
-            while (t >= rend) {   // ends at the last request, whose range ends at T[part] > t
+            while (t >= rend) {   // ends at the last request, whose range ends at Tall[part] > t
                 ++r;
                 rbeg = rend;
-                rend = r + 1 < n ? __ldg(off + r + 1) : T[part];
+                rend = r + 1 < n ? __ldg(off + r + 1) : Tall[part];
             }
             rr = r;
             j = (part == 1 ? d.Ccols : d.H) + (t - rbeg);
@@ -707,7 +727,8 @@ struct TaskCursor {
 
 template <int U, bool kAdapt>
 __global__ void __launch_bounds__(HP<U>::kThreads, kMinBlocks) k_hash_probe(const __grid_constant__ DevState d,
-                                                                   const uint32_t *__restrict__ tokens, uint64_t E) {
+                                                                   const uint32_t *__restrict__ tokens, uint64_t E,
+                                                                   uint32_t r0, uint32_t r1) {
     pdl_enter();
     extern __shared__ __align__(16) uint4 s_stage[];
     constexpr int S = HP<U>::kStages;
@@ -747,7 +768,7 @@ __global__ void __launch_bounds__(HP<U>::kThreads, kMinBlocks) k_hash_probe(cons
             }
         };
         TaskCursor cur_t;
-        cur_t.init(gw, nhw, n, ncol, nhr, total);
+        cur_t.init(d, gw, nhw, n, ncol, nhr, total, r0, r1);
         // m[s]: the warp's k-th task + s; the copies of m[0 .. S-2] are
         // issued, m[S-1] is looked up and issued next
         TaskMeta m[S];
@@ -774,6 +795,7 @@ __global__ void __launch_bounds__(HP<U>::kThreads, kMinBlocks) k_hash_probe(cons
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
                 const uint32_t b0 = cur.j * kSegBlocks, seg = cur.segoff + cur.j;
+                DM_CHECK(seg < d.max_segs && cur.bo + b0 + cnb <= d.max_blocks, d.err);
                 uint64_t P[2], tot1, sum2;
                 hash_loaded<U, true, kAdapt>(hl, v, b0, cnb, min(d.Kf2, cur.nblk), lane, P, tot1, sum2,
                                              kAdapt ? d.p2local + cur.bo + b0 : nullptr);
@@ -871,7 +893,8 @@ __global__ void __launch_bounds__(HP<U>::kThreads, kMinBlocks) k_hash_probe(cons
 // Launch shape of the routing kernel per device and block size: its
 // shared-memory stages are set up once, the grid fills every SM.
 template <int U, bool kAdapt>
-static cudaError_t launch_hash_probe_u(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st) {
+static cudaError_t launch_hash_probe_u(const DevState &d, const dm_batch &b, uint64_t E, uint32_t r0, uint32_t r1,
+                                       cudaStream_t st) {
     static std::atomic<int> grids[kGridDevices];
     int dev = 0;
     DM_TRY(cudaGetDevice(&dev));
@@ -887,25 +910,27 @@ static cudaError_t launch_hash_probe_u(const DevState &d, const dm_batch &b, uin
         grid = sms * (per > 0 ? per : 1);
         grids[dev].store(grid, std::memory_order_relaxed);
     }
-    DM_TRY(launch_pdl(k_hash_probe<U, kAdapt>, grid, HP<U>::kThreads, HP<U>::kSmem, st, d, b.tokens, E));
+    DM_TRY(launch_pdl(k_hash_probe<U, kAdapt>, grid, HP<U>::kThreads, HP<U>::kSmem, st, d, b.tokens, E, r0, r1));
     return cudaGetLastError();
 }
 
 template <bool kAdapt>
-static cudaError_t launch_hash_probe_t(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st) {
+static cudaError_t launch_hash_probe_t(const DevState &d, const dm_batch &b, uint64_t E, uint32_t r0, uint32_t r1,
+                                       cudaStream_t st) {
     switch (d.B) {
-        case 4: return launch_hash_probe_u<1, kAdapt>(d, b, E, st);
-        case 8: return launch_hash_probe_u<2, kAdapt>(d, b, E, st);
-        case 16: return launch_hash_probe_u<4, kAdapt>(d, b, E, st);
-        case 32: return launch_hash_probe_u<8, kAdapt>(d, b, E, st);
-        case 64: return launch_hash_probe_u<16, kAdapt>(d, b, E, st);
+        case 4: return launch_hash_probe_u<1, kAdapt>(d, b, E, r0, r1, st);
+        case 8: return launch_hash_probe_u<2, kAdapt>(d, b, E, r0, r1, st);
+        case 16: return launch_hash_probe_u<4, kAdapt>(d, b, E, r0, r1, st);
+        case 32: return launch_hash_probe_u<8, kAdapt>(d, b, E, r0, r1, st);
+        case 64: return launch_hash_probe_u<16, kAdapt>(d, b, E, r0, r1, st);
         default: return cudaErrorInvalidValue;
     }
 }
 
-cudaError_t launch_hash_probe(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st) {
-    if (b.n == 0) return cudaSuccess;
-    return d.ad_step ? launch_hash_probe_t<true>(d, b, E, st) : launch_hash_probe_t<false>(d, b, E, st);
+cudaError_t launch_hash_probe(const DevState &d, const dm_batch &b, uint64_t E, uint32_t r0, uint32_t r1,
+                              cudaStream_t st) {
+    if (b.n == 0 || r0 >= r1) return cudaSuccess;
+    return d.ad_step ? launch_hash_probe_t<true>(d, b, E, r0, r1, st) : launch_hash_probe_t<false>(d, b, E, r0, r1, st);
 }
 
 // Carries of every segment of the batch and the route outputs (the
@@ -920,6 +945,69 @@ __global__ void k_carries(DevState d, dm_route_out o, uint32_t n) {
 cudaError_t launch_carries(const DevState &d, const dm_route_out &o, uint32_t n, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
     DM_TRY(launch_pdl(k_carries, (n + 7) / 8, 256, 0, st, d, o, n));
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Sharded routing: what the routing kernel produced for requests r0 .. r1-1
+// (the local prefix values of their blocks, their segments' f1 totals and
+// owners, and per request the hash length, both candidates and both first
+// misses), packed into one buffer in that order (8-byte values first, then
+// 4-byte ones) or unpacked from it.  Every replica lays the batch out the
+// same way, so the ranges line up.
+__device__ __forceinline__ void shard_span(const DevState &d, uint32_t r0, uint32_t r1, uint64_t &b0, uint64_t &nb,
+                                           uint64_t &s0, uint64_t &ns) {
+    const uint32_t n = d.info->n;
+    b0 = d.r_blkoff[r0];
+    nb = (r1 < n ? d.r_blkoff[r1] : d.info->total_blocks) - b0;
+    s0 = d.r_segoff[r0];
+    ns = (r1 < n ? d.r_segoff[r1] : d.info->total_segs) - s0;
+}
+
+template <bool kExport>
+__global__ void k_shard_copy(DevState d, uint32_t r0, uint32_t r1, uint8_t *buf, uint64_t cap, uint64_t *bytes) {
+    pdl_enter();
+    if (has_err(d.err)) return;
+    uint64_t b0, nb, s0, ns;
+    shard_span(d, r0, r1, b0, nb, s0, ns);
+    const uint64_t nr = r1 - r0;
+    const uint64_t need = 8 * (nb + ns) + 4 * (ns + 5 * nr);
+    if (kExport && bytes && blockIdx.x == 0 && threadIdx.x == 0) *bytes = need;
+    if (need > cap) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) set_err(d.err, DM_ERR_CAPACITY);
+        return;
+    }
+    uint64_t *p64 = reinterpret_cast<uint64_t *>(buf);
+    uint32_t *p32 = reinterpret_cast<uint32_t *>(buf + 8 * (nb + ns));
+    uint32_t *const rq[5] = {d.r_K, d.r_c1, d.r_c2, d.r_m1, d.r_m2};
+    const uint64_t total = nb + ns + ns + 5 * nr;
+    for (uint64_t i = uint64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+         i += uint64_t(gridDim.x) * blockDim.x) {
+        if (i < nb) {
+            if (kExport) p64[i] = d.plocal[b0 + i];
+            else d.plocal[b0 + i] = p64[i];
+        } else if (i < nb + ns) {
+            const uint64_t k = i - nb;
+            if (kExport) p64[i] = d.seg_total[s0 + k];
+            else d.seg_total[s0 + k] = p64[i];
+        } else if (i < nb + 2 * ns) {
+            const uint64_t k = i - nb - ns;
+            if (kExport) p32[k] = d.seg_req[s0 + k];
+            else d.seg_req[s0 + k] = p32[k];
+        } else {
+            const uint64_t k = i - nb - 2 * ns, a = k / nr, r = r0 + k % nr;
+            if (kExport) p32[ns + k] = rq[a][r];
+            else rq[a][r] = p32[ns + k];
+        }
+    }
+}
+
+cudaError_t launch_shard_copy(const DevState &d, bool exp, uint32_t r0, uint32_t r1, uint8_t *buf, uint64_t cap,
+                              uint64_t *bytes, cudaStream_t st) {
+    if (r0 >= r1) return cudaSuccess;
+    const int grid = 2 * hash_grid_size();
+    if (exp) DM_TRY(launch_pdl(k_shard_copy<true>, grid, 256, 0, st, d, r0, r1, buf, cap, bytes));
+    else DM_TRY(launch_pdl(k_shard_copy<false>, grid, 256, 0, st, d, r0, r1, buf, cap, bytes));
     return cudaGetLastError();
 }
 

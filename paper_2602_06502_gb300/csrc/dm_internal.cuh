@@ -352,6 +352,29 @@ __device__ __forceinline__ bool has_err(const uint32_t *err) {
     return *(volatile const uint32_t *)err != 0u;
 }
 
+// Debug builds (-DDM_DEBUG, libdualmap_debug.so): DM_CHECK records
+// DM_ERR_BOUNDS when an index invariant that the release build relies on
+// does not hold, and DM_CLAMP also keeps the access inside its buffer.
+// Nothing traps: the call ends with the sticky status.  Release builds
+// compile both to nothing (DM_CLAMP to the index itself).
+#ifdef DM_DEBUG
+#define DM_CHECK(cond, err)                                     \
+    do {                                                        \
+        if (!(cond)) ::dm::set_err((err), DM_ERR_BOUNDS);       \
+    } while (0)
+__device__ __forceinline__ uint64_t dm_clamp(uint64_t i, uint64_t n, uint32_t *err) {
+    if (i < n) return i;
+    set_err(err, DM_ERR_BOUNDS);
+    return n ? n - 1 : 0;
+}
+#define DM_CLAMP(i, n, err) ::dm::dm_clamp((i), (n), (err))
+#else
+#define DM_CHECK(cond, err) \
+    do {                    \
+    } while (0)
+#define DM_CLAMP(i, n, err) (i)
+#endif
+
 __device__ __forceinline__ uint64_t shfl_u64(uint64_t v, int src) {
     return __shfl_sync(0xffffffffu, v, src);
 }
@@ -777,7 +800,10 @@ cudaError_t launch_setup_plain_drain(const DevState &d, const dm_batch &b, uint6
                                      cudaStream_t st);
 cudaError_t launch_route_d(const DevState &d, const dm_batch &b, const dm_route_out_d &o, uint64_t seq0,
                            cudaStream_t st);
-cudaError_t launch_hash_probe(const DevState &d, const dm_batch &b, uint64_t E, cudaStream_t st);
+cudaError_t launch_shard_copy(const DevState &d, bool exp, uint32_t r0, uint32_t r1, uint8_t *buf, uint64_t cap,
+                              uint64_t *bytes, cudaStream_t st);
+cudaError_t launch_hash_probe(const DevState &d, const dm_batch &b, uint64_t E, uint32_t r0, uint32_t r1,
+                              cudaStream_t st);
 cudaError_t launch_carries(const DevState &d, const dm_route_out &o, uint32_t n, cudaStream_t st);
 cudaError_t launch_adapt_update(const DevState &d, uint64_t *new_set, uint64_t n_live, uint64_t T, cudaStream_t st);
 cudaError_t launch_choice(const DevState &d, const dm_route_out &o, uint32_t n, uint64_t seq0,

@@ -12,11 +12,13 @@ import os
 import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(HERE, "libdualmap.so")
+# DM_LIBRARY=debug loads the debug build (bounds checks, DM_ERR_BOUNDS);
+# it is made by build.build(debug=True).  Read once, at the first lib() call.
+LIB_PATH = os.path.join(HERE, "libdualmap_debug.so" if os.environ.get("DM_LIBRARY") == "debug" else "libdualmap.so")
 
 DM_OK, DM_ERR_INVALID_ARG, DM_ERR_CAPACITY, DM_ERR_NO_INSTANCES = 0, 1, 2, 3
 DM_ERR_DUPLICATE_ID, DM_ERR_UNKNOWN_ID, DM_ERR_ORDER, DM_ERR_CUDA = 4, 5, 6, 7
-DM_ERR_TIMEOUT, DM_ERR_OOM = 8, 9
+DM_ERR_TIMEOUT, DM_ERR_OOM, DM_ERR_BOUNDS = 8, 9, 10
 STAGES = ["setup", "drain", "hash", "probe", "choice", "commit", "rebalance"]
 
 # dm_choice_rule
@@ -108,6 +110,10 @@ SIGNATURES = {
     "dm_route_batch_host": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
     "dm_route_batch_d": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out_d)]),
     "dm_route_batch_host_async": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
+    "dm_route_shard_begin": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.c_uint32, C.c_uint32]),
+    "dm_shard_export": (C.c_int, [C.c_void_p, C.c_uint32, C.c_uint32, C.c_void_p, C.c_uint64, C.c_void_p]),
+    "dm_shard_import": (C.c_int, [C.c_void_p, C.c_uint32, C.c_uint32, C.c_void_p, C.c_uint64]),
+    "dm_route_shard_finish": (C.c_int, [C.c_void_p, C.POINTER(dm_batch), C.POINTER(dm_route_out)]),
     "dm_rebalance": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.POINTER(C.c_uint32)]),
     "dm_rebalance_async": (C.c_int, [C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]),
     "dm_commit_cache": (C.c_int, [C.c_void_p]),
@@ -205,6 +211,22 @@ def dm_route_batch(h, batch, out):
 
 def dm_route_batch_d(h, batch, out):
     return lib().dm_route_batch_d(h, C.byref(batch), C.byref(out))
+
+
+def dm_route_shard_begin(h, batch, r0, r1):
+    return lib().dm_route_shard_begin(h, C.byref(batch), r0, r1)
+
+
+def dm_shard_export(h, r0, r1, buf_dev, cap, bytes_dev):
+    return lib().dm_shard_export(h, r0, r1, _ptr(buf_dev), cap, _ptr(bytes_dev))
+
+
+def dm_shard_import(h, r0, r1, buf_dev, nbytes):
+    return lib().dm_shard_import(h, r0, r1, _ptr(buf_dev), nbytes)
+
+
+def dm_route_shard_finish(h, batch, out):
+    return lib().dm_route_shard_finish(h, C.byref(batch), C.byref(out))
 
 
 def dm_route_batch_host(h, batch, out):
