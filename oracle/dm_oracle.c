@@ -203,8 +203,13 @@ typedef struct {
  *   expected to meet the TTFT SLO");
  * OR_RB_DOUBLE_OVERLOAD: a call migrates only after a routed batch in which
  *   some request's estimated TTFT exceeded the SLO on both candidates (the
- *   trigger "both candidate instances ... identified as overloaded"). */
-enum { OR_RB_SLO_TARGET = 1, OR_RB_DOUBLE_OVERLOAD = 2 };
+ *   trigger "both candidate instances ... identified as overloaded");
+ * OR_RB_FRESH_HITS: a migration candidate's TTFT on its other candidate j
+ *   uses the hit found by probing j's cache as it stands at the rebalance
+ *   call with the request's own block keys (the benefit's TTFT estimate
+ *   queries the instance's KV metadata afresh), instead of the hit stored
+ *   when the request was routed; queue entries keep their keys for this. */
+enum { OR_RB_SLO_TARGET = 1, OR_RB_DOUBLE_OVERLOAD = 2, OR_RB_FRESH_HITS = 4 };
 
 enum { OR_RULE_DUALMAP = 0, OR_RULE_CACHE_AFFINITY = 1, OR_RULE_LEAST_LOADED = 2,
        OR_RULE_MIN_TTFT = 3, OR_RULE_PREBLE = 4, OR_RULE_GLOBAL_CACHE_AFFINITY = 5,
@@ -235,6 +240,8 @@ typedef struct {
     uint64_t work, remaining;
     uint64_t moved_in_call;  /* rebalance call id that moved it here; 0 = none */
     uint64_t arrival;        /* batch time the request arrived with */
+    uint64_t *keys;          /* OR_RB_FRESH_HITS: the prompt's block keys (owned), else NULL */
+    uint32_t nblk;
 } q_entry;
 
 typedef struct {
@@ -617,6 +624,7 @@ static void q_drain(or_state *s, uint32_t id, uint64_t delta, uint64_t t0)
             run += h->remaining;
             s->W[id] -= h->remaining;
             record_ttft(s, t0 + run - h->arrival);
+            free(h->keys);
             q->head++;
             q->len--;
         } else {
@@ -651,7 +659,10 @@ void or_destroy(or_state *s)
     clear_pending(s);
     for (uint32_t i = 0; i < s->cfg.max_instances; i++) {
         if (s->cache) lru_free(&s->cache[i]);
-        if (s->q) free(s->q[i].e);
+        if (s->q) {
+            for (uint64_t k = 0; k < s->q[i].len; k++) free(s->q[i].e[s->q[i].head + k].keys);
+            free(s->q[i].e);
+        }
     }
     free(s->cache);
     free(s->q);
@@ -1084,7 +1095,14 @@ static int route_choose(or_state *s, const uint32_t *lengths, uint32_t n, uint64
         e.work = e.remaining = (uint64_t)cf->cost_us_per_token * (lengths[r] - hch);
         e.moved_in_call = 0;
         e.arrival = t_batch;
-        if (q_push(&s->q[ch], &e)) return OR_ERR_OOM;
+        e.keys = NULL;
+        e.nblk = s->pend_nblk[r];
+        if ((cf->rebalance_flags & OR_RB_FRESH_HITS) && e.nblk) {
+            e.keys = (uint64_t *)malloc((size_t)e.nblk * sizeof(uint64_t));
+            if (!e.keys) return OR_ERR_OOM;
+            memcpy(e.keys, s->pend_keys[r], (size_t)e.nblk * sizeof(uint64_t));
+        }
+        if (q_push(&s->q[ch], &e)) { free(e.keys); return OR_ERR_OOM; }
         s->W[ch] += e.work;
         s->pend_final[r] = ch;
         s->m_requests++;
@@ -1287,7 +1305,14 @@ int or_route_batch_d(or_state *s, uint32_t d, const uint32_t *tokens, const uint
         e.work = e.remaining = (uint64_t)cf->cost_us_per_token * (L - hch);
         e.moved_in_call = 0;
         e.arrival = t_batch;
-        if (q_push(&s->q[ch], &e)) return OR_ERR_OOM;
+        e.keys = NULL;
+        e.nblk = s->pend_nblk[r];
+        if ((cf->rebalance_flags & OR_RB_FRESH_HITS) && e.nblk) {
+            e.keys = (uint64_t *)malloc((size_t)e.nblk * sizeof(uint64_t));
+            if (!e.keys) return OR_ERR_OOM;
+            memcpy(e.keys, s->pend_keys[r], (size_t)e.nblk * sizeof(uint64_t));
+        }
+        if (q_push(&s->q[ch], &e)) { free(e.keys); return OR_ERR_OOM; }
         s->W[ch] += e.work;
         s->pend_final[r] = ch;
         s->m_requests++;
@@ -1346,6 +1371,16 @@ static int is_hot(const or_state *s, uint32_t i, uint64_t sumW, uint32_t N)
     return lhs > rhs;
 }
 
+/* Hit tokens of queue entry e on its candidate j: probed afresh against j's
+ * cache with OR_RB_FRESH_HITS (when the entry kept its keys), else the hit
+ * stored when it was routed. */
+static uint32_t other_hit(const or_state *s, const q_entry *e, uint32_t j)
+{
+    if ((s->cfg.rebalance_flags & OR_RB_FRESH_HITS) && e->keys)
+        return s->cfg.block_tokens * leading_hits(&s->cache[j], e->keys, e->nblk);
+    return j == e->c1 ? e->h1 : e->h2;
+}
+
 int or_rebalance(or_state *s, uint64_t *mig_seq, uint32_t *mig_from, uint32_t *mig_to,
                  uint32_t cap, uint32_t *n_out)
 {
@@ -1386,7 +1421,7 @@ int or_rebalance(or_state *s, uint64_t *mig_seq, uint32_t *mig_from, uint32_t *m
             ahead += e->remaining;
             if (e->remaining != e->work || e->moved_in_call == call) continue;
             uint32_t j = e->c1 == i ? e->c2 : e->c1;
-            uint32_t hj = j == e->c1 ? e->h1 : e->h2;
+            uint32_t hj = other_hit(s, e, j);
             uint64_t ttft_j = s->W[j] + (uint64_t)cf->cost_us_per_token * (e->L - hj);
             cand[nc].benefit = (int64_t)(ttft_i - ttft_j);
             cand[nc].seq = e->seq;
@@ -1402,7 +1437,7 @@ int or_rebalance(or_state *s, uint64_t *mig_seq, uint32_t *mig_from, uint32_t *m
             q_entry e = q->e[q->head + k];
             uint32_t j = e.c1 == i ? e.c2 : e.c1;
             if (s->state[j] != INST_LIVE) continue;
-            uint32_t hj = j == e.c1 ? e.h1 : e.h2;
+            uint32_t hj = other_hit(s, &e, j);
             uint64_t new_work = (uint64_t)cf->cost_us_per_token * (e.L - hj);
             uint64_t ttft_j = s->W[j] + new_work;
             if (!(cand[a].ttft_i > ttft_j && ttft_j < cf->slo_us)) continue;

@@ -55,7 +55,7 @@ class or_config(C.Structure):
 RULE_DUALMAP, RULE_CACHE_AFFINITY, RULE_LEAST_LOADED, RULE_MIN_TTFT, RULE_PREBLE = 0, 1, 2, 3, 4
 RULE_GLOBAL_CACHE_AFFINITY, RULE_GLOBAL_LEAST_LOADED, RULE_GLOBAL_MIN_TTFT, RULE_GLOBAL_PREBLE = 5, 6, 7, 8
 HIST_BUCKETS = 976
-RB_SLO_TARGET, RB_DOUBLE_OVERLOAD = 1, 2
+RB_SLO_TARGET, RB_DOUBLE_OVERLOAD, RB_FRESH_HITS = 1, 2, 4
 METRIC_KEYS = ["requests", "prompt_tokens", "hit_tokens", "switched", "est_slo_met", "completed",
                "ttft_sum_us", "ttft_max_us", "slo_met", "ttft_p50_us", "ttft_p90_us", "ttft_p99_us",
                "cv_samples"]

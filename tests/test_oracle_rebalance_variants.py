@@ -1,9 +1,11 @@
 """Pins of the oracle's rebalancing variants, the paper's own wording of
 hotspot-aware rebalancing (Sec. 3.3, App. A.1.2): migrate "until all
 requests in the overloaded instance's queue are expected to meet the TTFT
-SLO" (overloaded = queued work above the SLO), and start migrating "whenever
-both candidate instances of a request are identified as overloaded".
-Expected values are worked out by hand."""
+SLO" (overloaded = queued work above the SLO), start migrating "whenever
+both candidate instances of a request are identified as overloaded", and
+estimate a candidate's TTFT on the other instance from that instance's
+cache as it stands at the call (fresh hits) rather than from the hit
+stored at routing time.  Expected values are worked out by hand."""
 
 import numpy as np
 import pytest
@@ -102,8 +104,66 @@ def test_double_overload_trigger_gates_the_rule():
     assert results["loud", 0][0]
 
 
-def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
-    """Hotspot-aware rebalancing written out again in plain Python."""
+def test_fresh_hits_see_a_prefix_cached_after_routing():
+    """Request X (4 blocks, 64 tokens) is routed while nothing is cached: both
+    stored hits are 0 and it queues on i (equal hits: the less loaded, tie
+    c1).  Behind it on i an entry B of 1,000 us (alternative 2, no hits).
+    After the commit, X's four keys are also touched on its other candidate
+    j.  Stored hits: X's benefit on j is 64 - (0 + 64) = 0 and B's 1,064 -
+    1,000 = 64, so only B moves (then W_i = 64 is still hot, and X's move
+    would not lower its TTFT).  Fresh hits: X's hit on j is 64 tokens, so
+    its TTFT there is 0 and its benefit 64, tied with B's and first by
+    sequence number: X moves to j, then B moves to 2."""
+    probe = mk(0, 10 ** 9)
+    prompt = _prompt_with_candidates(probe, {0, 1})
+    keys, _ = probe.prompt_keys(prompt)
+    results = {}
+    for flags in (0, O.RB_FRESH_HITS):
+        o = mk(flags, 10 ** 9)
+        rc, out = o.route_batch(prompt, [0], [64], 0)
+        assert rc == 0 and int(out["hit1"][0]) == int(out["hit2"][0]) == 0
+        i = int(out["chosen"][0])
+        j = int(out["cand2"][0]) if i == int(out["cand1"][0]) else int(out["cand1"][0])
+        assert i == int(out["cand1"][0])
+        assert o.commit() == 0
+        for k in keys:
+            assert o.debug_touch(j, int(k)) == 0
+        o.debug_enqueue(i, 100, 1000, i, 2, 0, 0, 1000)
+        rc, n, (seq, fr, to) = o.rebalance()
+        assert rc == 0
+        results[flags] = list(zip(seq.tolist(), fr.tolist(), to.tolist())), o.loads().tolist()
+        xseq = 0
+        if flags:
+            assert results[flags][0] == [(xseq, i, j), (100, i, 2)]
+            assert results[flags][1][j] == 0 and results[flags][1][2] == 1000 and results[flags][1][i] == 0
+        else:
+            assert results[flags][0] == [(100, i, 2)]
+            assert results[flags][1][i] == 64 and results[flags][1][2] == 1000
+
+
+def test_fresh_hits_equal_stored_hits_before_any_commit():
+    """Between a batch's routing and its commit the caches do not change, so
+    the fresh and the stored hits agree and so do the migrations."""
+    from tracegen import Trace, workload
+    w = workload("tiny", n_requests=400, batch=100, capacity=2000, zipf_s=1.3, rho=1.5)
+    tr = Trace(w)
+    got = {}
+    for flags in (0, O.RB_FRESH_HITS):
+        o = O.Oracle(**O.config_from_workload(w), rebalance_flags=flags)
+        for i in range(w["n_instances"]):
+            assert o.add_instance(i) == 0
+        s, e, off, lens, nt = tr.batch_layout(0)
+        assert o.route_batch(tr.batch_tokens(0), off, lens, tr.batch_time(0))[0] == 0
+        rc, n, (seq, fr, to) = o.rebalance()
+        assert rc == 0
+        got[flags] = (seq.tolist(), to.tolist(), o.loads().tolist())
+    assert got[0] == got[O.RB_FRESH_HITS]
+
+
+def _model_rebalance(queues, live, flags, both_over, slo, cost, call, cached=None, B=16, seen=None):
+    """Hotspot-aware rebalancing written out again in plain Python.  With
+    RB_FRESH_HITS a candidate's hit on j is B x the leading run of its keys
+    in cached[j] (instance j's resident keys at the call)."""
     W = {i: sum(e["rem"] for e in q) for i, q in queues.items()}
     if flags & O.RB_DOUBLE_OVERLOAD and not both_over:
         return []
@@ -112,6 +172,17 @@ def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
 
     def over(i):
         return W[i] > slo if flags & O.RB_SLO_TARGET else 2 * N * W[i] > 3 * sumW
+
+    def hit_of(e, j):
+        stored = e["h1"] if j == e["c1"] else e["h2"]
+        if not flags & O.RB_FRESH_HITS:
+            return stored
+        run = 0
+        while run < len(e["keys"]) and int(e["keys"][run]) in cached[j]:
+            run += 1
+        if seen is not None and B * run != stored:
+            seen.append(e["seq"])
+        return B * run
 
     hot = sorted((i for i in live if over(i)), key=lambda i: (-W[i], i))
     moves = []
@@ -123,7 +194,7 @@ def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
             if e["rem"] != e["work"] or e["moved"] == call:
                 continue
             j = e["c2"] if e["c1"] == i else e["c1"]
-            hj = e["h1"] if j == e["c1"] else e["h2"]
+            hj = hit_of(e, j)
             cands.append((-(ttft_i - (W[j] + cost * (e["L"] - hj))), e["seq"], ttft_i))
         for _, seq, ttft_i in sorted(cands):
             if not over(i):
@@ -132,7 +203,7 @@ def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
             j = e["c2"] if e["c1"] == i else e["c1"]
             if j not in live:
                 continue
-            hj = e["h1"] if j == e["c1"] else e["h2"]
+            hj = hit_of(e, j)
             nw = cost * (e["L"] - hj)
             if not (ttft_i > W[j] + nw and W[j] + nw < slo):
                 continue
@@ -147,7 +218,8 @@ def _model_rebalance(queues, live, flags, both_over, slo, cost, call):
     return moves
 
 
-@pytest.mark.parametrize("flags", [0, O.RB_SLO_TARGET, O.RB_DOUBLE_OVERLOAD, 3])
+@pytest.mark.parametrize("flags", [0, O.RB_SLO_TARGET, O.RB_DOUBLE_OVERLOAD, 3, O.RB_FRESH_HITS,
+                                   O.RB_FRESH_HITS | O.RB_SLO_TARGET])
 def test_variants_match_an_independent_model_on_a_trace(flags):
     """A skewed 16-instance workload with a 5 ms SLO, rebalancing after
     every batch: the migrations of every call and the loads after it equal
@@ -164,7 +236,7 @@ def test_variants_match_an_independent_model_on_a_trace(flags):
         assert o.add_instance(i) == 0
     queues = {i: [] for i in range(n)}
     live = set(range(n))
-    t_prev, seq, total, ttfts = None, 0, 0, []
+    t_prev, seq, total, ttfts, seen = None, 0, 0, [], []
     for b in range(len(tr.batches)):
         s, e, off, lens, nt = tr.batch_layout(b)
         t = tr.batch_time(b)
@@ -185,10 +257,13 @@ def test_variants_match_an_independent_model_on_a_trace(flags):
             c1, c2, ch = int(out["cand1"][r]), int(out["cand2"][r]), int(out["chosen"][r])
             h1, h2, L = int(out["hit1"][r]), int(out["hit2"][r]), int(lens[r])
             wk = cost * (L - (h1 if ch == c1 else h2))
-            queues[ch].append(dict(seq=seq, L=L, c1=c1, c2=c2, h1=h1, h2=h2, work=wk, rem=wk, moved=0, arr=t))
+            keys = o.prompt_keys(tr.request_tokens(s + r))[0] if flags & O.RB_FRESH_HITS else []
+            queues[ch].append(dict(seq=seq, L=L, c1=c1, c2=c2, h1=h1, h2=h2, work=wk, rem=wk, moved=0, arr=t,
+                                   keys=keys))
             both |= int(out["ttft1"][r]) > slo and int(out["ttft2"][r]) > slo
             seq += 1
-        want = _model_rebalance(queues, live, flags, both, slo, cost, b + 1)
+        cached = {i: set(o.cache(i)[0].tolist()) for i in range(n)} if flags & O.RB_FRESH_HITS else None
+        want = _model_rebalance(queues, live, flags, both, slo, cost, b + 1, cached, w["block_tokens"], seen)
         rc, nm, (mseq, mfr, mto) = o.rebalance()
         assert rc == 0
         assert list(zip(mseq.tolist(), mfr.tolist(), mto.tolist())) == want, b
@@ -196,6 +271,8 @@ def test_variants_match_an_independent_model_on_a_trace(flags):
         total += len(want)
         assert o.commit() == 0
     assert total > 0
+    if flags & O.RB_FRESH_HITS:
+        assert seen          # some candidate's fresh hit differed from its stored one
     m, _ = o.metrics()
     assert (m["completed"], m["ttft_sum_us"], m["ttft_max_us"]) == (len(ttfts), sum(ttfts), max(ttfts))
     assert m["slo_met"] == sum(x <= slo for x in ttfts)
