@@ -187,6 +187,14 @@ typedef struct {
      * DM_ERR_INVALID_ARG otherwise, and dm_route_batch and dm_rebalance
      * return DM_ERR_INVALID_ARG on such a handle). */
     uint32_t candidates;
+    /* With DM_REBALANCE_FRESH_HITS: the capacity, in blocks, of each
+     * instance's ring of its queued requests' block keys (rounded up to a
+     * power of two; device memory: 8 bytes x this x max_instances).  It must
+     * hold the keys of every request queued on an instance at once: a
+     * routing or rebalance call that would outgrow it records
+     * DM_ERR_CAPACITY (sticky).  Required > 0 with that flag
+     * (DM_ERR_INVALID_ARG otherwise), ignored without it. */
+    uint64_t rebalance_key_blocks;
     /* Seed of all hash key material (SplitMix64). */
     uint64_t seed;
     /* cudaStream_t for all work of this handle; NULL = legacy default stream. */
@@ -261,9 +269,18 @@ enum {
  * DM_REBALANCE_DOUBLE_OVERLOAD: dm_rebalance migrates only if, in the last
  * routed batch, some request's estimated TTFT exceeded the SLO on both of
  * its candidates (App. A.1.2: rebalancing starts "whenever both candidate
- * instances of a request are identified as overloaded"). */
+ * instances of a request are identified as overloaded").
+ * DM_REBALANCE_FRESH_HITS: a migration candidate's TTFT on its other
+ * candidate uses the cached-prefix length found by probing that instance's
+ * index as it stands at the call, with the request's own block keys (kept
+ * for every queued request in per-instance rings, see
+ * dm_config.rebalance_key_blocks), instead of the length found when it was
+ * routed (Sec. 3.3's benefit with a fresh query of the instance's KV
+ * metadata).  With the pair rules (choice_rule < 5) and two candidates only
+ * (DM_ERR_INVALID_ARG otherwise). */
 #define DM_REBALANCE_SLO_TARGET 1u
 #define DM_REBALANCE_DOUBLE_OVERLOAD 2u
+#define DM_REBALANCE_FRESH_HITS 4u
 
 /* Create a scheduler with no instances (the global scheduler of Sec. 3.1;
  * the paper describes no construction step, so this lifecycle call and

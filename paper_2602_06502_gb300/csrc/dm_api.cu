@@ -228,7 +228,12 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     if (c.max_queue && (c.max_queue & (c.max_queue - 1))) return DM_ERR_INVALID_ARG;
     if (c.index_slots_log2 > 32) return DM_ERR_INVALID_ARG;   // index homes are logged as u32
     if (c.choice_rule > DM_RULE_PREBLE) return DM_ERR_INVALID_ARG;
-    if (c.rebalance_flags > (DM_REBALANCE_SLO_TARGET | DM_REBALANCE_DOUBLE_OVERLOAD)) return DM_ERR_INVALID_ARG;
+    if (c.rebalance_flags > (DM_REBALANCE_SLO_TARGET | DM_REBALANCE_DOUBLE_OVERLOAD | DM_REBALANCE_FRESH_HITS))
+        return DM_ERR_INVALID_ARG;
+    if ((c.rebalance_flags & DM_REBALANCE_FRESH_HITS) &&   // keys are queued by the pair-rule choice kernel
+        (!c.rebalance_key_blocks || c.rebalance_key_blocks > (1ull << 40) || c.choice_rule >= DM_RULE_LEAST_LOADED ||
+         (c.candidates && c.candidates != 2)))
+        return DM_ERR_INVALID_ARG;
     if (c.candidates > dm::kMaxD) return DM_ERR_INVALID_ARG;
     if (c.candidates && c.candidates != 2 && (c.choice_rule != DM_RULE_DUALMAP || c.adapt_step_blocks))
         return DM_ERR_INVALID_ARG;
@@ -388,6 +393,14 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.rb_seq, d.rb_cap));
     A(dalloc(h, &d.rb_ttft, d.rb_cap));
     A(dalloc(h, &d.rb_pos, d.rb_cap));
+    if (c.rebalance_flags & DM_REBALANCE_FRESH_HITS) {   // queued requests' keys, for fresh rebalancing probes
+        d.KQ = pow2_at_least(c.rebalance_key_blocks);
+        A(dalloc(h, &d.kring, M * d.KQ));
+        A(dalloc(h, &d.kr_head, M));
+        A(dalloc(h, &d.kr_tail, M));
+        A(dalloc(h, &d.r_koff, c.max_batch));
+        A(dalloc(h, &d.rb_hq, d.Q));
+    }
     A(dalloc(h, &d.r_hoff, c.max_batch));
     A(dalloc(h, &d.r_toff, c.max_batch));
     A(dalloc(h, &d.seg_pub, d.max_segs));
@@ -439,6 +452,11 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(cudaMemsetAsync(d.seg_pub, 0, d.max_segs * sizeof(dm::SegPub), h->st));
     A(cudaMemsetAsync(d.inst_state, 0, M, h->st));
     A(cudaMemsetAsync(d.W, 0, M * 8, h->st));
+    if (d.KQ) {
+        A(cudaMemsetAsync(d.kr_head, 0, M * 8, h->st));
+        A(cudaMemsetAsync(d.kr_tail, 0, M * 8, h->st));
+        A(cudaMemsetAsync(d.kring, 0, M * d.KQ * 8, h->st));
+    }
     A(cudaMemsetAsync(d.metrics, 0, sizeof(dm::DevMetrics), h->st));
     if (c.adapt_step_blocks) {
         A(cudaMemsetAsync(d.ad_set, 0, (d.ad_set_mask + 1) * 8, h->st));

@@ -265,6 +265,11 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
             e.h2 = h2;
             e.moved = 0;
             e.arrival = t_batch;
+            // its keys' ring position: the instance's ring tail at the batch's
+            // start plus this batch's earlier blocks queued there (the same
+            // order as its touch records)
+            e.koff = d.KQ ? d.kr_tail[ch] + (S.pt[k] >> 32) : 0;
+            if (d.KQ) d.r_koff[r] = e.koff;
             DM_CHECK(ch < d.M, d.err);
             d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
         }
@@ -276,6 +281,11 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
         d.W[i] = W[i];
         d.q_tail[i] = (uint32_t)PT[i];
         d.log_adv[i] = PT[i] >> 32;
+        if (d.KQ) {   // the batch's keys on instance i take its ring's next positions
+            const uint64_t nt = d.kr_tail[i] + (PT[i] >> 32);
+            if (nt - d.kr_head[i] > d.KQ) set_err(d.err, DM_ERR_CAPACITY);
+            d.kr_tail[i] = nt;
+        }
         if ((live_bits >> k) & 1u) {
             S1 += W[i];
             S2 += (unsigned __int128)W[i] * W[i];
@@ -486,6 +496,7 @@ __global__ void __launch_bounds__(1024) k_choice_global(DevState d, dm_route_out
             e.h2 = s_h2[rr];
             e.moved = 0;
             e.arrival = t_batch;
+            e.koff = 0;
             DM_CHECK(ch < d.M, d.err);
             d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
         }
@@ -729,6 +740,7 @@ __global__ void __launch_bounds__(1024) k_choice_d(DevState d, dm_route_out_d o,
             e.h2 = nd > 1 ? h[1] : h[0];
             e.moved = 0;
             e.arrival = t_batch;
+            e.koff = 0;
             DM_CHECK(ch < d.M, d.err);
             d.q[uint64_t(ch) * d.Q + (slot & (d.Q - 1))] = e;
         }

@@ -482,6 +482,7 @@ struct TouchSeg {
     uint8_t *st;
     uint32_t *lh;           // index home of each record
     uint32_t cnt, f;        // blocks in the segment, final instance
+    uint64_t kpos;          // DM_REBALANCE_FRESH_HITS: ring position of its first block's key on f
 };
 
 __device__ __forceinline__ TouchSeg touch_seg_load(const DevState &d, uint32_t seg, uint64_t clock_base) {
@@ -501,6 +502,7 @@ __device__ __forceinline__ TouchSeg touch_seg_load(const DevState &d, uint32_t s
     g.lh = d.loghome[f];
     g.cnt = min(nblk - first, kSegBlocks);
     g.f = f;
+    g.kpos = d.KQ ? d.r_koff[r] + first : 0;
     // the segment's records lie inside the instance's log window
     DM_CHECK(f < d.M && g.p_first + 1 - g.front <= d.logcap && g.pidx + g.cnt <= d.max_blocks, d.err);
     return g;
@@ -547,6 +549,11 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             if (v1) {
                 g.lg[p1 & lmask] = Rec{k1, g.stamp_first - lane - 32};
                 g.lh[p1 & lmask] = (uint32_t)h1;
+            }
+            if (d.KQ) {   // the queued request's keys, for fresh rebalancing probes
+                uint64_t *kr = d.kring + uint64_t(g.f) * d.KQ;
+                if (v0) kr[(g.kpos + lane) & (d.KQ - 1)] = k0;
+                if (v1) kr[(g.kpos + lane + 32) & (d.KQ - 1)] = k1;
             }
             const Slot c0s = v0 ? slot_cas(&g.t[h0], Slot{0, 0}, Slot{k0, p0 + 1}) : Slot{0, 0};
             const Slot c1s = v1 ? slot_cas(&g.t[h1], Slot{0, 0}, Slot{k1, p1 + 1}) : Slot{0, 0};

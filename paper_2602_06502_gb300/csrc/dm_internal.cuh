@@ -31,6 +31,7 @@ struct QEntry {
     uint32_t L, c1, c2, h1, h2;
     uint32_t moved;   // 0, or the rebalance call that moved it here, or kTomb
     uint64_t arrival; // batch time the request arrived with
+    uint64_t koff;    // DM_REBALANCE_FRESH_HITS: ring position of its first block key on this instance
 };
 
 // Serving metrics (dm_metrics before the percentiles), updated by the
@@ -248,6 +249,13 @@ struct DevState {
     // to the kernel's last CTA
     SegPub *seg_pub;
     uint32_t *r_m1, *r_m2;
+    // DM_REBALANCE_FRESH_HITS (KQ = 0 otherwise): per instance a ring of KQ
+    // block keys of its queued requests (instance i's at kring + i KQ), with
+    // monotonic head and tail positions; per request of the pending batch
+    // the ring position of its keys on its final instance
+    uint64_t KQ;
+    uint64_t *kring, *kr_head, *kr_tail, *r_koff;
+    uint32_t *rb_hq;                // rebalance scratch: a candidate's hit on its other candidate, per queue slot
     uint64_t *fix_list;             // queue entries of route tasks (request, tries)
     uint64_t *seg_total, *seg_carry, *plocal;
     uint64_t *p2local;              // adaptive only: per block < Kf2, in-segment prefix of its f2 digests
@@ -667,6 +675,7 @@ __device__ __forceinline__ void drain_queue(const DevState &d, uint32_t i, uint6
     if (lane == 0) {
         d.q_head[i] = head;
         d.W[i] -= used;
+        if (d.KQ) d.kr_head[i] = head != tail ? qb[head & (d.Q - 1)].koff : d.kr_tail[i];
     }
 }
 

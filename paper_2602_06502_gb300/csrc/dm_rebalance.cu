@@ -6,8 +6,10 @@
 // queued request that has not started, was not moved in this call and could
 // still pass the move test, with
 // TTFT_{r,i} = work queued up to and including r and TTFT_{r,j} = W_j +
-// cost * (L - h_{r,j}) for its other candidate j; sorts them by (benefit
-// desc, sequence asc); then one thread walks the list, moving r to j while i
+// cost * (L - h_{r,j}) for its other candidate j (h_{r,j} stored at routing,
+// or with DM_REBALANCE_FRESH_HITS probed now from the request's keys); sorts
+// them by (benefit desc, sequence asc); then one thread walks the list,
+// moving r to j while i
 // is still hot, the benefit (re-evaluated with the current W_j) is positive
 // and TTFT_{r,j} < SLO.  Moved requests leave a tombstone (zero work) in the
 // source queue and are appended to the target queue.
@@ -76,6 +78,50 @@ __device__ __forceinline__ uint64_t block_excl_u64(uint64_t v, uint64_t *s, uint
     return r;
 }
 
+// DM_REBALANCE_FRESH_HITS: the leading run (blocks) of a queued request's
+// keys, held at ring positions koff .. koff+nblk-1 of `ring` (KQ entries),
+// that is resident on instance j now (its index and log front at the call;
+// App. A.3.2's metadata query).  The resident keys are closed under prefixes
+// (touches run from a prompt's last block down into an exact LRU), so the
+// first block of every 64-block segment is tested, 32 segments per round,
+// and then the one segment that holds the run's end.  Whole warp.
+static __device__ __noinline__ uint32_t ring_leading_run(const DevState &d, const uint64_t *ring, uint64_t koff,
+                                                  uint32_t nblk, uint32_t j, int lane) {
+    const Slot *t = d.table[j];
+    const uint64_t front = d.log_front[j], mask = d.S - 1, km = d.KQ - 1;
+    const uint32_t nseg = (nblk + kSegBlocks - 1) / kSegBlocks;
+    uint32_t js = nseg;   // first segment whose first block is missing (nseg: none)
+    for (uint32_t s0 = 0; s0 < nseg; s0 += 32) {
+        const uint32_t sg = s0 + lane;
+        bool miss = false;
+        if (sg < nseg) {
+            const uint64_t key = ring[(koff + uint64_t(sg) * kSegBlocks) & km];
+            const uint64_t home = group_home(key, 0, mask);   // a segment's first block anchors its own group
+            miss = !resident_at(t, mask, key, home, front, load_slot(t + home), d.err, d.loop_limit);
+        }
+        const uint32_t bal = __ballot_sync(0xffffffffu, miss);
+        if (bal) {
+            js = s0 + __ffs(bal) - 1;
+            break;
+        }
+    }
+    if (js == 0) return 0;
+    // the run ends in segment js - 1, or at block 64 js
+    const uint32_t c0 = (js - 1) * kSegBlocks, cn = min(kSegBlocks, nblk - c0);
+    uint32_t first = 0xFFFFFFFFu;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const uint32_t b = 32 * k + lane;
+        const uint64_t key = b < cn ? ring[(koff + c0 + b) & km] : 0;
+        const uint64_t home = group_home(group_anchor(key, lane), c0 + b, mask);
+        const bool miss = b < cn && !resident_at(t, mask, key, home, front, load_slot(t + home), d.err, d.loop_limit);
+        const uint32_t bal = __ballot_sync(0xffffffffu, miss);
+        if (bal && first == 0xFFFFFFFFu) first = c0 + 32 * k + __ffs(bal) - 1;
+    }
+    if (first != 0xFFFFFFFFu) return first;
+    return js < nseg ? js * kSegBlocks : nblk;
+}
+
 constexpr uint32_t kRbStage = 1024;   // candidates staged per sequential pass
 
 // Sequential-pass staging of one chunk of sorted candidates.
@@ -83,8 +129,10 @@ struct RbChunk {
     uint64_t seq[kRbStage], work[kRbStage], ttft_i[kRbStage], new_work[kRbStage];
     uint32_t pos[kRbStage], L[kRbStage], c1[kRbStage], c2[kRbStage], h1[kRbStage], h2[kRbStage];
     uint32_t j[kRbStage];
-    // moves decided in this chunk: candidate index and target slot
+    // moves decided in this chunk: candidate index and target slot, and
+    // (DM_REBALANCE_FRESH_HITS) the ring position of its keys on the target
     uint32_t mv_k[kRbStage], mv_slot[kRbStage];
+    uint64_t mv_koff[kRbStage];
 };
 
 // Dynamic shared memory layout: per instance W (u64), queue tails (u32),
@@ -154,6 +202,7 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
     // hot list (ids in ascending order), then ranks by (W desc, id asc);
     // none when the double-overload trigger did not fire
     const bool slo_target = (d.rb_flags & DM_REBALANCE_SLO_TARGET) != 0;
+    const bool fresh = (d.rb_flags & DM_REBALANCE_FRESH_HITS) != 0 && d.KQ != 0;
     const bool armed = !(d.rb_flags & DM_REBALANCE_DOUBLE_OVERLOAD) || d.info->both_over;
     uint32_t nhot = 0;
     for (uint32_t base = 0; base < M; base += blockDim.x) {
@@ -194,10 +243,29 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
             const uint64_t ex = block_excl_u64(valid ? e.remaining : 0, s_u, &tot_rem);
             const uint64_t ttft_i = ahead + ex + (valid ? e.remaining : 0);
             bool elig = valid && e.moved != kTomb && e.moved != call && e.remaining == e.work;
+            const uint32_t jj = e.c1 == i ? e.c2 : e.c1;
+            uint32_t hj = jj == e.c1 ? e.h1 : e.h2;   // the hit stored at routing
+            if (fresh) {
+                // probe the other candidate's index now, a warp per entry in
+                // turn; the pending batch's own entries keep their stored
+                // hit (no commit since their routing: the same probe)
+                const bool need = elig && st[jj] == 1 && !(e.seq >= seq0 && e.seq < seq0 + n);
+                const int lane = threadIdx.x & 31;
+                for (uint32_t m = __ballot_sync(0xffffffffu, need); m; m &= m - 1) {
+                    const int src = __ffs(m) - 1;
+                    const uint64_t ko = __shfl_sync(0xffffffffu, e.koff, src);
+                    const uint32_t nb = __shfl_sync(0xffffffffu, e.L, src) / d.B;
+                    const uint32_t tj = __shfl_sync(0xffffffffu, jj, src);
+                    // its keys lie in the live part of the ring (written by an earlier commit)
+                    DM_CHECK(ko >= d.kr_head[i] && ko + nb <= d.kr_tail[i], d.err);
+                    const uint32_t run = ring_leading_run(d, d.kring + uint64_t(i) * d.KQ, ko, nb, tj, lane);
+                    if (lane == src) hj = run * d.B;
+                }
+                if (elig) d.rb_hq[p & (d.Q - 1)] = hj;
+            }
             uint64_t key = 0;
             if (elig) {
-                const uint32_t j = e.c1 == i ? e.c2 : e.c1;
-                const uint32_t hj = j == e.c1 ? e.h1 : e.h2;
+                const uint32_t j = jj;
                 const uint64_t ttft_j = W[j] + cost * (e.L - hj);
                 const int64_t B = (int64_t)(ttft_i - ttft_j);
                 key = ~(uint64_t(B) ^ 0x8000000000000000ull);   // ascending = benefit descending
@@ -222,6 +290,7 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
             ahead += tot_rem;
             p0 += min((uint32_t)blockDim.x, (uint32_t)(tail - p0));
         }
+        __syncthreads();   // the candidates written in the last pass, before any thread reads them
         if (ncand > d.rb_cap) {
             if (threadIdx.x == 0) set_err(d.err, DM_ERR_CAPACITY);
             return;
@@ -263,7 +332,7 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
                 const uint32_t p = d.rb_pos[c0 + k];
                 const QEntry e = qi[p & (d.Q - 1)];
                 const uint32_t j = e.c1 == i ? e.c2 : e.c1;
-                const uint32_t hj = j == e.c1 ? e.h1 : e.h2;
+                const uint32_t hj = fresh ? d.rb_hq[p & (d.Q - 1)] : (j == e.c1 ? e.h1 : e.h2);
                 Ch.seq[k] = e.seq;
                 Ch.work[k] = e.work;
                 Ch.ttft_i[k] = d.rb_ttft[c0 + k];
@@ -292,6 +361,12 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
                     if (!(Ch.ttft_i[k] > ttft_j && ttft_j < d.slo)) continue;
                     const uint32_t slot = tails[j];
                     if (slot - d.q_head[j] >= d.Q) { set_err(d.err, DM_ERR_CAPACITY); stop = 1; break; }
+                    if (fresh) {   // its keys move to the target's ring
+                        const uint64_t kt = d.kr_tail[j], nb = Ch.L[k] / d.B;
+                        if (kt + nb - d.kr_head[j] > d.KQ) { set_err(d.err, DM_ERR_CAPACITY); stop = 1; break; }
+                        d.kr_tail[j] = kt + nb;
+                        Ch.mv_koff[nmv] = kt;
+                    }
                     tails[j] = slot + 1;
                     W[i] -= Ch.work[k];
                     sumW -= Ch.work[k];
@@ -324,14 +399,29 @@ __global__ void __launch_bounds__(1024) k_rebalance(DevState d, uint32_t n, uint
                 e.h2 = Ch.h2[k];
                 e.moved = call;
                 e.arrival = src->arrival;   // TTFT still counts from the original arrival
+                e.koff = fresh ? Ch.mv_koff[t] : 0;
                 d.q[uint64_t(j) * d.Q + (Ch.mv_slot[t] & (d.Q - 1))] = e;
                 if (e.seq >= seq0 && e.seq < seq0 + n) {
                     d.r_final[e.seq - seq0] = j;
                     d.info->final_dirty = 1;
+                    if (fresh) d.r_koff[e.seq - seq0] = e.koff;   // the commit writes its keys there
                 }
                 if (cnt0 + t < cap) out[cnt0 + t] = dm_migration{e.seq, i, j};
             }
             __syncthreads();
+            if (fresh) {   // an earlier batch's moved request: its keys follow it
+                for (uint32_t t = 0; t < s_nmv; ++t) {
+                    const uint32_t k = Ch.mv_k[t];
+                    if (Ch.seq[k] >= seq0 && Ch.seq[k] < seq0 + n) continue;
+                    const uint64_t from = qi[Ch.pos[k] & (d.Q - 1)].koff, to = Ch.mv_koff[t];
+                    const uint64_t *sr = d.kring + uint64_t(i) * d.KQ;
+                    uint64_t *dr = d.kring + uint64_t(Ch.j[k]) * d.KQ;
+                    const uint32_t nb = Ch.L[k] / d.B;
+                    for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x)
+                        dr[(to + b) & (d.KQ - 1)] = sr[(from + b) & (d.KQ - 1)];
+                }
+                __syncthreads();
+            }
             if (threadIdx.x == 0) s_cnt = cnt0 + s_nmv;
             __syncthreads();
         }

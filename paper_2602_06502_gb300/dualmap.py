@@ -28,7 +28,7 @@ DM_RULE_CACHE_AFFINITY, DM_RULE_LEAST_LOADED, DM_RULE_MIN_TTFT, DM_RULE_PREBLE =
 RULE_NAMES = ["dualmap", "pair_cache_affinity", "pair_least_loaded", "pair_min_ttft", "pair_preble",
               "cache_affinity", "least_loaded", "min_ttft", "preble"]
 DM_HIST_BUCKETS = 976
-DM_REBALANCE_SLO_TARGET, DM_REBALANCE_DOUBLE_OVERLOAD = 1, 2
+DM_REBALANCE_SLO_TARGET, DM_REBALANCE_DOUBLE_OVERLOAD, DM_REBALANCE_FRESH_HITS = 1, 2, 4
 
 
 class dm_config(C.Structure):
@@ -55,6 +55,7 @@ class dm_config(C.Structure):
         ("rebuild_pool", C.c_uint32),
         ("test_loop_limit", C.c_uint32),
         ("candidates", C.c_uint32),
+        ("rebalance_key_blocks", C.c_uint64),
         ("seed", C.c_uint64),
         ("stream", C.c_void_p),
     ]

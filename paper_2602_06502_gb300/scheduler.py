@@ -19,7 +19,8 @@ class Scheduler:
                  capacity=65536, slo_us=2_000_000, cost_us=1, hot_num=3, hot_den=2, max_batch=4096,
                  max_batch_tokens=1 << 24, max_touch_per_instance=0, max_queue=0, index_slots_log2=0, seed=0,
                  choice_rule=0, adapt_step_blocks=0, adapt_max_blocks=0, adapt_window=1, rebalance_flags=0,
-                 rebuild_pool=0, test_loop_limit=0, candidates=0, stream=None, device="cuda"):
+                 rebuild_pool=0, test_loop_limit=0, candidates=0, rebalance_key_blocks=0, stream=None,
+                 device="cuda"):
         self.device = torch.device(device)
         self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
         self.cfg = D.dm_config(block_tokens=block_tokens, route_prefix_blocks=route_prefix_blocks,
@@ -30,7 +31,8 @@ class Scheduler:
                                max_queue=max_queue, index_slots_log2=index_slots_log2, choice_rule=choice_rule,
                                adapt_step_blocks=adapt_step_blocks, adapt_max_blocks=adapt_max_blocks,
                                adapt_window=adapt_window, rebalance_flags=rebalance_flags, rebuild_pool=rebuild_pool,
-                               test_loop_limit=test_loop_limit, candidates=candidates, seed=seed,
+                               test_loop_limit=test_loop_limit, candidates=candidates,
+                               rebalance_key_blocks=rebalance_key_blocks, seed=seed,
                                stream=C.c_void_p(self.stream.cuda_stream))
         self.h = D.dm_create(self.cfg)
         self.M = max_instances

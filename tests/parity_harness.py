@@ -17,7 +17,8 @@ class Pair:
     """An oracle and a GPU scheduler built from the same workload dict."""
 
     def __init__(self, w, max_instances=None, max_batch_tokens=None, max_touch=0, max_queue=0, capacity=None,
-                 index_slots_log2=0, choice_rule=0, adapt=None, rebalance_flags=0, rebuild_pool=0):
+                 index_slots_log2=0, choice_rule=0, adapt=None, rebalance_flags=0, rebuild_pool=0,
+                 rebalance_key_blocks=0):
         import torch
         from paper_2602_06502_gb300.scheduler import Scheduler
         self.torch = torch
@@ -36,7 +37,8 @@ class Pair:
                              cost_us=w["cost_us"], max_batch=w["batch"], max_batch_tokens=mbt,
                              max_touch_per_instance=max_touch, max_queue=max_queue,
                              index_slots_log2=index_slots_log2, seed=w["seed"], choice_rule=choice_rule,
-                             rebalance_flags=rebalance_flags, rebuild_pool=rebuild_pool, **ad)
+                             rebalance_flags=rebalance_flags, rebuild_pool=rebuild_pool,
+                             rebalance_key_blocks=rebalance_key_blocks, **ad)
         self.dev = torch.device("cuda:0")
         self.n_migrations = 0
         self.n_switched = 0
@@ -90,7 +92,7 @@ class Pair:
         assert rc == 0
         self.gpu.rebalance()
         gn, (gseq, gfr, gto) = self.gpu.migrations()
-        assert gn == n, f"{tag}: {gn} vs {n} migrations"
+        assert gn == n, f"{tag}: {gn} vs {n} migrations (GPU status {self.gpu.last_error()}; oracle {seq.tolist()})"
         assert np.array_equal(gseq, seq) and np.array_equal(gfr, fr) and np.array_equal(gto, to), tag
         self.n_migrations += n
         return n

@@ -289,6 +289,78 @@ def test_rebalance_variants_tiny(flags):
     assert p.n_migrations > 0
 
 
+@pytest.mark.parametrize("flags", [4, 5, 7])
+def test_rebalance_fresh_hits(flags):
+    """DM_REBALANCE_FRESH_HITS (with the SLO target, and with both other
+    variants): every migration candidate's hit on its other candidate is
+    probed afresh from its keys in the per-instance key rings; migrations,
+    loads, queues and resident keys bit for bit with the oracle, on the
+    skewed workload (where fresh and stored hits differ) and on a small-cache
+    tiny trace with evictions between the routing and the rebalance of
+    requests queued earlier."""
+    w = workload("scaling", n_requests=3000, batch=50, n_instances=16, vnodes=32, n_prefix=100, zipf_s=1.2,
+                 len_lo=400, len_hi=512, prefix_lo=384, prefix_hi=384, scale_every=0, rho=1.0, slo_us=5000)
+    p = Pair(w, max_instances=16, rebalance_flags=flags, rebalance_key_blocks=1 << 16)
+    run_trace(p, Trace(w), rebalance=True, state_every=10)
+    assert p.n_migrations > 0
+    w = workload("tiny", n_requests=2000, batch=100, capacity=700, zipf_s=1.3, rho=1.2, slo_us=20_000)
+    p = Pair(w, max_touch=2600, rebalance_flags=flags, rebalance_key_blocks=1 << 16)
+    run_trace(p, Trace(w), rebalance=True, state_every=5)
+
+
+def test_rebalance_fresh_hits_change_migrations():
+    """On a skewed workload at rho 1.2 with a 20 ms SLO the fresh hits change
+    which requests move (the oracle shows it); the GPU's fresh-hit run is in
+    parity with the oracle call by call.  A key ring too small for the
+    queued requests' keys is a sticky DM_ERR_CAPACITY, not a silent
+    overwrite."""
+    from oracle import oracle as O
+    from paper_2602_06502_gb300 import dualmap as D
+    w = workload("scaling", n_requests=3000, batch=50, n_instances=16, vnodes=32, n_prefix=100, zipf_s=1.2,
+                 len_lo=400, len_hi=512, prefix_lo=384, prefix_hi=384, scale_every=0, rho=1.2, slo_us=20000)
+    tr = Trace(w)
+    lists = {}
+    for flags in (0, O.RB_FRESH_HITS):
+        o = O.Oracle(**O.config_from_workload(w, max_instances=16), rebalance_flags=flags)
+        for i in range(16):
+            assert o.add_instance(i) == 0
+        got = []
+        for b in range(len(tr.batches)):
+            s, e, off, lens, nt = tr.batch_layout(b)
+            assert o.route_batch(tr.batch_tokens(b), off, lens, tr.batch_time(b))[0] == 0
+            rc, n, (seq, fr, to) = o.rebalance()
+            got += list(zip(seq.tolist(), fr.tolist(), to.tolist()))
+            assert o.commit() == 0
+        lists[flags] = got
+    assert lists[0] != lists[O.RB_FRESH_HITS]
+    p = Pair(w, max_instances=16, rebalance_flags=D.DM_REBALANCE_FRESH_HITS, rebalance_key_blocks=1 << 16)
+    run_trace(p, tr, rebalance=True, state_every=10)
+    assert p.n_migrations == len(lists[O.RB_FRESH_HITS])
+    from paper_2602_06502_gb300.scheduler import Scheduler
+    g = Scheduler(block_tokens=16, route_prefix_blocks=16, vnodes=32, max_instances=16, capacity=4096, slo_us=5000,
+                  max_batch=64, max_batch_tokens=1 << 16, rebalance_flags=D.DM_REBALANCE_FRESH_HITS,
+                  rebalance_key_blocks=64)
+    for i in range(4):
+        assert g.add_instance(i) == 0
+    import torch
+    tr = Trace(w)
+    s, e, off, lens, nt = tr.batch_layout(0)
+    dev = torch.device("cuda:0")
+    tok = torch.from_numpy(tr.batch_tokens(0).view(np.int32)).to(dev)
+    g.route(tok, torch.from_numpy(off.view(np.int64)).to(dev), torch.from_numpy(lens.view(np.int32)).to(dev),
+            e - s, nt, tr.batch_time(0), check=False)
+    assert g.last_error() == D.DM_ERR_CAPACITY      # 50 prompts of ~28 blocks on 4 instances: over 64 per ring
+
+
+def test_rebalance_fresh_hits_arguments():
+    from paper_2602_06502_gb300 import dualmap as D
+    from paper_2602_06502_gb300.scheduler import Scheduler
+    for kw in (dict(rebalance_key_blocks=0), dict(rebalance_key_blocks=1024, choice_rule=D.DM_RULE_MIN_TTFT),
+               dict(rebalance_key_blocks=1024, candidates=3)):
+        with pytest.raises(D.DualMapError):
+            Scheduler(max_instances=8, rebalance_flags=D.DM_REBALANCE_FRESH_HITS, **kw)
+
+
 # -- features combined ------------------------------------------------------------------
 
 @pytest.mark.parametrize("rule,flags", [(7, 3), (3, 1)])
