@@ -562,7 +562,7 @@ struct CtaQueue {
     uint32_t seq[kQCap];
     uint32_t head, tail;
     uint32_t hash_done;   // hashing warps out of tasks
-    uint32_t busy;        // probing warps inside a task
+    uint32_t busy;        // warps inside a route task
 };
 
 __device__ __forceinline__ uint64_t qentry(uint32_t r, uint32_t tries) {
@@ -836,17 +836,20 @@ __global__ void __launch_bounds__(HP<U>::kThreads, kMinBlocks) k_hash_probe(cons
         for (uint32_t s = 0; s < (uint32_t)S; ++s)
             if ((pend >> s) & 1) mbar_wait(bar + s, (par >> s) & 1, kWaitLimit);
         if (lane == 0) atomicAdd(&q.hash_done, 1u);
-    } else {
-        // ---- probing warp: work off the CTA's queue ----
-        // (bounded: kIdleLimit idle polls in a row, a few seconds at most,
-        // then the call ends with DM_ERR_TIMEOUT)
+    }
+    {
+        // ---- route tasks: the CTA's queue, worked off by its route warp
+        // from the start and by its hashing warps once their segments are
+        // done, which matters when a batch has many short prompts (bounded:
+        // kIdleLimit idle polls in a row, a few seconds at most, then the
+        // call ends with DM_ERR_TIMEOUT) ----
         constexpr uint32_t kIdleLimit = 1u << 22;
         for (uint32_t idle = 0;;) {
             uint64_t e = lane == 0 ? q_pop(q) : 0;
             e = shfl_u64(e, 0);
             if (e == 0) {
-                // done once the hashing warps are done, no probing warp holds
-                // a task (it might queue it again) and the queue is empty
+                // done once the hashing warps are done, no warp holds a task
+                // (it might queue it again) and the queue is empty
                 const bool fin = *(volatile uint32_t *)&q.hash_done == kHashWarps &&
                                  *(volatile uint32_t *)&q.busy == 0 &&
                                  *(volatile uint32_t *)&q.head == *(volatile uint32_t *)&q.tail;
