@@ -408,7 +408,6 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.r_m2, c.max_batch));
     A(dalloc(h, &d.fix_list, c.max_batch));   // every route task at most once
     A(dalloc(h, &d.defer, d.max_segs * dm::kSegBlocks));
-    A(dalloc(h, &d.defer_n, d.max_segs));
     // two sets of batch scratch: routing and dm_hash_prompts
     for (DevState *x : {&h->d, &h->dh}) {
         if (x == &h->dh) {
@@ -424,8 +423,6 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
         A(dalloc(h, &x->seg_total, d.max_segs));
         A(dalloc(h, &x->seg_carry, d.max_segs));
         A(dalloc(h, &x->seg_total2, d.max_segs));
-        A(dalloc(h, &x->seg_newly, d.max_segs));
-        A(dalloc(h, &x->seg_claims, d.max_segs));
         A(dalloc(h, &x->plocal, d.max_blocks));
         if (x == &h->d && c.adapt_step_blocks) A(dalloc(h, &x->p2local, d.max_blocks));
         A(dalloc(h, &x->r_K, c.max_batch));
@@ -512,8 +509,6 @@ static void sync_copy(dm_handle *h) {
     h->dh.r_tokoff = keep.r_tokoff; h->dh.r_blkoff = keep.r_blkoff; h->dh.seg_req = keep.seg_req;
     h->dh.seg_total = keep.seg_total; h->dh.seg_carry = keep.seg_carry; h->dh.plocal = keep.plocal;
     h->dh.seg_total2 = keep.seg_total2;
-    h->dh.seg_newly = keep.seg_newly;
-    h->dh.seg_claims = keep.seg_claims;
     h->dh.r_c1 = keep.r_c1; h->dh.r_c2 = keep.r_c2;
     h->dh.r_final = keep.r_final; h->dh.r_touchoff = keep.r_touchoff;
     h->dh.info = keep.info;

@@ -513,12 +513,18 @@ __device__ __forceinline__ TouchSeg touch_seg_load(const DevState &d, uint32_t s
 // (request, final instance, offsets: one dependent chain per 32 segments
 // instead of per segment); then, segment by segment, lane l touches blocks l
 // and l+32: both home-slot CAS are issued before either result is used, and
-// the next segment's plocal values are loaded while they are in flight.  No
-// CTA barriers: a warp never waits for another.
+// the next segment's plocal values are loaded while they are in flight.
+// Touches that one or two atomics did not settle are deferred to the end of
+// the 32 segments, where the warp's lanes take them one each, whatever their
+// segment, and walk the key's probe order (touch_resolve: a CAS claim or a
+// position max, concurrent with every other touch of the key, so the order
+// in which warps get there does not matter).  No CTA barriers: a warp never
+// waits for another.
 constexpr int kTouchThreads = 256;
 __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
     pdl_enter();
     __shared__ TouchSeg s_seg[kTouchThreads / 32][32];
+    __shared__ uint32_t s_add[kTouchThreads / 32][2][32];   // deferred outcomes per segment: newly, claims
     if (has_err(d.err)) return;
     const int lane = threadIdx.x & 31;
     const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
@@ -533,6 +539,7 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
         TouchSeg *sg = s_seg[threadIdx.x >> 5];
         if ((uint32_t)lane < nc) sg[lane] = touch_seg_load(d, c0 + lane, clock_base);
         __syncwarp();
+        uint32_t my_newly = 0, my_claims = 0, my_nd = 0;   // lane l: segment c0 + l
         uint64_t x0 = lane < (int)sg[0].cnt ? d.plocal[sg[0].pidx + lane] : 0;
         uint64_t x1 = lane + 32 < (int)sg[0].cnt ? d.plocal[sg[0].pidx + lane + 32] : 0;
         for (uint32_t i = 0; i < nc; ++i) {
@@ -626,58 +633,71 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
             // found: the key sits at the preferred slot of the recorded bucket
             // (its home, or the next bucket after a move) with position x
             if (need0)
-                dq[__popc(m0 & below)] = Deferred{k0, p0, x0, (uint32_t)h0, g.f,
-                                                  (mv0 ? r0.key : c0s.key) == k0 ? 1u : 0u, mv0 ? 1u : 0u};
+                dq[__popc(m0 & below)] = Deferred{k0, p0, x0, (uint32_t)h0,
+                                                  (uint16_t)((mv0 ? r0.key : c0s.key) == k0), (uint16_t)mv0};
             if (need1)
-                dq[__popc(m0) + __popc(m1 & below)] = Deferred{k1, p1, x1, (uint32_t)h1, g.f,
-                                                               (mv1 ? r1.key : c1s.key) == k1 ? 1u : 0u, mv1 ? 1u : 0u};
+                dq[__popc(m0) + __popc(m1 & below)] = Deferred{k1, p1, x1, (uint32_t)h1,
+                                                               (uint16_t)((mv1 ? r1.key : c1s.key) == k1),
+                                                               (uint16_t)mv1};
             newly = __reduce_add_sync(0xffffffffu, newly);
             claims = __reduce_add_sync(0xffffffffu, claims);
-            if (lane == 0) {   // summed per request by k_req_counts (no hot-counter atomics)
-                d.seg_newly[c0 + i] = newly;
-                d.seg_claims[c0 + i] = claims;
-                d.defer_n[c0 + i] = __popc(m0) + __popc(m1);
+            if (lane == (int)i) {
+                my_newly = newly;
+                my_claims = claims;
+                my_nd = __popc(m0) + __popc(m1);
+            }
+        }
+        if (__ballot_sync(0xffffffffu, my_nd != 0)) {
+            // the deferred touches of these segments, numbered segment by
+            // segment: lane l takes touch e0 + l
+            uint32_t *add_n = s_add[threadIdx.x >> 5][0], *add_c = s_add[threadIdx.x >> 5][1];
+            add_n[lane] = 0;
+            add_c[lane] = 0;
+            uint32_t incl = my_nd;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t u = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += u;
+            }
+            const uint32_t excl = incl - my_nd, E = __shfl_sync(0xffffffffu, incl, 31);
+            __syncwarp();
+            for (uint32_t e0 = 0; e0 < E; e0 += 32) {
+                const uint32_t e = e0 + lane;
+                uint32_t sj = 0;   // its segment: the number of segments whose touches end at or before e
+#pragma unroll
+                for (uint32_t step = 16; step; step >>= 1)
+                    if (__shfl_sync(0xffffffffu, incl, sj + step - 1) <= e) sj += step;
+                const uint32_t first = __shfl_sync(0xffffffffu, excl, sj);
+                if (e < E) {
+                    const TouchSeg &g = sg[sj];
+                    const Deferred en = d.defer[uint64_t(c0 + sj) * kSegBlocks + (e - first)];
+                    // the slot as the touch saw it last (another key: any value
+                    // other than 0 and the key)
+                    const Slot old = en.found ? Slot{en.key, en.x} : Slot{en.key == 1 ? 2ull : en.key ^ 1ull, 0};
+                    bool cl = false;
+                    uint32_t nw = 0;
+                    const uint64_t o = touch_resolve(g.t, mask, en.key, en.p + 1, en.home, old, d.err, &cl,
+                                                     en.bucket, d.loop_limit);
+                    touch_outcome(o, en.p, g.front, g.st, lmask, nw);
+                    if (nw) atomicAdd(&add_n[sj], nw);
+                    if (cl) atomicAdd(&add_c[sj], 1u);
+                }
+            }
+            __syncwarp();
+            my_newly += add_n[lane];
+            my_claims += add_c[lane];
+        }
+        {   // keys made resident and index slots taken, per final instance:
+            // one atomic per instance for these 32 segments (mostly of one request)
+            const uint32_t fi = (uint32_t)lane < nc ? sg[lane].f : 0xffffffffu;
+            const uint32_t peers = __match_any_sync(0xffffffffu, fi);
+            const uint32_t sa = __reduce_add_sync(peers, my_newly), sb = __reduce_add_sync(peers, my_claims);
+            if ((uint32_t)lane < nc && lane == __ffs(peers) - 1) {
+                if (sa) atomicAdd(reinterpret_cast<unsigned long long *>(&d.live[fi]), (unsigned long long)sa);
+                if (sb) atomicAdd(reinterpret_cast<unsigned long long *>(&d.used[fi]), (unsigned long long)sb);
             }
         }
         __syncwarp();   // the slots are refilled for the next 32 segments
-    }
-}
-
-// Second pass over the deferred touches, a warp per segment: raise the
-// position of a found key (atomic max), or walk the probe order of a key
-// whose home slot holds another key.  Every record still ends up marked
-// stale exactly once unless it is its key's latest: the first pass settled
-// only touches whose outcome its own atomic fixed (a claim of an empty slot,
-// a raise, a later position already there), and the maxima taken here order
-// the rest.
-__global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
-    pdl_enter();
-    if (has_err(d.err)) return;
-    const int lane = threadIdx.x & 31;
-    const uint32_t nw = (gridDim.x * blockDim.x) >> 5;
-    const uint32_t total_segs = d.info->total_segs;
-    const uint64_t mask = d.S - 1, lmask = d.logcap - 1;
-    for (uint32_t seg = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; seg < total_segs; seg += nw) {
-        const uint32_t n = d.defer_n[seg];
-        if (n == 0) continue;
-        uint32_t newly = 0, claims = 0;
-        for (uint32_t j = lane; j < n; j += 32) {
-            const Deferred e = d.defer[uint64_t(seg) * kSegBlocks + j];
-            // the home slot as the first pass saw it (another key: any value
-            // other than 0 and e.key)
-            const Slot old = e.found ? Slot{e.key, e.x} : Slot{e.key == 1 ? 2ull : e.key ^ 1ull, 0};
-            bool cl = false;
-            const uint64_t o =
-                touch_resolve(d.table[e.f], mask, e.key, e.p + 1, e.home, old, d.err, &cl, e.bucket, d.loop_limit);
-            touch_outcome(o, e.p, d.log_front[e.f], d.stale[e.f], lmask, newly);
-            claims += cl;
-        }
-        newly = __reduce_add_sync(0xffffffffu, newly);
-        claims = __reduce_add_sync(0xffffffffu, claims);
-        if (lane == 0) {   // this warp alone owns the segment's counters here
-            d.seg_newly[seg] += newly;
-            d.seg_claims[seg] += claims;
-        }
     }
 }
 
@@ -686,31 +706,7 @@ __global__ void __launch_bounds__(256) k_touch_deferred(DevState d) {
 // by moving its log front just past the excess_i-th non-stale record; the
 // stale flags it passes are reset (those positions will hold new records).
 // A cluster of CTAs walks an instance's log from the front (k_evict below);
-// first the touch passes' per-segment counts are summed per request.
-
-// Warp per request: sum the touch kernel's counts over the request's
-// (contiguous) segments, one atomic per request and counter.
-__global__ void k_req_counts(DevState d, uint32_t n) {
-    pdl_enter();
-    if (has_err(d.err)) return;
-    const int lane = threadIdx.x & 31;
-    const uint32_t r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (r >= n) return;
-    const uint32_t s0 = d.r_segoff[r];
-    const uint32_t ns = (d.r_nblk[r] + kSegBlocks - 1) / kSegBlocks;
-    uint32_t a = 0, b = 0;
-    for (uint32_t j = lane; j < ns; j += 32) {
-        a += d.seg_newly[s0 + j];
-        b += d.seg_claims[s0 + j];
-    }
-    a = __reduce_add_sync(0xffffffffu, a);
-    b = __reduce_add_sync(0xffffffffu, b);
-    if (lane == 0) {
-        const uint32_t f = d.r_final[r];
-        if (a) atomicAdd(reinterpret_cast<unsigned long long *>(&d.live[f]), (unsigned long long)a);
-        if (b) atomicAdd(reinterpret_cast<unsigned long long *>(&d.used[f]), (unsigned long long)b);
-    }
-}
+// the touch kernel has added the batch's newly resident keys to live_i.
 
 constexpr int kEvThreads = 1024;
 constexpr uint32_t kEvCluster = 4;                                // CTAs sharing one instance's walk
@@ -885,16 +881,13 @@ cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
         configured = smem;
     }
     static const int g_a = full_grid(k_maint_a, kMtThreads), g_c = full_grid(k_maint_c, kMtThreads),
-                     g_t = full_grid(k_commit_touch, kTouchThreads),
-                     g_d = full_grid(k_touch_deferred, 256), g_ev = evict_grid();
+                     g_t = full_grid(k_commit_touch, kTouchThreads), g_ev = evict_grid();
     DM_TRY(launch_pdl(k_maint_plan, 1, 1024, smem, st, d, n));
     DM_TRY(launch_pdl(k_maint_a, g_a, kMtThreads, 0, st, d));
     DM_TRY(launch_pdl(k_compact_scan, (d.M + 7) / 8, 256, 0, st, d));
     DM_TRY(launch_pdl(k_maint_c, g_c, kMtThreads, 0, st, d));
     DM_TRY(launch_pdl(k_commit_prep, 1, 1024, smem, st, d, n));
     DM_TRY(launch_pdl(k_commit_touch, g_t, kTouchThreads, 0, st, d));
-    DM_TRY(launch_pdl(k_touch_deferred, g_d, 256, 0, st, d));
-    DM_TRY(launch_pdl(k_req_counts, (n + 7) / 8, 256, 0, st, d, n));
     DM_TRY(launch_pdl(k_evict, g_ev, kEvThreads, 0, st, d));
     return cudaGetLastError();
 }

@@ -119,14 +119,15 @@ struct Rec {
     uint64_t key, stamp;
 };
 
-// A touch the commit's first pass could not settle (40 bytes): the key is at
-// its home slot with an older position (found = 1, x = the position value
-// seen last) or the preferred slot of bucket `bucket` of its probe order (0:
-// the home bucket) holds another key (found = 0).  The second pass finishes
-// it from there.
+// A touch that the commit's first atomics did not settle (32 bytes): the
+// preferred slot of bucket `bucket` of the key's probe order (0: the home
+// bucket) holds the key with an older position (found = 1, x = the position
+// value seen last) or another key (found = 0).  The touch kernel finishes it
+// from there at the end of its 32 segments.
 struct Deferred {
     uint64_t key, p, x;     // p: log position of the touch's record
-    uint32_t home, f, found, bucket;
+    uint32_t home;
+    uint16_t found, bucket;
 };
 
 // One node count of the adaptive prefix tree's current window (16 bytes):
@@ -261,9 +262,7 @@ struct DevState {
     uint64_t *p2local;              // adaptive only: per block < Kf2, in-segment prefix of its f2 digests
     uint32_t *r_K;                  // per request: the hash prefix length it was routed with
     uint64_t *seg_total2;           // per segment: f2 digest sum over its blocks < K
-    uint32_t *seg_newly, *seg_claims;   // per segment: keys made resident / index slots taken by the commit
-    Deferred *defer;                // kSegBlocks per segment: touches left to the commit's second pass
-    uint32_t *defer_n;              // per segment: deferred touches
+    Deferred *defer;                // kSegBlocks per segment: touches the commit's first atomics left open
     uint32_t *r_c1, *r_c2, *r_final;
     uint64_t *r_touchoff;           // per request: offset among its instance's records of the batch
     uint64_t *log_adv;              // per id: log records the pending batch appends
