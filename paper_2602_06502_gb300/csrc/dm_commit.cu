@@ -25,7 +25,7 @@ namespace cg = cooperative_groups;
 namespace dm {
 
 constexpr int kMtThreads = 256;
-constexpr uint32_t kPrepChunk = 2048;
+constexpr uint32_t kPrepChunk = 1024;
 constexpr uint32_t kFlagCompact = 1, kFlagRebuild = 2;
 constexpr uint32_t kZeroChunk = 4096;   // slots or flag bytes cleared per chunk
 
@@ -172,12 +172,17 @@ __device__ __forceinline__ uint32_t owner_of(const uint32_t *off, uint32_t M, ui
 //         compaction (log would overflow) or a rebuild (index would pass half
 //         full), and the chunk lists of both;
 //   a     grid: clear the second index (rebuild) / stale flags (compaction),
-//         count live records per 1024-record chunk of the log;
-//   scan  warp per compacting instance: chunk counts -> destination offsets;
+//         count live records per 1024-record chunk of the log; the last CTA
+//         to finish turns the counts into destination offsets (a warp per
+//         compacting instance);
 //   c     grid: walk the live records; compaction copies them in order into
 //         the second log (and repoints their index slots, or inserts them
 //         into the second index when rebuilding too); a rebuild alone
-//         inserts them with their current positions.
+//         inserts them with their current positions.  The last CTA to
+//         finish (CTA 0 when there was nothing to walk) swaps the new logs
+//         and indices in and lays out the commit's records.
+// Kernels a and c do nothing else when the plan asks for no maintenance, the
+// usual case; "last CTA" is an atomic count of finished CTAs, no CTA waits.
 
 __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
     pdl_enter();
@@ -261,7 +266,42 @@ __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
         d.mr_chunk_off[d.M] = cz;
         d.info->mc_chunks = cw;
         d.info->mr_chunks = cz;
+        d.info->mt_done_a = 0;
+        d.info->mt_done_c = 0;
         if (cw > d.mc_cap) set_err(d.err, DM_ERR_CAPACITY);
+    }
+}
+
+// True in the one CTA of the grid that finishes last (count: a counter the
+// plan kernel zeroed).  Called by all threads of every CTA that gets here.
+__device__ __forceinline__ bool last_cta(uint32_t *count) {
+    __shared__ uint32_t s_last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        s_last = atomicAdd(count, 1u) + 1 == gridDim.x;
+    }
+    __syncthreads();
+    if (s_last) __threadfence();
+    return s_last != 0;
+}
+
+// Warp per compacting instance: chunk counts -> exclusive destination
+// offsets (the counts of other CTAs are read from L2).
+__device__ void compact_scan_cta(const DevState &d) {
+    const int lane = threadIdx.x & 31;
+    for (uint32_t i = threadIdx.x >> 5; i < d.M; i += blockDim.x >> 5) {
+        if (!(d.mt_flags[i] & kFlagCompact)) continue;
+        const uint32_t c0 = d.mc_chunk_off[i], c1 = d.mc_chunk_off[i + 1];
+        uint64_t carry = 0;
+        for (uint32_t cb = c0; cb < c1; cb += 32) {
+            const uint32_t c = cb + lane;
+            const uint64_t v = c < c1 ? __ldcg(&d.mc_chunk_live[c]) : 0;
+            const uint64_t inc = warp_incl_scan(v, lane);
+            if (c < c1) d.mc_chunk_live[c] = (uint32_t)(carry + inc - v);
+            carry += shfl_u64(inc, 31);
+        }
+        if (lane == 0) d.mt_newtail[i] = d.log_front[i] + carry;
     }
 }
 
@@ -315,29 +355,16 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
         }
         __syncthreads();
     }
+    if (nw && last_cta(&d.info->mt_done_a)) compact_scan_cta(d);
 }
 
-// Warp per compacting instance: chunk counts -> exclusive destination offsets.
-__global__ void k_compact_scan(DevState d) {
-    pdl_enter();
-    if (has_err(d.err)) return;
-    const int lane = threadIdx.x & 31;
-    const uint32_t i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (i >= d.M || !(d.mt_flags[i] & kFlagCompact)) return;
-    const uint32_t c0 = d.mc_chunk_off[i], c1 = d.mc_chunk_off[i + 1];
-    uint64_t carry = 0;
-    for (uint32_t cb = c0; cb < c1; cb += 32) {
-        const uint32_t c = cb + lane;
-        const uint64_t v = c < c1 ? d.mc_chunk_live[c] : 0;
-        const uint64_t inc = warp_incl_scan(v, lane);
-        if (c < c1) d.mc_chunk_live[c] = (uint32_t)(carry + inc - v);
-        carry += shfl_u64(inc, 31);
-    }
-    if (lane == 0) d.mt_newtail[i] = d.log_front[i] + carry;
-}
+__device__ void commit_prep_cta(const DevState &d, uint32_t n, uint64_t *adv);
 
-__global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
+// n: requests of the batch (for the record layout); dynamic smem: one u64
+// per instance.
+__global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d, uint32_t n) {
     pdl_enter();
+    extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_i, s_w[kMtThreads / 32];
     if (has_err(d.err)) return;
     const uint32_t nw = d.info->mc_chunks;
@@ -381,6 +408,8 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
             __syncthreads();
         }
     }
+    if (nw ? last_cta(&d.info->mt_done_c) : blockIdx.x == 0)
+        commit_prep_cta(d, n, reinterpret_cast<uint64_t *>(smem));
 }
 
 // ---------------------------------------------------------------------------
@@ -388,14 +417,11 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_c(DevState d) {
 // this commit and advance its tail.  The choice kernel already placed every
 // request among its instance's records; only when a rebalance moved a
 // request of this batch are the offsets recomputed (arrival order per final
-// instance).  Single CTA; dynamic smem holds one u64 per instance.
-__global__ void __launch_bounds__(1024) k_commit_prep(DevState d, uint32_t n) {
-    pdl_enter();
-    extern __shared__ __align__(16) unsigned char smem[];
+// instance).  One CTA, after every CTA of k_maint_c; adv: one u64 per
+// instance in shared memory.
+__device__ void commit_prep_cta(const DevState &d, uint32_t n, uint64_t *adv) {
     __shared__ uint32_t s_f[kPrepChunk], s_nb[kPrepChunk];
     __shared__ uint64_t s_off[kPrepChunk];
-    if (has_err(d.err)) return;
-    uint64_t *adv = reinterpret_cast<uint64_t *>(smem);
     for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
         const uint32_t fl = d.mt_flags[i];
         if (fl & kFlagCompact) {
@@ -873,7 +899,7 @@ cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
     const size_t smem = sizeof(uint64_t) * d.M;
     static size_t configured = 0;
     if (smem > configured) {
-        cudaError_t e = cudaFuncSetAttribute(k_commit_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(k_maint_c, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(k_maint_plan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 
@@ -884,9 +910,7 @@ cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
                      g_t = full_grid(k_commit_touch, kTouchThreads), g_ev = evict_grid();
     DM_TRY(launch_pdl(k_maint_plan, 1, 1024, smem, st, d, n));
     DM_TRY(launch_pdl(k_maint_a, g_a, kMtThreads, 0, st, d));
-    DM_TRY(launch_pdl(k_compact_scan, (d.M + 7) / 8, 256, 0, st, d));
-    DM_TRY(launch_pdl(k_maint_c, g_c, kMtThreads, 0, st, d));
-    DM_TRY(launch_pdl(k_commit_prep, 1, 1024, smem, st, d, n));
+    DM_TRY(launch_pdl(k_maint_c, g_c, kMtThreads, smem, st, d, n));
     DM_TRY(launch_pdl(k_commit_touch, g_t, kTouchThreads, 0, st, d));
     DM_TRY(launch_pdl(k_evict, g_ev, kEvThreads, 0, st, d));
     return cudaGetLastError();

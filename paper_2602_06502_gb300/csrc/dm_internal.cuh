@@ -166,6 +166,8 @@ struct BatchInfo {
     uint32_t both_over;     // a request of this batch estimated TTFT > SLO on both candidates
     uint32_t fix_n;         // routing: entries of the last CTA's list
     uint32_t cta_done;      // routing: CTAs of the routing kernel that finished
+    uint32_t mt_done_a;     // commit: CTAs of k_maint_a that finished
+    uint32_t mt_done_c;     // commit: CTAs of k_maint_c that finished
 };
 
 struct Ring {
