@@ -439,11 +439,11 @@ def main():
     met, _ = D.dm_get_metrics(g.h)
     stage_ms = {k: v[0] / max(v[1], 1) for k, v in st_all.items()}
     # route: setup (with the queue drain), hash + ring lookup + probes (one
-    # kernel), choice (with the segment carries) (3); commit: maint_plan,
-    # maint_a, compact_scan, maint_c, commit_prep, commit_touch,
-    # touch_deferred, req_counts, evict (9); rebalance (1)
+    # kernel), choice (with the segment carries) (3); commit: maint_a (with
+    # the maintenance plan), maint_c (with the commit prep), commit_touch,
+    # evict (4); rebalance (1)
     # (the cluster-wide rules add the carries and the all-instance probe kernels)
-    launches_per_step = 3 + 9 + (1 if w.get("rebalance") else 0) + (2 if rule >= D.DM_RULE_LEAST_LOADED else 0)
+    launches_per_step = 3 + 4 + (1 if w.get("rebalance") else 0) + (2 if rule >= D.DM_RULE_LEAST_LOADED else 0)
     if args.adapt:   # window end: the update kernel, once per window
         launches_per_step += 1.0 / kw["adapt_window"]
     clocks = sampler.summary(wall0, wall1)

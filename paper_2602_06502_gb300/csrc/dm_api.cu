@@ -366,7 +366,6 @@ dm_status dm_create(const dm_config *cfg, dm_handle **out) {
     A(dalloc(h, &d.log_tail, M));
     A(dalloc(h, &d.live, M));
     A(dalloc(h, &d.used, M));
-    A(dalloc(h, &d.touch_cnt, M));
     A(dalloc(h, &d.log_adv, M));
     A(dalloc(h, &d.log_base, M));
     A(dalloc(h, &d.clock, 1));

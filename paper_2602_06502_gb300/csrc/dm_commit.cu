@@ -168,9 +168,11 @@ __device__ __forceinline__ uint32_t owner_of(const uint32_t *off, uint32_t M, ui
 
 // ---------------------------------------------------------------------------
 // Maintenance before the touches.
-//   plan  one CTA: blocks each instance receives, which instances need a
-//         compaction (log would overflow) or a rebuild (index would pass half
-//         full), and the chunk lists of both;
+//   plan  blocks each instance receives, which instances need a compaction
+//         (log would overflow) or a rebuild (index would pass half full),
+//         and the chunk lists of both: every CTA of kernel a computes the
+//         same plan from the same inputs in its shared memory, CTA 0 also
+//         stores it for the kernels after;
 //   a     grid: clear the second index (rebuild) / stale flags (compaction),
 //         count live records per 1024-record chunk of the log; the last CTA
 //         to finish turns the counts into destination offsets (a warp per
@@ -184,67 +186,98 @@ __device__ __forceinline__ uint32_t owner_of(const uint32_t *off, uint32_t M, ui
 // Kernels a and c do nothing else when the plan asks for no maintenance, the
 // usual case; "last CTA" is an atomic count of finished CTAs, no CTA waits.
 
-__global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
-    pdl_enter();
-    extern __shared__ __align__(16) unsigned char smem[];
+// The plan in shared memory (dynamic, plan_smem(M) bytes).
+struct PlanSm {
+    uint64_t *cnt;       // M: blocks each instance receives
+    uint32_t *fl;        // M: kFlagCompact | kFlagRebuild
+    uint32_t *mc, *mr;   // M + 1: chunk offsets of the log walk and of the clearing
+    uint32_t *rk;        // M: pool slot of a rebuilding instance
+};
+__device__ __forceinline__ PlanSm plan_sm(unsigned char *smem, uint32_t M) {
+    PlanSm p;
+    p.cnt = reinterpret_cast<uint64_t *>(smem);
+    p.fl = reinterpret_cast<uint32_t *>(p.cnt + M);
+    p.mc = p.fl + M;
+    p.mr = p.mc + M + 1;
+    p.rk = p.mr + M + 1;
+    return p;
+}
+static size_t plan_smem(uint32_t M) { return size_t(M) * 24 + 8; }
+
+// The plan, computed by a whole CTA; `store`: also write it to global
+// memory (flags, chunk offsets, pool slots and buffers, the rotation start
+// the commit prep installs, the counters of this commit).
+__device__ void maint_plan_cta(const DevState &d, uint32_t n, const PlanSm &P, bool store) {
     __shared__ uint32_t s_w[33];
-    if (has_err(d.err)) return;
-    unsigned long long *cntv = reinterpret_cast<unsigned long long *>(smem);
-    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) cntv[i] = 0;
+    __shared__ uint32_t s_served, s_last;
+    // blocks each instance receives: the choice kernel's count, unless a
+    // rebalance has moved a request of the batch since
+    const bool dirty = d.info->final_dirty != 0;
+    for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) P.cnt[i] = dirty ? 0 : d.log_adv[i];
     __syncthreads();
-    for (uint32_t r = threadIdx.x; r < n; r += blockDim.x)
-        atomicAdd(&cntv[d.r_final[r]], (unsigned long long)d.r_nblk[r]);
+    for (uint32_t r0 = threadIdx.x; dirty && r0 < n; r0 += 4 * blockDim.x) {   // four loads in flight per thread
+        uint32_t f[4], nb[4];
+#pragma unroll
+        for (uint32_t u = 0; u < 4; ++u) {
+            const uint32_t r = r0 + u * blockDim.x;
+            f[u] = r < n ? d.r_final[r] : 0;
+            nb[u] = r < n ? d.r_nblk[r] : 0;
+        }
+#pragma unroll
+        for (uint32_t u = 0; u < 4; ++u)
+            if (nb[u]) atomicAdd(reinterpret_cast<unsigned long long *>(&P.cnt[f[u]]), (unsigned long long)nb[u]);
+    }
     __syncthreads();
     // 1) what each instance needs: compaction if its log would overflow,
     //    a rebuild if its index would pass rb_thr taken slots
     for (uint32_t i = threadIdx.x; i < d.M; i += blockDim.x) {
         uint32_t fl = 0;
         if (d.table[i]) {
-            const uint64_t cnt = cntv[i];
+            const uint64_t cnt = P.cnt[i];
             if (cnt > d.T) set_err(d.err, DM_ERR_CAPACITY);
             if (d.log_tail[i] - d.log_front[i] + cnt > d.logcap) fl |= kFlagCompact;
             if (d.used[i] + cnt > d.rb_thr) fl |= kFlagRebuild;
-            d.touch_cnt[i] = cnt;
         }
-        d.mt_flags[i] = fl;
+        P.fl[i] = fl;
     }
+    if (threadIdx.x == 0) { s_served = 0; s_last = 0; }
     __syncthreads();
     // 2) rebuilds take spare buffers from the pool, in id order from a
     //    rotating start; those beyond the pool wait for a later commit (each
     //    waits at most ceil(M / pool) commits; dm_create checks the index
-    //    has that much headroom above half full)
-    __shared__ uint32_t s_served, s_last;
-    if (threadIdx.x == 0) { s_served = 0; s_last = 0; }
-    __syncthreads();
+    //    has that much headroom above half full).  The new start is
+    //    installed by the commit prep, after every CTA has read the old one.
     const uint32_t rr = *d.rb_rr;
     for (uint32_t base = 0; base < d.M; base += blockDim.x) {
         const uint32_t k = base + threadIdx.x;
         const uint32_t i = k < d.M ? (rr + k) % d.M : 0;
-        const bool want = k < d.M && (d.mt_flags[i] & kFlagRebuild);
+        const bool want = k < d.M && (P.fl[i] & kFlagRebuild);
         uint32_t tot;
         const uint32_t rank = s_served + block_excl_u32(want ? 1u : 0u, s_w, tot);
         if (want) {
             if (rank < d.pool_n) {
-                d.rb_slot[i] = rank;
-                d.table_alt[i] = d.pool[rank];
+                P.rk[i] = rank;
+                if (store) {
+                    d.rb_slot[i] = rank;
+                    d.table_alt[i] = d.pool[rank];
+                }
                 atomicMax(&s_last, k);   // the last position served
             } else {
-                d.mt_flags[i] &= ~kFlagRebuild;
+                P.fl[i] &= ~kFlagRebuild;
             }
         }
         __syncthreads();
         if (threadIdx.x == 0) s_served += tot;
         __syncthreads();
     }
-    if (threadIdx.x == 0 && s_served) *d.rb_rr = (rr + s_last + 1) % d.M;
-    __syncthreads();
+    if (store && threadIdx.x == 0) d.info->rb_rr_next = s_served ? (rr + s_last + 1) % d.M : rr;
     // 3) chunk offsets of the work the final flags ask for
     uint32_t cw = 0, cz = 0;
     for (uint32_t base = 0; base < d.M; base += blockDim.x) {
         const uint32_t i = base + threadIdx.x;
         uint32_t nw = 0, nz = 0, fl = 0;
         if (i < d.M && d.table[i]) {
-            fl = d.mt_flags[i];
+            fl = P.fl[i];
             const uint64_t len = d.log_tail[i] - d.log_front[i];
             if (fl & kFlagCompact) nz += (uint32_t)((d.logcap + kZeroChunk - 1) / kZeroChunk);
             if (fl & kFlagRebuild) nz += (uint32_t)((d.S + kZeroChunk - 1) / kZeroChunk);
@@ -254,22 +287,31 @@ __global__ void __launch_bounds__(1024) k_maint_plan(DevState d, uint32_t n) {
         const uint32_t ew = block_excl_u32(nw, s_w, tw);
         const uint32_t ez = block_excl_u32(nz, s_w, tz);
         if (i < d.M) {
-            d.mc_chunk_off[i] = cw + ew;
-            d.mr_chunk_off[i] = cz + ez;
-            d.mt_flags[i] = fl;
+            P.mc[i] = cw + ew;
+            P.mr[i] = cz + ez;
+            P.fl[i] = fl;
+            if (store) {
+                d.mc_chunk_off[i] = cw + ew;
+                d.mr_chunk_off[i] = cz + ez;
+                d.mt_flags[i] = fl;
+            }
         }
         cw += tw;
         cz += tz;
     }
     if (threadIdx.x == 0) {
-        d.mc_chunk_off[d.M] = cw;
-        d.mr_chunk_off[d.M] = cz;
-        d.info->mc_chunks = cw;
-        d.info->mr_chunks = cz;
-        d.info->mt_done_a = 0;
-        d.info->mt_done_c = 0;
-        if (cw > d.mc_cap) set_err(d.err, DM_ERR_CAPACITY);
+        P.mc[d.M] = cw;
+        P.mr[d.M] = cz;
+        if (store) {
+            d.mc_chunk_off[d.M] = cw;
+            d.mr_chunk_off[d.M] = cz;
+            d.info->mc_chunks = cw;
+            d.info->mr_chunks = cz;
+            d.info->mt_done_c = 0;
+            if (cw > d.mc_cap) set_err(d.err, DM_ERR_CAPACITY);
+        }
     }
+    __syncthreads();
 }
 
 // True in the one CTA of the grid that finishes last (count: a counter the
@@ -288,11 +330,11 @@ __device__ __forceinline__ bool last_cta(uint32_t *count) {
 
 // Warp per compacting instance: chunk counts -> exclusive destination
 // offsets (the counts of other CTAs are read from L2).
-__device__ void compact_scan_cta(const DevState &d) {
+__device__ void compact_scan_cta(const DevState &d, const PlanSm &P) {
     const int lane = threadIdx.x & 31;
     for (uint32_t i = threadIdx.x >> 5; i < d.M; i += blockDim.x >> 5) {
-        if (!(d.mt_flags[i] & kFlagCompact)) continue;
-        const uint32_t c0 = d.mc_chunk_off[i], c1 = d.mc_chunk_off[i + 1];
+        if (!(P.fl[i] & kFlagCompact)) continue;
+        const uint32_t c0 = P.mc[i], c1 = P.mc[i + 1];
         uint64_t carry = 0;
         for (uint32_t cb = c0; cb < c1; cb += 32) {
             const uint32_t c = cb + lane;
@@ -305,23 +347,27 @@ __device__ void compact_scan_cta(const DevState &d) {
     }
 }
 
-__global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
+// n: requests of the batch; dynamic smem: plan_smem(M) bytes.
+__global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d, uint32_t n) {
     pdl_enter();
+    extern __shared__ __align__(16) unsigned char smem[];
     __shared__ uint32_t s_i, s_cnt[kMtThreads / 32];
     if (has_err(d.err)) return;
+    const PlanSm P = plan_sm(smem, d.M);
+    maint_plan_cta(d, n, P, blockIdx.x == 0);
     // clearing: a rebuilding instance's chunks cover its second index first,
     // a compacting instance's (then) its second stale-flag array
-    const uint32_t nz = d.info->mr_chunks;
+    const uint32_t nz = P.mr[d.M];
     for (uint32_t c = blockIdx.x; c < nz; c += gridDim.x) {
-        if (threadIdx.x == 0) s_i = owner_of(d.mr_chunk_off, d.M, c);
+        if (threadIdx.x == 0) s_i = owner_of(P.mr, d.M, c);
         __syncthreads();
         const uint32_t i = s_i;
-        const uint32_t fl = d.mt_flags[i];
-        uint64_t k = uint64_t(c - d.mr_chunk_off[i]) * kZeroChunk;
+        const uint32_t fl = P.fl[i];
+        uint64_t k = uint64_t(c - P.mr[i]) * kZeroChunk;
         const uint64_t tab = (fl & kFlagRebuild) ? d.S : 0;
         const uint64_t tab_chunks_end = (tab + kZeroChunk - 1) / kZeroChunk * kZeroChunk;
         if (k < tab_chunks_end) {
-            Slot *t = d.table_alt[i];
+            Slot *t = d.pool[P.rk[i]];
             for (uint32_t q = threadIdx.x; q < kZeroChunk; q += kMtThreads)
                 if (k + q < tab) t[k + q] = Slot{0, 0};
         } else {
@@ -332,15 +378,16 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
         }
         __syncthreads();
     }
-    // live records per log chunk of every instance being maintained
-    const uint32_t nw = d.info->mc_chunks;
+    // live records per log chunk of every instance being maintained (none
+    // when the chunk list would not fit: the plan has recorded the error)
+    const uint32_t nw = P.mc[d.M] <= d.mc_cap ? P.mc[d.M] : 0;
     const uint64_t lmask = d.logcap - 1;
     for (uint32_t c = blockIdx.x; c < nw; c += gridDim.x) {
-        if (threadIdx.x == 0) s_i = owner_of(d.mc_chunk_off, d.M, c);
+        if (threadIdx.x == 0) s_i = owner_of(P.mc, d.M, c);
         __syncthreads();
         const uint32_t i = s_i;
         const uint64_t tail = d.log_tail[i];
-        const uint64_t base = d.log_front[i] + uint64_t(c - d.mc_chunk_off[i]) * kEvChunk;
+        const uint64_t base = d.log_front[i] + uint64_t(c - P.mc[i]) * kEvChunk;
         const uint8_t *st = d.stale[i];
         uint32_t cnt = 0;
         for (uint32_t k = threadIdx.x; k < kEvChunk; k += kMtThreads)
@@ -355,7 +402,10 @@ __global__ void __launch_bounds__(kMtThreads) k_maint_a(DevState d) {
         }
         __syncthreads();
     }
-    if (nw && last_cta(&d.info->mt_done_a)) compact_scan_cta(d);
+    if (nw && last_cta(&d.info->mt_done_a)) {
+        compact_scan_cta(d, P);
+        if (threadIdx.x == 0) d.info->mt_done_a = 0;   // for the next commit
+    }
 }
 
 __device__ void commit_prep_cta(const DevState &d, uint32_t n, uint64_t *adv);
@@ -478,6 +528,7 @@ __device__ void commit_prep_cta(const DevState &d, uint32_t n, uint64_t *adv) {
     if (threadIdx.x == 0) {
         d.info->clock_base = *d.clock;
         *d.clock += d.info->total_blocks;
+        *d.rb_rr = d.info->rb_rr_next;
     }
 }
 
@@ -896,21 +947,22 @@ static int evict_grid() {
 
 cudaError_t launch_commit(const DevState &d, uint32_t n, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
-    const size_t smem = sizeof(uint64_t) * d.M;
+    const size_t smem_a = plan_smem(d.M), smem_c = sizeof(uint64_t) * d.M;
     static size_t configured = 0;
-    if (smem > configured) {
-        cudaError_t e = cudaFuncSetAttribute(k_maint_c, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (smem_a > configured) {   // smem_a > smem_c
+        cudaError_t e = cudaFuncSetAttribute(k_maint_a, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_a);
         if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_maint_plan, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-
+            e = cudaFuncSetAttribute(k_maint_c, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_c);
         if (e != cudaSuccess) return e;
-        configured = smem;
+        configured = smem_a;
     }
-    static const int g_a = full_grid(k_maint_a, kMtThreads), g_c = full_grid(k_maint_c, kMtThreads),
-                     g_t = full_grid(k_commit_touch, kTouchThreads), g_ev = evict_grid();
-    DM_TRY(launch_pdl(k_maint_plan, 1, 1024, smem, st, d, n));
-    DM_TRY(launch_pdl(k_maint_a, g_a, kMtThreads, 0, st, d));
-    DM_TRY(launch_pdl(k_maint_c, g_c, kMtThreads, smem, st, d, n));
+    // every CTA of k_maint_a reads the whole batch for its plan: two per SM
+    static const int g_a = full_grid(k_maint_a, kMtThreads) < 2 * sm_count() ? full_grid(k_maint_a, kMtThreads)
+                                                                                : 2 * sm_count(),
+                     g_c = full_grid(k_maint_c, kMtThreads), g_t = full_grid(k_commit_touch, kTouchThreads),
+                     g_ev = evict_grid();
+    DM_TRY(launch_pdl(k_maint_a, g_a, kMtThreads, smem_a, st, d, n));
+    DM_TRY(launch_pdl(k_maint_c, g_c, kMtThreads, smem_c, st, d, n));
     DM_TRY(launch_pdl(k_commit_touch, g_t, kTouchThreads, 0, st, d));
     DM_TRY(launch_pdl(k_evict, g_ev, kEvThreads, 0, st, d));
     return cudaGetLastError();

@@ -168,6 +168,7 @@ struct BatchInfo {
     uint32_t cta_done;      // routing: CTAs of the routing kernel that finished
     uint32_t mt_done_a;     // commit: CTAs of k_maint_a that finished
     uint32_t mt_done_c;     // commit: CTAs of k_maint_c that finished
+    uint32_t rb_rr_next;    // commit: rotation start of the rebuild order after this commit
 };
 
 struct Ring {
@@ -229,7 +230,6 @@ struct DevState {
     uint8_t **stale_alt;
     uint32_t **loghome_alt;
     uint64_t *log_front, *log_tail, *live, *used;
-    uint64_t *touch_cnt;            // per id: blocks touched by the pending commit
     // maintenance plan: per id flags / new log tail, chunk offsets and counts
     uint32_t *mt_flags;
     uint64_t *mt_newtail;
@@ -787,6 +787,14 @@ __device__ __forceinline__ void adaptive_positions(const DevState &d, uint32_t r
     pos1 = fmix64(P1K ^ d.Sr1);
     pos2 = fmix64(P2K ^ d.Sr2);
     Kout = K;
+}
+
+// Streaming multiprocessors of the current device.
+inline int sm_count() {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return sms > 0 ? sms : 1;
 }
 
 // Grid of a grid-stride kernel: every SM filled to the kernel's occupancy.
