@@ -414,6 +414,7 @@ def main():
     # duration is the whole hash+probe path of the metric
     achieved = bytes_per_launch / hash_avg_s / 1e9
     prompt_gbps = achieved
+    rebuilds, compactions = D.dm_get_maint_counts(g.h)   # over the warm-up and timed steps
 
     # per-stage breakdown: a fresh handle replays the same steps with every
     # stage timed (events between kernels stop their launch overlap, so this
@@ -513,6 +514,8 @@ def main():
                         "completed": met["completed"], "requests": met["requests"],
                         "note": "scheduler time model over the stage-breakdown replay"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": int(round(launches_per_step * K)), "clocks": clocks,
+            "maintenance": {"index_rebuilds": rebuilds, "log_compactions": compactions,
+                            "steps": W + K, "note": "commits of the headline run that rebuilt an index or compacted a log"},
         }
         print(json.dumps(line), flush=True)
     if world > 1:

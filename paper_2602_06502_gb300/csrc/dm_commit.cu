@@ -785,12 +785,10 @@ __global__ void __launch_bounds__(kTouchThreads, 4) k_commit_touch(DevState d) {
 // A cluster of CTAs walks an instance's log from the front (k_evict below);
 // the touch kernel has added the batch's newly resident keys to live_i.
 
-constexpr int kEvThreads = 1024;
+constexpr int kEvThreads = 512;
 constexpr uint32_t kEvCluster = 4;                                // CTAs sharing one instance's walk
-constexpr uint32_t kEvVec = 4;                                    // 16-byte flag loads per thread and round
-constexpr uint32_t kEvPer = 16 * kEvVec;                          // records per thread and round
-constexpr uint64_t kEvCtaSpan = uint64_t(kEvThreads) * kEvPer;    // records per CTA and round
-constexpr uint64_t kEvRound = kEvCtaSpan * kEvCluster;            // records per cluster and round
+constexpr uint32_t kEvVec = 4;                                    // 16-byte flag loads per thread and round, at most
+constexpr uint32_t kEvPer = 16 * kEvVec;                          // records per thread and round, at most
 
 // A cluster of kEvCluster CTAs per instance (persistent: clusters loop over
 // instances).  Per round each CTA counts the non-stale records of its own
@@ -840,14 +838,21 @@ __global__ void __cluster_dims__(kEvCluster, 1, 1) __launch_bounds__(kEvThreads)
         // front in the first round do not count
         uint64_t base = front & ~uint64_t(kEvPer - 1);
         for (uint64_t it = 0; remaining > 0 && base < tail && it < kSpinLimit; ++it) {
-            const uint64_t p0 = base + r * kEvCtaSpan + uint64_t(threadIdx.x) * kEvPer;
-            // records [lo, hi) of the thread's kEvPer are after the front and before the tail
-            const uint32_t lo = front > p0 ? (uint32_t)min(front - p0, (uint64_t)kEvPer) : 0u;
-            const uint32_t hi = tail > p0 ? (uint32_t)min(tail - p0, (uint64_t)kEvPer) : 0u;
+            // a round reads about twice the records still to evict (stale
+            // ones lie between them), 1-4 flag vectors per thread; the
+            // choice depends on `remaining` alone, the same in every CTA
+            const uint64_t vspan = uint64_t(kEvThreads) * kEvCluster * 16;
+            const uint64_t want = (2 * remaining + vspan - 1) / vspan;
+            const uint32_t vec = want >= kEvVec ? kEvVec : (want < 1 ? 1u : (uint32_t)want);
+            const uint32_t per = 16 * vec;
+            const uint64_t p0 = base + r * (uint64_t(kEvThreads) * per) + uint64_t(threadIdx.x) * per;
+            // records [lo, hi) of the thread's `per` are after the front and before the tail
+            const uint32_t lo = front > p0 ? (uint32_t)min(front - p0, (uint64_t)per) : 0u;
+            const uint32_t hi = tail > p0 ? (uint32_t)min(tail - p0, (uint64_t)per) : 0u;
             uint64_t live_bits = 0;
 #pragma unroll
             for (uint32_t k = 0; k < kEvVec; ++k) {
-                if (16 * k >= hi) continue;
+                if (k >= vec || 16 * k >= hi) continue;
                 const uint4 v = *reinterpret_cast<const uint4 *>(st + ((p0 + 16 * k) & lmask));
                 const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
@@ -911,7 +916,7 @@ __global__ void __cluster_dims__(kEvCluster, 1, 1) __launch_bounds__(kEvThreads)
                 }
             }
             remaining -= min(remaining, all);
-            base += kEvRound;
+            base += uint64_t(kEvThreads) * per * kEvCluster;
             front = min(base, tail);
         }
         if (r == 0 && threadIdx.x == 0) {
