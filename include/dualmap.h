@@ -449,9 +449,9 @@ DM_API dm_status dm_hash_prompts(dm_handle *h, const dm_batch *batch, uint64_t *
  * DM_NOALLOC_MAX_BLOCKS; device-side checks (prompt lengths and offsets, the
  * exact block count) are reported by the return value: every call
  * synchronises `stream` (a cudaStream_t, NULL = legacy default stream) and
- * reads the device error word back before returning.  The first call on each
- * device looks up the array's device address and should come before any
- * stream capture on that device; the address is kept for the life of the
+ * reads the device error word back before returning, so no call may be made
+ * while any stream on that device is capturing.  The first call on each
+ * device looks up the array's device address; the address is kept for the life of the
  * process, so after a cudaDeviceReset of a device the entry point must not be
  * called on that device again.  Every call uses the same array: calls whose
  * work overlaps on the GPU (other host threads, other streams) race and
