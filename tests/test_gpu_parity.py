@@ -136,11 +136,17 @@ def test_tiny_trace_parity(seed):
 
 def test_tiny_trace_with_rebalance_and_small_cache():
     """Eviction every batch, log compaction and index rebuilds (small C and
-    touch bound), rebalancing after every batch."""
+    touch bound), rebalancing after every batch: commits whose plan must
+    recount the blocks per instance because a rebalance moved a request of
+    the batch meet commits that compact or rebuild."""
+    from paper_2602_06502_gb300 import dualmap as D
     w = workload("tiny", n_requests=2000, batch=100, capacity=700, zipf_s=1.3, rho=1.2)
     tr = Trace(w)
     p = Pair(w, max_touch=2600)
     run_trace(p, tr, rebalance=True, state_every=5)
+    rebuilds, compactions = D.dm_get_maint_counts(p.gpu.h)
+    print(f"{p.n_migrations} migrations, {rebuilds} index rebuilds, {compactions} log compactions")
+    assert p.n_migrations > 0 and rebuilds + compactions > 0
 
 
 def test_multiturn_parity():
@@ -637,7 +643,8 @@ def test_rebuilds_share_a_one_buffer_pool():
 
 def test_eviction_of_more_than_one_round():
     """Each commit evicts about 327k records per instance, more than one
-    eviction round (4 CTAs x 65,536 records) covers."""
+    eviction round covers (a round reads 32k-128k records: four CTAs of 512
+    threads, 16-64 records each, sized to twice what is left to evict)."""
     rng = np.random.default_rng(22)
     w = _mk(n_instances=2, vnodes=16, capacity=1000, batch=80)
     p = Pair(w, max_instances=3, max_touch=1 << 20, max_batch_tokens=1 << 24)
