@@ -1560,7 +1560,7 @@ int or_debug_enqueue(or_state *s, uint32_t id, uint64_t seq, uint32_t L, uint32_
                      uint32_t h1, uint32_t h2, uint64_t work, uint64_t remaining)
 {
     if (id >= s->cfg.max_instances) return OR_ERR_INVALID_ARG;
-    q_entry e = {seq, L, c1, c2, h1, h2, work, remaining, 0, s->t_prev};
+    q_entry e = {seq, L, c1, c2, h1, h2, work, remaining, 0, s->t_prev, NULL, 0};
     int rc = q_push(&s->q[id], &e);
     if (!rc) s->W[id] += remaining;
     if (seq >= s->next_seq) s->next_seq = seq + 1;
