@@ -169,7 +169,8 @@ __device__ __forceinline__ uint32_t owner_of(const uint32_t *off, uint32_t M, ui
 // ---------------------------------------------------------------------------
 // Maintenance before the touches.
 //   plan  blocks each instance receives, which instances need a compaction
-//         (log would overflow) or a rebuild (index would pass half full),
+//         (log would overflow) or a rebuild (index would pass its rebuild
+//         threshold),
 //         and the chunk lists of both: every CTA of kernel a computes the
 //         same plan from the same inputs in its shared memory, CTA 0 also
 //         stores it for the kernels after;
