@@ -57,8 +57,8 @@ __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
 // Finish the touch of `key` at position value p1 (1 + log position), given
 // `old`, the result of CAS({0,0} -> {key, p1}) at its home slot.  An empty
 // slot was claimed by that CAS; a slot holding the key has its position
-// raised to p1 unless a larger one is already there (CAS loop: only a larger
-// value is written); a slot of another key moves on along the key's probe
+// raised to p1 unless a larger one is already there (a 64-bit atomic max on
+// the position word: the slot's key never changes); a slot of another key moves on along the key's probe
 // order, using a snapshot of the bucket to skip the slots other keys hold
 // (slots never empty again, so only empty or matching ones are candidates).
 // Every touch of a key follows the same order, so concurrent first touches
