@@ -14,7 +14,7 @@
 // key is resident iff that record is at or after the log front, so evicting
 // the k oldest keys is moving the front past the k-th non-stale record: no
 // per-key write at all.  Evicted keys keep their index slots until the index
-// passes half full, when it is rebuilt from the log's live records; a log
+// passes its rebuild threshold, when it is rebuilt from the log's live records; a log
 // about to overflow is compacted.  Both write into second buffers and swap.
 #include <cooperative_groups.h>
 
@@ -29,16 +29,16 @@ constexpr uint32_t kPrepChunk = 1024;
 constexpr uint32_t kFlagCompact = 1, kFlagRebuild = 2;
 constexpr uint32_t kZeroChunk = 4096;   // slots or flag bytes cleared per chunk
 
-// 16-byte compare-and-swap of a whole index slot; returns its previous
-// contents.  Every slot update of the touch passes goes through this, so key
-// and position change together and never tear (whole-bucket reads are plain
-// 16-byte loads used only to pick the next slot to try).
 // Raise the position word of a slot whose key is set (keys never change once
 // set, and positions only grow): returns the value it had before.
 __device__ __forceinline__ uint64_t pos_max(Slot *s, uint64_t p1) {
     return atomicMax(reinterpret_cast<unsigned long long *>(&s->pos1), (unsigned long long)p1);
 }
 
+// 16-byte compare-and-swap of a whole index slot; returns its previous
+// contents.  Every claim of a slot by the touch kernel goes through this, so
+// key and position are set together and never tear (whole-bucket reads are
+// plain 16-byte loads used only to pick the next slot to try).
 __device__ __forceinline__ Slot slot_cas(Slot *s, Slot expect, Slot desired) {
     Slot old;
     asm volatile(
