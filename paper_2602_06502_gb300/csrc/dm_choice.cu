@@ -201,6 +201,9 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
                 const int64_t thr = valid ? S.thr[k] : 0;
                 const bool tieb = (ab >> 30) & 1u;
                 const uint64_t xa = (ab >> 31) ? ua : 0, xb = (ab >> 31) ? ub : 0;
+                const uint64_t inc = valid ? (uint64_t(S.nb[k]) << 32) + 1 : 0;   // PT step of this request
+                uint64_t oWa = 0, oWb = 0, oP = 0;   // the lane's decision, stored once the window is done
+                bool opb = false;
                 uint32_t done = __ballot_sync(0xffffffffu, !valid);
                 while (done != 0xffffffffu) {
                     const bool ready = !((done >> lane) & 1u) && (conf & ~done) == 0;
@@ -216,14 +219,20 @@ __global__ void __launch_bounds__(1024) k_choice(DevState d, dm_route_out o, uin
                         const uint32_t ch = pb ? b : a;
                         const uint64_t Pold = pb ? Pb : Pa;
                         W[ch] = pb ? Wb + ub : Wa + ua;
-                        PT[ch] = Pold + (uint64_t(S.nb[k]) << 32) + 1;
-                        S.Wa[k] = Wa;
-                        S.Wb[k] = Wb;
-                        S.pt[k] = Pold;
-                        S.pickb[k] = pb;
+                        PT[ch] = Pold + inc;
+                        oWa = Wa;
+                        oWb = Wb;
+                        oP = Pold;
+                        opb = pb;
                     }
                     __syncwarp();
                     done |= __ballot_sync(0xffffffffu, ready);
+                }
+                if (valid) {
+                    S.Wa[k] = oWa;
+                    S.Wb[k] = oWb;
+                    S.pt[k] = oP;
+                    S.pickb[k] = opb;
                 }
             }
         }
