@@ -1,6 +1,7 @@
 """Multi-process logic of bench.py on CPU: replicas agree on the slowest
 rank's time through a gloo all-reduce, the job throughput aggregates all
-replicas, and the reference arm does no work on ranks other than 0."""
+replicas, the reference arm does no work on ranks other than 0, and on rank
+0 it routes exactly the steps it is given."""
 
 import os
 import subprocess
@@ -52,3 +53,16 @@ def test_reference_arm_other_ranks_exit_without_work():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2"],
                        env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_reference_arm_times_exactly_the_steps_it_is_given():
+    """The oracle arm routes exactly W warm-up and K timed whole batches (the
+    same steps as the GPU arm) and says so in its line."""
+    import json
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "3", "--warmup", "2"], capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads([l for l in r.stdout.splitlines() if l.startswith("{")][-1])
+    assert line["impl"] == "reference" and line["steps"] == 3 and line["warmup"] == 2
+    assert line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
