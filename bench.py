@@ -362,20 +362,35 @@ def main():
         probe_b = need[0]
         src = host["tok"][probe_b]
         dst = torch.empty_like(src, device=dev)
-        best = 0.0
-        for _ in range(5):
-            c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            c0.record()
-            dst.copy_(src, non_blocking=True)
-            c1.record()
-            torch.cuda.synchronize()
-            best = max(best, src.numel() * 4 / (c0.elapsed_time(c1) / 1e3) / 1e9)
+        def copy_gbps(a, reps):
+            out = []
+            for _ in range(reps):
+                c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                c0.record()
+                dst.copy_(a, non_blocking=True)
+                c1.record()
+                torch.cuda.synchronize()
+                out.append(a.numel() * 4 / (c0.elapsed_time(c1) / 1e3) / 1e9)
+            return out
+        probe = copy_gbps(src, 5)
+        best = max(probe)
+        # the loop uploads each pinned buffer once; a buffer pinned now and
+        # uploaded three times shows what a first upload costs
+        try:
+            fresh = torch.empty_like(src, pin_memory=True)
+            fresh.copy_(tokens[:fresh.numel()])
+            fresh_gbps = copy_gbps(fresh, 3)
+            del fresh
+        except Exception as ex:   # a diagnostic only
+            fresh_gbps = str(ex)[:200]
         del dst
         e2e_val = job_throughput(ne, te * 1e3, world)
         bound = best * 1e9 / (h2d / Ke) * (ne / Ke) * world
         e2e = {"value": e2e_val, "unit": "req/s", "h2d_bytes_per_step": h2d // Ke,
                "d2h_bytes_per_step": d2h // Ke, "steps": Ke, "h2d_pinned_GBps": best,
-               "h2d_bound_req_s": bound, "frac_of_h2d_bound": e2e_val / bound}
+               "h2d_bound_req_s": bound, "frac_of_h2d_bound": e2e_val / bound,
+               "h2d_probe_GBps": probe, "h2d_fresh_buffer_GBps": fresh_gbps,
+               "loop_upload_GBps": (h2d / Ke) / (te / Ke) / 1e9}
 
     # -- device-resident run -------------------------------------------------
     g = make_sched()
